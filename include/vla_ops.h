@@ -1,0 +1,48 @@
+/*
+ * vla_ops.h — single-kernel entry points of libvla.so, for checking one operation of the
+ * hot path at a time.  Same conventions as vla.h (device pointers, asynchronous on
+ * `cuda_stream`, host-checkable errors returned at once); each returns a vla_status.
+ */
+#ifndef VLA_OPS_H_
+#define VLA_OPS_H_
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* C[M, N] (f32, row stride ldc) = (A + A_lo)[M, K] · W[N, K]^T with A, A_lo, W bf16
+ * row-major (row strides lda, ldw elements, multiples of 8), fp32 accumulation on the tcgen05
+ * tensor cores.  A_lo may be NULL (then C = A · W^T); otherwise the activation is the
+ * unevaluated bf16 pair A + A_lo, the form in which the hot path feeds every projection.
+ * This is the contraction of every projection of the decoder layer (§3.1: the Llama-2
+ * backbone's q/k/v, o, gate/up and down projections).  `block_n` in {128, 256} is the output
+ * tile width; `splits` >= 1 splits K across CTAs (partials in `workspace`, f32
+ * [splits, M, N], required when splits > 1, then summed in a fixed order).
+ * Requires M, N, K >= 1. */
+int vla_op_gemm_bf16(const void* A, const void* A_lo, int lda, const void* W, int ldw, float* C,
+                     int ldc, int M, int N, int K, int block_n, int splits, float* workspace,
+                     void* cuda_stream);
+
+/* The fused action head (§3.1 action bins; Eq. 1 log-probs; Algorithm 1 f) on B given
+ * hidden states h (f32 [B, d], row stride ldh): RMSNorm with final_norm (bf16 [d], eps),
+ * logits z = y · head_rows^T (head_rows bf16 [256, d] = the last 256 lm_head rows), then the
+ * sampler of vla_decode_actions with uniforms (f32 [B, 256]) at `temperature`.
+ * forced (int32 [B] bin indices 0..255, or NULL) selects whose log-prob is returned.
+ * Outputs (device, [B]): bins_out int32 (sampled bin k), logprobs_out f32, actions_out f32,
+ * logits_out f32 [B, 256] (may be NULL).  status: device uint32 word, OR-ed with
+ * VLA_STATUS_* bits. */
+int vla_op_action_head(const float* h, int ldh, int B, int d, const void* final_norm,
+                       const void* head_rows, float eps, const float* uniforms,
+                       float temperature, const int32_t* forced, int32_t* bins_out,
+                       float* logprobs_out, float* actions_out, float* logits_out,
+                       uint32_t* status, void* cuda_stream);
+
+/* Number of SMs the kernels size their persistent grids for (device property). */
+int vla_op_num_sms(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* VLA_OPS_H_ */

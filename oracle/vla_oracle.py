@@ -25,7 +25,7 @@ Readings where the paper is silent (listed in the design notes with their reason
 action ids are the last 256 vocabulary ids in ascending bin order; bin k maps to the
 centre -1 + (2k+1)/256; sampling is restricted to the 256 bins; the log-prob is that of
 the tempered 256-way softmax; T = 0 means greedy with T = 1 log-probs; ties go to the
-lowest bin; Gumbel-max with caller-supplied uniforms u (clamped to [2^-25, 1-2^-25]);
+lowest bin; Gumbel-max with caller-supplied uniforms u (clamped to [2^-24, 1-2^-24], the fp32-representable ends of (0,1));
 RoPE is the rotate-half form with theta = 1e4; RMSNorm eps = 1e-6; the 7th action token's
 KV is written as the first row of the next turn's chunk.
 
@@ -43,8 +43,8 @@ import numpy as np
 import torch
 
 F64 = torch.float64
-U_MIN = 2.0 ** -25
-U_MAX = 1.0 - 2.0 ** -25
+U_MIN = 2.0 ** -24
+U_MAX = 1.0 - 2.0 ** -24
 
 
 @dataclass(frozen=True)
@@ -146,29 +146,64 @@ class Weights:
         return lw
 
 
-def layer_forward(shape: Shape, lw: dict, h, pos, k_cache, v_cache):
+def round_bf16(x: torch.Tensor) -> torch.Tensor:
+    """Round to the nearest bf16 value (attribution mode only)."""
+    return x.to(torch.float32).to(torch.bfloat16).to(F64)
+
+
+def round_bf16_pair(x: torch.Tensor) -> torch.Tensor:
+    """x -> hi + lo with hi = bf16(x), lo = bf16(x - hi) (attribution mode only)."""
+    hi = round_bf16(x)
+    return hi + round_bf16(x - hi)
+
+
+def round_f16(x: torch.Tensor) -> torch.Tensor:
+    """Round to the nearest fp16 value (attribution mode only)."""
+    return x.to(torch.float32).to(torch.float16).to(F64)
+
+
+def _same(x):
+    return x
+
+
+@dataclass(frozen=True)
+class Rounding:
+    """Where an implementation stores activations at reduced precision.  The oracle proper
+    uses EXACT (no rounding); the attribution mode mirrors the GPU path so that rounding
+    error can be told apart from bugs."""
+    act: object = _same   # GEMM input activations (norm outputs, attention output, SwiGLU)
+    q: object = _same     # queries after RoPE
+    kv: object = _same    # keys (after RoPE) and values as cached
+
+
+EXACT = Rounding()
+GPU_PATH = Rounding(act=round_bf16_pair, q=lambda x: x.to(torch.float32).to(F64), kv=round_f16)
+
+
+def layer_forward(shape: Shape, lw: dict, h, pos, k_cache, v_cache, rnd: Rounding = EXACT):
     """One decoder layer over the chunk rows h [n, d] at positions pos [n].
 
     k_cache / v_cache: [m, H, hd] post-RoPE keys / values already in the context
     (positions 0 .. m-1); returns (h_out, k_all, v_all) with the chunk appended.
+    `rnd` is EXACT for the oracle proper (attribution runs pass GPU_PATH).
     """
     n = h.shape[0]
     d, H, hd, F = shape.d_model, shape.n_heads, shape.head_dim, shape.d_ffn
-    y = rms_norm(h, lw["attn_norm"], shape.rms_eps)
+    y = rnd.act(rms_norm(h, lw["attn_norm"], shape.rms_eps))
     qkv = y @ lw["wqkv"].T
     q = qkv[:, 0:d].reshape(n, H, hd)
     k = qkv[:, d:2 * d].reshape(n, H, hd)
-    v = qkv[:, 2 * d:3 * d].reshape(n, H, hd)
-    q = apply_rope(q, pos, shape.rope_theta)
-    k = apply_rope(k, pos, shape.rope_theta)
+    v = rnd.kv(qkv[:, 2 * d:3 * d].reshape(n, H, hd))
+    q = rnd.q(apply_rope(q, pos, shape.rope_theta))
+    k = rnd.kv(apply_rope(k, pos, shape.rope_theta))
     k_all = torch.cat([k_cache, k], dim=0)
     v_all = torch.cat([v_cache, v], dim=0)
     k_pos = torch.arange(k_all.shape[0], dtype=torch.long)
-    o = causal_attention(q, k_all, v_all, pos, k_pos)
+    o = rnd.act(causal_attention(q, k_all, v_all, pos, k_pos))
     h = h + o.reshape(n, d) @ lw["wo"].T
-    y = rms_norm(h, lw["ffn_norm"], shape.rms_eps)
+    y = rnd.act(rms_norm(h, lw["ffn_norm"], shape.rms_eps))
     gu = y @ lw["w_gate_up"].T
-    h = h + (silu(gu[:, :F]) * gu[:, F:]) @ lw["w_down"].T
+    h = h + rnd.act(silu(gu[:, :F]) * gu[:, F:]) @ lw["w_down"].T
     return h, k_all, v_all
 
 
@@ -252,8 +287,11 @@ class Oracle:
     """
 
     def __init__(self, shape: Shape, weights: Dict[str, torch.Tensor], n_envs: int,
-                 cache_f64: bool = True):
+                 cache_f64: bool = True, rounding: Rounding = EXACT):
+        """rounding: EXACT for the oracle proper; attribution runs pass GPU_PATH (not the
+        parity gate) to separate rounding error from bugs."""
         self.shape = shape
+        self.rnd = rounding
         self.W = Weights(shape, weights, cache_f64)
         self.envs = [self._fresh() for _ in range(n_envs)]
 
@@ -281,7 +319,8 @@ class Oracle:
             lw = self.W.layer(l)
             for j, b in enumerate(env_ids):
                 e = self.envs[b]
-                hs[j], e.k[l], e.v[l] = layer_forward(sh, lw, hs[j], poss[j], e.k[l], e.v[l])
+                hs[j], e.k[l], e.v[l] = layer_forward(sh, lw, hs[j], poss[j], e.k[l], e.v[l],
+                                                      self.rnd)
         for b, x in zip(env_ids, chunks):
             e = self.envs[b]
             e.rows.extend(list(x))

@@ -1,0 +1,23 @@
+// Internal interface of the attention kernels (attention.cu).
+#pragma once
+#include "common.cuh"
+
+namespace vla {
+
+// A tile of up to 64 consecutive query rows of one env: packed rows row0 .. row0+nrows-1
+// at positions pos0 .. pos0+nrows-1.
+struct AttnTile {
+  int env, row0, nrows, pos0;
+};
+
+// q: f32 [rows, H*hd]; out: bf16 hi/lo pair [rows, H*hd]; keys from the fp16 cache of `layer`.
+int attn_chunk_launch(const float* q, bf16* out_hi, bf16* out_lo, const AttnTile* tiles,
+                      int n_tiles, KVLayout kv, int layer, int H, int hd, cudaStream_t stream);
+
+// One query per env row b (rows[b] gives env and position); key range split into chunks of
+// `chunk` keys; partials in part_o [B*H*S*hd] f32 and part_ml [B*H*S] (S = ceil(max_ctx/chunk)).
+int attn_decode_launch(const float* q, bf16* out_hi, bf16* out_lo, const RowInfo* rows, int B,
+                       int max_ctx, KVLayout kv, int layer, int H, int hd, int chunk,
+                       float* part_o, float2* part_ml, cudaStream_t stream);
+
+}  // namespace vla

@@ -1,0 +1,103 @@
+// Shared device/host helpers of libvla.so (sm_103a).
+#pragma once
+
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_fp16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "../../include/vla.h"
+
+namespace vla {
+
+using bf16 = __nv_bfloat16;
+using f16 = __half;  // KV-cache element type
+
+// ----------------------------------------------------------------------------- launch log
+// Every kernel launch goes through note_launch() so the handle can report how many of its
+// kernels ran (the host counter is per process; handles keep their own copy too).
+extern int64_t g_launch_count;
+inline void note_launch() { ++g_launch_count; }
+
+// ----------------------------------------------------------------------------- row info
+// One entry per row of a packed chunk: env, absolute position, source kind, source index.
+enum RowKind : int { ROW_VISUAL = 0, ROW_TEXT = 1, ROW_TOKEN = 2 };
+struct RowInfo {
+  int env, pos, kind, idx;
+};
+
+// KV cache geometry: [layer][env][2 (K,V)][H][cap][hd] fp16.
+struct KVLayout {
+  f16* base;          // whole cache
+  int64_t layer_stride;
+  int64_t env_stride;  // 2 * H * cap * hd
+  int64_t kv_stride;   // H * cap * hd (V follows K)
+  int64_t head_stride; // cap * hd
+  int cap;
+};
+
+// ----------------------------------------------------------------------------- bf16 helpers
+__device__ __forceinline__ float bf2f(bf16 x) { return __bfloat162float(x); }
+__device__ __forceinline__ bf16 f2bf(float x) { return __float2bfloat16_rn(x); }
+
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+  __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<uint32_t*>(&v);
+}
+__device__ __forceinline__ float2 unpack_bf16x2(uint32_t v) {
+  __nv_bfloat162 b = *reinterpret_cast<__nv_bfloat162*>(&v);
+  return __bfloat1622float2(b);
+}
+
+__device__ __forceinline__ uint32_t pack_f16x2(float lo, float hi) {
+  __half2 v = __floats2half2_rn(lo, hi);
+  return *reinterpret_cast<uint32_t*>(&v);
+}
+__device__ __forceinline__ float2 unpack_f16x2(uint32_t v) {
+  __half2 b = *reinterpret_cast<__half2*>(&v);
+  return __half22float2(b);
+}
+
+// A GEMM input activation x is stored as an unevaluated pair of bf16 values:
+// hi = bf16(x), lo = bf16(x - hi), so hi + lo carries ~16 mantissa bits.  The GEMM multiplies
+// both halves by the bf16 weights into one fp32 accumulator.
+__device__ __forceinline__ void split_bf16(float x, bf16& hi, bf16& lo) {
+  hi = __float2bfloat16_rn(x);
+  lo = __float2bfloat16_rn(x - __bfloat162float(hi));
+}
+// Packs two consecutive values into (hi pair, lo pair) words.
+__device__ __forceinline__ void split_pack2(float a, float b, uint32_t& hi, uint32_t& lo) {
+  bf16 ha, la, hb, lb;
+  split_bf16(a, ha, la);
+  split_bf16(b, hb, lb);
+  __nv_bfloat162 h2 = __halves2bfloat162(ha, hb), l2 = __halves2bfloat162(la, lb);
+  hi = *reinterpret_cast<uint32_t*>(&h2);
+  lo = *reinterpret_cast<uint32_t*>(&l2);
+}
+
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+__device__ __forceinline__ float warp_max(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+  return v;
+}
+
+__device__ __forceinline__ float silu_f(float x) { return x / (1.0f + expf(-x)); }
+
+}  // namespace vla
+
+// ----------------------------------------------------------------------------- host macros
+#define VLA_CUDA_TRY(expr)                                   \
+  do {                                                       \
+    cudaError_t _e = (expr);                                 \
+    if (_e != cudaSuccess) return ::vla::cuda_fail(_e, #expr); \
+  } while (0)
+
+namespace vla {
+int cuda_fail(cudaError_t e, const char* what);  // records the message, returns VLA_ERR_CUDA
+}

@@ -1,0 +1,813 @@
+// Host engine behind the C ABI of include/vla.h: KV cache and workspace ownership, chunk
+// bookkeeping for multi-turn trajectories, the 7-token decode loop and the teacher-forced
+// score pass.
+//
+// Paper mapping: Algorithm 1 (rollout phase: π_θ generates v_out, f extracts a_t, Eq. 1
+// sums token log-probs), §3.3 (a trajectory is one multi-turn context), Eq. 2 (the PPO
+// ratio re-scores stored actions), §3.5 (large-batch decoding on one inference GPU).
+#include <algorithm>
+#include <cmath>
+#include <cstdio>
+#include <cstring>
+#include <string>
+#include <vector>
+
+#include "../../include/vla.h"
+#include "../../include/vla_ops.h"
+#include "attention.h"
+#include "gemm.h"
+#include "misc.h"
+
+namespace vla {
+
+namespace {
+thread_local std::string t_err;  // last error of this thread (for calls without a handle)
+}
+
+int cuda_fail(cudaError_t e, const char* what) {
+  char buf[512];
+  snprintf(buf, sizeof(buf), "CUDA error %d (%s) at %s", static_cast<int>(e),
+           cudaGetErrorString(e), what);
+  t_err = buf;
+  return VLA_ERR_CUDA;
+}
+
+static int set_err(std::string* dst, int code, const std::string& msg) {
+  t_err = msg;
+  if (dst) *dst = msg;
+  return code;
+}
+
+static int query_num_sms() {
+  int dev = 0, n = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return 148;
+  if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0)
+    return 148;
+  return n;
+}
+
+// GEMM tiling / split-K plan for an M x N x K projection.
+struct Plan {
+  int block_n, splits;
+};
+static Plan plan_gemm(int M, int N, int K, int epi, int d, int num_sms) {
+  const int tiles_m = (M + 127) / 128;
+  int bn = 256;
+  if (epi == EPI_QKV && (d % 256)) bn = 128;
+  const int n_eff = (epi == EPI_SWIGLU) ? N / 2 : N;
+  const int bn_eff = (epi == EPI_SWIGLU) ? bn / 2 : bn;
+  int64_t units = static_cast<int64_t>(tiles_m) * ((n_eff + bn_eff - 1) / bn_eff);
+  if (units >= num_sms) return {bn, 1};
+  // Few tiles (decode-sized M): narrower tiles and split-K so every SM streams weights.
+  bn = 128;
+  units = static_cast<int64_t>(tiles_m) * ((N + bn - 1) / bn);
+  const int kbt = (K + 63) / 64;
+  int splits = static_cast<int>((num_sms + units / 2) / units);
+  splits = std::max(1, std::min(splits, kbt / 2));
+  if (splits == 1 && units < num_sms) {
+    // keep the fused epilogue when split-K would not help
+    bn = 128;
+    if (epi == EPI_QKV && (d % 128)) bn = 256;
+  }
+  return {bn, splits};
+}
+
+struct EventPair {
+  cudaEvent_t a, b;
+  int cls;
+};
+
+}  // namespace vla
+
+using namespace vla;
+
+struct vla_handle {
+  vla_config cfg{};
+  int dev = 0;
+  cudaStream_t stream = nullptr;
+  int num_sms = 148;
+  int max_tokens = 0;
+  // borrowed weights
+  const bf16* embed = nullptr;
+  std::vector<const bf16*> attn_norm, wqkv, wo, ffn_norm, wgu, wdown;
+  const bf16* final_norm = nullptr;
+  const bf16* head_rows = nullptr;
+  // owned device memory
+  f16* kv = nullptr;      // KV cache [L][B][2][H][cap][hd] fp16
+  KVLayout kvl{};
+  float* h = nullptr;    // residual stream f32 [T, d]
+  bf16* y = nullptr;     // RMSNorm output, bf16 pair: hi [T, d] then lo [T, d]
+  float* q = nullptr;    // RoPE'd queries f32 [T, d]
+  bf16* ao = nullptr;    // attention output, bf16 pair [2][T, d]
+  bf16* u = nullptr;     // SwiGLU output, bf16 pair [2][T, F]
+  float* ws = nullptr;
+  size_t ws_bytes = 0;
+  float* h_last = nullptr;
+  float* head_in = nullptr;
+  float2* rope = nullptr;
+  RowInfo* rows = nullptr;
+  AttnTile* tiles = nullptr;
+  int* sidx = nullptr;
+  int* didx = nullptr;
+  int* fed = nullptr;
+  int* pending = nullptr;
+  uint32_t* status = nullptr;
+  float* part_o = nullptr;
+  float2* part_ml = nullptr;
+  int attn_chunk = 256;
+  int max_tiles = 0;
+  // pinned host staging (ring of slots, each guarded by an event)
+  static constexpr int kSlots = 4;
+  void* stage_host[kSlots] = {};
+  cudaEvent_t stage_ev[kSlots] = {};
+  size_t stage_bytes = 0;
+  int stage_next = 0;
+  // host state per env
+  std::vector<int> len, len_prefill;
+  std::vector<uint8_t> has_pending, prefilled;
+  int active_batch = 0;
+  std::string err;
+  // measurement
+  uint32_t prof_mask = 0;
+  std::vector<EventPair> ev_used, ev_free;
+  int64_t prof_launches[VLA_KCLASS_COUNT] = {};
+  double prof_ms[VLA_KCLASS_COUNT] = {};
+  double prof_flops[VLA_KCLASS_COUNT] = {};
+  double prof_bytes[VLA_KCLASS_COUNT] = {};
+  int64_t launches_at_create = 0;
+};
+
+namespace vla {
+namespace {
+
+int fail(vla_handle* h, int code, const std::string& msg) { return set_err(h ? &h->err : nullptr, code, msg); }
+
+// Returns a pinned staging slot whose previous upload has completed.
+void* stage_slot(vla_handle* h, int* slot) {
+  const int s = h->stage_next;
+  h->stage_next = (s + 1) % vla_handle::kSlots;
+  cudaEventSynchronize(h->stage_ev[s]);
+  *slot = s;
+  return h->stage_host[s];
+}
+
+int upload(vla_handle* h, void* dst, const void* src_host, size_t bytes) {
+  if (!bytes) return VLA_OK;
+  VLA_CUDA_TRY(cudaMemcpyAsync(dst, src_host, bytes, cudaMemcpyHostToDevice, h->stream));
+  return VLA_OK;
+}
+
+// ---- measurement helpers
+// Returns the index of the event pair bracketing the next launch, or -1 when class `cls`
+// is not being timed.
+int prof_begin(vla_handle* h, int cls) {
+  if (!(h->prof_mask & (1u << cls))) return -1;
+  if (h->ev_free.empty()) {
+    EventPair e{};
+    if (cudaEventCreate(&e.a) != cudaSuccess || cudaEventCreate(&e.b) != cudaSuccess) return -1;
+    h->ev_free.push_back(e);
+  }
+  h->ev_used.push_back(h->ev_free.back());
+  h->ev_free.pop_back();
+  EventPair& p = h->ev_used.back();
+  p.cls = cls;
+  cudaEventRecord(p.a, h->stream);
+  return static_cast<int>(h->ev_used.size()) - 1;
+}
+void prof_end(vla_handle* h, int ev, int cls, double flops, double bytes) {
+  h->prof_launches[cls] += 1;
+  h->prof_flops[cls] += flops;
+  h->prof_bytes[cls] += bytes;
+  if (ev >= 0) cudaEventRecord(h->ev_used[ev].b, h->stream);
+}
+void prof_harvest(vla_handle* h) {
+  cudaStreamSynchronize(h->stream);
+  for (auto& e : h->ev_used) {
+    float ms = 0.f;
+    if (cudaEventElapsedTime(&ms, e.a, e.b) == cudaSuccess) h->prof_ms[e.cls] += ms;
+    h->ev_free.push_back(e);
+  }
+  h->ev_used.clear();
+}
+
+// A is the bf16 hi/lo pair: hi at A, lo at A + a_plane.
+int run_gemm(vla_handle* h, int cls, const bf16* A, size_t a_plane, int lda, const bf16* W, int ldw,
+             int M, int N, int K, EpiArgs epi) {
+  const Plan pl = plan_gemm(M, N, K, epi.kind, h->cfg.d_model, h->num_sms);
+  GemmArgs g;
+  g.A = A;
+  g.A_lo = A + a_plane;
+  g.lda = lda;
+  g.B = W;
+  g.ldb = ldw;
+  g.M = M;
+  g.N = N;
+  g.K = K;
+  g.block_n = pl.block_n;
+  g.splits = pl.splits;
+  g.workspace = h->ws;
+  g.workspace_bytes = h->ws_bytes;
+  epi.status = h->status;
+  g.epi = epi;
+  if (gemm_workspace_bytes(g) > h->ws_bytes) {
+    g.splits = 1;
+  }
+  if (h->ev_used.size() > 8192) prof_harvest(h);
+  int ev = prof_begin(h, cls);
+  GemmCost cost{0, 0};
+  const int rc = gemm_launch(g, h->stream, h->num_sms, &cost);
+  prof_end(h, ev, cls, cost.flops, cost.bytes);
+  if (rc != VLA_OK) return fail(h, rc, t_err.empty() ? "gemm launch failed" : t_err);
+  return VLA_OK;
+}
+
+// All decoder layers over M rows already assembled in h->h (Llama-2 layer, §3.1).
+// decode == true: one query per env row (rows[b] gives env and position), split-K attention.
+int forward_layers(vla_handle* h, int M, const RowInfo* rows_dev, bool decode, int n_tiles,
+                   int max_ctx) {
+  const vla_config& c = h->cfg;
+  const int d = c.d_model, F = c.d_ffn, H = c.n_heads, hd = c.head_dim;
+  const int gcls = decode ? VLA_KCLASS_GEMM_DECODE : VLA_KCLASS_GEMM_PREFILL;
+  const size_t pd = static_cast<size_t>(h->max_tokens) * d;   // hi -> lo plane offsets
+  const size_t pf = static_cast<size_t>(h->max_tokens) * F;
+  int rc;
+  for (int l = 0; l < c.n_layers; ++l) {
+    int ev = prof_begin(h, VLA_KCLASS_OTHER);
+    if ((rc = rmsnorm_launch(h->h, h->attn_norm[l], M, d, c.rms_eps, h->y, h->y + pd, h->stream))) return fail(h, rc, t_err);
+    prof_end(h, ev, VLA_KCLASS_OTHER, 0, 6.0 * M * d);
+
+    EpiArgs e;
+    e.kind = EPI_QKV;
+    e.out_f32 = h->q;
+    e.rows = rows_dev;
+    e.kv = h->kvl;
+    e.layer = l;
+    e.rope = h->rope;
+    e.d = d;
+    e.hd = hd;
+    if ((rc = run_gemm(h, gcls, h->y, pd, d, h->wqkv[l], d, M, 3 * d, d, e))) return rc;
+
+    if (decode) {
+      ev = prof_begin(h, VLA_KCLASS_ATTN_DECODE);
+      rc = attn_decode_launch(h->q, h->ao, h->ao + pd, rows_dev, M, max_ctx, h->kvl, l, H, hd,
+                              h->attn_chunk, h->part_o, h->part_ml, h->stream);
+      prof_end(h, ev, VLA_KCLASS_ATTN_DECODE, 0, 0);
+    } else {
+      ev = prof_begin(h, VLA_KCLASS_ATTN_PREFILL);
+      rc = attn_chunk_launch(h->q, h->ao, h->ao + pd, h->tiles, n_tiles, h->kvl, l, H, hd, h->stream);
+      prof_end(h, ev, VLA_KCLASS_ATTN_PREFILL, 0, 0);
+    }
+    if (rc) return fail(h, rc, t_err);
+
+    EpiArgs eo;
+    eo.kind = EPI_RESID;
+    eo.resid = h->h;
+    eo.ldr = d;
+    if ((rc = run_gemm(h, gcls, h->ao, pd, d, h->wo[l], d, M, d, d, eo))) return rc;
+
+    ev = prof_begin(h, VLA_KCLASS_OTHER);
+    if ((rc = rmsnorm_launch(h->h, h->ffn_norm[l], M, d, c.rms_eps, h->y, h->y + pd, h->stream))) return fail(h, rc, t_err);
+    prof_end(h, ev, VLA_KCLASS_OTHER, 0, 6.0 * M * d);
+
+    EpiArgs eg;
+    eg.kind = EPI_SWIGLU;
+    eg.out_hi = h->u;
+    eg.out_lo = h->u + pf;
+    eg.ldo = F;
+    if ((rc = run_gemm(h, gcls, h->y, pd, d, h->wgu[l], d, M, 2 * F, d, eg))) return rc;
+
+    EpiArgs ed;
+    ed.kind = EPI_RESID;
+    ed.resid = h->h;
+    ed.ldr = d;
+    if ((rc = run_gemm(h, gcls, h->u, pf, F, h->wdown[l], F, M, d, F, ed))) return rc;
+  }
+  return VLA_OK;
+}
+
+bool finite_nonneg(float t) { return std::isfinite(t) && t >= 0.f; }
+
+}  // namespace
+}  // namespace vla
+
+// =================================================================================== C ABI
+extern "C" {
+
+int vla_create(const vla_config* cfg, const vla_weights* w, void* cuda_stream, vla_handle** out) {
+  if (out) *out = nullptr;
+  if (!cfg || !w || !out) return set_err(nullptr, VLA_ERR_ARG, "vla_create: NULL argument");
+  const vla_config& c = *cfg;
+  if (c.n_layers < 1 || c.d_model < 1 || c.n_heads < 1 || c.head_dim < 1 || c.d_ffn < 1 ||
+      c.vocab < 1 || c.max_batch < 1 || c.kv_capacity < 1 || c.max_tokens < 1 ||
+      !(c.rms_eps >= 0.f) || !(c.rope_theta > 0.f))
+    return set_err(nullptr, VLA_ERR_ARG, "vla_create: non-positive size in config");
+  if (c.head_dim != 64 && c.head_dim != 128)
+    return set_err(nullptr, VLA_ERR_UNSUPPORTED, "vla_create: head_dim must be 64 or 128");
+  if (c.n_heads * c.head_dim != c.d_model || c.d_model % 128 || c.d_ffn % 8)
+    return set_err(nullptr, VLA_ERR_UNSUPPORTED,
+                   "vla_create: need n_heads*head_dim == d_model, d_model % 128 == 0, d_ffn % 8 == 0");
+  if (c.n_action_bins != 256 || c.vocab < 256 || c.action_dim < 1 || c.action_dim > 16)
+    return set_err(nullptr, VLA_ERR_UNSUPPORTED,
+                   "vla_create: need n_action_bins == 256, vocab >= 256, 1 <= action_dim <= 16");
+  if (!w->embed || !w->attn_norm || !w->wqkv || !w->wo || !w->ffn_norm || !w->w_gate_up ||
+      !w->w_down || !w->final_norm || !w->lm_head)
+    return set_err(nullptr, VLA_ERR_ARG, "vla_create: NULL weight pointer");
+  for (int l = 0; l < c.n_layers; ++l)
+    if (!w->attn_norm[l] || !w->wqkv[l] || !w->wo[l] || !w->ffn_norm[l] || !w->w_gate_up[l] ||
+        !w->w_down[l])
+      return set_err(nullptr, VLA_ERR_ARG, "vla_create: NULL per-layer weight pointer");
+
+  vla_handle* h = new vla_handle();
+  h->cfg = c;
+  h->stream = static_cast<cudaStream_t>(cuda_stream);
+  cudaGetDevice(&h->dev);
+  h->num_sms = query_num_sms();
+  const int A = c.action_dim, B = c.max_batch, d = c.d_model, F = c.d_ffn, L = c.n_layers;
+  h->max_tokens = std::max(c.max_tokens, std::max(B, (A - 1) * B));
+  h->embed = static_cast<const bf16*>(w->embed);
+  for (int l = 0; l < L; ++l) {
+    h->attn_norm.push_back(static_cast<const bf16*>(w->attn_norm[l]));
+    h->wqkv.push_back(static_cast<const bf16*>(w->wqkv[l]));
+    h->wo.push_back(static_cast<const bf16*>(w->wo[l]));
+    h->ffn_norm.push_back(static_cast<const bf16*>(w->ffn_norm[l]));
+    h->wgu.push_back(static_cast<const bf16*>(w->w_gate_up[l]));
+    h->wdown.push_back(static_cast<const bf16*>(w->w_down[l]));
+  }
+  h->final_norm = static_cast<const bf16*>(w->final_norm);
+  h->head_rows = static_cast<const bf16*>(w->lm_head) + static_cast<size_t>(c.vocab - 256) * d;
+  h->len.assign(B, 0);
+  h->len_prefill.assign(B, 0);
+  h->has_pending.assign(B, 0);
+  h->prefilled.assign(B, 0);
+  h->launches_at_create = g_launch_count;
+
+  // KV cache geometry [layer][env][K,V][H][cap][hd]
+  const int64_t cap = c.kv_capacity;
+  h->kvl.cap = c.kv_capacity;
+  h->kvl.head_stride = cap * c.head_dim;
+  h->kvl.kv_stride = static_cast<int64_t>(c.n_heads) * h->kvl.head_stride;
+  h->kvl.env_stride = 2 * h->kvl.kv_stride;
+  h->kvl.layer_stride = static_cast<int64_t>(B) * h->kvl.env_stride;
+
+  // split-K workspace: worst case over the decode / score projection shapes
+  size_t ws = 0;
+  std::vector<int> Ms = {B, (A - 1) * B};
+  for (int M = 128; M <= h->max_tokens; M += 128) Ms.push_back(M);
+  for (int M : Ms) {
+    if (M < 1 || M > h->max_tokens) continue;
+    const int shapes[4][4] = {{3 * d, d, EPI_QKV, 0}, {d, d, EPI_RESID, 0}, {2 * F, d, EPI_SWIGLU, 0}, {d, F, EPI_RESID, 0}};
+    for (auto& s : shapes) {
+      const Plan pl = plan_gemm(M, s[0], s[1], s[2], d, h->num_sms);
+      const int sp = gemm_effective_splits(s[1], pl.splits);
+      if (sp > 1) ws = std::max(ws, static_cast<size_t>(sp) * M * s[0] * sizeof(float));
+    }
+  }
+  h->ws_bytes = ws;
+  const int max_S = (c.kv_capacity + h->attn_chunk - 1) / h->attn_chunk;
+  h->max_tiles = h->max_tokens / 64 + B + 1;
+  const size_t T = h->max_tokens;
+
+  auto alloc = [&](void** p, size_t bytes) -> bool {
+    if (!bytes) return true;
+    return cudaMalloc(p, bytes) == cudaSuccess;
+  };
+  bool ok = alloc(reinterpret_cast<void**>(&h->kv), static_cast<size_t>(L) * h->kvl.layer_stride * sizeof(f16)) &&
+            alloc(reinterpret_cast<void**>(&h->h), T * d * sizeof(float)) &&
+            alloc(reinterpret_cast<void**>(&h->y), 2 * T * d * sizeof(bf16)) &&
+            alloc(reinterpret_cast<void**>(&h->q), T * d * sizeof(float)) &&
+            alloc(reinterpret_cast<void**>(&h->ao), 2 * T * d * sizeof(bf16)) &&
+            alloc(reinterpret_cast<void**>(&h->u), 2 * T * F * sizeof(bf16)) &&
+            alloc(reinterpret_cast<void**>(&h->ws), ws) &&
+            alloc(reinterpret_cast<void**>(&h->h_last), static_cast<size_t>(B) * d * sizeof(float)) &&
+            alloc(reinterpret_cast<void**>(&h->head_in), static_cast<size_t>(B) * A * d * sizeof(float)) &&
+            alloc(reinterpret_cast<void**>(&h->rope), static_cast<size_t>(cap) * (c.head_dim / 2) * sizeof(float2)) &&
+            alloc(reinterpret_cast<void**>(&h->rows), T * sizeof(RowInfo)) &&
+            alloc(reinterpret_cast<void**>(&h->tiles), static_cast<size_t>(h->max_tiles) * sizeof(AttnTile)) &&
+            alloc(reinterpret_cast<void**>(&h->sidx), std::max(T, static_cast<size_t>(B) * A) * sizeof(int)) &&
+            alloc(reinterpret_cast<void**>(&h->didx), std::max(T, static_cast<size_t>(B) * A) * sizeof(int)) &&
+            alloc(reinterpret_cast<void**>(&h->fed), static_cast<size_t>(B) * A * sizeof(int)) &&
+            alloc(reinterpret_cast<void**>(&h->pending), static_cast<size_t>(B) * sizeof(int)) &&
+            alloc(reinterpret_cast<void**>(&h->status), sizeof(uint32_t)) &&
+            alloc(reinterpret_cast<void**>(&h->part_o), static_cast<size_t>(B) * c.n_heads * max_S * c.head_dim * sizeof(float)) &&
+            alloc(reinterpret_cast<void**>(&h->part_ml), static_cast<size_t>(B) * c.n_heads * max_S * sizeof(float2));
+  if (!ok) {
+    cudaGetLastError();
+    vla_destroy(h);
+    return set_err(nullptr, VLA_ERR_OOM, "vla_create: device allocation failed");
+  }
+  h->kvl.base = h->kv;
+  // pinned staging
+  h->stage_bytes = T * sizeof(RowInfo) + static_cast<size_t>(h->max_tiles) * sizeof(AttnTile) +
+                   2 * std::max(T, static_cast<size_t>(B) * A) * sizeof(int) + 1024;
+  for (int s = 0; s < vla_handle::kSlots; ++s) {
+    if (cudaMallocHost(&h->stage_host[s], h->stage_bytes) != cudaSuccess ||
+        cudaEventCreateWithFlags(&h->stage_ev[s], cudaEventDisableTiming) != cudaSuccess) {
+      cudaGetLastError();
+      vla_destroy(h);
+      return set_err(nullptr, VLA_ERR_OOM, "vla_create: pinned host allocation failed");
+    }
+  }
+  // RoPE table in fp64 on the host: angle = pos * theta^(-2i/hd)
+  {
+    const int half = c.head_dim / 2;
+    std::vector<float2> tab(static_cast<size_t>(cap) * half);
+    for (int64_t p = 0; p < cap; ++p)
+      for (int i = 0; i < half; ++i) {
+        const double ang = static_cast<double>(p) *
+                           std::pow(static_cast<double>(c.rope_theta), -2.0 * i / c.head_dim);
+        tab[p * half + i] = make_float2(static_cast<float>(std::cos(ang)), static_cast<float>(std::sin(ang)));
+      }
+    if (cudaMemcpy(h->rope, tab.data(), tab.size() * sizeof(float2), cudaMemcpyHostToDevice) != cudaSuccess ||
+        cudaMemset(h->status, 0, sizeof(uint32_t)) != cudaSuccess ||
+        cudaMemset(h->pending, 0, static_cast<size_t>(B) * sizeof(int)) != cudaSuccess) {
+      const int rc = cuda_fail(cudaGetLastError(), "vla_create: initial copies");
+      vla_destroy(h);
+      return rc;
+    }
+  }
+  *out = h;
+  return VLA_OK;
+}
+
+int vla_prefill(vla_handle* h, int batch, const void* visual, int n_visual, const int32_t* token_ids,
+                const int32_t* lengths, int max_len) {
+  if (!h) return set_err(nullptr, VLA_ERR_ARG, "vla_prefill: NULL handle");
+  const vla_config& c = h->cfg;
+  if (batch < 1 || batch > c.max_batch) return fail(h, VLA_ERR_ARG, "vla_prefill: batch outside [1, max_batch]");
+  if (n_visual < 0 || max_len < 0 || !lengths) return fail(h, VLA_ERR_ARG, "vla_prefill: bad n_visual / max_len / lengths");
+  if (n_visual > 0 && !visual) return fail(h, VLA_ERR_ARG, "vla_prefill: NULL visual");
+  int64_t total = 0;
+  bool any_text = false;
+  std::vector<int> chunk(batch);
+  for (int b = 0; b < batch; ++b) {
+    if (lengths[b] < 0 || lengths[b] > max_len) return fail(h, VLA_ERR_ARG, "vla_prefill: length outside [0, max_len]");
+    any_text |= lengths[b] > 0;
+    chunk[b] = (h->has_pending[b] ? 1 : 0) + n_visual + lengths[b];
+    if (chunk[b] < 1) return fail(h, VLA_ERR_ARG, "vla_prefill: empty chunk");
+    if (static_cast<int64_t>(h->len[b]) + chunk[b] + (c.action_dim - 1) > c.kv_capacity)
+      return fail(h, VLA_ERR_CAPACITY, "vla_prefill: KV capacity of an env would be exceeded");
+    total += chunk[b];
+  }
+  if (any_text && !token_ids) return fail(h, VLA_ERR_ARG, "vla_prefill: NULL token_ids");
+  if (total > h->max_tokens) return fail(h, VLA_ERR_CAPACITY, "vla_prefill: more rows than max_tokens");
+  cudaSetDevice(h->dev);
+
+  // host-side row table, attention tiles and last-row indices
+  int slot;
+  uint8_t* st = static_cast<uint8_t*>(stage_slot(h, &slot));
+  RowInfo* rows = reinterpret_cast<RowInfo*>(st);
+  AttnTile* tiles = reinterpret_cast<AttnTile*>(rows + total);
+  int n_tiles = 0;
+  std::vector<int> last(batch);
+  int r = 0;
+  for (int b = 0; b < batch; ++b) {
+    const int r0 = r;
+    int pos = h->len[b];
+    if (h->has_pending[b]) rows[r++] = RowInfo{b, pos++, ROW_TOKEN, b};
+    for (int j = 0; j < n_visual; ++j) rows[r++] = RowInfo{b, pos++, ROW_VISUAL, b * n_visual + j};
+    for (int j = 0; j < lengths[b]; ++j) rows[r++] = RowInfo{b, pos++, ROW_TEXT, b * max_len + j};
+    for (int t0 = 0; t0 < chunk[b]; t0 += 64)
+      tiles[n_tiles++] = AttnTile{b, r0 + t0, std::min(64, chunk[b] - t0), h->len[b] + t0};
+    last[b] = r - 1;
+  }
+  int* sidx = reinterpret_cast<int*>(tiles + n_tiles);
+  for (int b = 0; b < batch; ++b) sidx[b] = last[b];
+  int rc;
+  if ((rc = upload(h, h->rows, rows, total * sizeof(RowInfo))) ||
+      (rc = upload(h, h->tiles, tiles, n_tiles * sizeof(AttnTile))) ||
+      (rc = upload(h, h->sidx, sidx, batch * sizeof(int))))
+    return fail(h, rc, t_err);
+  cudaEventRecord(h->stage_ev[slot], h->stream);
+
+  int ev = prof_begin(h, VLA_KCLASS_OTHER);
+  rc = assemble_launch(h->rows, static_cast<int>(total), static_cast<const bf16*>(visual), token_ids,
+                       h->pending, h->embed, c.d_model, c.vocab, h->h, h->status, h->stream);
+  prof_end(h, ev, VLA_KCLASS_OTHER, 0, 6.0 * total * c.d_model);
+  if (rc) return fail(h, rc, t_err);
+  if ((rc = forward_layers(h, static_cast<int>(total), h->rows, false, n_tiles, 0))) return rc;
+  if ((rc = gather_rows_launch(h->h, h->sidx, batch, c.d_model, h->h_last, h->stream))) return fail(h, rc, t_err);
+
+  for (int b = 0; b < batch; ++b) {
+    h->len[b] += chunk[b];
+    h->len_prefill[b] = h->len[b];
+    h->has_pending[b] = 0;
+    h->prefilled[b] = 1;
+  }
+  h->active_batch = batch;
+  return VLA_OK;
+}
+
+static int check_turn_state(vla_handle* h, const char* who) {
+  if (h->active_batch < 1) return fail(h, VLA_ERR_STATE, std::string(who) + ": no prefill yet");
+  for (int b = 0; b < h->active_batch; ++b)
+    if (!h->prefilled[b]) return fail(h, VLA_ERR_STATE, std::string(who) + ": env reset since the last prefill");
+  return VLA_OK;
+}
+
+int vla_decode_actions(vla_handle* h, const float* uniforms, float temperature, const int32_t* forced_tokens,
+                       int32_t* tokens_out, float* logprobs_out, float* actions_out, float* logits_out) {
+  if (!h) return set_err(nullptr, VLA_ERR_ARG, "vla_decode_actions: NULL handle");
+  if (!finite_nonneg(temperature)) return fail(h, VLA_ERR_ARG, "vla_decode_actions: temperature must be finite and >= 0");
+  if ((temperature > 0.f && !uniforms) || !tokens_out || !logprobs_out || !actions_out)
+    return fail(h, VLA_ERR_ARG, "vla_decode_actions: NULL buffer");
+  int rc;
+  if ((rc = check_turn_state(h, "vla_decode_actions"))) return rc;
+  cudaSetDevice(h->dev);
+  const vla_config& c = h->cfg;
+  const int B = h->active_batch, A = c.action_dim, d = c.d_model;
+
+  // decode rows of steps 1..A-1: env b at position len_prefill[b] + i - 1, fed token of step i-1
+  int slot;
+  RowInfo* rows = static_cast<RowInfo*>(stage_slot(h, &slot));
+  for (int i = 1; i < A; ++i)
+    for (int b = 0; b < B; ++b)
+      rows[(i - 1) * B + b] = RowInfo{b, h->len_prefill[b] + i - 1, ROW_TOKEN, b * A + (i - 1)};
+  if ((rc = upload(h, h->rows, rows, static_cast<size_t>(A - 1) * B * sizeof(RowInfo)))) return fail(h, rc, t_err);
+  cudaEventRecord(h->stage_ev[slot], h->stream);
+  int max_len_p = 0;
+  for (int b = 0; b < B; ++b) max_len_p = std::max(max_len_p, h->len_prefill[b]);
+
+  HeadArgs ha;
+  ha.B = B;
+  ha.n_pos = 1;
+  ha.A = A;
+  ha.final_norm = h->final_norm;
+  ha.head_rows = h->head_rows;
+  ha.d = d;
+  ha.ldh = d;
+  ha.eps = c.rms_eps;
+  ha.temperature = temperature;
+  ha.uniforms = temperature > 0.f ? uniforms : nullptr;
+  ha.forced = forced_tokens;
+  ha.forced_base = c.vocab - 256;
+  ha.token_base = c.vocab - 256;
+  ha.tokens_out = tokens_out;
+  ha.lp_out = logprobs_out;
+  ha.act_out = actions_out;
+  ha.logits_out = logits_out;
+  ha.fed_out = h->fed;
+  ha.status = h->status;
+
+  for (int i = 0; i < A; ++i) {
+    if (i > 0) {
+      const RowInfo* rows_i = h->rows + static_cast<size_t>(i - 1) * B;
+      int ev = prof_begin(h, VLA_KCLASS_OTHER);
+      rc = assemble_launch(rows_i, B, nullptr, nullptr, h->fed, h->embed, d, c.vocab, h->h, h->status, h->stream);
+      prof_end(h, ev, VLA_KCLASS_OTHER, 0, 6.0 * B * d);
+      if (rc) return fail(h, rc, t_err);
+      if ((rc = forward_layers(h, B, rows_i, true, 0, max_len_p + i))) return rc;
+    }
+    ha.h = (i == 0) ? h->h_last : h->h;
+    ha.step = i;
+    int ev = prof_begin(h, VLA_KCLASS_HEAD);
+    rc = action_head_launch(ha, h->stream);
+    prof_end(h, ev, VLA_KCLASS_HEAD, 2.0 * B * 256 * d, 2.0 * 256 * d + 4.0 * B * d);
+    if (rc) return fail(h, rc, t_err);
+  }
+  // the last token stays pending
+  if (cudaMemcpy2DAsync(h->pending, sizeof(int), h->fed + (A - 1), A * sizeof(int), sizeof(int), B,
+                        cudaMemcpyDeviceToDevice, h->stream) != cudaSuccess)
+    return fail(h, cuda_fail(cudaGetLastError(), "pending copy"), t_err);
+  for (int b = 0; b < B; ++b) {
+    h->len[b] = h->len_prefill[b] + (A - 1);
+    h->has_pending[b] = 1;
+  }
+  return VLA_OK;
+}
+
+int vla_score_actions(vla_handle* h, const int32_t* tokens, float temperature, float* logprobs_out,
+                      float* logits_out) {
+  if (!h) return set_err(nullptr, VLA_ERR_ARG, "vla_score_actions: NULL handle");
+  if (!finite_nonneg(temperature)) return fail(h, VLA_ERR_ARG, "vla_score_actions: temperature must be finite and >= 0");
+  if (!tokens || !logprobs_out) return fail(h, VLA_ERR_ARG, "vla_score_actions: NULL buffer");
+  int rc;
+  if ((rc = check_turn_state(h, "vla_score_actions"))) return rc;
+  cudaSetDevice(h->dev);
+  const vla_config& c = h->cfg;
+  const int B = h->active_batch, A = c.action_dim, d = c.d_model;
+  const int n = A - 1;  // teacher-forced rows per env
+  const int M = n * B;
+
+  int slot;
+  uint8_t* st = static_cast<uint8_t*>(stage_slot(h, &slot));
+  RowInfo* rows = reinterpret_cast<RowInfo*>(st);
+  AttnTile* tiles = reinterpret_cast<AttnTile*>(rows + M);
+  int* sidx = reinterpret_cast<int*>(tiles + B);
+  int* didx = sidx + M;
+  int n_tiles = 0;
+  for (int b = 0; b < B; ++b) {
+    for (int j = 0; j < n; ++j) {
+      rows[b * n + j] = RowInfo{b, h->len_prefill[b] + j, ROW_TOKEN, b * A + j};
+      sidx[b * n + j] = b * n + j;
+      didx[b * n + j] = b * A + 1 + j;
+    }
+    if (n > 0) tiles[n_tiles++] = AttnTile{b, b * n, n, h->len_prefill[b]};
+  }
+  if ((rc = upload(h, h->rows, rows, M * sizeof(RowInfo))) ||
+      (rc = upload(h, h->tiles, tiles, n_tiles * sizeof(AttnTile))) ||
+      (rc = upload(h, h->sidx, sidx, M * sizeof(int))) ||
+      (rc = upload(h, h->didx, didx, M * sizeof(int))))
+    return fail(h, rc, t_err);
+  cudaEventRecord(h->stage_ev[slot], h->stream);
+
+  if (M > 0) {
+    int ev = prof_begin(h, VLA_KCLASS_OTHER);
+    rc = assemble_launch(h->rows, M, nullptr, nullptr, tokens, h->embed, d, c.vocab, h->h, h->status, h->stream);
+    prof_end(h, ev, VLA_KCLASS_OTHER, 0, 6.0 * M * d);
+    if (rc) return fail(h, rc, t_err);
+    if ((rc = forward_layers(h, M, h->rows, false, n_tiles, 0))) return rc;
+  }
+  // head inputs: row b*A = prefill's last hidden, rows b*A+1+j = chunk rows
+  if (cudaMemcpy2DAsync(h->head_in, static_cast<size_t>(A) * d * sizeof(float), h->h_last, d * sizeof(float),
+                        d * sizeof(float), B, cudaMemcpyDeviceToDevice, h->stream) != cudaSuccess)
+    return fail(h, cuda_fail(cudaGetLastError(), "head input copy"), t_err);
+  if (M > 0 && (rc = scatter_rows_launch(h->h, h->sidx, h->didx, M, d, h->head_in, h->stream)))
+    return fail(h, rc, t_err);
+
+  HeadArgs ha;
+  ha.h = h->head_in;
+  ha.ldh = d;
+  ha.B = B;
+  ha.n_pos = A;
+  ha.step = 0;
+  ha.A = A;
+  ha.final_norm = h->final_norm;
+  ha.head_rows = h->head_rows;
+  ha.d = d;
+  ha.eps = c.rms_eps;
+  ha.temperature = temperature;
+  ha.uniforms = nullptr;
+  ha.forced = tokens;
+  ha.forced_base = c.vocab - 256;
+  ha.token_base = c.vocab - 256;
+  ha.lp_out = logprobs_out;
+  ha.logits_out = logits_out;
+  ha.status = h->status;
+  int ev = prof_begin(h, VLA_KCLASS_HEAD);
+  rc = action_head_launch(ha, h->stream);
+  prof_end(h, ev, VLA_KCLASS_HEAD, 2.0 * B * A * 256 * d, 2.0 * 256 * d + 4.0 * B * A * d);
+  if (rc) return fail(h, rc, t_err);
+  if (cudaMemcpy2DAsync(h->pending, sizeof(int), tokens + (A - 1), A * sizeof(int), sizeof(int), B,
+                        cudaMemcpyDeviceToDevice, h->stream) != cudaSuccess)
+    return fail(h, cuda_fail(cudaGetLastError(), "pending copy"), t_err);
+  for (int b = 0; b < B; ++b) {
+    h->len[b] = h->len_prefill[b] + (A - 1);
+    h->has_pending[b] = 1;
+  }
+  return VLA_OK;
+}
+
+int vla_reset(vla_handle* h, const uint8_t* env_mask) {
+  if (!h) return set_err(nullptr, VLA_ERR_ARG, "vla_reset: NULL handle");
+  for (int b = 0; b < h->cfg.max_batch; ++b) {
+    if (env_mask && !env_mask[b]) continue;
+    h->len[b] = 0;
+    h->len_prefill[b] = 0;
+    h->has_pending[b] = 0;
+    h->prefilled[b] = 0;
+  }
+  return VLA_OK;
+}
+
+int vla_sync(vla_handle* h) {
+  if (!h) return set_err(nullptr, VLA_ERR_ARG, "vla_sync: NULL handle");
+  cudaSetDevice(h->dev);
+  cudaError_t e = cudaStreamSynchronize(h->stream);
+  if (e != cudaSuccess) return fail(h, cuda_fail(e, "vla_sync: stream"), t_err);
+  uint32_t st = 0;
+  e = cudaMemcpy(&st, h->status, sizeof(uint32_t), cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess) return fail(h, cuda_fail(e, "vla_sync: status read"), t_err);
+  if (st) {
+    cudaMemset(h->status, 0, sizeof(uint32_t));
+    std::string msg = "device status:";
+    if (st & VLA_STATUS_BAD_TOKEN) msg += " token id out of range;";
+    if (st & VLA_STATUS_NONFINITE) msg += " non-finite logit;";
+    if (st & VLA_STATUS_TIMEOUT) msg += " GEMM pipeline wait timed out;";
+    if (st & VLA_STATUS_BAD_FORCED) msg += " forced/scored token is not an action-bin id;";
+    char buf[32];
+    snprintf(buf, sizeof(buf), " (0x%x)", st);
+    return fail(h, VLA_ERR_DEVICE_STATUS, msg + buf);
+  }
+  return VLA_OK;
+}
+
+int vla_context_length(const vla_handle* h, int env) {
+  if (!h || env < 0 || env >= h->cfg.max_batch) return -1;
+  return h->len[env];
+}
+
+const char* vla_last_error(const vla_handle* h) { return h ? h->err.c_str() : t_err.c_str(); }
+
+void vla_destroy(vla_handle* h) {
+  if (!h) return;
+  cudaSetDevice(h->dev);
+  cudaStreamSynchronize(h->stream);
+  void* bufs[] = {h->kv, h->h, h->y, h->q, h->ao, h->u, h->ws, h->h_last, h->head_in, h->rope,
+                  h->rows, h->tiles, h->sidx, h->didx, h->fed, h->pending, h->status, h->part_o,
+                  h->part_ml};
+  for (void* p : bufs)
+    if (p) cudaFree(p);
+  for (int s = 0; s < vla_handle::kSlots; ++s) {
+    if (h->stage_host[s]) cudaFreeHost(h->stage_host[s]);
+    if (h->stage_ev[s]) cudaEventDestroy(h->stage_ev[s]);
+  }
+  for (auto& e : h->ev_used) {
+    cudaEventDestroy(e.a);
+    cudaEventDestroy(e.b);
+  }
+  for (auto& e : h->ev_free) {
+    cudaEventDestroy(e.a);
+    cudaEventDestroy(e.b);
+  }
+  delete h;
+}
+
+int vla_profile(vla_handle* h, uint32_t class_mask) {
+  if (!h) return set_err(nullptr, VLA_ERR_ARG, "vla_profile: NULL handle");
+  prof_harvest(h);
+  h->prof_mask = class_mask;
+  for (int i = 0; i < VLA_KCLASS_COUNT; ++i) {
+    h->prof_launches[i] = 0;
+    h->prof_ms[i] = h->prof_flops[i] = h->prof_bytes[i] = 0.0;
+  }
+  return VLA_OK;
+}
+
+int vla_profile_read(vla_handle* h, int64_t* launches, double* ms, double* flops, double* bytes) {
+  if (!h) return set_err(nullptr, VLA_ERR_ARG, "vla_profile_read: NULL handle");
+  prof_harvest(h);
+  for (int i = 0; i < VLA_KCLASS_COUNT; ++i) {
+    if (launches) launches[i] = h->prof_launches[i];
+    if (ms) ms[i] = h->prof_ms[i];
+    if (flops) flops[i] = h->prof_flops[i];
+    if (bytes) bytes[i] = h->prof_bytes[i];
+  }
+  return VLA_OK;
+}
+
+int64_t vla_launch_count(const vla_handle* h) {
+  return h ? g_launch_count - h->launches_at_create : g_launch_count;
+}
+
+// ---------------------------------------------------------------------------------- ops
+int vla_op_gemm_bf16(const void* A, const void* A_lo, int lda, const void* W, int ldw, float* C, int ldc,
+                     int M, int N, int K, int block_n, int splits, float* workspace, void* cuda_stream) {
+  if (!A || !W || !C || M < 1 || N < 1 || K < 1 || ldc < N)
+    return set_err(nullptr, VLA_ERR_ARG, "vla_op_gemm_bf16: bad argument");
+  GemmArgs g;
+  g.A = static_cast<const bf16*>(A);
+  g.A_lo = static_cast<const bf16*>(A_lo);
+  g.lda = lda;
+  g.B = static_cast<const bf16*>(W);
+  g.ldb = ldw;
+  g.M = M;
+  g.N = N;
+  g.K = K;
+  g.block_n = block_n;
+  g.splits = splits;
+  g.workspace = workspace;
+  g.workspace_bytes = workspace ? gemm_workspace_bytes(g) : 0;
+  g.epi.kind = EPI_F32;
+  g.epi.out_f32 = C;
+  g.epi.ldo = ldc;
+  if (splits > 1 && gemm_effective_splits(K, splits) > 1 && !workspace)
+    return set_err(nullptr, VLA_ERR_ARG, "vla_op_gemm_bf16: splits > 1 needs a workspace");
+  const int rc = gemm_launch(g, static_cast<cudaStream_t>(cuda_stream), query_num_sms(), nullptr);
+  if (rc != VLA_OK && rc != VLA_ERR_CUDA) return set_err(nullptr, rc, "vla_op_gemm_bf16: unsupported arguments");
+  return rc;
+}
+
+int vla_op_action_head(const float* hs, int ldh, int B, int d, const void* final_norm, const void* head_rows,
+                       float eps, const float* uniforms, float temperature, const int32_t* forced,
+                       int32_t* bins_out, float* logprobs_out, float* actions_out, float* logits_out,
+                       uint32_t* status, void* cuda_stream) {
+  if (!hs || B < 1 || d < 8 || ldh < d || !final_norm || !head_rows || !logprobs_out || !status ||
+      !finite_nonneg(temperature) || (temperature > 0.f && !uniforms))
+    return set_err(nullptr, VLA_ERR_ARG, "vla_op_action_head: bad argument");
+  HeadArgs ha;
+  ha.h = hs;
+  ha.ldh = ldh;
+  ha.B = B;
+  ha.n_pos = 1;
+  ha.step = 0;
+  ha.A = 1;
+  ha.final_norm = static_cast<const bf16*>(final_norm);
+  ha.head_rows = static_cast<const bf16*>(head_rows);
+  ha.d = d;
+  ha.eps = eps;
+  ha.temperature = temperature;
+  ha.uniforms = temperature > 0.f ? uniforms : nullptr;
+  ha.forced = forced;
+  ha.forced_base = 0;
+  ha.token_base = 0;
+  ha.bins_out = bins_out;
+  ha.lp_out = logprobs_out;
+  ha.act_out = actions_out;
+  ha.logits_out = logits_out;
+  ha.status = status;
+  return action_head_launch(ha, static_cast<cudaStream_t>(cuda_stream));
+}
+
+int vla_op_num_sms(void) { return query_num_sms(); }
+
+}  // extern "C"

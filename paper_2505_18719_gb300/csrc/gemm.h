@@ -1,0 +1,59 @@
+// Internal interface of the tcgen05 GEMM (gemm_tc.cu) used by the engine and the op API.
+#pragma once
+#include "common.cuh"
+
+namespace vla {
+
+// Epilogue of Y[M, N] = A[M, K] · B[N, K]^T (fp32 accumulator in TMEM).
+enum EpiKind : int {
+  EPI_F32 = 0,     // out_f32[m * ldo + n] = y
+  EPI_RESID = 1,   // resid[m * ldr + n] += y               (O-proj, down-proj)
+  EPI_SWIGLU = 2,  // u = silu(y_gate) * y_up, f < F = N / 2, stored as the bf16 pair
+                   // out_hi / out_lo [m * ldo + f]
+  EPI_QKV = 3,     // RoPE(q) -> out_f32 [M, d]; RoPE(k), v -> fp16 KV cache
+  EPI_PARTIAL = 4  // internal: split-K partial sums to the workspace
+};
+
+struct EpiArgs {
+  int kind = EPI_F32;
+  float* out_f32 = nullptr;
+  bf16* out_hi = nullptr;
+  bf16* out_lo = nullptr;
+  int ldo = 0;
+  float* resid = nullptr;
+  int ldr = 0;
+  const RowInfo* rows = nullptr;  // EPI_QKV: env / position of each row
+  KVLayout kv{};
+  int layer = 0;
+  const float2* rope = nullptr;   // EPI_QKV: [cap][hd/2] (cos, sin)
+  int d = 0, hd = 0;
+  uint32_t* status = nullptr;
+};
+
+struct GemmArgs {
+  const bf16* A = nullptr;     // [M, K], row stride lda
+  const bf16* A_lo = nullptr;  // optional low half of A (same layout): Y = (A + A_lo) · B^T
+  int lda = 0;
+  const bf16* B = nullptr;  // [N, K], row stride ldb (SwiGLU: [2F, K] rows gate | up, N = 2F)
+  int ldb = 0;
+  int M = 0, N = 0, K = 0;
+  int block_n = 256;        // 128 or 256
+  int splits = 1;           // split-K factor (> 1 needs workspace)
+  float* workspace = nullptr;
+  size_t workspace_bytes = 0;
+  EpiArgs epi;
+};
+
+// Algorithmic cost of one GEMM call (for the roofline report).
+struct GemmCost {
+  double flops, bytes;
+};
+
+// Effective split count (no empty split) for a requested one.
+int gemm_effective_splits(int K, int splits);
+// Workspace bytes the call needs (0 when splits == 1).
+size_t gemm_workspace_bytes(const GemmArgs& a);
+// Launch; returns VLA_OK or an error code (host checks only; kernels report via status).
+int gemm_launch(const GemmArgs& a, cudaStream_t stream, int num_sms, GemmCost* cost);
+
+}  // namespace vla

@@ -1,0 +1,830 @@
+// tcgen05 / TMEM / TMA GEMM for sm_103a with the decoder layer's fused epilogues.
+//
+// Y[M, N] = A[M, K] · B[N, K]^T, bf16 operands (both K-major), fp32 accumulation in TMEM.
+// With a split A (the activation carried as a bf16 pair hi + lo), each K step issues two
+// MMAs, hi·B and lo·B, into the same accumulator, so the product sees ~16 mantissa bits of
+// the activation while the weights stay bf16.
+// This is every projection of the Llama-2 backbone of the policy (paper §3.1): q|k|v, o,
+// gate|up and down.  Epilogues fuse what follows each projection in the layer: RoPE and
+// the KV-cache write after q|k|v, the residual add after o and down, SwiGLU after gate|up.
+//
+// Kernel structure (one persistent CTA per SM, 192 threads):
+//   warp 0      TMA producer: 128x64 A tile(s) + BNx64 B tile per stage, 128-byte swizzle,
+//               STAGES-deep ring guarded by full/empty mbarriers.
+//   warp 1      allocates 2*BN TMEM columns (two accumulators); lane 0 issues
+//               tcgen05.mma.cta_group::1.kind::f16 (M=128, N=BN, K=16) and commits
+//               stage releases / accumulator-ready to mbarriers.
+//   warps 2-5   epilogue: tcgen05.ld 32x32b (one TMEM lane = one output row per thread),
+//               fused math, global stores; releases the accumulator to the MMA warp so
+//               the next tile's main loop overlaps this tile's epilogue.
+// Work units (m-tile, n-tile, k-split) are rastered in groups of 16 m-tiles so that the
+// tiles in flight share A and B in L2.  Every mbarrier wait is bounded (globaltimer): on
+// timeout the CTA records VLA_STATUS_TIMEOUT, drains its own copies and MMAs, frees TMEM and
+// exits.  No TMA multicast and no clusters are used.
+#include <cstdio>
+#include <cstring>
+#include <mutex>
+
+#include "gemm.h"
+
+namespace vla {
+
+namespace {
+
+constexpr int BM = 128;
+constexpr int BK = 64;  // 64 bf16 = 128 bytes = one swizzle atom row
+constexpr int kThreads = 192;
+constexpr uint64_t kWaitLimitNs = 1000000000ull;  // 1 s per wait
+constexpr int kGroupM = 16;
+
+// ----------------------------------------------------------------------------- PTX helpers
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+__device__ __forceinline__ uint64_t globaltimer() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count));
+}
+__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
+               : "memory");
+}
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map, uint32_t bar,
+                                            int c0, int c1) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%3, %4}], [%2];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(bar), "r"(c0), "r"(c1)
+      : "memory");
+}
+__device__ __forceinline__ void tc_fence_before() {
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tc_fence_after() {
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tc_commit(uint32_t bar) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
+                   bar)
+               : "memory");
+}
+__device__ __forceinline__ void tc_mma(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc,
+                                       uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+// 32 lanes x 32 bit, 16 consecutive columns -> 16 registers of this thread's row.
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, "
+      "%11, %12, %13, %14, %15}, [%16];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]),
+        "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+      : "r"(taddr));
+}
+__device__ __forceinline__ void tmem_wait_ld() {
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+
+// Shared-memory matrix descriptor: K-major operand, 128-byte swizzle, rows of 128 bytes,
+// 8-row core-matrix groups 1024 bytes apart (SBO); LBO unused for this layout.
+__device__ __forceinline__ uint64_t make_sdesc(uint32_t saddr) {
+  uint64_t d = 0;
+  d |= static_cast<uint64_t>((saddr & 0x3FFFFu) >> 4);
+  d |= static_cast<uint64_t>(1) << 16;            // LBO (ignored for swizzled K-major)
+  d |= static_cast<uint64_t>(1024 >> 4) << 32;    // SBO
+  d |= static_cast<uint64_t>(1) << 46;            // descriptor version (sm_100 family)
+  d |= static_cast<uint64_t>(2) << 61;            // SWIZZLE_128B
+  return d;
+}
+
+// Instruction descriptor, kind::f16: D f32, A/B bf16, both K-major, M = 128, N = BN.
+template <int BN>
+__device__ __forceinline__ constexpr uint32_t make_idesc() {
+  return (1u << 4) | (1u << 7) | (1u << 10) | (static_cast<uint32_t>(BN >> 3) << 17) |
+         (static_cast<uint32_t>(BM >> 4) << 24);
+}
+
+struct Params {
+  int M, N, K;          // N: columns of B used (SwiGLU: 2F)
+  int tiles_m, tiles_n, splits, kb_total, kb_per_split;
+  EpiArgs epi;
+};
+
+// Bounded wait.  Returns false when this CTA is aborting (timeout here or elsewhere).
+__device__ __forceinline__ bool wait_bounded(uint32_t bar, uint32_t parity, volatile int* abort_flag,
+                                             uint32_t* status) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = globaltimer();
+  uint32_t n = 0;
+  while (true) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if (((++n) & 63u) == 0) {
+      if (*abort_flag) return false;
+      if (globaltimer() - t0 > kWaitLimitNs) {
+        *abort_flag = 1;
+        if (status) atomicOr(status, VLA_STATUS_TIMEOUT);
+        return false;
+      }
+    }
+  }
+}
+// Wait used while draining: ignores the abort flag, bounded by time only.
+__device__ __forceinline__ void wait_drain(uint32_t bar, uint32_t parity) {
+  const uint64_t t0 = globaltimer();
+  while (!mbar_try_wait(bar, parity)) {
+    if (globaltimer() - t0 > kWaitLimitNs) return;
+  }
+}
+
+__device__ __forceinline__ void unit_coords(const Params& p, int u, int& m_blk, int& n_blk,
+                                            int& split) {
+  const int ncols = p.tiles_n * p.splits;        // (n-tile, split) pairs
+  const int per_group = kGroupM * ncols;
+  const int g = u / per_group;
+  const int r = u - g * per_group;
+  const int first_m = g * kGroupM;
+  const int gsize = min(kGroupM, p.tiles_m - first_m);
+  m_blk = first_m + r % gsize;
+  const int col = r / gsize;
+  n_blk = col / p.splits;
+  split = col - n_blk * p.splits;
+}
+
+// ----------------------------------------------------------------------------- epilogues
+__device__ __forceinline__ void store_bf16x16(bf16* dst, const float (&v)[16]) {
+  uint4 a, b;
+  a.x = pack_bf16x2(v[0], v[1]);
+  a.y = pack_bf16x2(v[2], v[3]);
+  a.z = pack_bf16x2(v[4], v[5]);
+  a.w = pack_bf16x2(v[6], v[7]);
+  b.x = pack_bf16x2(v[8], v[9]);
+  b.y = pack_bf16x2(v[10], v[11]);
+  b.z = pack_bf16x2(v[12], v[13]);
+  b.w = pack_bf16x2(v[14], v[15]);
+  reinterpret_cast<uint4*>(dst)[0] = a;
+  reinterpret_cast<uint4*>(dst)[1] = b;
+}
+
+// 16 values as bf16 hi/lo pairs (two 32-byte stores each).
+__device__ __forceinline__ void store_split16(bf16* hi_dst, bf16* lo_dst, const float (&v)[16]) {
+  uint32_t h[8], l[8];
+#pragma unroll
+  for (int i = 0; i < 8; ++i) split_pack2(v[2 * i], v[2 * i + 1], h[i], l[i]);
+  reinterpret_cast<uint4*>(hi_dst)[0] = make_uint4(h[0], h[1], h[2], h[3]);
+  reinterpret_cast<uint4*>(hi_dst)[1] = make_uint4(h[4], h[5], h[6], h[7]);
+  reinterpret_cast<uint4*>(lo_dst)[0] = make_uint4(l[0], l[1], l[2], l[3]);
+  reinterpret_cast<uint4*>(lo_dst)[1] = make_uint4(l[4], l[5], l[6], l[7]);
+}
+__device__ __forceinline__ void store_f16x16(f16* dst, const float (&v)[16]) {
+  uint4 a, b;
+  a.x = pack_f16x2(v[0], v[1]);
+  a.y = pack_f16x2(v[2], v[3]);
+  a.z = pack_f16x2(v[4], v[5]);
+  a.w = pack_f16x2(v[6], v[7]);
+  b.x = pack_f16x2(v[8], v[9]);
+  b.y = pack_f16x2(v[10], v[11]);
+  b.z = pack_f16x2(v[12], v[13]);
+  b.w = pack_f16x2(v[14], v[15]);
+  reinterpret_cast<uint4*>(dst)[0] = a;
+  reinterpret_cast<uint4*>(dst)[1] = b;
+}
+__device__ __forceinline__ void store_f32x16(float* dst, const float (&v)[16]) {
+#pragma unroll
+  for (int i = 0; i < 4; ++i)
+    reinterpret_cast<float4*>(dst)[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+}
+
+__device__ __forceinline__ void ld16f(uint32_t taddr, float (&v)[16]) {
+  uint32_t r[16];
+  tmem_ld16(taddr, r);
+  tmem_wait_ld();
+#pragma unroll
+  for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+// Plain epilogues: F32 / RESID / PARTIAL, 16 columns at a time.
+template <int BN, int EPI>
+__device__ __forceinline__ void epilogue_plain(const Params& p, uint32_t trow, int m, int n0,
+                                               int split) {
+  const bool row_ok = m < p.M;
+#pragma unroll 1
+  for (int c = 0; c < BN; c += 16) {
+    float v[16];
+    ld16f(trow + c, v);
+    const int n = n0 + c;
+    if (!row_ok || n >= p.N) continue;
+    float* dst;
+    int ld;
+    if (EPI == EPI_F32) {
+      dst = p.epi.out_f32 + static_cast<size_t>(m) * p.epi.ldo + n;
+      ld = p.epi.ldo;
+    } else if (EPI == EPI_RESID) {
+      dst = p.epi.resid + static_cast<size_t>(m) * p.epi.ldr + n;
+      ld = p.epi.ldr;
+    } else {  // PARTIAL: workspace [splits][M][N]
+      dst = p.epi.out_f32 + (static_cast<size_t>(split) * p.M + m) * p.N + n;
+      ld = p.N;
+    }
+    const bool vec = (n + 16 <= p.N) && ((ld & 3) == 0) &&
+                     ((reinterpret_cast<uintptr_t>(dst) & 15) == 0);
+    if (vec) {
+      float4* d4 = reinterpret_cast<float4*>(dst);
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        float4 o;
+        if (EPI == EPI_RESID) {
+          o = d4[i];
+          o.x += v[4 * i];
+          o.y += v[4 * i + 1];
+          o.z += v[4 * i + 2];
+          o.w += v[4 * i + 3];
+        } else {
+          o = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+        }
+        d4[i] = o;
+      }
+    } else {
+      for (int i = 0; i < 16 && n + i < p.N; ++i) {
+        if (EPI == EPI_RESID)
+          dst[i] += v[i];
+        else
+          dst[i] = v[i];
+      }
+    }
+  }
+}
+
+// SwiGLU: tile columns [0, BN/2) are gate features f0.., [BN/2, BN) the matching up features.
+template <int BN>
+__device__ __forceinline__ void epilogue_swiglu(const Params& p, uint32_t trow, int m, int f0) {
+  const int F = p.N >> 1;
+  const bool row_ok = m < p.M;
+#pragma unroll 1
+  for (int j = 0; j < BN / 2; j += 16) {
+    float g[16], u[16];
+    ld16f(trow + j, g);
+    ld16f(trow + BN / 2 + j, u);
+    const int f = f0 + j;
+    if (!row_ok || f >= F) continue;
+    float o[16];
+#pragma unroll
+    for (int i = 0; i < 16; ++i) o[i] = silu_f(g[i]) * u[i];
+    const size_t off = static_cast<size_t>(m) * p.epi.ldo + f;
+    if (f + 16 <= F && ((p.epi.ldo & 7) == 0)) {
+      store_split16(p.epi.out_hi + off, p.epi.out_lo + off, o);
+    } else {
+      for (int i = 0; i < 16 && f + i < F; ++i) {
+        bf16 hi, lo;
+        split_bf16(o[i], hi, lo);
+        p.epi.out_hi[off + i] = hi;
+        p.epi.out_lo[off + i] = lo;
+      }
+    }
+  }
+}
+
+// q|k|v with RoPE (rotate-half: pair (i, i + hd/2) rotated by pos * theta^(-2i/hd)) and the
+// KV-cache write.  q goes to an fp32 buffer, K and V to the fp16 cache.  The tile lies inside
+// one of the q / k / v sections (BN divides d) and holds BN / hd whole heads.
+template <int BN>
+__device__ __forceinline__ void epilogue_qkv(const Params& p, uint32_t trow, int m, int n0) {
+  const int d = p.epi.d, hd = p.epi.hd, half = hd >> 1;
+  const int sec = n0 / d;              // 0 q, 1 k, 2 v
+  const int head0 = (n0 - sec * d) / hd;
+  const bool row_ok = m < p.M;
+  RowInfo ri{0, 0, 0, 0};
+  if (row_ok) ri = p.epi.rows[m];
+  const KVLayout& kv = p.epi.kv;
+  f16* kv_row = nullptr;
+  if (row_ok && sec > 0) {
+    kv_row = kv.base + static_cast<int64_t>(p.epi.layer) * kv.layer_stride +
+             static_cast<int64_t>(ri.env) * kv.env_stride + (sec == 2 ? kv.kv_stride : 0) +
+             static_cast<int64_t>(ri.pos) * hd;
+  }
+  const int heads = BN / hd;
+#pragma unroll 1
+  for (int hh = 0; hh < heads; ++hh) {
+    const int head = head0 + hh;
+    const uint32_t tcol = trow + hh * hd;
+    if (sec == 2) {
+      f16* dst = row_ok ? kv_row + static_cast<int64_t>(head) * kv.head_stride : nullptr;
+#pragma unroll 1
+      for (int j = 0; j < hd; j += 16) {
+        float v[16];
+        ld16f(tcol + j, v);
+        if (row_ok) store_f16x16(dst + j, v);
+      }
+    } else {
+#pragma unroll 1
+      for (int j = 0; j < half; j += 16) {
+        float a[16], b[16];
+        ld16f(tcol + j, a);
+        ld16f(tcol + half + j, b);
+        if (!row_ok) continue;
+        const float2* cs = p.epi.rope + static_cast<size_t>(ri.pos) * half + j;
+        float ra[16], rb[16];
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+          const float2 t = cs[i];
+          ra[i] = a[i] * t.x - b[i] * t.y;
+          rb[i] = b[i] * t.x + a[i] * t.y;
+        }
+        if (sec == 0) {
+          float* dst = p.epi.out_f32 + static_cast<size_t>(m) * d + head * hd;
+          store_f32x16(dst + j, ra);
+          store_f32x16(dst + half + j, rb);
+        } else {
+          f16* dst = kv_row + static_cast<int64_t>(head) * kv.head_stride;
+          store_f16x16(dst + j, ra);
+          store_f16x16(dst + half + j, rb);
+        }
+      }
+    }
+  }
+}
+
+// ----------------------------------------------------------------------------- the kernel
+template <int BN, int STAGES, int EPI, bool SPLIT>
+__global__ void __launch_bounds__(kThreads, 1)
+    gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmA2,
+                   const __grid_constant__ CUtensorMap tmB, const __grid_constant__ CUtensorMap tmB2,
+                   const Params p) {
+  constexpr int A_BYTES = BM * BK * 2;
+  constexpr int A_TOTAL = SPLIT ? 2 * A_BYTES : A_BYTES;
+  constexpr int B_BYTES = BN * BK * 2;
+  constexpr int STAGE_BYTES = A_TOTAL + B_BYTES;
+  constexpr uint32_t TMEM_COLS = 2 * BN;
+  constexpr uint32_t IDESC = make_idesc<BN>();
+  constexpr bool SWIGLU = (EPI == EPI_SWIGLU);
+
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~static_cast<uintptr_t>(1023));
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + STAGES * STAGE_BYTES);
+  // bars: full[STAGES], empty[STAGES], tfull[2], tempty[2], drain
+  const uint32_t full0 = smem_u32(bars);
+  const uint32_t empty0 = full0 + 8 * STAGES;
+  const uint32_t tfull0 = empty0 + 8 * STAGES;
+  const uint32_t tempty0 = tfull0 + 16;
+  const uint32_t drain_bar = tempty0 + 16;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * STAGES + 5);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < STAGES; ++s) {
+      mbar_init(full0 + 8 * s, 1);
+      mbar_init(empty0 + 8 * s, 1);
+    }
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(tfull0 + 8 * a, 1);
+      mbar_init(tempty0 + 8 * a, 4);
+    }
+    mbar_init(drain_bar, 1);
+    *abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmA)) : "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmB)) : "memory");
+    if (SPLIT)
+      asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmA2)) : "memory");
+  }
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                     smem_u32(tmem_slot)),
+                 "r"(TMEM_COLS)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+  const int units = p.tiles_m * p.tiles_n * p.splits;
+  uint32_t* status = p.epi.status;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ------------------------------------------------------------ TMA producer
+      int stage = 0;
+      uint32_t phase = 0;
+      uint32_t issued = 0, issued_phase = 0;
+      bool ok = true;
+      for (int u = blockIdx.x; u < units && ok; u += gridDim.x) {
+        int m_blk, n_blk, split;
+        unit_coords(p, u, m_blk, n_blk, split);
+        const int kb0 = split * p.kb_per_split;
+        const int kb1 = min(kb0 + p.kb_per_split, p.kb_total);
+        for (int kb = kb0; kb < kb1; ++kb) {
+          if (!wait_bounded(empty0 + 8 * stage, phase ^ 1u, abort_flag, status)) {
+            ok = false;
+            break;
+          }
+          const uint32_t fb = full0 + 8 * stage;
+          const uint32_t sa = smem_u32(smem + stage * STAGE_BYTES);
+          const uint32_t sb = sa + A_TOTAL;
+          mbar_arrive_expect_tx(fb, STAGE_BYTES);
+          tma_load_2d(sa, &tmA, fb, kb * BK, m_blk * BM);
+          if (SPLIT) tma_load_2d(sa + A_BYTES, &tmA2, fb, kb * BK, m_blk * BM);
+          if (SWIGLU) {
+            tma_load_2d(sb, &tmB, fb, kb * BK, n_blk * (BN / 2));
+            tma_load_2d(sb + (BN / 2) * BK * 2, &tmB2, fb, kb * BK, n_blk * (BN / 2));
+          } else {
+            tma_load_2d(sb, &tmB, fb, kb * BK, n_blk * BN);
+          }
+          issued |= 1u << stage;
+          issued_phase = (issued_phase & ~(1u << stage)) | (phase << stage);
+          if (++stage == STAGES) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+      }
+      // Drain: every stage's last issued copy has landed before the CTA may exit.
+      for (int s = 0; s < STAGES; ++s)
+        if (issued & (1u << s)) wait_drain(full0 + 8 * s, (issued_phase >> s) & 1u);
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      // ------------------------------------------------------------ MMA issuer
+      int stage = 0;
+      uint32_t phase = 0;
+      int it = 0;
+      bool ok = true;
+      for (int u = blockIdx.x; u < units && ok; u += gridDim.x, ++it) {
+        int m_blk, n_blk, split;
+        unit_coords(p, u, m_blk, n_blk, split);
+        const int kb0 = split * p.kb_per_split;
+        const int kb1 = min(kb0 + p.kb_per_split, p.kb_total);
+        const int acc = it & 1;
+        const uint32_t acc_phase = (it >> 1) & 1;
+        if (!wait_bounded(tempty0 + 8 * acc, acc_phase ^ 1u, abort_flag, status)) break;
+        tc_fence_after();
+        const uint32_t d_tmem = tmem_base + acc * BN;
+        for (int kb = kb0; kb < kb1; ++kb) {
+          if (!wait_bounded(full0 + 8 * stage, phase, abort_flag, status)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t sa = smem_u32(smem + stage * STAGE_BYTES);
+          const uint32_t sb = sa + A_TOTAL;
+#pragma unroll
+          for (int k = 0; k < BK / 16; ++k) {
+            const uint64_t bdesc = make_sdesc(sb + k * 32);
+            tc_mma(d_tmem, make_sdesc(sa + k * 32), bdesc, IDESC, (kb > kb0 || k > 0) ? 1u : 0u);
+            if (SPLIT) tc_mma(d_tmem, make_sdesc(sa + A_BYTES + k * 32), bdesc, IDESC, 1u);
+          }
+          tc_commit(empty0 + 8 * stage);
+          if (++stage == STAGES) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+        if (ok) tc_commit(tfull0 + 8 * acc);
+      }
+      // Drain: all MMAs issued by this thread have completed before TMEM is freed.
+      tc_commit(drain_bar);
+      wait_drain(drain_bar, 0);
+    }
+  } else {
+    // -------------------------------------------------------------- epilogue warps 2..5
+    const int q = warp & 3;  // TMEM lane quarter this warp may access
+    int it = 0;
+    for (int u = blockIdx.x; u < units; u += gridDim.x, ++it) {
+      int m_blk, n_blk, split;
+      unit_coords(p, u, m_blk, n_blk, split);
+      const int acc = it & 1;
+      const uint32_t acc_phase = (it >> 1) & 1;
+      int ok = 1;
+      if (lane == 0) ok = wait_bounded(tfull0 + 8 * acc, acc_phase, abort_flag, status) ? 1 : 0;
+      ok = __shfl_sync(0xffffffffu, ok, 0);
+      if (!ok) break;
+      tc_fence_after();
+      const int m = m_blk * BM + q * 32 + lane;
+      const uint32_t trow = tmem_base + (static_cast<uint32_t>(q * 32) << 16) + acc * BN;
+      if (EPI == EPI_SWIGLU)
+        epilogue_swiglu<BN>(p, trow, m, n_blk * (BN / 2));
+      else if (EPI == EPI_QKV)
+        epilogue_qkv<BN>(p, trow, m, n_blk * BN);
+      else
+        epilogue_plain<BN, EPI>(p, trow, m, n_blk * BN, split);
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(tempty0 + 8 * acc);
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem_base),
+                 "r"(TMEM_COLS)
+                 : "memory");
+  }
+}
+
+// ----------------------------------------------------------------------------- split-K sums
+// Fixed summation order s = 0 .. S-1, so results do not depend on the launch.
+__global__ void reduce_f32_kernel(const float* __restrict__ ws, int S, int M, int N, float* out,
+                                  int ldo, int resid) {
+  const int64_t total = static_cast<int64_t>(M) * N;
+  for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < total;
+       i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+    float acc = 0.f;
+    for (int s = 0; s < S; ++s) acc += ws[s * total + i];
+    const int m = static_cast<int>(i / N), n = static_cast<int>(i - static_cast<int64_t>(m) * N);
+    float* o = out + static_cast<size_t>(m) * ldo + n;
+    if (resid)
+      *o += acc;
+    else
+      *o = acc;
+  }
+}
+
+__global__ void reduce_swiglu_kernel(const float* __restrict__ ws, int S, int M, int F,
+                                     bf16* out_hi, bf16* out_lo, int ldo) {
+  const int64_t total = static_cast<int64_t>(M) * F;
+  const int64_t plane = static_cast<int64_t>(M) * 2 * F;
+  for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < total;
+       i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+    const int m = static_cast<int>(i / F), f = static_cast<int>(i - static_cast<int64_t>(m) * F);
+    const int64_t base = static_cast<int64_t>(m) * 2 * F + f;
+    float g = 0.f, u = 0.f;
+    for (int s = 0; s < S; ++s) {
+      g += ws[s * plane + base];
+      u += ws[s * plane + base + F];
+    }
+    bf16 hi, lo;
+    split_bf16(silu_f(g) * u, hi, lo);
+    out_hi[static_cast<size_t>(m) * ldo + f] = hi;
+    out_lo[static_cast<size_t>(m) * ldo + f] = lo;
+  }
+}
+
+// One thread per (row, q|k|v section, head, i < hd/2): sums the pair (i, i + hd/2).
+__global__ void reduce_qkv_kernel(const float* __restrict__ ws, int S, int M, EpiArgs e) {
+  const int d = e.d, hd = e.hd, half = hd >> 1, H = d / hd;
+  const int64_t N = 3LL * d;
+  const int64_t plane = static_cast<int64_t>(M) * N;
+  const int64_t total = static_cast<int64_t>(M) * 3 * H * half;
+  for (int64_t t = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; t < total;
+       t += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+    const int i = static_cast<int>(t % half);
+    int64_t r = t / half;
+    const int head = static_cast<int>(r % H);
+    r /= H;
+    const int sec = static_cast<int>(r % 3);
+    const int m = static_cast<int>(r / 3);
+    const int64_t c = sec * static_cast<int64_t>(d) + head * hd + i;
+    float a = 0.f, b = 0.f;
+    for (int s = 0; s < S; ++s) {
+      a += ws[s * plane + static_cast<int64_t>(m) * N + c];
+      b += ws[s * plane + static_cast<int64_t>(m) * N + c + half];
+    }
+    const RowInfo ri = e.rows[m];
+    if (sec < 2) {
+      const float2 cs = e.rope[static_cast<size_t>(ri.pos) * half + i];
+      const float ra = a * cs.x - b * cs.y;
+      const float rb = b * cs.x + a * cs.y;
+      a = ra;
+      b = rb;
+    }
+    if (sec == 0) {
+      float* dst = e.out_f32 + static_cast<size_t>(m) * d + head * hd;
+      dst[i] = a;
+      dst[i + half] = b;
+    } else {
+      f16* dst = e.kv.base + static_cast<int64_t>(e.layer) * e.kv.layer_stride +
+                 static_cast<int64_t>(ri.env) * e.kv.env_stride + (sec == 2 ? e.kv.kv_stride : 0) +
+                 static_cast<int64_t>(head) * e.kv.head_stride + static_cast<int64_t>(ri.pos) * hd;
+      dst[i] = __float2half_rn(a);
+      dst[i + half] = __float2half_rn(b);
+    }
+  }
+}
+
+// ----------------------------------------------------------------------------- host side
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                  const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                  const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(p);
+  });
+  return fn;
+}
+
+// 2-D bf16 map over [rows, cols] (row stride ld elements), box {64, box_rows}, 128B swizzle.
+bool make_map(CUtensorMap* m, const void* ptr, int64_t rows, int64_t cols, int64_t ld,
+              int box_rows) {
+  EncodeTiledFn fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[2] = {static_cast<cuuint64_t>(cols), static_cast<cuuint64_t>(rows)};
+  cuuint64_t strides[1] = {static_cast<cuuint64_t>(ld) * 2};
+  cuuint32_t box[2] = {static_cast<cuuint32_t>(BK), static_cast<cuuint32_t>(box_rows)};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ptr), dims, strides,
+                  box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                  CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
+struct Maps {
+  CUtensorMap a, a2, b, b2;
+};
+
+template <int BN, int EPI, bool SPLIT>
+int launch_kernel(const Maps& m, const Params& p, int grid, cudaStream_t stream) {
+  // ~192 KB of stages: BN=256 -> 4 (3 split), BN=128 -> 6 (4 split)
+  constexpr int STAGE = (SPLIT ? 2 : 1) * BM * BK * 2 + BN * BK * 2;
+  constexpr int STAGES = (196608 / STAGE) < 8 ? (196608 / STAGE) : 8;
+  constexpr int smem = STAGES * STAGE + 1024 + 256;
+  static bool attr_set = false;
+  auto kern = gemm_tc_kernel<BN, STAGES, EPI, SPLIT>;
+  if (!attr_set) {
+    VLA_CUDA_TRY(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem));
+    attr_set = true;
+  }
+  kern<<<grid, kThreads, smem, stream>>>(m.a, m.a2, m.b, m.b2, p);
+  note_launch();
+  VLA_CUDA_TRY(cudaGetLastError());
+  return VLA_OK;
+}
+
+template <int BN, bool SPLIT>
+int dispatch_epi(int epi, const Maps& m, const Params& p, int grid, cudaStream_t s) {
+  switch (epi) {
+    case EPI_F32: return launch_kernel<BN, EPI_F32, SPLIT>(m, p, grid, s);
+    case EPI_RESID: return launch_kernel<BN, EPI_RESID, SPLIT>(m, p, grid, s);
+    case EPI_SWIGLU: return launch_kernel<BN, EPI_SWIGLU, SPLIT>(m, p, grid, s);
+    case EPI_QKV: return launch_kernel<BN, EPI_QKV, SPLIT>(m, p, grid, s);
+    case EPI_PARTIAL: return launch_kernel<BN, EPI_PARTIAL, SPLIT>(m, p, grid, s);
+  }
+  return VLA_ERR_ARG;
+}
+
+int blocks_for(int64_t n) {
+  int64_t b = (n + 255) / 256;
+  if (b > 4096) b = 4096;
+  return static_cast<int>(b < 1 ? 1 : b);
+}
+
+}  // namespace
+
+int gemm_effective_splits(int K, int splits) {
+  const int kbt = (K + BK - 1) / BK;
+  if (splits < 1) splits = 1;
+  if (splits > kbt) splits = kbt;
+  const int kbps = (kbt + splits - 1) / splits;
+  return (kbt + kbps - 1) / kbps;
+}
+
+size_t gemm_workspace_bytes(const GemmArgs& a) {
+  const int s = gemm_effective_splits(a.K, a.splits);
+  if (s <= 1) return 0;
+  return static_cast<size_t>(s) * a.M * a.N * sizeof(float);
+}
+
+int gemm_launch(const GemmArgs& a, cudaStream_t stream, int num_sms, GemmCost* cost) {
+  if (a.M < 1 || a.N < 1 || a.K < 1 || !a.A || !a.B) return VLA_ERR_ARG;
+  if (a.block_n != 128 && a.block_n != 256) return VLA_ERR_ARG;
+  if ((a.lda % 8) || (a.ldb % 8) || a.lda < a.K || a.ldb < a.K) return VLA_ERR_ARG;
+  if ((reinterpret_cast<uintptr_t>(a.A) & 15) || (reinterpret_cast<uintptr_t>(a.B) & 15) ||
+      (reinterpret_cast<uintptr_t>(a.A_lo) & 15))
+    return VLA_ERR_ARG;
+  const bool split = a.A_lo != nullptr;
+  const int BN = a.block_n;
+  const int epi = a.epi.kind;
+  const bool swiglu = (epi == EPI_SWIGLU);
+  if (swiglu && (a.N & 1)) return VLA_ERR_ARG;
+  if (epi == EPI_QKV && (a.epi.d % BN || BN % a.epi.hd || a.N != 3 * a.epi.d)) return VLA_ERR_ARG;
+
+  const int splits = gemm_effective_splits(a.K, a.splits);
+  const int kbt = (a.K + BK - 1) / BK;
+  Params p{};
+  p.M = a.M;
+  p.N = a.N;
+  p.K = a.K;
+  p.tiles_m = (a.M + BM - 1) / BM;
+  p.splits = splits;
+  p.kb_total = kbt;
+  p.kb_per_split = (kbt + splits - 1) / splits;
+  p.epi = a.epi;
+
+  Maps maps;
+  CUtensorMap &ma = maps.a, &mb = maps.b, &mb2 = maps.b2;
+  if (!make_map(&ma, a.A, a.M, a.K, a.lda, BM)) return cuda_fail(cudaErrorInvalidValue, "tensor map A");
+  maps.a2 = ma;
+  if (split && !make_map(&maps.a2, a.A_lo, a.M, a.K, a.lda, BM))
+    return cuda_fail(cudaErrorInvalidValue, "tensor map A (low half)");
+  int run_epi = epi;
+  if (splits > 1) {
+    // Split-K: plain tiles of B into the workspace, then a fixed-order reduction applying
+    // the epilogue.
+    if (!a.workspace || a.workspace_bytes < gemm_workspace_bytes(a)) return VLA_ERR_ARG;
+    run_epi = EPI_PARTIAL;
+    p.epi.out_f32 = a.workspace;
+    p.tiles_n = (a.N + BN - 1) / BN;
+    if (!make_map(&mb, a.B, a.N, a.K, a.ldb, BN)) return cuda_fail(cudaErrorInvalidValue, "tensor map B");
+    mb2 = mb;
+  } else if (swiglu) {
+    const int F = a.N / 2;
+    p.tiles_n = (F + BN / 2 - 1) / (BN / 2);
+    const bf16* up = a.B + static_cast<size_t>(F) * a.ldb;
+    if ((reinterpret_cast<uintptr_t>(up) & 15)) return VLA_ERR_ARG;
+    if (!make_map(&mb, a.B, F, a.K, a.ldb, BN / 2) || !make_map(&mb2, up, F, a.K, a.ldb, BN / 2))
+      return cuda_fail(cudaErrorInvalidValue, "tensor map B (gate/up)");
+  } else {
+    p.tiles_n = (a.N + BN - 1) / BN;
+    if (!make_map(&mb, a.B, a.N, a.K, a.ldb, BN)) return cuda_fail(cudaErrorInvalidValue, "tensor map B");
+    mb2 = mb;
+  }
+  const int64_t units = static_cast<int64_t>(p.tiles_m) * p.tiles_n * p.splits;
+  const int grid = static_cast<int>(units < num_sms ? units : num_sms);
+  int rc;
+  if (split)
+    rc = (BN == 256) ? dispatch_epi<256, true>(run_epi, maps, p, grid, stream)
+                     : dispatch_epi<128, true>(run_epi, maps, p, grid, stream);
+  else
+    rc = (BN == 256) ? dispatch_epi<256, false>(run_epi, maps, p, grid, stream)
+                     : dispatch_epi<128, false>(run_epi, maps, p, grid, stream);
+  if (rc != VLA_OK) return rc;
+
+  if (splits > 1) {
+    const float* ws = a.workspace;
+    switch (epi) {
+      case EPI_F32:
+      case EPI_RESID: {
+        float* out = (epi == EPI_F32) ? a.epi.out_f32 : a.epi.resid;
+        const int ld = (epi == EPI_F32) ? a.epi.ldo : a.epi.ldr;
+        reduce_f32_kernel<<<blocks_for(static_cast<int64_t>(a.M) * a.N), 256, 0, stream>>>(
+            ws, splits, a.M, a.N, out, ld, epi == EPI_RESID);
+        break;
+      }
+      case EPI_SWIGLU:
+        reduce_swiglu_kernel<<<blocks_for(static_cast<int64_t>(a.M) * a.N / 2), 256, 0, stream>>>(
+            ws, splits, a.M, a.N / 2, a.epi.out_hi, a.epi.out_lo, a.epi.ldo);
+        break;
+      case EPI_QKV:
+        reduce_qkv_kernel<<<blocks_for(static_cast<int64_t>(a.M) * a.N / 2), 256, 0, stream>>>(
+            ws, splits, a.M, a.epi);
+        break;
+      default:
+        return VLA_ERR_ARG;
+    }
+    note_launch();
+    VLA_CUDA_TRY(cudaGetLastError());
+  }
+  if (cost) {
+    // Algorithmic work of the model's product: 2MNK flops (the low-half MMAs of a split A are
+    // not counted); bytes = A + B read once, output written once (+ read for the residual).
+    cost->flops = 2.0 * a.M * static_cast<double>(a.N) * a.K;
+    double out_bytes;
+    switch (epi) {
+      case EPI_RESID: out_bytes = 8.0 * a.M * a.N; break;
+      case EPI_SWIGLU: out_bytes = 2.0 * a.M * (a.N / 2); break;
+      case EPI_QKV: out_bytes = 2.0 * a.M * a.N; break;
+      default: out_bytes = 4.0 * a.M * a.N;
+    }
+    cost->bytes = 2.0 * (static_cast<double>(a.M) * a.K + static_cast<double>(a.N) * a.K) + out_bytes;
+  }
+  return VLA_OK;
+}
+
+}  // namespace vla

@@ -1,0 +1,128 @@
+// Row kernels of the hot path: chunk assembly (Algorithm 1: the state h(o_t) ‖ v_t^in, plus
+// the pending action token of the previous turn in a multi-turn trajectory, §3.3), RMSNorm
+// of the Llama-2 backbone (§3.1; fp32 math, output as the bf16 hi/lo pair the GEMM reads)
+// and row gathers.  All HBM-bound; one CTA per row, vector accesses.
+#include "misc.h"
+
+namespace vla {
+
+int64_t g_launch_count = 0;
+
+namespace {
+
+__global__ void __launch_bounds__(256) assemble_kernel(const RowInfo* __restrict__ rows,
+                                                       const bf16* __restrict__ visual,
+                                                       const int* __restrict__ ids,
+                                                       const int* __restrict__ tokens,
+                                                       const bf16* __restrict__ embed, int d,
+                                                       int vocab, float* __restrict__ h,
+                                                       uint32_t* status) {
+  const RowInfo ri = rows[blockIdx.x];
+  const bf16* src;
+  if (ri.kind == ROW_VISUAL) {
+    src = visual + static_cast<size_t>(ri.idx) * d;
+  } else {
+    int id = (ri.kind == ROW_TEXT) ? ids[ri.idx] : tokens[ri.idx];
+    if (id < 0 || id >= vocab) {
+      if (threadIdx.x == 0) atomicOr(status, VLA_STATUS_BAD_TOKEN);
+      id = 0;
+    }
+    src = embed + static_cast<size_t>(id) * d;
+  }
+  float* dst = h + static_cast<size_t>(blockIdx.x) * d;
+  for (int c = threadIdx.x * 8; c < d; c += blockDim.x * 8) {
+    const uint4 v = *reinterpret_cast<const uint4*>(src + c);
+    const float2 a = unpack_bf16x2(v.x), b = unpack_bf16x2(v.y);
+    const float2 e = unpack_bf16x2(v.z), f = unpack_bf16x2(v.w);
+    reinterpret_cast<float4*>(dst + c)[0] = make_float4(a.x, a.y, b.x, b.y);
+    reinterpret_cast<float4*>(dst + c)[1] = make_float4(e.x, e.y, f.x, f.y);
+  }
+}
+
+__global__ void __launch_bounds__(256) rmsnorm_kernel(const float* __restrict__ h,
+                                                      const bf16* __restrict__ w, int d,
+                                                      float eps, bf16* __restrict__ y_hi,
+                                                      bf16* __restrict__ y_lo) {
+  __shared__ float red[8];
+  const float* row = h + static_cast<size_t>(blockIdx.x) * d;
+  float ss = 0.f;
+  for (int c = threadIdx.x * 4; c < d; c += blockDim.x * 4) {
+    const float4 v = *reinterpret_cast<const float4*>(row + c);
+    ss += v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w;
+  }
+  ss = warp_sum(ss);
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = ss;
+  __syncthreads();
+  float tot = 0.f;
+  for (int i = 0; i < (blockDim.x >> 5); ++i) tot += red[i];
+  const float r = rsqrtf(tot / static_cast<float>(d) + eps);
+  const size_t off = static_cast<size_t>(blockIdx.x) * d;
+  for (int c = threadIdx.x * 4; c < d; c += blockDim.x * 4) {
+    const float4 v = *reinterpret_cast<const float4*>(row + c);
+    const uint2 ww = *reinterpret_cast<const uint2*>(w + c);
+    const float2 w0 = unpack_bf16x2(ww.x), w1 = unpack_bf16x2(ww.y);
+    uint2 hi, lo;
+    split_pack2(v.x * r * w0.x, v.y * r * w0.y, hi.x, lo.x);
+    split_pack2(v.z * r * w1.x, v.w * r * w1.y, hi.y, lo.y);
+    *reinterpret_cast<uint2*>(y_hi + off + c) = hi;
+    *reinterpret_cast<uint2*>(y_lo + off + c) = lo;
+  }
+}
+
+__global__ void gather_rows_kernel(const float* __restrict__ src, const int* __restrict__ idx,
+                                   int d, float* __restrict__ dst) {
+  const float* s = src + static_cast<size_t>(idx[blockIdx.x]) * d;
+  float* o = dst + static_cast<size_t>(blockIdx.x) * d;
+  for (int c = threadIdx.x * 4; c < d; c += blockDim.x * 4)
+    *reinterpret_cast<float4*>(o + c) = *reinterpret_cast<const float4*>(s + c);
+}
+
+__global__ void scatter_rows_kernel(const float* __restrict__ src, const int* __restrict__ sidx,
+                                    const int* __restrict__ didx, int d, float* __restrict__ dst) {
+  const float* s = src + static_cast<size_t>(sidx[blockIdx.x]) * d;
+  float* o = dst + static_cast<size_t>(didx[blockIdx.x]) * d;
+  for (int c = threadIdx.x * 4; c < d; c += blockDim.x * 4)
+    *reinterpret_cast<float4*>(o + c) = *reinterpret_cast<const float4*>(s + c);
+}
+
+}  // namespace
+
+int assemble_launch(const RowInfo* rows, int n_rows, const bf16* visual, const int* ids,
+                    const int* tokens, const bf16* embed, int d, int vocab, float* h,
+                    uint32_t* status, cudaStream_t s) {
+  if (n_rows <= 0) return VLA_OK;
+  assemble_kernel<<<n_rows, 256, 0, s>>>(rows, visual, ids, tokens, embed, d, vocab, h, status);
+  note_launch();
+  VLA_CUDA_TRY(cudaGetLastError());
+  return VLA_OK;
+}
+
+int rmsnorm_launch(const float* h, const bf16* w, int M, int d, float eps, bf16* y_hi,
+                   bf16* y_lo, cudaStream_t s) {
+  if (M <= 0) return VLA_OK;
+  rmsnorm_kernel<<<M, 256, 0, s>>>(h, w, d, eps, y_hi, y_lo);
+  note_launch();
+  VLA_CUDA_TRY(cudaGetLastError());
+  return VLA_OK;
+}
+
+int gather_rows_launch(const float* src, const int* idx, int n, int d, float* dst, cudaStream_t s) {
+  if (n <= 0) return VLA_OK;
+  gather_rows_kernel<<<n, 256, 0, s>>>(src, idx, d, dst);
+  note_launch();
+  VLA_CUDA_TRY(cudaGetLastError());
+  return VLA_OK;
+}
+
+}  // namespace vla
+
+namespace vla {
+int scatter_rows_launch(const float* src, const int* sidx, const int* didx, int n, int d, float* dst,
+                        cudaStream_t s) {
+  if (n <= 0) return VLA_OK;
+  scatter_rows_kernel<<<n, 256, 0, s>>>(src, sidx, didx, d, dst);
+  note_launch();
+  VLA_CUDA_TRY(cudaGetLastError());
+  return VLA_OK;
+}
+}  // namespace vla

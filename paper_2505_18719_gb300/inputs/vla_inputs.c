@@ -75,8 +75,8 @@ static void run_range(const job_t* j) {
   } else if (j->kind == K_UNIFORM_F32) {
     float* o = (float*)j->out;
     for (int64_t e = j->begin; e < j->end; ++e) {
-      uint64_t m = draw(j->key, (uint64_t)e) >> 40; /* 24 bits */
-      o[e] = (float)(((double)m + 0.5) * 0x1p-24);  /* exact in fp32, in (0,1) */
+      uint64_t m = draw(j->key, (uint64_t)e) >> 41; /* 23 bits */
+      o[e] = (float)(((double)m + 0.5) * 0x1p-23);  /* (2m+1) 2^-24: exact in fp32, in (0,1) */
     }
   } else {
     int32_t* o = (int32_t*)j->out;
@@ -138,7 +138,7 @@ void vla_gen_normal_bf16(uint16_t* out, int64_t n, uint64_t seed, uint64_t strea
   run_parallel(j, n);
 }
 
-/* out[i] = (m + 0.5) * 2^-24, m uniform in [0, 2^24): strictly inside (0, 1). */
+/* out[i] = (m + 0.5) * 2^-23, m uniform in [0, 2^23): exact in fp32, in [2^-24, 1 - 2^-24]. */
 void vla_gen_uniform_f32(float* out, int64_t n, uint64_t seed, uint64_t stream) {
   job_t j = {K_UNIFORM_F32, out, 0, 0, stream_key(seed, stream), 0, 0, 0, 0};
   run_parallel(j, n);

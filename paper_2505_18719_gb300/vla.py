@@ -1,0 +1,271 @@
+"""ctypes binding of libvla.so (include/vla.h, include/vla_ops.h): argument marshalling only.
+
+Every step of the hot path runs in the CUDA library.  There is no fallback: if the library
+is missing or fails to load, importing this module's functions raises.
+
+Functions keep the C names (``vla_create``, ``vla_prefill``, ``vla_decode_actions``,
+``vla_score_actions``, ``vla_reset``, ``vla_sync``, ``vla_last_error``, ``vla_destroy``,
+...).  ``Policy`` is a convenience wrapper that holds torch device tensors and a handle.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from typing import Dict, Optional, Sequence
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(HERE, "libvla.so")
+
+VLA_OK = 0
+VLA_ERR_ARG = -1
+VLA_ERR_CAPACITY = -2
+VLA_ERR_STATE = -3
+VLA_ERR_CUDA = -4
+VLA_ERR_OOM = -5
+VLA_ERR_DEVICE_STATUS = -6
+VLA_ERR_UNSUPPORTED = -7
+
+VLA_STATUS_BAD_TOKEN = 0x1
+VLA_STATUS_NONFINITE = 0x2
+VLA_STATUS_TIMEOUT = 0x4
+VLA_STATUS_BAD_FORCED = 0x8
+
+KCLASS = ("gemm_prefill", "gemm_decode", "attn_prefill", "attn_decode", "head", "other")
+
+
+class VlaConfig(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_int) for n in ("n_layers", "d_model", "n_heads", "head_dim", "d_ffn",
+                                             "vocab", "n_action_bins", "action_dim", "max_batch",
+                                             "kv_capacity", "max_tokens")] + \
+               [("rms_eps", ctypes.c_float), ("rope_theta", ctypes.c_float)]
+
+
+class VlaWeights(ctypes.Structure):
+    _fields_ = [("embed", ctypes.c_void_p),
+                ("attn_norm", ctypes.POINTER(ctypes.c_void_p)),
+                ("wqkv", ctypes.POINTER(ctypes.c_void_p)),
+                ("wo", ctypes.POINTER(ctypes.c_void_p)),
+                ("ffn_norm", ctypes.POINTER(ctypes.c_void_p)),
+                ("w_gate_up", ctypes.POINTER(ctypes.c_void_p)),
+                ("w_down", ctypes.POINTER(ctypes.c_void_p)),
+                ("final_norm", ctypes.c_void_p),
+                ("lm_head", ctypes.c_void_p)]
+
+
+class VlaError(RuntimeError):
+    def __init__(self, code: int, msg: str):
+        super().__init__(f"vla error {code}: {msg}")
+        self.code = code
+
+
+_lib = None
+
+
+def load(path: str = LIB_PATH):
+    """Load libvla.so (raises if it is missing: build it with paper_2505_18719_gb300.build)."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(path):
+        raise FileNotFoundError(f"{path} is missing; run `python -c 'import __graft_entry__ as g; g.build()'`")
+    lib = ctypes.CDLL(path)
+    vp, i32, f32, u32, i64 = ctypes.c_void_p, ctypes.c_int, ctypes.c_float, ctypes.c_uint32, ctypes.c_int64
+    sig = {
+        "vla_create": (i32, [ctypes.POINTER(VlaConfig), ctypes.POINTER(VlaWeights), vp, ctypes.POINTER(vp)]),
+        "vla_prefill": (i32, [vp, i32, vp, i32, vp, ctypes.POINTER(ctypes.c_int32), i32]),
+        "vla_decode_actions": (i32, [vp, vp, f32, vp, vp, vp, vp, vp]),
+        "vla_score_actions": (i32, [vp, vp, f32, vp, vp]),
+        "vla_reset": (i32, [vp, vp]),
+        "vla_sync": (i32, [vp]),
+        "vla_context_length": (i32, [vp, i32]),
+        "vla_last_error": (ctypes.c_char_p, [vp]),
+        "vla_destroy": (None, [vp]),
+        "vla_profile": (i32, [vp, u32]),
+        "vla_profile_read": (i32, [vp, vp, vp, vp, vp]),
+        "vla_launch_count": (i64, [vp]),
+        "vla_op_gemm_bf16": (i32, [vp, vp, i32, vp, i32, vp, i32, i32, i32, i32, i32, i32, vp, vp]),
+        "vla_op_action_head": (i32, [vp, i32, i32, i32, vp, vp, f32, vp, f32, vp, vp, vp, vp, vp, vp, vp]),
+        "vla_op_num_sms": (i32, []),
+    }
+    for name, (res, args) in sig.items():
+        f = getattr(lib, name)
+        f.restype = res
+        f.argtypes = args
+    _lib = lib
+    return lib
+
+
+# ---------------------------------------------------------------------------- C-named wrappers
+def vla_last_error(handle=None) -> str:
+    s = load().vla_last_error(handle)
+    return s.decode() if s else ""
+
+
+def _check(rc: int, handle=None):
+    if rc != VLA_OK:
+        raise VlaError(rc, vla_last_error(handle))
+    return rc
+
+
+def vla_create(cfg: VlaConfig, weights: VlaWeights, stream: int = 0):
+    h = ctypes.c_void_p()
+    rc = load().vla_create(ctypes.byref(cfg), ctypes.byref(weights), ctypes.c_void_p(stream or None),
+                           ctypes.byref(h))
+    _check(rc)
+    return h
+
+
+def vla_prefill(h, batch: int, visual_ptr: int, n_visual: int, ids_ptr: int, lengths: Sequence[int],
+                max_len: int) -> int:
+    lens = (ctypes.c_int32 * len(lengths))(*[int(x) for x in lengths])
+    return load().vla_prefill(h, batch, visual_ptr or None, n_visual, ids_ptr or None, lens, max_len)
+
+
+def vla_decode_actions(h, uniforms_ptr: int, temperature: float, forced_ptr: int, tokens_ptr: int,
+                       logprobs_ptr: int, actions_ptr: int, logits_ptr: int = 0) -> int:
+    return load().vla_decode_actions(h, uniforms_ptr or None, float(temperature), forced_ptr or None,
+                                     tokens_ptr or None, logprobs_ptr or None, actions_ptr or None,
+                                     logits_ptr or None)
+
+
+def vla_score_actions(h, tokens_ptr: int, temperature: float, logprobs_ptr: int, logits_ptr: int = 0) -> int:
+    return load().vla_score_actions(h, tokens_ptr or None, float(temperature), logprobs_ptr or None,
+                                    logits_ptr or None)
+
+
+def vla_reset(h, env_mask: Optional[Sequence[int]] = None) -> int:
+    if env_mask is None:
+        return load().vla_reset(h, None)
+    m = (ctypes.c_uint8 * len(env_mask))(*[1 if x else 0 for x in env_mask])
+    return load().vla_reset(h, m)
+
+
+def vla_sync(h) -> int:
+    return load().vla_sync(h)
+
+
+def vla_context_length(h, env: int) -> int:
+    return load().vla_context_length(h, env)
+
+
+def vla_destroy(h) -> None:
+    load().vla_destroy(h)
+
+
+def vla_profile(h, class_mask: int) -> int:
+    return load().vla_profile(h, class_mask)
+
+
+def vla_profile_read(h) -> Dict[str, dict]:
+    n = len(KCLASS)
+    la = (ctypes.c_int64 * n)()
+    ms = (ctypes.c_double * n)()
+    fl = (ctypes.c_double * n)()
+    by = (ctypes.c_double * n)()
+    _check(load().vla_profile_read(h, la, ms, fl, by), h)
+    return {KCLASS[i]: {"launches": la[i], "ms": ms[i], "flops": fl[i], "bytes": by[i]} for i in range(n)}
+
+
+def vla_launch_count(h=None) -> int:
+    return load().vla_launch_count(h)
+
+
+def vla_op_gemm_bf16(A_ptr, A_lo_ptr, lda, W_ptr, ldw, C_ptr, ldc, M, N, K, block_n=256, splits=1,
+                     ws_ptr=0, stream=0) -> int:
+    return load().vla_op_gemm_bf16(A_ptr, A_lo_ptr or None, lda, W_ptr, ldw, C_ptr, ldc, M, N, K,
+                                   block_n, splits, ws_ptr or None, stream or None)
+
+
+def vla_op_action_head(h_ptr, ldh, B, d, final_norm_ptr, head_rows_ptr, eps, uniforms_ptr, temperature,
+                       forced_ptr, bins_ptr, lp_ptr, act_ptr, logits_ptr, status_ptr, stream=0) -> int:
+    return load().vla_op_action_head(h_ptr, ldh, B, d, final_norm_ptr, head_rows_ptr, float(eps),
+                                     uniforms_ptr or None, float(temperature), forced_ptr or None,
+                                     bins_ptr or None, lp_ptr, act_ptr or None, logits_ptr or None,
+                                     status_ptr, stream or None)
+
+
+def vla_op_num_sms() -> int:
+    return load().vla_op_num_sms()
+
+
+# ---------------------------------------------------------------------------- convenience
+class Policy:
+    """A handle plus the torch device tensors it borrows (weights) or fills (outputs).
+
+    torch is used only to hold device memory and to name the stream; all compute is in
+    libvla.so.
+    """
+
+    def __init__(self, shape, weights_dev: Dict, max_batch: int, kv_capacity: int, max_tokens: int,
+                 stream=None):
+        import torch
+        self.torch = torch
+        self.shape = shape
+        self.w = weights_dev
+        L = shape.n_layers
+        cfg = VlaConfig(shape.n_layers, shape.d_model, shape.n_heads, shape.head_dim, shape.d_ffn,
+                        shape.vocab, shape.n_bins, shape.action_dim, max_batch, kv_capacity, max_tokens,
+                        shape.rms_eps, shape.rope_theta)
+        arr = lambda name: (ctypes.c_void_p * L)(*[weights_dev[name][l].data_ptr() for l in range(L)])
+        self._keep = {n: arr(n) for n in ("attn_norm", "wqkv", "wo", "ffn_norm", "w_gate_up", "w_down")}
+        cast = lambda a: ctypes.cast(a, ctypes.POINTER(ctypes.c_void_p))
+        wts = VlaWeights(weights_dev["embed"].data_ptr(), cast(self._keep["attn_norm"]),
+                         cast(self._keep["wqkv"]), cast(self._keep["wo"]), cast(self._keep["ffn_norm"]),
+                         cast(self._keep["w_gate_up"]), cast(self._keep["w_down"]),
+                         weights_dev["final_norm"].data_ptr(), weights_dev["lm_head"].data_ptr())
+        self.stream = stream if stream is not None else torch.cuda.current_stream()
+        self.h = vla_create(cfg, wts, self.stream.cuda_stream)
+        self.max_batch = max_batch
+        self.B = 0
+
+    def close(self):
+        if self.h:
+            vla_destroy(self.h)
+            self.h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def check(self, rc):
+        return _check(rc, self.h)
+
+    def prefill(self, visual, ids, lengths):
+        """visual bf16 [B, Nv, d] (device), ids int32 [B, L] (device), lengths host ints."""
+        B = len(lengths)
+        nv = visual.shape[1] if visual is not None else 0
+        self.check(vla_prefill(self.h, B, visual.data_ptr() if visual is not None else 0, nv,
+                               ids.data_ptr() if ids is not None else 0, list(lengths),
+                               ids.shape[1] if ids is not None else 0))
+        self.B = B
+
+    def decode(self, uniforms, temperature: float, forced=None, want_logits: bool = True):
+        t = self.torch
+        B, A = self.B, self.shape.action_dim
+        dev = uniforms.device if uniforms is not None else t.device("cuda")
+        out = {"tokens": t.empty(B, A, dtype=t.int32, device=dev),
+               "logprobs": t.empty(B, A, dtype=t.float32, device=dev),
+               "actions": t.empty(B, A, dtype=t.float32, device=dev),
+               "logits": t.empty(B, A, 256, dtype=t.float32, device=dev) if want_logits else None}
+        self.check(vla_decode_actions(self.h, uniforms.data_ptr() if uniforms is not None else 0, temperature,
+                                      forced.data_ptr() if forced is not None else 0, out["tokens"].data_ptr(),
+                                      out["logprobs"].data_ptr(), out["actions"].data_ptr(),
+                                      out["logits"].data_ptr() if want_logits else 0))
+        return out
+
+    def score(self, tokens, temperature: float, want_logits: bool = True):
+        t = self.torch
+        B, A = self.B, self.shape.action_dim
+        out = {"logprobs": t.empty(B, A, dtype=t.float32, device=tokens.device),
+               "logits": t.empty(B, A, 256, dtype=t.float32, device=tokens.device) if want_logits else None}
+        self.check(vla_score_actions(self.h, tokens.data_ptr(), temperature, out["logprobs"].data_ptr(),
+                                     out["logits"].data_ptr() if want_logits else 0))
+        return out
+
+    def reset(self, mask=None):
+        self.check(vla_reset(self.h, mask))
+
+    def sync(self):
+        self.check(vla_sync(self.h))

@@ -1,0 +1,59 @@
+"""The C-ABI library loads and exports every symbol its headers declare; host-side argument
+checks return their documented codes without touching a GPU (CPU only)."""
+import ctypes
+import os
+import re
+
+import pytest
+
+from paper_2505_18719_gb300 import build as B
+from paper_2505_18719_gb300 import vla as V
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    B.build()
+    return V.load()
+
+
+def declared_functions():
+    names = []
+    for hdr in ("vla.h", "vla_ops.h"):
+        src = open(os.path.join(ROOT, "include", hdr)).read()
+        src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+        names += re.findall(r"\b(vla_[a-z0-9_]+)\s*\(", src)
+    return sorted(set(names))
+
+
+def test_every_declared_symbol_is_exported(lib):
+    names = declared_functions()
+    assert "vla_create" in names and "vla_decode_actions" in names and "vla_op_gemm_bf16" in names
+    for n in names:
+        assert hasattr(lib, n), n
+
+
+def test_host_argument_errors_without_gpu(lib):
+    h = ctypes.c_void_p()
+    assert lib.vla_create(None, None, None, ctypes.byref(h)) == V.VLA_ERR_ARG
+    assert h.value is None
+    assert "NULL" in V.vla_last_error(None)
+    cfg = V.VlaConfig(2, 256, 4, 48, 688, 32064, 256, 7, 4, 128, 512, 1e-6, 1e4)  # head_dim 48
+    w = V.VlaWeights()
+    assert lib.vla_create(ctypes.byref(cfg), ctypes.byref(w), None, ctypes.byref(h)) == V.VLA_ERR_UNSUPPORTED
+    cfg.head_dim = 64
+    cfg.n_action_bins = 128
+    assert lib.vla_create(ctypes.byref(cfg), ctypes.byref(w), None, ctypes.byref(h)) == V.VLA_ERR_UNSUPPORTED
+    cfg.n_action_bins = 256
+    assert lib.vla_create(ctypes.byref(cfg), ctypes.byref(w), None, ctypes.byref(h)) == V.VLA_ERR_ARG  # NULL weights
+    assert lib.vla_prefill(None, 1, None, 0, None, None, 0) == V.VLA_ERR_ARG
+    assert lib.vla_decode_actions(None, None, 1.0, None, None, None, None, None) == V.VLA_ERR_ARG
+    assert lib.vla_score_actions(None, None, 1.0, None, None) == V.VLA_ERR_ARG
+    assert lib.vla_reset(None, None) == V.VLA_ERR_ARG
+    assert lib.vla_sync(None) == V.VLA_ERR_ARG
+    assert lib.vla_context_length(None, 0) == -1
+    lib.vla_destroy(None)  # no-op
+    assert lib.vla_op_gemm_bf16(None, None, 0, None, 0, None, 0, 0, 0, 0, 256, 1, None, None) == V.VLA_ERR_ARG
+    assert lib.vla_op_action_head(None, 0, 0, 0, None, None, 1e-6, None, 1.0, None, None, None, None,
+                                  None, None, None) == V.VLA_ERR_ARG

@@ -1,0 +1,100 @@
+"""Single-kernel parity through the C ABI (vla_ops.h): the tcgen05 GEMM and the action head
+against fp64 CPU references, on ragged shapes that span several tiles."""
+import math
+import types
+
+import numpy as np
+import pytest
+import torch
+
+import oracle.vla_oracle as O
+from paper_2505_18719_gb300 import inputs as I
+from paper_2505_18719_gb300 import vla as V
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def lib():
+    from paper_2505_18719_gb300 import build
+    build.build()
+    return V.load()
+
+
+GEMM_CASES = [
+    # M, N, K, block_n, splits, split A (hi/lo pair)
+    (1, 128, 64, 128, 1, False),
+    (4, 256, 256, 256, 1, True),
+    (130, 384, 688, 128, 1, False),     # ragged M and K tails
+    (130, 384, 688, 128, 1, True),
+    (300, 512, 1024, 256, 1, True),
+    (257, 200, 136, 128, 2, True),      # ragged N, split-K
+    (64, 384, 4096, 128, 5, False),     # decode-like: few tiles, split-K
+    (64, 384, 4096, 128, 5, True),
+    (1000, 768, 256, 256, 1, False),    # many tiles (persistent loop, both accumulators)
+    (2304, 1024, 512, 256, 1, True),    # > 16 m-tiles: grouped raster
+]
+
+
+@pytest.mark.parametrize("M,N,K,bn,splits,split_a", GEMM_CASES)
+def test_gemm_matches_fp64(M, N, K, bn, splits, split_a):
+    A = I.normal_bf16((M, K), 99, 1000 + M, 1.0)
+    A_lo = I.normal_bf16((M, K), 99, 3000 + M, 2.0 ** -9)   # a realistic low half
+    W = I.normal_bf16((N, K), 99, 2000 + N, 1.0)
+    Ad, Ald, Wd = A.cuda(), A_lo.cuda(), W.cuda()
+    C = torch.full((M, N), float("nan"), dtype=torch.float32, device="cuda")
+    ws = torch.empty(max(1, splits * M * N), dtype=torch.float32, device="cuda")
+    rc = V.vla_op_gemm_bf16(Ad.data_ptr(), Ald.data_ptr() if split_a else 0, K, Wd.data_ptr(), K,
+                            C.data_ptr(), N, M, N, K, bn, splits, ws.data_ptr(), 0)
+    assert rc == 0, V.vla_last_error()
+    torch.cuda.synchronize()
+    Aref = A.double() + A_lo.double() if split_a else A.double()
+    ref = Aref @ W.double().T
+    err = (C.cpu().double() - ref).abs().max().item()
+    # exact bf16 products, fp32 sums: error ~ sqrt(K) * |sum| * 2^-24
+    assert err < 2e-5 * math.sqrt(K) * 8, err
+
+
+def test_gemm_rejects_bad_strides():
+    A = torch.zeros(8, 12, dtype=torch.bfloat16, device="cuda")
+    C = torch.zeros(8, 8, dtype=torch.float32, device="cuda")
+    rc = V.vla_op_gemm_bf16(A.data_ptr(), 0, 12, A.data_ptr(), 12, C.data_ptr(), 8, 8, 8, 12, 128, 1, 0, 0)
+    assert rc == V.VLA_ERR_ARG          # 12 * 2 bytes is not a multiple of 16
+
+
+@pytest.mark.parametrize("T", [0.0, 1.0, 1.5])
+@pytest.mark.parametrize("forced", [False, True])
+def test_action_head_matches_fp64(T, forced):
+    B, d = 16, 4096
+    h = I.normal_bf16((B, d), 7, 1, 1.0).float() * 3.0
+    fn = I.normal_bf16((d,), 7, 2, 0.1, 1.0)
+    rows = I.normal_bf16((256, d), 7, 3, 0.02)
+    u = I.uniform_f32((B, 256), 7, 4)
+    fb = I.randint_i32((B,), 7, 5, 0, 255)
+    dev = {k: v.cuda() for k, v in dict(h=h, fn=fn, rows=rows, u=u, fb=fb).items()}
+    bins = torch.empty(B, dtype=torch.int32, device="cuda")
+    lp = torch.empty(B, dtype=torch.float32, device="cuda")
+    act = torch.empty(B, dtype=torch.float32, device="cuda")
+    logits = torch.empty(B, 256, dtype=torch.float32, device="cuda")
+    status = torch.zeros(1, dtype=torch.int32, device="cuda")
+    rc = V.vla_op_action_head(dev["h"].data_ptr(), d, B, d, dev["fn"].data_ptr(), dev["rows"].data_ptr(),
+                              1e-6, dev["u"].data_ptr(), T, dev["fb"].data_ptr() if forced else 0,
+                              bins.data_ptr(), lp.data_ptr(), act.data_ptr(), logits.data_ptr(),
+                              status.data_ptr(), 0)
+    assert rc == 0
+    torch.cuda.synchronize()
+    assert int(status.item()) == 0
+    W = types.SimpleNamespace(final_norm=O.f64(fn), head_rows=O.f64(rows))
+    sh = O.Shape(1, d, 32, 128, 8, 32064)
+    checked = 0
+    for b in range(B):
+        z = O.head_logits(sh, W, O.f64(h[b]))
+        k, lps, margin = O.sample_bins(z, T, u[b])
+        assert np.max(np.abs(logits[b].cpu().numpy() - z.numpy())) < 1e-4
+        want = int(fb[b]) if forced else k
+        assert abs(lp[b].item() - float(lps[want])) < 1e-4
+        if margin > 0.05:
+            checked += 1
+            assert int(bins[b].item()) == k
+            assert act[b].item() == O.bin_centre(k)
+    assert checked >= B // 2

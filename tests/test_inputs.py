@@ -23,8 +23,9 @@ def test_distributions():
     assert abs(x.mean()) < 1e-4 and abs(x.std() - 0.02) < 2e-4
     u = I.uniform_f32((1_000_000,), 1, 2).numpy()
     assert u.min() > 0 and u.max() < 1 and abs(u.mean() - 0.5) < 2e-3
-    m = u * 2 ** 24 - 0.5
-    assert np.array_equal(m, np.round(m))           # (m + 0.5) 2^-24, m integer
+    m = u.astype(np.float64) * 2 ** 23 - 0.5
+    assert np.array_equal(m, np.round(m))           # (m + 0.5) 2^-23, m integer, exact in fp32
+    assert u.min() >= 2.0 ** -24 and u.max() <= 1 - 2.0 ** -24
     r = I.randint_i32((100_000,), 1, 3, 16, 48).numpy()
     assert r.min() == 16 and r.max() == 48
     assert np.all(np.bincount(r - 16, minlength=33) > 2500)
