@@ -25,6 +25,22 @@ int vla_op_gemm_bf16(const void* A, const void* A_lo, int lda, const void* W, in
                      int ldc, int M, int N, int K, int block_n, int splits, float* workspace,
                      void* cuda_stream);
 
+/* vla_op_gemm_bf16 without a caller workspace: the paper has no counterpart; this entry
+ * point exists for callers that cannot allocate device memory (all device memory owned by
+ * another allocator, or a loop that must not pay the synchronisation of cudaMalloc/cudaFree).
+ * Same arguments and result as vla_op_gemm_bf16 (its C within the same tolerance), but the
+ * split-K partials live in a file-scope 8 MiB device array inside libvla.so, which every
+ * device that loads the library holds until the process exits.  It allocates nothing.
+ *  - splits * M * N * 4 bytes must fit in 8 MiB, else VLA_ERR_CAPACITY and nothing runs.
+ *  - The first call on each device looks up the array's device address (with that device
+ *    current); make that first call before any stream capture.
+ *  - All calls share the one array: calls that overlap on the GPU (other streams, other
+ *    threads) race on it.  Serialise them, e.g. on one stream.
+ *  - Nothing carries over between calls: every partial is rewritten before it is read. */
+int vla_op_gemm_bf16_noalloc(const void* A, const void* A_lo, int lda, const void* W, int ldw,
+                             float* C, int ldc, int M, int N, int K, int block_n, int splits,
+                             void* cuda_stream);
+
 /* The fused action head (§3.1 action bins; Eq. 1 log-probs; Algorithm 1 f) on B given
  * hidden states h (f32 [B, d], row stride ldh): RMSNorm with final_norm (bf16 [d], eps),
  * logits z = y · head_rows^T (head_rows bf16 [256, d] = the last 256 lm_head rows), then the

@@ -100,4 +100,5 @@ __device__ __forceinline__ float silu_f(float x) { return x / (1.0f + expf(-x));
 
 namespace vla {
 int cuda_fail(cudaError_t e, const char* what);  // records the message, returns VLA_ERR_CUDA
+int record_error(int code, const char* msg);      // records the message, returns `code`
 }

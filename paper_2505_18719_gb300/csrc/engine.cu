@@ -32,6 +32,11 @@ int cuda_fail(cudaError_t e, const char* what) {
   return VLA_ERR_CUDA;
 }
 
+int record_error(int code, const char* msg) {
+  t_err = msg;
+  return code;
+}
+
 static int set_err(std::string* dst, int code, const std::string& msg) {
   t_err = msg;
   if (dst) *dst = msg;

@@ -828,3 +828,84 @@ int gemm_launch(const GemmArgs& a, cudaStream_t stream, int num_sms, GemmCost* c
 }
 
 }  // namespace vla
+
+// ============================================================================= no-allocation
+// Split-K GEMM whose partial sums live in a fixed, file-scope device array instead of a
+// caller-provided workspace.  It serves callers that cannot allocate device memory, e.g.
+// code running where every device byte belongs to another allocator (a host framework's
+// memory pool, a plugin without access to it) or a control loop that must not pay the
+// device-wide synchronisation of cudaMalloc / cudaFree.  The array is 8 MiB; every device
+// that loads this library keeps it until the process exits.
+namespace vla {
+namespace {
+
+constexpr size_t kNoAllocScratchFloats = static_cast<size_t>(2) << 20;  // 8 MiB of fp32
+__device__ __align__(256) float g_noalloc_scratch[kNoAllocScratchFloats];
+
+constexpr int kMaxDevices = 64;
+std::mutex g_noalloc_mu;
+float* g_noalloc_ptr[kMaxDevices] = {};
+
+// Device address of the scratch array on the current device.  In host code the array's
+// name is only a host-side stand-in, so the address is looked up once per device (with that
+// device current) and cached.
+int noalloc_scratch(float** out) {
+  int dev = 0;
+  VLA_CUDA_TRY(cudaGetDevice(&dev));
+  if (dev < 0 || dev >= kMaxDevices) return record_error(VLA_ERR_UNSUPPORTED, "no-alloc GEMM: device index >= 64");
+  std::lock_guard<std::mutex> lock(g_noalloc_mu);
+  if (!g_noalloc_ptr[dev]) {
+    void* p = nullptr;
+    VLA_CUDA_TRY(cudaGetSymbolAddress(&p, g_noalloc_scratch));
+    g_noalloc_ptr[dev] = static_cast<float*>(p);
+  }
+  *out = g_noalloc_ptr[dev];
+  return VLA_OK;
+}
+
+}  // namespace
+}  // namespace vla
+
+extern "C" int vla_op_gemm_bf16_noalloc(const void* A, const void* A_lo, int lda, const void* W,
+                                        int ldw, float* C, int ldc, int M, int N, int K,
+                                        int block_n, int splits, void* cuda_stream) {
+  using namespace vla;
+  if (!A || !W || !C || M < 1 || N < 1 || K < 1 || ldc < N)
+    return record_error(VLA_ERR_ARG, "vla_op_gemm_bf16_noalloc: bad argument");
+  GemmArgs g;
+  g.A = static_cast<const bf16*>(A);
+  g.A_lo = static_cast<const bf16*>(A_lo);
+  g.lda = lda;
+  g.B = static_cast<const bf16*>(W);
+  g.ldb = ldw;
+  g.M = M;
+  g.N = N;
+  g.K = K;
+  g.block_n = block_n;
+  g.splits = splits;
+  g.epi.kind = EPI_F32;
+  g.epi.out_f32 = C;
+  g.epi.ldo = ldc;
+  const size_t need = gemm_workspace_bytes(g);
+  if (need > kNoAllocScratchFloats * sizeof(float))
+    return record_error(VLA_ERR_CAPACITY,
+                        "vla_op_gemm_bf16_noalloc: splits * M * N * 4 bytes exceeds the 8 MiB "
+                        "static scratch; lower splits or use vla_op_gemm_bf16 with a workspace");
+  if (need > 0) {
+    // Every partial of every split is written before the reduction reads it, so the
+    // previous call's contents never leak into this one and nothing needs clearing.
+    int rc = noalloc_scratch(&g.workspace);
+    if (rc != VLA_OK) return rc;
+    g.workspace_bytes = kNoAllocScratchFloats * sizeof(float);
+  }
+  int dev = 0;
+  cudaGetDevice(&dev);
+  int n_sms = 0;
+  if (cudaDeviceGetAttribute(&n_sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n_sms <= 0)
+    n_sms = 148;
+  const int rc = gemm_launch(g, static_cast<cudaStream_t>(cuda_stream), n_sms, nullptr);
+  if (rc != VLA_OK && rc != VLA_ERR_CUDA)
+    return record_error(rc, "vla_op_gemm_bf16_noalloc: unsupported arguments");
+  return rc;
+}
+

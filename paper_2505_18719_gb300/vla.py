@@ -84,6 +84,7 @@ def load(path: str = LIB_PATH):
         "vla_profile_read": (i32, [vp, vp, vp, vp, vp]),
         "vla_launch_count": (i64, [vp]),
         "vla_op_gemm_bf16": (i32, [vp, vp, i32, vp, i32, vp, i32, i32, i32, i32, i32, i32, vp, vp]),
+        "vla_op_gemm_bf16_noalloc": (i32, [vp, vp, i32, vp, i32, vp, i32, i32, i32, i32, i32, i32, vp]),
         "vla_op_action_head": (i32, [vp, i32, i32, i32, vp, vp, f32, vp, f32, vp, vp, vp, vp, vp, vp, vp]),
         "vla_op_num_sms": (i32, []),
     }
@@ -174,6 +175,14 @@ def vla_op_gemm_bf16(A_ptr, A_lo_ptr, lda, W_ptr, ldw, C_ptr, ldc, M, N, K, bloc
                      ws_ptr=0, stream=0) -> int:
     return load().vla_op_gemm_bf16(A_ptr, A_lo_ptr or None, lda, W_ptr, ldw, C_ptr, ldc, M, N, K,
                                    block_n, splits, ws_ptr or None, stream or None)
+
+
+def vla_op_gemm_bf16_noalloc(A_ptr, A_lo_ptr, lda, W_ptr, ldw, C_ptr, ldc, M, N, K, block_n=256,
+                             splits=1, stream=0) -> int:
+    """vla_op_gemm_bf16 for callers that cannot allocate: split-K partials in the library's
+    fixed 8 MiB device scratch (see include/vla_ops.h)."""
+    return load().vla_op_gemm_bf16_noalloc(A_ptr, A_lo_ptr or None, lda, W_ptr, ldw, C_ptr, ldc, M, N,
+                                           K, block_n, splits, stream or None)
 
 
 def vla_op_action_head(h_ptr, ldh, B, d, final_norm_ptr, head_rows_ptr, eps, uniforms_ptr, temperature,
