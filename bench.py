@@ -149,6 +149,68 @@ def run_reference(args):
 
 METRIC = "action tokens/sec (batched decode, 7B shape) and prefill tok/s; % of HBM/TC roofline"
 
+# Single-kernel cases (7B shapes) for profiling one kernel in isolation, e.g. under ncu.
+CASES = {
+    # name: (M, N, K, block_n, splits, split A)
+    "gemm_prefill_qkv": (4608, 12288, 4096, 256, 1, True),     # 16 envs x 288-token prefixes
+    "gemm_prefill_down": (4608, 4096, 11008, 256, 1, True),
+    "gemm_decode_qkv": (64, 12288, 4096, 128, 2, True),        # one decode step, 64 envs
+    "gemm_decode_o": (64, 4096, 4096, 128, 5, True),
+    # weight-streaming decode GEMM (swap-AB, stream-K): block_n / splits unused
+    "gemv_decode_qkv": (64, 12288, 4096, 0, 0, True),
+    "gemv_decode_gate_up": (64, 22016, 4096, 0, 0, True),
+    "gemv_decode_down": (64, 4096, 11008, 0, 0, True),
+}
+
+
+def run_case(args):
+    """Time one GEMM shape through vla_op_gemm_bf16 (CUDA events, device-resident operands)."""
+    import torch
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2505_18719_gb300 import inputs as I
+    from paper_2505_18719_gb300 import vla as V
+    M, N, K, bn, splits, split_a = CASES[args.case]
+    A = I.normal_bf16((M, K), 1, 1, 1.0).cuda()
+    A_lo = I.normal_bf16((M, K), 1, 2, 2.0 ** -9).cuda()
+    W = I.normal_bf16((N, K), 1, 3, 0.02).cuda()
+    C = torch.empty(M, N, dtype=torch.float32, device="cuda")
+    stream = torch.cuda.current_stream()
+    if args.case.startswith("gemv"):
+        nbytes = V.vla_op_gemm_decode_workspace_bytes(M, N, K)
+        ws = torch.empty(max(1, nbytes // 4), dtype=torch.float32, device="cuda")
+
+        def launch():
+            rc = V.vla_op_gemm_decode_bf16(A.data_ptr(), A_lo.data_ptr(), K, W.data_ptr(), K, C.data_ptr(), N,
+                                           M, N, K, ws.data_ptr(), nbytes, stream.cuda_stream)
+            assert rc == 0, V.vla_last_error()
+    else:
+        ws = torch.empty(max(1, splits * M * N), dtype=torch.float32, device="cuda")
+
+        def launch():
+            rc = V.vla_op_gemm_bf16(A.data_ptr(), A_lo.data_ptr() if split_a else 0, K, W.data_ptr(), K,
+                                    C.data_ptr(), N, M, N, K, bn, splits, ws.data_ptr(), stream.cuda_stream)
+            assert rc == 0, V.vla_last_error()
+
+    for _ in range(args.warmup):
+        launch()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        launch()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1) / args.steps
+    hbm, tf_burst, _, kind = peaks()
+    flops = 2.0 * M * N * K
+    bytes_ = 2.0 * (M * K * (2 if split_a else 1) + N * K) + 4.0 * M * N
+    print(json.dumps({"case": args.case, "M": M, "N": N, "K": K, "block_n": bn, "splits": splits,
+                      "split_a": split_a, "ms": ms, "tflops": flops / ms / 1e9,
+                      "tc_frac_of_burst": flops / ms / 1e9 / tf_burst, "gbs": bytes_ / ms / 1e6,
+                      "hbm_frac": bytes_ / ms / 1e6 / hbm, "peaks": kind}))
+    return 0
+
 
 def main():
     ap = argparse.ArgumentParser()
@@ -158,9 +220,12 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--workload", default=WORKLOAD)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--case", choices=sorted(CASES), help="time one kernel shape instead of the hot path")
     args = ap.parse_args()
     if args.impl == "reference":
         return run_reference(args)
+    if args.case:
+        return run_case(args)
 
     import torch
     world, rank, local = dist_setup()
@@ -250,9 +315,16 @@ def main():
     e[3].record(stream)
     pol.sync()
     t_pre, t_dec, t_sc = e[0].elapsed_time(e[1]), e[1].elapsed_time(e[2]), e[2].elapsed_time(e[3])
+    # one more step with every kernel class bracketed by events (outside the timed region)
+    V.vla_profile(h, (1 << len(V.KCLASS)) - 1)
+    step(vis_d, ids_d, u_d)
+    per_class = V.vla_profile_read(h)
+    V.vla_profile(h, 0)
     prefill_tokens = sum(lengths) + B * wl.n_visual
     phase = {"prefill_ms": t_pre, "decode_ms": t_dec, "score_ms": t_sc,
-             "prefill_tok_s": prefill_tokens / (t_pre / 1e3), "decode_action_tok_s": B * A / (t_dec / 1e3)}
+             "prefill_tok_s": prefill_tokens / (t_pre / 1e3), "decode_action_tok_s": B * A / (t_dec / 1e3),
+             "kernel_classes_ms": {k: round(v["ms"], 3) for k, v in per_class.items()},
+             "kernel_classes_launches": {k: v["launches"] for k, v in per_class.items()}}
 
     # ---- e2e through the C ABI with host buffers
     vis_h = inp.visual.pin_memory()

@@ -6,6 +6,7 @@
 #ifndef VLA_OPS_H_
 #define VLA_OPS_H_
 
+#include <stddef.h>
 #include <stdint.h>
 
 #ifdef __cplusplus
@@ -24,6 +25,17 @@ extern "C" {
 int vla_op_gemm_bf16(const void* A, const void* A_lo, int lda, const void* W, int ldw, float* C,
                      int ldc, int M, int N, int K, int block_n, int splits, float* workspace,
                      void* cuda_stream);
+
+/* The decode-step projection (§3.1 projections at decode batch sizes, Algorithm 1 rollout):
+ * C[M, N] (f32) = (A + A_lo)[M, K] · W[N, K]^T for M <= 128 activation rows, bf16 operands,
+ * A_lo required.  Streams W from HBM once: swap-AB tcgen05 MMAs (W rows are the MMA's M),
+ * stream-K over the 128-row weight tiles, fp32 partials in `workspace` (at least
+ * vla_op_gemm_decode_workspace_bytes(M, N, K) bytes), fixed-order reduction into C.
+ * VLA_ERR_ARG for M > 128, NULL pointers or a short workspace. */
+int vla_op_gemm_decode_bf16(const void* A, const void* A_lo, int lda, const void* W, int ldw,
+                            float* C, int ldc, int M, int N, int K, float* workspace,
+                            size_t workspace_bytes, void* cuda_stream);
+size_t vla_op_gemm_decode_workspace_bytes(int M, int N, int K);
 
 /* vla_op_gemm_bf16 without a caller workspace: the paper has no counterpart; this entry
  * point exists for callers that cannot allocate device memory (all device memory owned by

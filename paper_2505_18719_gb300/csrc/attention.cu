@@ -4,9 +4,10 @@
 //
 //  * attn_chunk: query rows of one env at consecutive positions (a prefill chunk, or the
 //    6 teacher-forced action rows of the score pass) against keys 0..pos of that env.
-//    One CTA per (64-row tile, head); K/V blocks of 64 keys staged in shared memory; online
-//    softmax in the exp2 domain; fp32 math on the fp32 queries and fp16 K/V; the output is
-//    written as the bf16 hi/lo pair the O-projection GEMM reads.
+//    One CTA per (64-row tile, head); mma.sync tensor-core flash attention with fp32
+//    accumulation on fp16 K/V, the fp32 queries and the softmax weights each taken as an
+//    fp16 hi/lo pair; the output is written as the bf16 hi/lo pair the O-projection GEMM
+//    reads.
 //  * attn_decode: one query per env (the decode step) with the key range split across CTAs
 //    (flash-decoding); each CTA writes its partial (max, sum, unnormalised output) and a
 //    combine kernel merges the splits in a fixed order.  16 lanes x 16 bytes read one
@@ -20,122 +21,244 @@ namespace vla {
 
 namespace {
 
-constexpr int kTileRows = 64;
-constexpr int kKeyBlock = 64;
+
+// ------------------------------------------------------------------------ chunk (tensor core)
+// Flash-attention over one 64-row query tile of one env and one head: S = Q K^T and O += P V
+// on mma.sync m16n8k16 (fp16 inputs, fp32 accumulation), online softmax in the exp2 domain.
+// 4 warps x 16 query rows; K/V blocks of 64 keys double-buffered in shared memory with
+// cp.async (rows past the last visible key are zero-filled, never read from the cache).
+__device__ __forceinline__ void mma16816(float (&c)[4], const uint32_t (&a)[4], uint32_t b0,
+                                         uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, "
+      "{%8,%9}, {%0,%1,%2,%3};"
+      : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2,
+                                        uint32_t& r3) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
+               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+               : "r"(addr));
+}
+__device__ __forceinline__ void ldsm_x4_t(uint32_t addr, uint32_t& r0, uint32_t& r1, uint32_t& r2,
+                                          uint32_t& r3) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];"
+               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+               : "r"(addr));
+}
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, bool valid) {
+  const int n = valid ? 16 : 0;  // 0 source bytes -> 16 zero bytes
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(n)
+               : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+}
+// (a, b) -> fp16 pairs hi = fp16(x), lo = fp16(x - hi): P V is taken as P_hi V + P_lo V so the
+// softmax weights keep ~22 bits.
+__device__ __forceinline__ void split_h2(float a, float b, uint32_t& hi, uint32_t& lo) {
+  const __half ha = __float2half_rn(a), hb = __float2half_rn(b);
+  __half2 h2 = __halves2half2(ha, hb);
+  __half2 l2 = __floats2half2_rn(a - __half2float(ha), b - __half2float(hb));
+  hi = *reinterpret_cast<uint32_t*>(&h2);
+  lo = *reinterpret_cast<uint32_t*>(&l2);
+}
 
 template <int HD>
-__global__ void __launch_bounds__(256) attn_chunk_kernel(const float* __restrict__ q,
-                                                         bf16* __restrict__ out_hi,
-                                                         bf16* __restrict__ out_lo,
-                                                         const AttnTile* __restrict__ tiles,
-                                                         KVLayout kv, int layer, int H,
-                                                         float scale_log2) {
-  constexpr int PER_LANE = HD / 32;  // output dims per lane
-  constexpr int KS = HD + 1;          // padded key row (conflict-free column reads)
-  extern __shared__ float sm[];
-  float* Qs = sm;                         // [64][HD]
-  float* Ks = Qs + kTileRows * HD;        // [64][HD+1]
-  float* Vs = Ks + kKeyBlock * KS;        // [64][HD]
+__global__ void __launch_bounds__(128) attn_chunk_mma_kernel(const float* __restrict__ q,
+                                                             bf16* __restrict__ out_hi,
+                                                             bf16* __restrict__ out_lo,
+                                                             const AttnTile* __restrict__ tiles,
+                                                             KVLayout kv, int layer, int H,
+                                                             float scale_log2) {
+  constexpr int KB = 64;       // keys per block
+  constexpr int LD = HD + 8;   // padded row (halves): 16-byte rows land in distinct banks
+  constexpr int CPR = HD / 8;  // 16-byte chunks per row
+  constexpr int NT_D = HD / 8; // n-tiles over the head dim
+  extern __shared__ __align__(16) f16 sm_h[];
+  f16* Ks = sm_h;              // [2][KB][LD]
+  f16* Vs = Ks + 2 * KB * LD;  // [2][KB][LD]
 
   const AttnTile t = tiles[blockIdx.x];
   const int head = blockIdx.y;
   const int d = H * HD;
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-
-  // Q tile, pre-scaled by log2(e)/sqrt(hd)
-  for (int i = threadIdx.x; i < kTileRows * HD; i += blockDim.x) {
-    const int r = i / HD, c = i - r * HD;
-    float v = 0.f;
-    if (r < t.nrows) v = q[static_cast<size_t>(t.row0 + r) * d + head * HD + c] * scale_log2;
-    Qs[i] = v;
-  }
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int g = lane >> 2, tq = lane & 3;
   const f16* kbase = kv.base + static_cast<int64_t>(layer) * kv.layer_stride +
                      static_cast<int64_t>(t.env) * kv.env_stride +
                      static_cast<int64_t>(head) * kv.head_stride;
   const f16* vbase = kbase + kv.kv_stride;
+  const int n_keys = t.pos0 + t.nrows;
+  const int n_blocks = (n_keys + KB - 1) / KB;
 
-  float m_i[8], l_i[8], o_i[8][PER_LANE];
+  auto load_block = [&](int blk, int buf) {
+    const int j0 = blk * KB;
+    const uint32_t ks = static_cast<uint32_t>(__cvta_generic_to_shared(Ks + buf * KB * LD));
+    const uint32_t vs = static_cast<uint32_t>(__cvta_generic_to_shared(Vs + buf * KB * LD));
+    for (int i = tid; i < KB * CPR; i += 128) {
+      const int r = i / CPR, c = (i - r * CPR) * 8;
+      const bool ok = j0 + r < n_keys;
+      const int64_t src = static_cast<int64_t>(ok ? j0 + r : 0) * HD + c;
+      cp_async16(ks + (r * LD + c) * 2, kbase + src, ok);
+      cp_async16(vs + (r * LD + c) * 2, vbase + src, ok);
+    }
+  };
+
+  load_block(0, 0);
+  cp_async_commit();
+
+  // this thread's two rows and their positions (rows past nrows reuse the last position;
+  // their results are never written)
+  const int r0 = warp * 16 + g, r1 = r0 + 8;
+  const int qpos0 = t.pos0 + min(r0, t.nrows - 1);
+  const int qpos1 = t.pos0 + min(r1, t.nrows - 1);
+  const int warp_last = t.pos0 + min(warp * 16 + 15, t.nrows - 1);
+  const bool warp_active = warp * 16 < t.nrows;
+
+  float o[NT_D][4];
 #pragma unroll
-  for (int r = 0; r < 8; ++r) {
-    m_i[r] = -INFINITY;
-    l_i[r] = 0.f;
+  for (int i = 0; i < NT_D; ++i) o[i][0] = o[i][1] = o[i][2] = o[i][3] = 0.f;
+  float m0 = -INFINITY, m1 = -INFINITY, l0 = 0.f, l1 = 0.f;
+  // Q A-fragments straight from the fp32 rows, as fp16 hi/lo pairs (S = Q_hi K + Q_lo K).
+  uint32_t qh[HD / 16][4], ql[HD / 16][4];
+  {
+    const int ra = min(r0, t.nrows - 1), rb = min(r1, t.nrows - 1);
+    const float* qa = q + static_cast<size_t>(t.row0 + ra) * d + head * HD + 2 * tq;
+    const float* qb = q + static_cast<size_t>(t.row0 + rb) * d + head * HD + 2 * tq;
 #pragma unroll
-    for (int c = 0; c < PER_LANE; ++c) o_i[r][c] = 0.f;
+    for (int kk = 0; kk < HD / 16; ++kk) {
+      const float2 x0 = *reinterpret_cast<const float2*>(qa + kk * 16);
+      const float2 x1 = *reinterpret_cast<const float2*>(qb + kk * 16);
+      const float2 x2 = *reinterpret_cast<const float2*>(qa + kk * 16 + 8);
+      const float2 x3 = *reinterpret_cast<const float2*>(qb + kk * 16 + 8);
+      split_h2(x0.x, x0.y, qh[kk][0], ql[kk][0]);
+      split_h2(x1.x, x1.y, qh[kk][1], ql[kk][1]);
+      split_h2(x2.x, x2.y, qh[kk][2], ql[kk][2]);
+      split_h2(x3.x, x3.y, qh[kk][3], ql[kk][3]);
+    }
   }
 
-  const int n_keys = t.pos0 + t.nrows;  // keys 0 .. last query position
-  for (int j0 = 0; j0 < n_keys; j0 += kKeyBlock) {
-    __syncthreads();
-    for (int i = threadIdx.x; i < kKeyBlock * (HD / 8); i += blockDim.x) {
-      const int r = i / (HD / 8), c8 = (i - r * (HD / 8)) * 8;
-      const int key = j0 + r;
-      uint4 kk = make_uint4(0, 0, 0, 0), vv = make_uint4(0, 0, 0, 0);
-      if (key < n_keys) {
-        kk = *reinterpret_cast<const uint4*>(kbase + static_cast<int64_t>(key) * HD + c8);
-        vv = *reinterpret_cast<const uint4*>(vbase + static_cast<int64_t>(key) * HD + c8);
-      }
-      const uint32_t kw[4] = {kk.x, kk.y, kk.z, kk.w};
-      const uint32_t vw[4] = {vv.x, vv.y, vv.z, vv.w};
-#pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        const float2 kf = unpack_f16x2(kw[e]);
-        const float2 vf = unpack_f16x2(vw[e]);
-        Ks[r * KS + c8 + 2 * e] = kf.x;
-        Ks[r * KS + c8 + 2 * e + 1] = kf.y;
-        Vs[r * HD + c8 + 2 * e] = vf.x;
-        Vs[r * HD + c8 + 2 * e + 1] = vf.y;
-      }
+  for (int blk = 0; blk < n_blocks; ++blk) {
+    if (blk + 1 < n_blocks) {
+      load_block(blk + 1, (blk + 1) & 1);
+      cp_async_commit();
+      cp_async_wait<1>();
+    } else {
+      cp_async_wait<0>();
     }
     __syncthreads();
+    const int j0 = blk * KB;
+    if (warp_active && j0 <= warp_last) {
+      const int buf = blk & 1;
+      const uint32_t ks = static_cast<uint32_t>(__cvta_generic_to_shared(Ks + buf * KB * LD));
+      const uint32_t vs = static_cast<uint32_t>(__cvta_generic_to_shared(Vs + buf * KB * LD));
+      float s[8][4];
 #pragma unroll
-    for (int rr = 0; rr < 8; ++rr) {
-      const int r = warp * 8 + rr;
-      if (r >= t.nrows) continue;  // warp-uniform
-      const int qpos = t.pos0 + r;
-      if (j0 > qpos) continue;     // whole block in the future (warp-uniform)
-      const float* qrow = Qs + r * HD;
-      float s0 = 0.f, s1 = 0.f;
-      const float* k0 = Ks + lane * KS;
-      const float* k1 = Ks + (lane + 32) * KS;
-#pragma unroll 8
-      for (int c = 0; c < HD; ++c) {
-        const float qv = qrow[c];
-        s0 = fmaf(qv, k0[c], s0);
-        s1 = fmaf(qv, k1[c], s1);
+      for (int nt = 0; nt < 8; ++nt) {
+        s[nt][0] = s[nt][1] = s[nt][2] = s[nt][3] = 0.f;
+        const int i = lane >> 3;
+#pragma unroll
+        for (int kk = 0; kk < HD / 16; kk += 2) {
+          uint32_t b0, b1, b2, b3;
+          const int key = nt * 8 + (lane & 7);
+          const int dim = (kk + (i >> 1)) * 16 + (i & 1) * 8;
+          ldsm_x4(ks + (key * LD + dim) * 2, b0, b1, b2, b3);
+          mma16816(s[nt], qh[kk], b0, b1);
+          mma16816(s[nt], ql[kk], b0, b1);
+          mma16816(s[nt], qh[kk + 1], b2, b3);
+          mma16816(s[nt], ql[kk + 1], b2, b3);
+        }
       }
-      if (j0 + lane > qpos) s0 = -INFINITY;
-      if (j0 + lane + 32 > qpos) s1 = -INFINITY;
-      const float mx = warp_max(fmaxf(s0, s1));
-      const float m_new = fmaxf(m_i[rr], mx);
-      const float alpha = exp2f(m_i[rr] - m_new);
-      const float p0 = exp2f(s0 - m_new), p1 = exp2f(s1 - m_new);
-      l_i[rr] = l_i[rr] * alpha + warp_sum(p0 + p1);
-      m_i[rr] = m_new;
+      // scale, causal mask, online softmax (rows r0: c 0,1; r1: c 2,3)
+      float mx0 = -INFINITY, mx1 = -INFINITY;
 #pragma unroll
-      for (int c = 0; c < PER_LANE; ++c) o_i[rr][c] *= alpha;
-      for (int jj = 0; jj < 32; ++jj) {
-        const float pa = __shfl_sync(0xffffffffu, p0, jj);
-        const float pb = __shfl_sync(0xffffffffu, p1, jj);
+      for (int nt = 0; nt < 8; ++nt) {
 #pragma unroll
-        for (int c = 0; c < PER_LANE; ++c) {
-          o_i[rr][c] = fmaf(pa, Vs[jj * HD + lane + 32 * c], o_i[rr][c]);
-          o_i[rr][c] = fmaf(pb, Vs[(jj + 32) * HD + lane + 32 * c], o_i[rr][c]);
+        for (int c = 0; c < 4; ++c) {
+          const int key = j0 + nt * 8 + 2 * tq + (c & 1);
+          const int qp = (c < 2) ? qpos0 : qpos1;
+          const float v = (key <= qp) ? s[nt][c] * scale_log2 : -INFINITY;
+          s[nt][c] = v;
+        }
+        mx0 = fmaxf(mx0, fmaxf(s[nt][0], s[nt][1]));
+        mx1 = fmaxf(mx1, fmaxf(s[nt][2], s[nt][3]));
+      }
+      mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 1));
+      mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 2));
+      mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 1));
+      mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 2));
+      const float mn0 = fmaxf(m0, mx0), mn1 = fmaxf(m1, mx1);  // finite: key j0 <= qpos
+      const float a0 = exp2f(m0 - mn0), a1 = exp2f(m1 - mn1);
+      m0 = mn0;
+      m1 = mn1;
+      float ps0 = 0.f, ps1 = 0.f;
+#pragma unroll
+      for (int nt = 0; nt < 8; ++nt) {
+        s[nt][0] = exp2f(s[nt][0] - mn0);
+        s[nt][1] = exp2f(s[nt][1] - mn0);
+        s[nt][2] = exp2f(s[nt][2] - mn1);
+        s[nt][3] = exp2f(s[nt][3] - mn1);
+        ps0 += s[nt][0] + s[nt][1];
+        ps1 += s[nt][2] + s[nt][3];
+      }
+      l0 = l0 * a0 + ps0;  // per-thread partial row sums; reduced across the quad at the end
+      l1 = l1 * a1 + ps1;
+#pragma unroll
+      for (int nt = 0; nt < NT_D; ++nt) {
+        o[nt][0] *= a0;
+        o[nt][1] *= a0;
+        o[nt][2] *= a1;
+        o[nt][3] *= a1;
+      }
+      // O += P V: P re-used from the S accumulators as the A operand, as an fp16 hi/lo pair
+#pragma unroll
+      for (int kk = 0; kk < 4; ++kk) {
+        uint32_t ph[4], pl[4];
+        split_h2(s[2 * kk][0], s[2 * kk][1], ph[0], pl[0]);
+        split_h2(s[2 * kk][2], s[2 * kk][3], ph[1], pl[1]);
+        split_h2(s[2 * kk + 1][0], s[2 * kk + 1][1], ph[2], pl[2]);
+        split_h2(s[2 * kk + 1][2], s[2 * kk + 1][3], ph[3], pl[3]);
+        const int i = lane >> 3;
+#pragma unroll
+        for (int nt = 0; nt < NT_D; nt += 2) {
+          uint32_t b0, b1, b2, b3;
+          const int key = kk * 16 + (i & 1) * 8 + (lane & 7);
+          const int dim = (nt + (i >> 1)) * 8;
+          ldsm_x4_t(vs + (key * LD + dim) * 2, b0, b1, b2, b3);
+          mma16816(o[nt], ph, b0, b1);
+          mma16816(o[nt], pl, b0, b1);
+          mma16816(o[nt + 1], ph, b2, b3);
+          mma16816(o[nt + 1], pl, b2, b3);
         }
       }
     }
+    __syncthreads();  // this buffer is refilled two blocks later
   }
+  if (!warp_active) return;
+  l0 += __shfl_xor_sync(0xffffffffu, l0, 1);
+  l0 += __shfl_xor_sync(0xffffffffu, l0, 2);
+  l1 += __shfl_xor_sync(0xffffffffu, l1, 1);
+  l1 += __shfl_xor_sync(0xffffffffu, l1, 2);
+  const float inv0 = 1.f / l0, inv1 = 1.f / l1;
 #pragma unroll
-  for (int rr = 0; rr < 8; ++rr) {
-    const int r = warp * 8 + rr;
-    if (r >= t.nrows) continue;
-    const float inv = 1.f / l_i[rr];
-    const size_t off = static_cast<size_t>(t.row0 + r) * d + head * HD;
-#pragma unroll
-    for (int c = 0; c < PER_LANE; ++c) {
-      bf16 hi, lo;
-      split_bf16(o_i[rr][c] * inv, hi, lo);
-      out_hi[off + lane + 32 * c] = hi;
-      out_lo[off + lane + 32 * c] = lo;
+  for (int nt = 0; nt < NT_D; ++nt) {
+    const int col = head * HD + nt * 8 + 2 * tq;
+    if (r0 < t.nrows) {
+      const size_t off = static_cast<size_t>(t.row0 + r0) * d + col;
+      uint32_t hi, lo;
+      split_pack2(o[nt][0] * inv0, o[nt][1] * inv0, hi, lo);
+      *reinterpret_cast<uint32_t*>(out_hi + off) = hi;
+      *reinterpret_cast<uint32_t*>(out_lo + off) = lo;
+    }
+    if (r1 < t.nrows) {
+      const size_t off = static_cast<size_t>(t.row0 + r1) * d + col;
+      uint32_t hi, lo;
+      split_pack2(o[nt][2] * inv1, o[nt][3] * inv1, hi, lo);
+      *reinterpret_cast<uint32_t*>(out_hi + off) = hi;
+      *reinterpret_cast<uint32_t*>(out_lo + off) = lo;
     }
   }
 }
@@ -183,15 +306,24 @@ __global__ void __launch_bounds__(128) attn_decode_kernel(const float* __restric
 #pragma unroll
   for (int e = 0; e < 8; ++e) o[e] = 0.f;
 
-  for (int key0 = k_begin + warp * KPI; key0 < k_end; key0 += 4 * KPI) {
-    const int key = key0 + sub;
-    const bool valid = key < k_end;
-    float s = -INFINITY;
-    uint4 vv = make_uint4(0, 0, 0, 0);
-    if (valid) {
-      const uint4 kk = *reinterpret_cast<const uint4*>(kbase + static_cast<int64_t>(key) * HD + part * 8);
-      vv = *reinterpret_cast<const uint4*>(vbase + static_cast<int64_t>(key) * HD + part * 8);
-      const uint32_t w[4] = {kk.x, kk.y, kk.z, kk.w};
+  // U key rows per lane group are loaded before any is used (memory-level parallelism)
+  constexpr int U = 4;
+  for (int key0 = k_begin + warp * KPI * U; key0 < k_end; key0 += 4 * KPI * U) {
+    uint4 kk[U], vv[U];
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const int key = key0 + u * KPI + sub;
+      kk[u] = make_uint4(0, 0, 0, 0);
+      vv[u] = make_uint4(0, 0, 0, 0);
+      if (key < k_end) {
+        kk[u] = *reinterpret_cast<const uint4*>(kbase + static_cast<int64_t>(key) * HD + part * 8);
+        vv[u] = *reinterpret_cast<const uint4*>(vbase + static_cast<int64_t>(key) * HD + part * 8);
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const bool valid = key0 + u * KPI + sub < k_end;
+      const uint32_t w[4] = {kk[u].x, kk[u].y, kk[u].z, kk[u].w};
       float acc = 0.f;
 #pragma unroll
       for (int e = 0; e < 4; ++e) {
@@ -199,28 +331,24 @@ __global__ void __launch_bounds__(128) attn_decode_kernel(const float* __restric
         acc = fmaf(qv[2 * e], f.x, acc);
         acc = fmaf(qv[2 * e + 1], f.y, acc);
       }
-      s = acc;
-    }
-    // reduce the dot product across the LPK lanes of this key row (all lanes take part)
-    // (a key row's LPK lanes share `valid`, and the xor offsets stay inside the group)
+      // reduce across the LPK lanes of this key row (a row's lanes share `valid`; the xor
+      // offsets stay inside the group)
 #pragma unroll
-    for (int off = LPK / 2; off > 0; off >>= 1) {
-      const float other = __shfl_xor_sync(0xffffffffu, s, off);
-      if (valid) s += other;
-    }
-    if (valid) {
-      const float m_new = fmaxf(m, s);
-      const float alpha = exp2f(m - m_new);
-      const float p = exp2f(s - m_new);
-      l = l * alpha + p;
-      const uint32_t w[4] = {vv.x, vv.y, vv.z, vv.w};
+      for (int off = LPK / 2; off > 0; off >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, off);
+      if (valid) {
+        const float m_new = fmaxf(m, acc);
+        const float alpha = exp2f(m - m_new);
+        const float p = exp2f(acc - m_new);
+        l = l * alpha + p;
+        const uint32_t v4[4] = {vv[u].x, vv[u].y, vv[u].z, vv[u].w};
 #pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        const float2 f = unpack_f16x2(w[e]);
-        o[2 * e] = fmaf(p, f.x, o[2 * e] * alpha);
-        o[2 * e + 1] = fmaf(p, f.y, o[2 * e + 1] * alpha);
+        for (int e = 0; e < 4; ++e) {
+          const float2 f = unpack_f16x2(v4[e]);
+          o[2 * e] = fmaf(p, f.x, o[2 * e] * alpha);
+          o[2 * e + 1] = fmaf(p, f.y, o[2 * e + 1] * alpha);
+        }
+        m = m_new;
       }
-      m = m_new;
     }
   }
   // per (warp, sub) partials -> shared memory
@@ -283,23 +411,23 @@ int attn_chunk_launch(const float* q, bf16* out_hi, bf16* out_lo, const AttnTile
   const float scale_log2 = 1.4426950408889634f / sqrtf(static_cast<float>(hd));
   dim3 grid(n_tiles, H);
   if (hd == 128) {
-    const int smem = (kTileRows * 128 + kKeyBlock * 129 + kKeyBlock * 128) * 4;
+    const int smem = (4 * 64) * (128 + 8) * 2;
     static bool set = false;
     if (!set) {
-      VLA_CUDA_TRY(cudaFuncSetAttribute(attn_chunk_kernel<128>,
+      VLA_CUDA_TRY(cudaFuncSetAttribute(attn_chunk_mma_kernel<128>,
                                         cudaFuncAttributeMaxDynamicSharedMemorySize, smem));
       set = true;
     }
-    attn_chunk_kernel<128><<<grid, 256, smem, stream>>>(q, out_hi, out_lo, tiles, kv, layer, H, scale_log2);
+    attn_chunk_mma_kernel<128><<<grid, 128, smem, stream>>>(q, out_hi, out_lo, tiles, kv, layer, H, scale_log2);
   } else if (hd == 64) {
-    const int smem = (kTileRows * 64 + kKeyBlock * 65 + kKeyBlock * 64) * 4;
+    const int smem = (4 * 64) * (64 + 8) * 2;
     static bool set = false;
     if (!set) {
-      VLA_CUDA_TRY(cudaFuncSetAttribute(attn_chunk_kernel<64>,
+      VLA_CUDA_TRY(cudaFuncSetAttribute(attn_chunk_mma_kernel<64>,
                                         cudaFuncAttributeMaxDynamicSharedMemorySize, smem));
       set = true;
     }
-    attn_chunk_kernel<64><<<grid, 256, smem, stream>>>(q, out_hi, out_lo, tiles, kv, layer, H, scale_log2);
+    attn_chunk_mma_kernel<64><<<grid, 128, smem, stream>>>(q, out_hi, out_lo, tiles, kv, layer, H, scale_log2);
   } else {
     return VLA_ERR_UNSUPPORTED;
   }
@@ -312,7 +440,9 @@ int attn_decode_launch(const float* q, bf16* out_hi, bf16* out_lo, const RowInfo
                        int max_ctx, KVLayout kv, int layer, int H, int hd, int chunk,
                        float* part_o, float2* part_ml, cudaStream_t stream) {
   if (B <= 0) return VLA_OK;
+  // equal key ranges (multiples of 16) no longer than `chunk`
   const int S = (max_ctx + chunk - 1) / chunk;
+  chunk = ((max_ctx + S - 1) / S + 15) / 16 * 16;
   const float scale_log2 = 1.4426950408889634f / sqrtf(static_cast<float>(hd));
   dim3 grid(S, H, B);
   if (hd == 128) {

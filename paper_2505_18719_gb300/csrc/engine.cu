@@ -119,7 +119,7 @@ struct vla_handle {
   uint32_t* status = nullptr;
   float* part_o = nullptr;
   float2* part_ml = nullptr;
-  int attn_chunk = 256;
+  int attn_chunk = 160;  // max keys per decode-attention CTA
   int max_tiles = 0;
   // pinned host staging (ring of slots, each guarded by an event)
   static constexpr int kSlots = 4;
@@ -214,13 +214,15 @@ int run_gemm(vla_handle* h, int cls, const bf16* A, size_t a_plane, int lda, con
   g.workspace_bytes = h->ws_bytes;
   epi.status = h->status;
   g.epi = epi;
-  if (gemm_workspace_bytes(g) > h->ws_bytes) {
+  const bool stream_k = M <= 128;  // decode-sized: weight-streaming swap-AB GEMM
+  if (!stream_k && gemm_workspace_bytes(g) > h->ws_bytes) {
     g.splits = 1;
   }
   if (h->ev_used.size() > 8192) prof_harvest(h);
   int ev = prof_begin(h, cls);
   GemmCost cost{0, 0};
-  const int rc = gemm_launch(g, h->stream, h->num_sms, &cost);
+  const int rc = stream_k ? gemv_launch(g, h->stream, h->num_sms, &cost)
+                          : gemm_launch(g, h->stream, h->num_sms, &cost);
   prof_end(h, ev, cls, cost.flops, cost.bytes);
   if (rc != VLA_OK) return fail(h, rc, t_err.empty() ? "gemm launch failed" : t_err);
   return VLA_OK;
@@ -243,7 +245,7 @@ int forward_layers(vla_handle* h, int M, const RowInfo* rows_dev, bool decode, i
 
     EpiArgs e;
     e.kind = EPI_QKV;
-    e.out_f32 = h->q;
+    e.out_q = h->q;
     e.rows = rows_dev;
     e.kv = h->kvl;
     e.layer = l;
@@ -362,6 +364,10 @@ int vla_create(const vla_config* cfg, const vla_weights* w, void* cuda_stream, v
     if (M < 1 || M > h->max_tokens) continue;
     const int shapes[4][4] = {{3 * d, d, EPI_QKV, 0}, {d, d, EPI_RESID, 0}, {2 * F, d, EPI_SWIGLU, 0}, {d, F, EPI_RESID, 0}};
     for (auto& s : shapes) {
+      if (M <= 128) {
+        ws = std::max(ws, gemv_workspace_bytes(M, s[0], s[1], h->num_sms));
+        continue;
+      }
       const Plan pl = plan_gemm(M, s[0], s[1], s[2], d, h->num_sms);
       const int sp = gemm_effective_splits(s[1], pl.splits);
       if (sp > 1) ws = std::max(ws, static_cast<size_t>(sp) * M * s[0] * sizeof(float));
@@ -780,6 +786,35 @@ int vla_op_gemm_bf16(const void* A, const void* A_lo, int lda, const void* W, in
   const int rc = gemm_launch(g, static_cast<cudaStream_t>(cuda_stream), query_num_sms(), nullptr);
   if (rc != VLA_OK && rc != VLA_ERR_CUDA) return set_err(nullptr, rc, "vla_op_gemm_bf16: unsupported arguments");
   return rc;
+}
+
+int vla_op_gemm_decode_bf16(const void* A, const void* A_lo, int lda, const void* W, int ldw, float* C,
+                            int ldc, int M, int N, int K, float* workspace, size_t workspace_bytes,
+                            void* cuda_stream) {
+  if (!A || !A_lo || !W || !C || M < 1 || M > 128 || N < 1 || K < 1 || ldc < N || !workspace)
+    return set_err(nullptr, VLA_ERR_ARG, "vla_op_gemm_decode_bf16: bad argument");
+  GemmArgs g;
+  g.A = static_cast<const bf16*>(A);
+  g.A_lo = static_cast<const bf16*>(A_lo);
+  g.lda = lda;
+  g.B = static_cast<const bf16*>(W);
+  g.ldb = ldw;
+  g.M = M;
+  g.N = N;
+  g.K = K;
+  g.workspace = workspace;
+  g.workspace_bytes = workspace_bytes;
+  g.epi.kind = EPI_F32;
+  g.epi.out_f32 = C;
+  g.epi.ldo = ldc;
+  const int rc = gemv_launch(g, static_cast<cudaStream_t>(cuda_stream), query_num_sms(), nullptr);
+  if (rc != VLA_OK && rc != VLA_ERR_CUDA)
+    return set_err(nullptr, rc, "vla_op_gemm_decode_bf16: unsupported arguments or workspace too small");
+  return rc;
+}
+
+size_t vla_op_gemm_decode_workspace_bytes(int M, int N, int K) {
+  return gemv_workspace_bytes(M, N, K, query_num_sms());
 }
 
 int vla_op_action_head(const float* hs, int ldh, int B, int d, const void* final_norm, const void* head_rows,

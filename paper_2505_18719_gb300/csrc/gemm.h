@@ -10,13 +10,14 @@ enum EpiKind : int {
   EPI_RESID = 1,   // resid[m * ldr + n] += y               (O-proj, down-proj)
   EPI_SWIGLU = 2,  // u = silu(y_gate) * y_up, f < F = N / 2, stored as the bf16 pair
                    // out_hi / out_lo [m * ldo + f]
-  EPI_QKV = 3,     // RoPE(q) -> out_f32 [M, d]; RoPE(k), v -> fp16 KV cache
+  EPI_QKV = 3,     // RoPE(q) -> out_q f32 [M, d]; RoPE(k), v -> fp16 KV cache
   EPI_PARTIAL = 4  // internal: split-K partial sums to the workspace
 };
 
 struct EpiArgs {
   int kind = EPI_F32;
   float* out_f32 = nullptr;
+  float* out_q = nullptr;
   bf16* out_hi = nullptr;
   bf16* out_lo = nullptr;
   int ldo = 0;
@@ -55,5 +56,11 @@ int gemm_effective_splits(int K, int splits);
 size_t gemm_workspace_bytes(const GemmArgs& a);
 // Launch; returns VLA_OK or an error code (host checks only; kernels report via status).
 int gemm_launch(const GemmArgs& a, cudaStream_t stream, int num_sms, GemmCost* cost);
+
+// Weight-streaming (decode) GEMM for M <= 128 rows with a split A (A_lo required): swap-AB
+// tcgen05 MMAs, stream-K over the weight tiles, partials in `workspace`
+// (gemv_workspace_bytes), then the epilogue of `a.epi` in a fixed-order reduction.
+size_t gemv_workspace_bytes(int M, int N, int K, int num_sms);
+int gemv_launch(const GemmArgs& a, cudaStream_t stream, int num_sms, GemmCost* cost);
 
 }  // namespace vla

@@ -75,6 +75,26 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map
       "l"(reinterpret_cast<uint64_t>(map)), "r"(bar), "r"(c0), "r"(c1)
       : "memory");
 }
+// Same with an L2 cache policy (createpolicy): weights streamed once per decode step are
+// loaded evict-first, the small activation tiles every CTA re-reads evict-last.
+__device__ __forceinline__ void tma_load_2d_hint(uint32_t dst, const CUtensorMap* map,
+                                                 uint32_t bar, int c0, int c1, uint64_t policy) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint"
+      " [%0], [%1, {%3, %4}], [%2], %5;" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(bar), "r"(c0), "r"(c1), "l"(policy)
+      : "memory");
+}
+__device__ __forceinline__ uint64_t policy_evict_first() {
+  uint64_t p;
+  asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
+  return p;
+}
+__device__ __forceinline__ uint64_t policy_evict_last() {
+  uint64_t p;
+  asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(p));
+  return p;
+}
 __device__ __forceinline__ void tc_fence_before() {
   asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
 }
@@ -308,7 +328,7 @@ __device__ __forceinline__ void epilogue_swiglu(const Params& p, uint32_t trow, 
 }
 
 // q|k|v with RoPE (rotate-half: pair (i, i + hd/2) rotated by pos * theta^(-2i/hd)) and the
-// KV-cache write.  q goes to an fp32 buffer, K and V to the fp16 cache.  The tile lies inside
+// KV-cache write.  q is stored fp32, K and V fp16 (cache).  The tile lies inside
 // one of the q / k / v sections (BN divides d) and holds BN / hd whole heads.
 template <int BN>
 __device__ __forceinline__ void epilogue_qkv(const Params& p, uint32_t trow, int m, int n0) {
@@ -354,7 +374,7 @@ __device__ __forceinline__ void epilogue_qkv(const Params& p, uint32_t trow, int
           rb[i] = b[i] * t.x + a[i] * t.y;
         }
         if (sec == 0) {
-          float* dst = p.epi.out_f32 + static_cast<size_t>(m) * d + head * hd;
+          float* dst = p.epi.out_q + static_cast<size_t>(m) * d + head * hd;
           store_f32x16(dst + j, ra);
           store_f32x16(dst + half + j, rb);
         } else {
@@ -550,16 +570,61 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 }
 
-// ----------------------------------------------------------------------------- split-K sums
-// Fixed summation order s = 0 .. S-1, so results do not depend on the launch.
-__global__ void reduce_f32_kernel(const float* __restrict__ ws, int S, int M, int N, float* out,
-                                  int ldo, int resid) {
+// ----------------------------------------------------------------------------- partial sums
+// Partials of a split GEMM are summed in a fixed order, so results do not depend on the
+// launch.  Two layouts:
+//  SplitSrc   split-K of the tile GEMM: ws[s][M][N], s = 0 .. S-1.
+//  StreamSrc  stream-K of the weight-streaming GEMM: ws[slot][128][BNX] (output row n of
+//             tile t = n / 128 at row n % 128, batch row m at column m); the CTAs whose
+//             iteration ranges cover tile t are c = t*KB / P .. ((t+1)*KB - 1) / P, and CTA c
+//             keeps tile t in slot c * max_seg + t - (c * P) / KB.
+struct SplitSrc {
+  const float* ws;
+  int S, M, N;
+  static constexpr bool kBatchFastest = false;
+  __device__ __forceinline__ float operator()(int m, int n) const {
+    float a = 0.f;
+    for (int s = 0; s < S; ++s) a += ws[(static_cast<size_t>(s) * M + m) * N + n];
+    return a;
+  }
+};
+struct StreamSrc {
+  const float* ws;
+  int BNX, KB, P, max_seg;
+  static constexpr bool kBatchFastest = true;
+  __device__ __forceinline__ float operator()(int m, int n) const {
+    const int t = n >> 7, r = n & 127;
+    const int c0 = (t * KB) / P, c1 = (t * KB + KB - 1) / P;
+    float a = 0.f;
+    for (int c = c0; c <= c1; ++c) {
+      const int slot = c * max_seg + t - (c * P) / KB;
+      a += ws[(static_cast<size_t>(slot) * 128 + r) * BNX + m];
+    }
+    return a;
+  }
+};
+
+// Linear index -> (row m, rest r) with the layout-friendly order.
+template <class Src>
+__device__ __forceinline__ void split_index(int64_t i, int M, int64_t R, int& m, int64_t& r) {
+  if (Src::kBatchFastest) {
+    m = static_cast<int>(i % M);
+    r = i / M;
+  } else {
+    m = static_cast<int>(i / R);
+    r = i - static_cast<int64_t>(m) * R;
+  }
+}
+
+template <class Src>
+__global__ void reduce_f32_kernel(Src src, int M, int N, float* out, int ldo, int resid) {
   const int64_t total = static_cast<int64_t>(M) * N;
   for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < total;
        i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
-    float acc = 0.f;
-    for (int s = 0; s < S; ++s) acc += ws[s * total + i];
-    const int m = static_cast<int>(i / N), n = static_cast<int>(i - static_cast<int64_t>(m) * N);
+    int m;
+    int64_t n;
+    split_index<Src>(i, M, N, m, n);
+    const float acc = src(m, static_cast<int>(n));
     float* o = out + static_cast<size_t>(m) * ldo + n;
     if (resid)
       *o += acc;
@@ -568,19 +633,16 @@ __global__ void reduce_f32_kernel(const float* __restrict__ ws, int S, int M, in
   }
 }
 
-__global__ void reduce_swiglu_kernel(const float* __restrict__ ws, int S, int M, int F,
-                                     bf16* out_hi, bf16* out_lo, int ldo) {
+template <class Src>
+__global__ void reduce_swiglu_kernel(Src src, int M, int F, bf16* out_hi, bf16* out_lo, int ldo) {
   const int64_t total = static_cast<int64_t>(M) * F;
-  const int64_t plane = static_cast<int64_t>(M) * 2 * F;
   for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < total;
        i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
-    const int m = static_cast<int>(i / F), f = static_cast<int>(i - static_cast<int64_t>(m) * F);
-    const int64_t base = static_cast<int64_t>(m) * 2 * F + f;
-    float g = 0.f, u = 0.f;
-    for (int s = 0; s < S; ++s) {
-      g += ws[s * plane + base];
-      u += ws[s * plane + base + F];
-    }
+    int m;
+    int64_t f;
+    split_index<Src>(i, M, F, m, f);
+    const float g = src(m, static_cast<int>(f));
+    const float u = src(m, static_cast<int>(f) + F);
     bf16 hi, lo;
     split_bf16(silu_f(g) * u, hi, lo);
     out_hi[static_cast<size_t>(m) * ldo + f] = hi;
@@ -589,25 +651,22 @@ __global__ void reduce_swiglu_kernel(const float* __restrict__ ws, int S, int M,
 }
 
 // One thread per (row, q|k|v section, head, i < hd/2): sums the pair (i, i + hd/2).
-__global__ void reduce_qkv_kernel(const float* __restrict__ ws, int S, int M, EpiArgs e) {
+template <class Src>
+__global__ void reduce_qkv_kernel(Src src, int M, EpiArgs e) {
   const int d = e.d, hd = e.hd, half = hd >> 1, H = d / hd;
-  const int64_t N = 3LL * d;
-  const int64_t plane = static_cast<int64_t>(M) * N;
-  const int64_t total = static_cast<int64_t>(M) * 3 * H * half;
+  const int64_t R = 3LL * H * half;
+  const int64_t total = static_cast<int64_t>(M) * R;
   for (int64_t t = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; t < total;
        t += static_cast<int64_t>(gridDim.x) * blockDim.x) {
-    const int i = static_cast<int>(t % half);
-    int64_t r = t / half;
+    int m;
+    int64_t r;
+    split_index<Src>(t, M, R, m, r);
+    const int i = static_cast<int>(r % half);
+    r /= half;
     const int head = static_cast<int>(r % H);
-    r /= H;
-    const int sec = static_cast<int>(r % 3);
-    const int m = static_cast<int>(r / 3);
-    const int64_t c = sec * static_cast<int64_t>(d) + head * hd + i;
-    float a = 0.f, b = 0.f;
-    for (int s = 0; s < S; ++s) {
-      a += ws[s * plane + static_cast<int64_t>(m) * N + c];
-      b += ws[s * plane + static_cast<int64_t>(m) * N + c + half];
-    }
+    const int sec = static_cast<int>(r / H);
+    const int c = sec * d + head * hd + i;
+    float a = src(m, c), b = src(m, c + half);
     const RowInfo ri = e.rows[m];
     if (sec < 2) {
       const float2 cs = e.rope[static_cast<size_t>(ri.pos) * half + i];
@@ -617,7 +676,7 @@ __global__ void reduce_qkv_kernel(const float* __restrict__ ws, int S, int M, Ep
       b = rb;
     }
     if (sec == 0) {
-      float* dst = e.out_f32 + static_cast<size_t>(m) * d + head * hd;
+      float* dst = e.out_q + static_cast<size_t>(m) * d + head * hd;
       dst[i] = a;
       dst[i + half] = b;
     } else {
@@ -627,6 +686,197 @@ __global__ void reduce_qkv_kernel(const float* __restrict__ ws, int S, int M, Ep
       dst[i] = __float2half_rn(a);
       dst[i + half] = __float2half_rn(b);
     }
+  }
+}
+
+// ----------------------------------------------------------------------------- decode GEMM
+// Weight-streaming GEMM for decode-sized batches (M <= 128 rows of activations), where the
+// projections are bound by reading the weights from HBM once.
+//  * swap-AB: the 128-row weight tile is the MMA's A operand and the batch (BNX rows, the
+//    activation pair hi / lo) is its N, so no MMA row is wasted on padding and the
+//    activation tiles cost smem fill BNX/128 of the weights';
+//  * stream-K: the (n-tile, k-block) iteration space is cut into equal contiguous ranges,
+//    one per CTA, so all SMs stream the same number of weight bytes; each run of one tile
+//    inside a range accumulates in TMEM and is written as one fp32 partial (StreamSrc);
+//  * weights are loaded evict-first, activations evict-last.
+struct GemvParams {
+  int N, K;
+  int tiles, kbt;       // 128-row tiles of W, 64-wide k-blocks per tile
+  int per_cta, max_seg; // stream-K range length and partial slots per CTA
+  float* ws;
+  uint32_t* status;
+};
+
+template <int BNX, int STAGES>
+__global__ void __launch_bounds__(kThreads, 1)
+    gemv_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUtensorMap tmX,
+                   const __grid_constant__ CUtensorMap tmX2, const GemvParams p) {
+  constexpr int W_BYTES = 128 * BK * 2;
+  constexpr int X_BYTES = BNX * BK * 2;
+  constexpr int STAGE_BYTES = W_BYTES + 2 * X_BYTES;
+  constexpr uint32_t TMEM_COLS = (2 * BNX < 32) ? 32 : 2 * BNX;
+  constexpr uint32_t IDESC = (1u << 4) | (1u << 7) | (1u << 10) |
+                             (static_cast<uint32_t>(BNX >> 3) << 17) | (static_cast<uint32_t>(128 >> 4) << 24);
+
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~static_cast<uintptr_t>(1023));
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + STAGES * STAGE_BYTES);
+  const uint32_t full0 = smem_u32(bars);
+  const uint32_t empty0 = full0 + 8 * STAGES;
+  const uint32_t tfull0 = empty0 + 8 * STAGES;
+  const uint32_t tempty0 = tfull0 + 16;
+  const uint32_t drain_bar = tempty0 + 16;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * STAGES + 5);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < STAGES; ++s) {
+      mbar_init(full0 + 8 * s, 1);
+      mbar_init(empty0 + 8 * s, 1);
+    }
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(tfull0 + 8 * a, 1);
+      mbar_init(tempty0 + 8 * a, 4);
+    }
+    mbar_init(drain_bar, 1);
+    *abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmW)) : "memory");
+  }
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                     smem_u32(tmem_slot)),
+                 "r"(TMEM_COLS)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+  const int total = p.tiles * p.kbt;
+  const int g_begin = blockIdx.x * p.per_cta;
+  const int g_end = min(g_begin + p.per_cta, total);
+  const int t_first = g_begin / p.kbt;
+  uint32_t* status = p.status;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      const uint64_t pol_w = policy_evict_first();
+      const uint64_t pol_x = policy_evict_last();
+      int stage = 0;
+      uint32_t phase = 0, issued = 0, issued_phase = 0;
+      bool ok = true;
+      for (int g = g_begin; g < g_end && ok;) {
+        const int t = g / p.kbt;
+        const int kb0 = g - t * p.kbt;
+        const int kb1 = min(p.kbt, kb0 + (g_end - g));
+        for (int kb = kb0; kb < kb1; ++kb) {
+          if (!wait_bounded(empty0 + 8 * stage, phase ^ 1u, abort_flag, status)) {
+            ok = false;
+            break;
+          }
+          const uint32_t fb = full0 + 8 * stage;
+          const uint32_t sw = smem_u32(smem + stage * STAGE_BYTES);
+          const uint32_t sx = sw + W_BYTES;
+          mbar_arrive_expect_tx(fb, STAGE_BYTES);
+          tma_load_2d_hint(sw, &tmW, fb, kb * BK, t * 128, pol_w);
+          tma_load_2d_hint(sx, &tmX, fb, kb * BK, 0, pol_x);
+          tma_load_2d_hint(sx + X_BYTES, &tmX2, fb, kb * BK, 0, pol_x);
+          issued |= 1u << stage;
+          issued_phase = (issued_phase & ~(1u << stage)) | (phase << stage);
+          if (++stage == STAGES) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+        g += kb1 - kb0;
+      }
+      for (int s = 0; s < STAGES; ++s)
+        if (issued & (1u << s)) wait_drain(full0 + 8 * s, (issued_phase >> s) & 1u);
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      int stage = 0;
+      uint32_t phase = 0;
+      int it = 0;
+      bool ok = true;
+      for (int g = g_begin; g < g_end && ok; ++it) {
+        const int t = g / p.kbt;
+        const int kb0 = g - t * p.kbt;
+        const int kb1 = min(p.kbt, kb0 + (g_end - g));
+        g += kb1 - kb0;
+        const int acc = it & 1;
+        const uint32_t acc_phase = (it >> 1) & 1;
+        if (!wait_bounded(tempty0 + 8 * acc, acc_phase ^ 1u, abort_flag, status)) break;
+        tc_fence_after();
+        const uint32_t d_tmem = tmem_base + acc * BNX;
+        for (int kb = kb0; kb < kb1; ++kb) {
+          if (!wait_bounded(full0 + 8 * stage, phase, abort_flag, status)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t sw = smem_u32(smem + stage * STAGE_BYTES);
+          const uint32_t sx = sw + W_BYTES;
+#pragma unroll
+          for (int k = 0; k < BK / 16; ++k) {
+            const uint64_t adesc = make_sdesc(sw + k * 32);
+            tc_mma(d_tmem, adesc, make_sdesc(sx + k * 32), IDESC, (kb > kb0 || k > 0) ? 1u : 0u);
+            tc_mma(d_tmem, adesc, make_sdesc(sx + X_BYTES + k * 32), IDESC, 1u);
+          }
+          tc_commit(empty0 + 8 * stage);
+          if (++stage == STAGES) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+        if (ok) tc_commit(tfull0 + 8 * acc);
+      }
+      tc_commit(drain_bar);
+      wait_drain(drain_bar, 0);
+    }
+  } else {
+    const int q = warp & 3;
+    int it = 0;
+    for (int g = g_begin; g < g_end; ++it) {
+      const int t = g / p.kbt;
+      const int kb0 = g - t * p.kbt;
+      const int kb1 = min(p.kbt, kb0 + (g_end - g));
+      g += kb1 - kb0;
+      const int acc = it & 1;
+      const uint32_t acc_phase = (it >> 1) & 1;
+      int ok = 1;
+      if (lane == 0) ok = wait_bounded(tfull0 + 8 * acc, acc_phase, abort_flag, status) ? 1 : 0;
+      ok = __shfl_sync(0xffffffffu, ok, 0);
+      if (!ok) break;
+      tc_fence_after();
+      const int r = q * 32 + lane;
+      const int slot = blockIdx.x * p.max_seg + (t - t_first);
+      float* dst = p.ws + (static_cast<size_t>(slot) * 128 + r) * BNX;
+      const uint32_t trow = tmem_base + (static_cast<uint32_t>(q * 32) << 16) + acc * BNX;
+#pragma unroll 1
+      for (int c = 0; c < BNX; c += 16) {
+        float v[16];
+        ld16f(trow + c, v);
+        store_f32x16(dst + c, v);
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(tempty0 + 8 * acc);
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem_base),
+                 "r"(TMEM_COLS)
+                 : "memory");
   }
 }
 
@@ -703,6 +953,90 @@ int blocks_for(int64_t n) {
   int64_t b = (n + 255) / 256;
   if (b > 4096) b = 4096;
   return static_cast<int>(b < 1 ? 1 : b);
+}
+
+
+// Applies the epilogue of `a` to summed partials.
+template <class Src>
+int launch_reduce(const Src& src, const GemmArgs& a, cudaStream_t stream) {
+  const int epi = a.epi.kind;
+  switch (epi) {
+    case EPI_F32:
+    case EPI_RESID: {
+      float* out = (epi == EPI_F32) ? a.epi.out_f32 : a.epi.resid;
+      const int ld = (epi == EPI_F32) ? a.epi.ldo : a.epi.ldr;
+      reduce_f32_kernel<Src><<<blocks_for(static_cast<int64_t>(a.M) * a.N), 256, 0, stream>>>(
+          src, a.M, a.N, out, ld, epi == EPI_RESID);
+      break;
+    }
+    case EPI_SWIGLU:
+      reduce_swiglu_kernel<Src><<<blocks_for(static_cast<int64_t>(a.M) * a.N / 2), 256, 0, stream>>>(
+          src, a.M, a.N / 2, a.epi.out_hi, a.epi.out_lo, a.epi.ldo);
+      break;
+    case EPI_QKV:
+      reduce_qkv_kernel<Src><<<blocks_for(static_cast<int64_t>(a.M) * a.N / 2), 256, 0, stream>>>(
+          src, a.M, a.epi);
+      break;
+    default:
+      return VLA_ERR_ARG;
+  }
+  note_launch();
+  VLA_CUDA_TRY(cudaGetLastError());
+  return VLA_OK;
+}
+
+GemmCost gemm_cost(const GemmArgs& a) {
+  // Algorithmic work of the model's product: 2MNK flops (the low-half MMAs of a split A are
+  // not counted); bytes = A + B read once, output written once (+ read for the residual).
+  GemmCost c;
+  c.flops = 2.0 * a.M * static_cast<double>(a.N) * a.K;
+  double out_bytes;
+  switch (a.epi.kind) {
+    case EPI_RESID: out_bytes = 8.0 * a.M * a.N; break;
+    case EPI_SWIGLU: out_bytes = 2.0 * a.M * (a.N / 2) * 2; break;
+    case EPI_QKV: out_bytes = 2.0 * a.M * a.N; break;
+    default: out_bytes = 4.0 * a.M * a.N;
+  }
+  const double a_bytes = 2.0 * a.M * static_cast<double>(a.K) * (a.A_lo ? 2 : 1);
+  c.bytes = a_bytes + 2.0 * static_cast<double>(a.N) * a.K + out_bytes;
+  return c;
+}
+
+// Stream-K plan of the weight-streaming GEMM.
+struct GemvPlan {
+  int bnx, grid, tiles, kbt, per_cta, max_seg;
+  size_t ws_bytes;
+};
+GemvPlan gemv_plan(int M, int N, int K, int num_sms) {
+  GemvPlan g{};
+  g.bnx = M <= 16 ? 16 : M <= 32 ? 32 : M <= 64 ? 64 : 128;
+  g.tiles = (N + 127) / 128;
+  g.kbt = (K + BK - 1) / BK;
+  const int total = g.tiles * g.kbt;
+  int grid = total < num_sms ? total : num_sms;
+  g.per_cta = (total + grid - 1) / grid;
+  g.grid = (total + g.per_cta - 1) / g.per_cta;
+  g.max_seg = (g.per_cta - 1) / g.kbt + 2;
+  g.ws_bytes = static_cast<size_t>(g.grid) * g.max_seg * 128 * g.bnx * sizeof(float);
+  return g;
+}
+
+template <int BNX>
+int launch_gemv(const CUtensorMap& w, const CUtensorMap& x, const CUtensorMap& x2,
+                const GemvParams& p, int grid, cudaStream_t stream) {
+  constexpr int STAGE = 128 * BK * 2 + 2 * BNX * BK * 2;
+  constexpr int STAGES = (196608 / STAGE) < 8 ? (196608 / STAGE) : 8;
+  constexpr int smem = STAGES * STAGE + 1024 + 256;
+  static bool attr_set = false;
+  auto kern = gemv_tc_kernel<BNX, STAGES>;
+  if (!attr_set) {
+    VLA_CUDA_TRY(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem));
+    attr_set = true;
+  }
+  kern<<<grid, kThreads, smem, stream>>>(w, x, x2, p);
+  note_launch();
+  VLA_CUDA_TRY(cudaGetLastError());
+  return VLA_OK;
 }
 
 }  // namespace
@@ -787,43 +1121,53 @@ int gemm_launch(const GemmArgs& a, cudaStream_t stream, int num_sms, GemmCost* c
   if (rc != VLA_OK) return rc;
 
   if (splits > 1) {
-    const float* ws = a.workspace;
-    switch (epi) {
-      case EPI_F32:
-      case EPI_RESID: {
-        float* out = (epi == EPI_F32) ? a.epi.out_f32 : a.epi.resid;
-        const int ld = (epi == EPI_F32) ? a.epi.ldo : a.epi.ldr;
-        reduce_f32_kernel<<<blocks_for(static_cast<int64_t>(a.M) * a.N), 256, 0, stream>>>(
-            ws, splits, a.M, a.N, out, ld, epi == EPI_RESID);
-        break;
-      }
-      case EPI_SWIGLU:
-        reduce_swiglu_kernel<<<blocks_for(static_cast<int64_t>(a.M) * a.N / 2), 256, 0, stream>>>(
-            ws, splits, a.M, a.N / 2, a.epi.out_hi, a.epi.out_lo, a.epi.ldo);
-        break;
-      case EPI_QKV:
-        reduce_qkv_kernel<<<blocks_for(static_cast<int64_t>(a.M) * a.N / 2), 256, 0, stream>>>(
-            ws, splits, a.M, a.epi);
-        break;
-      default:
-        return VLA_ERR_ARG;
-    }
-    note_launch();
-    VLA_CUDA_TRY(cudaGetLastError());
+    const SplitSrc src{a.workspace, splits, a.M, a.N};
+    if ((rc = launch_reduce(src, a, stream)) != VLA_OK) return rc;
   }
-  if (cost) {
-    // Algorithmic work of the model's product: 2MNK flops (the low-half MMAs of a split A are
-    // not counted); bytes = A + B read once, output written once (+ read for the residual).
-    cost->flops = 2.0 * a.M * static_cast<double>(a.N) * a.K;
-    double out_bytes;
-    switch (epi) {
-      case EPI_RESID: out_bytes = 8.0 * a.M * a.N; break;
-      case EPI_SWIGLU: out_bytes = 2.0 * a.M * (a.N / 2); break;
-      case EPI_QKV: out_bytes = 2.0 * a.M * a.N; break;
-      default: out_bytes = 4.0 * a.M * a.N;
-    }
-    cost->bytes = 2.0 * (static_cast<double>(a.M) * a.K + static_cast<double>(a.N) * a.K) + out_bytes;
+  if (cost) *cost = gemm_cost(a);
+  return VLA_OK;
+}
+
+
+size_t gemv_workspace_bytes(int M, int N, int K, int num_sms) {
+  if (M < 1 || M > 128) return 0;
+  return gemv_plan(M, N, K, num_sms).ws_bytes;
+}
+
+int gemv_launch(const GemmArgs& a, cudaStream_t stream, int num_sms, GemmCost* cost) {
+  if (a.M < 1 || a.M > 128 || a.N < 1 || a.K < 1 || !a.A || !a.A_lo || !a.B) return VLA_ERR_ARG;
+  if ((a.lda % 8) || (a.ldb % 8) || a.lda < a.K || a.ldb < a.K) return VLA_ERR_ARG;
+  if ((reinterpret_cast<uintptr_t>(a.A) & 15) || (reinterpret_cast<uintptr_t>(a.B) & 15) ||
+      (reinterpret_cast<uintptr_t>(a.A_lo) & 15))
+    return VLA_ERR_ARG;
+  if (a.epi.kind == EPI_SWIGLU && (a.N & 1)) return VLA_ERR_ARG;
+  if (a.epi.kind == EPI_QKV && (a.N != 3 * a.epi.d || 128 % a.epi.hd)) return VLA_ERR_ARG;
+  const GemvPlan pl = gemv_plan(a.M, a.N, a.K, num_sms);
+  if (!a.workspace || a.workspace_bytes < pl.ws_bytes) return VLA_ERR_ARG;
+  CUtensorMap mw, mx, mx2;
+  if (!make_map(&mw, a.B, a.N, a.K, a.ldb, 128) || !make_map(&mx, a.A, a.M, a.K, a.lda, pl.bnx) ||
+      !make_map(&mx2, a.A_lo, a.M, a.K, a.lda, pl.bnx))
+    return cuda_fail(cudaErrorInvalidValue, "tensor maps (decode GEMM)");
+  GemvParams p{};
+  p.N = a.N;
+  p.K = a.K;
+  p.tiles = pl.tiles;
+  p.kbt = pl.kbt;
+  p.per_cta = pl.per_cta;
+  p.max_seg = pl.max_seg;
+  p.ws = a.workspace;
+  p.status = a.epi.status;
+  int rc;
+  switch (pl.bnx) {
+    case 16: rc = launch_gemv<16>(mw, mx, mx2, p, pl.grid, stream); break;
+    case 32: rc = launch_gemv<32>(mw, mx, mx2, p, pl.grid, stream); break;
+    case 64: rc = launch_gemv<64>(mw, mx, mx2, p, pl.grid, stream); break;
+    default: rc = launch_gemv<128>(mw, mx, mx2, p, pl.grid, stream); break;
   }
+  if (rc != VLA_OK) return rc;
+  const StreamSrc src{a.workspace, pl.bnx, pl.kbt, pl.per_cta, pl.max_seg};
+  if ((rc = launch_reduce(src, a, stream)) != VLA_OK) return rc;
+  if (cost) *cost = gemm_cost(a);
   return VLA_OK;
 }
 

@@ -55,6 +55,37 @@ def test_gemm_matches_fp64(M, N, K, bn, splits, split_a):
     assert err < 2e-5 * math.sqrt(K) * 8, err
 
 
+DECODE_CASES = [
+    # M (<= 128 rows), N, K
+    (1, 128, 64),
+    (4, 768, 256),
+    (16, 3072, 1024),
+    (24, 200, 688),        # ragged N and K, score-sized M
+    (64, 12288, 4096),     # 7B q|k|v decode step
+    (64, 4096, 11008),     # 7B down-projection decode step
+    (100, 1376, 256),
+    (128, 4096, 4096),
+]
+
+
+@pytest.mark.parametrize("M,N,K", DECODE_CASES)
+def test_decode_gemm_matches_fp64(M, N, K):
+    A = I.normal_bf16((M, K), 98, 1000 + M, 1.0)
+    A_lo = I.normal_bf16((M, K), 98, 3000 + M, 2.0 ** -9)
+    W = I.normal_bf16((N, K), 98, 2000 + N, 1.0)
+    C = torch.full((M, N), float("nan"), dtype=torch.float32, device="cuda")
+    nbytes = V.vla_op_gemm_decode_workspace_bytes(M, N, K)
+    ws = torch.empty(max(1, nbytes // 4), dtype=torch.float32, device="cuda")
+    Ad, Ald, Wd = A.cuda(), A_lo.cuda(), W.cuda()
+    rc = V.vla_op_gemm_decode_bf16(Ad.data_ptr(), Ald.data_ptr(), K, Wd.data_ptr(), K, C.data_ptr(), N,
+                                   M, N, K, ws.data_ptr(), nbytes, 0)
+    assert rc == 0, V.vla_last_error()
+    torch.cuda.synchronize()
+    ref = (A.double() + A_lo.double()) @ W.double().T
+    err = (C.cpu().double() - ref).abs().max().item()
+    assert err < 2e-5 * math.sqrt(K) * 8, err
+
+
 def test_gemm_rejects_bad_strides():
     A = torch.zeros(8, 12, dtype=torch.bfloat16, device="cuda")
     C = torch.zeros(8, 8, dtype=torch.float32, device="cuda")
