@@ -90,6 +90,16 @@ class ClockSampler:
                 "reasons": reasons, "samples": len(self.samples)}
 
 
+def max_over_ranks(x: float, dist=None, device="cuda") -> float:
+    """Largest value over all ranks (the job is as slow as its slowest replica)."""
+    if dist is None or not dist.is_initialized() or dist.get_world_size() == 1:
+        return x
+    import torch
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
 def dist_setup():
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -270,13 +280,6 @@ def main():
         if dist is not None:
             dist.barrier()
 
-    def max_over_ranks(x):
-        if dist is None:
-            return x
-        t = torch.tensor([x], dtype=torch.float64, device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        return float(t.item())
-
     # ---- warm-up
     for _ in range(args.warmup):
         step(vis_d, ids_d, u_d)
@@ -295,7 +298,7 @@ def main():
         ev1.record(stream)
         torch.cuda.synchronize()
     barrier()
-    ms_total = max_over_ranks(ev0.elapsed_time(ev1))
+    ms_total = max_over_ranks(ev0.elapsed_time(ev1), dist)
     launches = V.vla_launch_count(h) - launches0
     prof = V.vla_profile_read(h)
     V.vla_profile(h, 0)
@@ -350,7 +353,7 @@ def main():
         e2e_step()
     ev1.record(stream)
     torch.cuda.synchronize()
-    e2e_ms = max_over_ranks(ev0.elapsed_time(ev1)) / args.steps
+    e2e_ms = max_over_ranks(ev0.elapsed_time(ev1), dist) / args.steps
     h2d = vis_h.numel() * 2 + ids_h.numel() * 4 + u_h.numel() * 4
     d2h = sum(t.numel() * 4 for t in out_h)
 
