@@ -170,7 +170,53 @@ CASES = {
     "gemv_decode_qkv": (64, 12288, 4096, 0, 0, True),
     "gemv_decode_gate_up": (64, 22016, 4096, 0, 0, True),
     "gemv_decode_down": (64, 4096, 11008, 0, 0, True),
+    "attn_decode": None,                                       # see run_attn_case
 }
+
+
+def run_attn_case(args):
+    """Decode attention for 64 envs x 32 heads at ~290 cached positions (one layer)."""
+    import torch
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2505_18719_gb300 import inputs as I
+    from paper_2505_18719_gb300 import vla as V
+    B, H, hd, cap = 64, 32, 128, 320
+    kv = I.normal_bf16((B, 2, H, cap, hd), 5, 1, 1.0).cuda().half()
+    q = I.normal_bf16((B, H, hd), 5, 2, 1.0).cuda().float()
+    ctx = I.randint_i32((B,), 5, 3, 273, 311)
+    env = torch.arange(B, dtype=torch.int32, device="cuda")
+    pos = (ctx - 1).cuda()
+    max_ctx = int(ctx.max())
+    keys = args.attn_keys
+    nbytes = V.vla_op_attn_decode_workspace_bytes(B, H, hd, max_ctx, keys)
+    ws = torch.empty(nbytes // 4 + 64, dtype=torch.float32, device="cuda")
+    oh = torch.empty(B, H * hd, dtype=torch.bfloat16, device="cuda")
+    ol = torch.empty_like(oh)
+    stream = torch.cuda.current_stream()
+
+    def launch():
+        rc = V.vla_op_attn_decode(q.data_ptr(), kv.data_ptr(), B, H, hd, cap, env.data_ptr(), pos.data_ptr(), B,
+                                  max_ctx, oh.data_ptr(), ol.data_ptr(), ws.data_ptr(), nbytes, stream.cuda_stream,
+                                  keys)
+        assert rc == 0, V.vla_last_error()
+
+    for _ in range(args.warmup):
+        launch()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        launch()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1) / args.steps
+    hbm, _, _, kind = peaks()
+    bytes_ = float(ctx.sum()) * 2 * H * hd * 2 + B * H * hd * (4 + 4)
+    print(json.dumps({"case": args.case, "B": B, "H": H, "hd": hd, "max_keys_per_cta": keys,
+                      "kv_positions": int(ctx.sum()), "ms": ms,
+                      "gbs": bytes_ / ms / 1e6, "hbm_frac": bytes_ / ms / 1e6 / hbm, "peaks": kind}))
+    return 0
 
 
 def run_case(args):
@@ -180,6 +226,8 @@ def run_case(args):
     __graft_entry__.build()
     from paper_2505_18719_gb300 import inputs as I
     from paper_2505_18719_gb300 import vla as V
+    if args.case == "attn_decode":
+        return run_attn_case(args)
     M, N, K, bn, splits, split_a = CASES[args.case]
     A = I.normal_bf16((M, K), 1, 1, 1.0).cuda()
     A_lo = I.normal_bf16((M, K), 1, 2, 2.0 ** -9).cuda()
@@ -231,6 +279,7 @@ def main():
     ap.add_argument("--workload", default=WORKLOAD)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--case", choices=sorted(CASES), help="time one kernel shape instead of the hot path")
+    ap.add_argument("--attn-keys", type=int, default=0, help="attn_decode case: max keys per CTA (0 = default)")
     args = ap.parse_args()
     if args.impl == "reference":
         return run_reference(args)

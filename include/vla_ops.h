@@ -67,6 +67,22 @@ int vla_op_action_head(const float* h, int ldh, int B, int d, const void* final_
                        float* logprobs_out, float* actions_out, float* logits_out,
                        uint32_t* status, void* cuda_stream);
 
+/* Decode-step causal attention (§3.1 self-attention over the env's whole multi-turn context,
+ * §3.3) for B single queries, flash-decoding over the fp16 KV cache:
+ *   q         f32 [B, H, hd] (already rotated);
+ *   kv        fp16 cache laid out [env][K,V][H][cap][hd] (one layer, max_env envs);
+ *   env, pos  int32 [B] each: query b reads env env[b], keys 0..pos[b] (pos[b] < cap);
+ *   max_keys_per_cta  longest key range one CTA handles (0 = the library's default, 160);
+ *   out_hi / out_lo  bf16 [B, H*hd]: the output o as the pair hi + lo;
+ *   workspace f32, at least vla_op_attn_decode_workspace_bytes(B, H, hd, max_ctx,
+ *             max_keys_per_cta) bytes, max_ctx >= every pos[b] + 1.
+ * hd in {64, 128}. */
+int vla_op_attn_decode(const float* q, const void* kv, int max_env, int H, int hd, int cap,
+                       const int32_t* env, const int32_t* pos, int B, int max_ctx,
+                       int max_keys_per_cta, void* out_hi, void* out_lo, float* workspace,
+                       size_t workspace_bytes, void* cuda_stream);
+size_t vla_op_attn_decode_workspace_bytes(int B, int H, int hd, int max_ctx, int max_keys_per_cta);
+
 /* Number of SMs the kernels size their persistent grids for (device property). */
 int vla_op_num_sms(void);
 

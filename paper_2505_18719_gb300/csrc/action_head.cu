@@ -31,6 +31,8 @@ __global__ void __launch_bounds__(256) action_head_kernel(const HeadArgs a) {
   __shared__ ArgMax red_a[8];
   __shared__ float red_m[8];
 
+  pdl_launch_dependents();
+  pdl_wait();
   const int b = blockIdx.x, j = blockIdx.y;
   const int i_act = a.step + j;               // action index
   const int out_i = b * a.A + i_act;          // [B, A] output slot
@@ -155,7 +157,7 @@ int action_head_launch(const HeadArgs& a, cudaStream_t s) {
     }
   }
   dim3 grid(a.B, a.n_pos);
-  action_head_kernel<<<grid, 256, smem, s>>>(a);
+  VLA_CUDA_TRY(launch_pdl(action_head_kernel, grid, dim3(256), smem, s, a));
   note_launch();
   VLA_CUDA_TRY(cudaGetLastError());
   return VLA_OK;

@@ -16,6 +16,7 @@
 // Keys visible to a query at position p are positions 0..p (all of them are in the cache:
 // chunk rows write their K/V in the QKV epilogue before attention runs).
 #include "attention.h"
+#include "ptx.cuh"
 
 namespace vla {
 
@@ -82,6 +83,8 @@ __global__ void __launch_bounds__(128) attn_chunk_mma_kernel(const float* __rest
   f16* Ks = sm_h;              // [2][KB][LD]
   f16* Vs = Ks + 2 * KB * LD;  // [2][KB][LD]
 
+  pdl_launch_dependents();
+  pdl_wait();
   const AttnTile t = tiles[blockIdx.x];
   const int head = blockIdx.y;
   const int d = H * HD;
@@ -264,6 +267,11 @@ __global__ void __launch_bounds__(128) attn_chunk_mma_kernel(const float* __rest
 }
 
 // ---------------------------------------------------------------------------------- decode
+// One query per (env, head, key range): 16 lanes x 16 bytes read one 128-element fp16 key row,
+// each lane group loads 4 key rows (K and V) before using any (memory-level parallelism), the
+// dot products reduce with xor shuffles inside the group, online softmax per lane group; the
+// groups of the CTA merge through shared memory into one partial (max, sum, unnormalised
+// output) per range, which the combine kernel merges across ranges in a fixed order.
 template <int HD>
 __global__ void __launch_bounds__(128) attn_decode_kernel(const float* __restrict__ q,
                                                           const RowInfo* __restrict__ rows,
@@ -271,11 +279,14 @@ __global__ void __launch_bounds__(128) attn_decode_kernel(const float* __restric
                                                           int chunk, int S, float scale_log2,
                                                           float* __restrict__ part_o,
                                                           float2* __restrict__ part_ml) {
-  constexpr int LPK = HD / 8;     // lanes per key row (8 bf16 = 16 bytes per lane)
+  constexpr int LPK = HD / 8;     // lanes per key row (8 fp16 = 16 bytes per lane)
   constexpr int KPI = 32 / LPK;   // key rows per warp instruction
+  constexpr int U = 4;            // key rows per lane group loaded ahead
   __shared__ float s_m[4][KPI], s_l[4][KPI];
   __shared__ float s_o[4][KPI][HD];
 
+  pdl_launch_dependents();
+  pdl_wait();
   const int split = blockIdx.x, head = blockIdx.y, b = blockIdx.z;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int sub = lane / LPK, part = lane - sub * LPK;
@@ -306,8 +317,6 @@ __global__ void __launch_bounds__(128) attn_decode_kernel(const float* __restric
 #pragma unroll
   for (int e = 0; e < 8; ++e) o[e] = 0.f;
 
-  // U key rows per lane group are loaded before any is used (memory-level parallelism)
-  constexpr int U = 4;
   for (int key0 = k_begin + warp * KPI * U; key0 < k_end; key0 += 4 * KPI * U) {
     uint4 kk[U], vv[U];
 #pragma unroll
@@ -384,6 +393,8 @@ template <int HD>
 __global__ void attn_combine_kernel(const float* __restrict__ part_o,
                                     const float2* __restrict__ part_ml, int H, int S,
                                     bf16* __restrict__ out_hi, bf16* __restrict__ out_lo) {
+  pdl_launch_dependents();
+  pdl_wait();
   const int bh = blockIdx.x;  // b * H + head
   const int c = threadIdx.x;
   float M = -INFINITY;
@@ -418,7 +429,8 @@ int attn_chunk_launch(const float* q, bf16* out_hi, bf16* out_lo, const AttnTile
                                         cudaFuncAttributeMaxDynamicSharedMemorySize, smem));
       set = true;
     }
-    attn_chunk_mma_kernel<128><<<grid, 128, smem, stream>>>(q, out_hi, out_lo, tiles, kv, layer, H, scale_log2);
+    VLA_CUDA_TRY(launch_pdl(attn_chunk_mma_kernel<128>, grid, dim3(128), smem, stream, q, out_hi, out_lo,
+                            tiles, kv, layer, H, scale_log2));
   } else if (hd == 64) {
     const int smem = (4 * 64) * (64 + 8) * 2;
     static bool set = false;
@@ -427,7 +439,8 @@ int attn_chunk_launch(const float* q, bf16* out_hi, bf16* out_lo, const AttnTile
                                         cudaFuncAttributeMaxDynamicSharedMemorySize, smem));
       set = true;
     }
-    attn_chunk_mma_kernel<64><<<grid, 128, smem, stream>>>(q, out_hi, out_lo, tiles, kv, layer, H, scale_log2);
+    VLA_CUDA_TRY(launch_pdl(attn_chunk_mma_kernel<64>, grid, dim3(128), smem, stream, q, out_hi, out_lo,
+                            tiles, kv, layer, H, scale_log2));
   } else {
     return VLA_ERR_UNSUPPORTED;
   }
@@ -442,19 +455,21 @@ int attn_decode_launch(const float* q, bf16* out_hi, bf16* out_lo, const RowInfo
   if (B <= 0) return VLA_OK;
   // equal key ranges (multiples of 16) no longer than `chunk`
   const int S = (max_ctx + chunk - 1) / chunk;
-  chunk = ((max_ctx + S - 1) / S + 15) / 16 * 16;
+  const int c = ((max_ctx + S - 1) / S + 15) / 16 * 16;
   const float scale_log2 = 1.4426950408889634f / sqrtf(static_cast<float>(hd));
   dim3 grid(S, H, B);
   if (hd == 128) {
-    attn_decode_kernel<128><<<grid, 128, 0, stream>>>(q, rows, kv, layer, H, chunk, S,
-                                                      scale_log2, part_o, part_ml);
+    VLA_CUDA_TRY(launch_pdl(attn_decode_kernel<128>, grid, dim3(128), 0, stream, q, rows, kv, layer, H,
+                            c, S, scale_log2, part_o, part_ml));
     note_launch();
-    attn_combine_kernel<128><<<B * H, 128, 0, stream>>>(part_o, part_ml, H, S, out_hi, out_lo);
+    VLA_CUDA_TRY(launch_pdl(attn_combine_kernel<128>, dim3(B * H), dim3(128), 0, stream, part_o, part_ml,
+                            H, S, out_hi, out_lo));
   } else if (hd == 64) {
-    attn_decode_kernel<64><<<grid, 128, 0, stream>>>(q, rows, kv, layer, H, chunk, S,
-                                                     scale_log2, part_o, part_ml);
+    VLA_CUDA_TRY(launch_pdl(attn_decode_kernel<64>, grid, dim3(128), 0, stream, q, rows, kv, layer, H,
+                            c, S, scale_log2, part_o, part_ml));
     note_launch();
-    attn_combine_kernel<64><<<B * H, 64, 0, stream>>>(part_o, part_ml, H, S, out_hi, out_lo);
+    VLA_CUDA_TRY(launch_pdl(attn_combine_kernel<64>, dim3(B * H), dim3(64), 0, stream, part_o, part_ml,
+                            H, S, out_hi, out_lo));
   } else {
     return VLA_ERR_UNSUPPORTED;
   }

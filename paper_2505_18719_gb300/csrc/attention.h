@@ -14,8 +14,8 @@ struct AttnTile {
 int attn_chunk_launch(const float* q, bf16* out_hi, bf16* out_lo, const AttnTile* tiles,
                       int n_tiles, KVLayout kv, int layer, int H, int hd, cudaStream_t stream);
 
-// One query per env row b (rows[b] gives env and position); key range split into chunks of
-// `chunk` keys; partials in part_o [B*H*S*hd] f32 and part_ml [B*H*S] (S = ceil(max_ctx/chunk)).
+// One query per env row b (rows[b] gives env and position); key range split into equal ranges
+// of at most `chunk` keys (chunk <= 256); partials in part_o [B*H*S*hd] f32 and part_ml [B*H*S] (S = ceil(max_ctx/chunk)).
 int attn_decode_launch(const float* q, bf16* out_hi, bf16* out_lo, const RowInfo* rows, int B,
                        int max_ctx, KVLayout kv, int layer, int H, int hd, int chunk,
                        float* part_o, float2* part_ml, cudaStream_t stream);

@@ -848,6 +848,51 @@ int vla_op_action_head(const float* hs, int ldh, int B, int d, const void* final
   return action_head_launch(ha, static_cast<cudaStream_t>(cuda_stream));
 }
 
+static const int kOpAttnChunk = 160;
+
+size_t vla_op_attn_decode_workspace_bytes(int B, int H, int hd, int max_ctx, int max_keys_per_cta) {
+  if (B < 1 || H < 1 || hd < 1 || max_ctx < 1) return 0;
+  const int chunk = max_keys_per_cta > 0 ? max_keys_per_cta : kOpAttnChunk;
+  const size_t S = (static_cast<size_t>(max_ctx) + chunk - 1) / chunk;
+  // RowInfo table, then partial outputs and (max, sum) pairs
+  return static_cast<size_t>(B) * sizeof(RowInfo) + 256 + static_cast<size_t>(B) * H * S * hd * sizeof(float) +
+         256 + static_cast<size_t>(B) * H * S * sizeof(float2) + 256 + 256;
+}
+
+int vla_op_attn_decode(const float* q, const void* kv, int max_env, int H, int hd, int cap, const int32_t* env,
+                       const int32_t* pos, int B, int max_ctx, int max_keys_per_cta, void* out_hi, void* out_lo,
+                       float* workspace, size_t workspace_bytes, void* cuda_stream) {
+  const int chunk = max_keys_per_cta > 0 ? max_keys_per_cta : kOpAttnChunk;
+  if (!q || !kv || !env || !pos || !out_hi || !out_lo || !workspace || B < 1 || H < 1 || cap < 1 ||
+      max_env < 1 || max_ctx < 1 || max_ctx > cap || (hd != 64 && hd != 128) || chunk < 16 ||
+      workspace_bytes < vla_op_attn_decode_workspace_bytes(B, H, hd, max_ctx, chunk))
+    return set_err(nullptr, VLA_ERR_ARG, "vla_op_attn_decode: bad argument");
+  cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
+  // Row table from env / pos (a strided device copy each, no host round trip).
+  RowInfo* rows = reinterpret_cast<RowInfo*>(workspace);
+  if (cudaMemsetAsync(rows, 0, static_cast<size_t>(B) * sizeof(RowInfo), st) != cudaSuccess ||
+      cudaMemcpy2DAsync(&rows[0].env, sizeof(RowInfo), env, sizeof(int32_t), sizeof(int32_t), B,
+                        cudaMemcpyDeviceToDevice, st) != cudaSuccess ||
+      cudaMemcpy2DAsync(&rows[0].pos, sizeof(RowInfo), pos, sizeof(int32_t), sizeof(int32_t), B,
+                        cudaMemcpyDeviceToDevice, st) != cudaSuccess)
+    return cuda_fail(cudaGetLastError(), "vla_op_attn_decode: row table");
+  char* base = reinterpret_cast<char*>(workspace) + ((static_cast<size_t>(B) * sizeof(RowInfo) + 255) / 256) * 256;
+  const size_t S = (static_cast<size_t>(max_ctx) + chunk - 1) / chunk;
+  float* part_o = reinterpret_cast<float*>(base);
+  float2* part_ml = reinterpret_cast<float2*>(base + ((static_cast<size_t>(B) * H * S * hd * sizeof(float) + 255) / 256) * 256);
+  KVLayout L{};
+  L.base = static_cast<f16*>(const_cast<void*>(kv));
+  L.cap = cap;
+  L.head_stride = static_cast<int64_t>(cap) * hd;
+  L.kv_stride = static_cast<int64_t>(H) * L.head_stride;
+  L.env_stride = 2 * L.kv_stride;
+  L.layer_stride = static_cast<int64_t>(max_env) * L.env_stride;
+  const int rc = attn_decode_launch(q, static_cast<bf16*>(out_hi), static_cast<bf16*>(out_lo), rows, B, max_ctx, L,
+                                    0, H, hd, chunk, part_o, part_ml, st);
+  if (rc != VLA_OK && rc != VLA_ERR_CUDA) return set_err(nullptr, rc, "vla_op_attn_decode: unsupported arguments");
+  return rc;
+}
+
 int vla_op_num_sms(void) { return query_num_sms(); }
 
 }  // extern "C"

@@ -26,6 +26,7 @@
 #include <mutex>
 
 #include "gemm.h"
+#include "ptx.cuh"
 
 namespace vla {
 
@@ -34,100 +35,7 @@ namespace {
 constexpr int BM = 128;
 constexpr int BK = 64;  // 64 bf16 = 128 bytes = one swizzle atom row
 constexpr int kThreads = 192;
-constexpr uint64_t kWaitLimitNs = 1000000000ull;  // 1 s per wait
 constexpr int kGroupM = 16;
-
-// ----------------------------------------------------------------------------- PTX helpers
-__device__ __forceinline__ uint32_t smem_u32(const void* p) {
-  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
-}
-__device__ __forceinline__ uint64_t globaltimer() {
-  uint64_t t;
-  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
-  return t;
-}
-__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
-  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count));
-}
-__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
-  uint32_t ok;
-  asm volatile(
-      "{\n\t.reg .pred p;\n\t"
-      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
-      "selp.u32 %0, 1, 0, p;\n\t}"
-      : "=r"(ok)
-      : "r"(bar), "r"(parity)
-      : "memory");
-  return ok != 0;
-}
-__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
-  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
-}
-__device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t bar, uint32_t bytes) {
-  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
-               : "memory");
-}
-__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map, uint32_t bar,
-                                            int c0, int c1) {
-  asm volatile(
-      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes"
-      " [%0], [%1, {%3, %4}], [%2];" ::"r"(dst),
-      "l"(reinterpret_cast<uint64_t>(map)), "r"(bar), "r"(c0), "r"(c1)
-      : "memory");
-}
-// Same with an L2 cache policy (createpolicy): weights streamed once per decode step are
-// loaded evict-first, the small activation tiles every CTA re-reads evict-last.
-__device__ __forceinline__ void tma_load_2d_hint(uint32_t dst, const CUtensorMap* map,
-                                                 uint32_t bar, int c0, int c1, uint64_t policy) {
-  asm volatile(
-      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint"
-      " [%0], [%1, {%3, %4}], [%2], %5;" ::"r"(dst),
-      "l"(reinterpret_cast<uint64_t>(map)), "r"(bar), "r"(c0), "r"(c1), "l"(policy)
-      : "memory");
-}
-__device__ __forceinline__ uint64_t policy_evict_first() {
-  uint64_t p;
-  asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
-  return p;
-}
-__device__ __forceinline__ uint64_t policy_evict_last() {
-  uint64_t p;
-  asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(p));
-  return p;
-}
-__device__ __forceinline__ void tc_fence_before() {
-  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
-}
-__device__ __forceinline__ void tc_fence_after() {
-  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-}
-__device__ __forceinline__ void tc_commit(uint32_t bar) {
-  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
-                   bar)
-               : "memory");
-}
-__device__ __forceinline__ void tc_mma(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc,
-                                       uint32_t idesc, uint32_t accumulate) {
-  asm volatile(
-      "{\n\t.reg .pred p;\n\t"
-      "setp.ne.b32 p, %4, 0;\n\t"
-      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
-      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
-      : "memory");
-}
-// 32 lanes x 32 bit, 16 consecutive columns -> 16 registers of this thread's row.
-__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
-  asm volatile(
-      "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, "
-      "%11, %12, %13, %14, %15}, [%16];"
-      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
-        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]),
-        "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
-      : "r"(taddr));
-}
-__device__ __forceinline__ void tmem_wait_ld() {
-  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
-}
 
 // Shared-memory matrix descriptor: K-major operand, 128-byte swizzle, rows of 128 bytes,
 // 8-row core-matrix groups 1024 bytes apart (SBO); LBO unused for this layout.
@@ -153,32 +61,6 @@ struct Params {
   int tiles_m, tiles_n, splits, kb_total, kb_per_split;
   EpiArgs epi;
 };
-
-// Bounded wait.  Returns false when this CTA is aborting (timeout here or elsewhere).
-__device__ __forceinline__ bool wait_bounded(uint32_t bar, uint32_t parity, volatile int* abort_flag,
-                                             uint32_t* status) {
-  if (mbar_try_wait(bar, parity)) return true;
-  const uint64_t t0 = globaltimer();
-  uint32_t n = 0;
-  while (true) {
-    if (mbar_try_wait(bar, parity)) return true;
-    if (((++n) & 63u) == 0) {
-      if (*abort_flag) return false;
-      if (globaltimer() - t0 > kWaitLimitNs) {
-        *abort_flag = 1;
-        if (status) atomicOr(status, VLA_STATUS_TIMEOUT);
-        return false;
-      }
-    }
-  }
-}
-// Wait used while draining: ignores the abort flag, bounded by time only.
-__device__ __forceinline__ void wait_drain(uint32_t bar, uint32_t parity) {
-  const uint64_t t0 = globaltimer();
-  while (!mbar_try_wait(bar, parity)) {
-    if (globaltimer() - t0 > kWaitLimitNs) return;
-  }
-}
 
 __device__ __forceinline__ void unit_coords(const Params& p, int u, int& m_blk, int& n_blk,
                                             int& split) {
@@ -401,6 +283,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   constexpr uint32_t IDESC = make_idesc<BN>();
   constexpr bool SWIGLU = (EPI == EPI_SWIGLU);
 
+  pdl_launch_dependents();
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
@@ -451,6 +334,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp == 0) {
     if (lane == 0) {
       // ------------------------------------------------------------ TMA producer
+      pdl_wait();  // everything this CTA reads or writes is ordered after this wait
       int stage = 0;
       uint32_t phase = 0;
       uint32_t issued = 0, issued_phase = 0;
@@ -574,8 +458,8 @@ __global__ void __launch_bounds__(kThreads, 1)
 // Partials of a split GEMM are summed in a fixed order, so results do not depend on the
 // launch.  Two layouts:
 //  SplitSrc   split-K of the tile GEMM: ws[s][M][N], s = 0 .. S-1.
-//  StreamSrc  stream-K of the weight-streaming GEMM: ws[slot][128][BNX] (output row n of
-//             tile t = n / 128 at row n % 128, batch row m at column m); the CTAs whose
+//  StreamSrc  stream-K of the weight-streaming GEMM: ws[slot][256][BNX] (output row n of
+//             tile t = n / 256 at row n % 256, batch row m at column m); the CTAs whose
 //             iteration ranges cover tile t are c = t*KB / P .. ((t+1)*KB - 1) / P, and CTA c
 //             keeps tile t in slot c * max_seg + t - (c * P) / KB.
 struct SplitSrc {
@@ -593,12 +477,12 @@ struct StreamSrc {
   int BNX, KB, P, max_seg;
   static constexpr bool kBatchFastest = true;
   __device__ __forceinline__ float operator()(int m, int n) const {
-    const int t = n >> 7, r = n & 127;
+    const int t = n >> 8, r = n & 255;
     const int c0 = (t * KB) / P, c1 = (t * KB + KB - 1) / P;
     float a = 0.f;
     for (int c = c0; c <= c1; ++c) {
       const int slot = c * max_seg + t - (c * P) / KB;
-      a += ws[(static_cast<size_t>(slot) * 128 + r) * BNX + m];
+      a += ws[(static_cast<size_t>(slot) * 256 + r) * BNX + m];
     }
     return a;
   }
@@ -618,6 +502,8 @@ __device__ __forceinline__ void split_index(int64_t i, int M, int64_t R, int& m,
 
 template <class Src>
 __global__ void reduce_f32_kernel(Src src, int M, int N, float* out, int ldo, int resid) {
+  pdl_launch_dependents();
+  pdl_wait();
   const int64_t total = static_cast<int64_t>(M) * N;
   for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < total;
        i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
@@ -635,6 +521,8 @@ __global__ void reduce_f32_kernel(Src src, int M, int N, float* out, int ldo, in
 
 template <class Src>
 __global__ void reduce_swiglu_kernel(Src src, int M, int F, bf16* out_hi, bf16* out_lo, int ldo) {
+  pdl_launch_dependents();
+  pdl_wait();
   const int64_t total = static_cast<int64_t>(M) * F;
   for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < total;
        i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
@@ -653,6 +541,8 @@ __global__ void reduce_swiglu_kernel(Src src, int M, int F, bf16* out_hi, bf16* 
 // One thread per (row, q|k|v section, head, i < hd/2): sums the pair (i, i + hd/2).
 template <class Src>
 __global__ void reduce_qkv_kernel(Src src, int M, EpiArgs e) {
+  pdl_launch_dependents();
+  pdl_wait();
   const int d = e.d, hd = e.hd, half = hd >> 1, H = d / hd;
   const int64_t R = 3LL * H * half;
   const int64_t total = static_cast<int64_t>(M) * R;
@@ -701,23 +591,29 @@ __global__ void reduce_qkv_kernel(Src src, int M, EpiArgs e) {
 //  * weights are loaded evict-first, activations evict-last.
 struct GemvParams {
   int N, K;
-  int tiles, kbt;       // 128-row tiles of W, 64-wide k-blocks per tile
+  int tiles, kbt;       // 256-row tiles of W, 64-wide k-blocks per tile
   int per_cta, max_seg; // stream-K range length and partial slots per CTA
   float* ws;
   uint32_t* status;
 };
 
+// TR = 256 weight rows per tile, as two M=128 MMAs sharing each activation tile, so the
+// activation fill per weight byte is BNX/256 * 2 and 4 stages keep 128 KB of weights in flight.
 template <int BNX, int STAGES>
 __global__ void __launch_bounds__(kThreads, 1)
     gemv_tc_kernel(const __grid_constant__ CUtensorMap tmW, const __grid_constant__ CUtensorMap tmX,
                    const __grid_constant__ CUtensorMap tmX2, const GemvParams p) {
-  constexpr int W_BYTES = 128 * BK * 2;
+  constexpr int TR = 256, NH = TR / 128;
+  constexpr int W_HALF = 128 * BK * 2;
+  constexpr int W_BYTES = NH * W_HALF;
   constexpr int X_BYTES = BNX * BK * 2;
   constexpr int STAGE_BYTES = W_BYTES + 2 * X_BYTES;
-  constexpr uint32_t TMEM_COLS = (2 * BNX < 32) ? 32 : 2 * BNX;
+  constexpr uint32_t TMEM_COLS = 2 * NH * BNX;
   constexpr uint32_t IDESC = (1u << 4) | (1u << 7) | (1u << 10) |
                              (static_cast<uint32_t>(BNX >> 3) << 17) | (static_cast<uint32_t>(128 >> 4) << 24);
+  static_assert(TMEM_COLS >= 32 && (TMEM_COLS & (TMEM_COLS - 1)) == 0, "TMEM allocation");
 
+  pdl_launch_dependents();
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
@@ -765,41 +661,54 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (warp == 0) {
     if (lane == 0) {
+      // ------------------------------------------------------------ TMA producer
+      // The weights do not depend on the previous kernel: the first STAGES weight tiles are
+      // requested before waiting for it, the activations only after.
       const uint64_t pol_w = policy_evict_first();
       const uint64_t pol_x = policy_evict_last();
-      int stage = 0;
-      uint32_t phase = 0, issued = 0, issued_phase = 0;
-      bool ok = true;
-      for (int g = g_begin; g < g_end && ok;) {
-        const int t = g / p.kbt;
-        const int kb0 = g - t * p.kbt;
-        const int kb1 = min(p.kbt, kb0 + (g_end - g));
-        for (int kb = kb0; kb < kb1; ++kb) {
-          if (!wait_bounded(empty0 + 8 * stage, phase ^ 1u, abort_flag, status)) {
-            ok = false;
-            break;
-          }
-          const uint32_t fb = full0 + 8 * stage;
-          const uint32_t sw = smem_u32(smem + stage * STAGE_BYTES);
-          const uint32_t sx = sw + W_BYTES;
-          mbar_arrive_expect_tx(fb, STAGE_BYTES);
-          tma_load_2d_hint(sw, &tmW, fb, kb * BK, t * 128, pol_w);
-          tma_load_2d_hint(sx, &tmX, fb, kb * BK, 0, pol_x);
-          tma_load_2d_hint(sx + X_BYTES, &tmX2, fb, kb * BK, 0, pol_x);
-          issued |= 1u << stage;
-          issued_phase = (issued_phase & ~(1u << stage)) | (phase << stage);
-          if (++stage == STAGES) {
-            stage = 0;
-            phase ^= 1u;
-          }
+      const int n = g_end - g_begin;
+      const int pre = n < STAGES ? n : STAGES;
+      uint32_t issued = 0, issued_phase = 0;
+      for (int i = 0; i < pre; ++i) {
+        const int g = g_begin + i, t = g / p.kbt, kb = g - t * p.kbt;
+        const uint32_t sw = smem_u32(smem + i * STAGE_BYTES);
+        mbar_arrive_expect_tx(full0 + 8 * i, STAGE_BYTES);
+        tma_load_2d_hint(sw, &tmW, full0 + 8 * i, kb * BK, t * TR, pol_w);
+        issued |= 1u << i;
+      }
+      pdl_wait();
+      for (int i = 0; i < pre; ++i) {
+        const int g = g_begin + i, t = g / p.kbt, kb = g - t * p.kbt;
+        (void)t;
+        const uint32_t sx = smem_u32(smem + i * STAGE_BYTES) + W_BYTES;
+        tma_load_2d_hint(sx, &tmX, full0 + 8 * i, kb * BK, 0, pol_x);
+        tma_load_2d_hint(sx + X_BYTES, &tmX2, full0 + 8 * i, kb * BK, 0, pol_x);
+      }
+      int stage = pre % STAGES;
+      uint32_t phase = (pre == STAGES) ? 1u : 0u;
+      for (int i = pre; i < n; ++i) {
+        const int g = g_begin + i, t = g / p.kbt, kb = g - t * p.kbt;
+        if (!wait_bounded(empty0 + 8 * stage, phase ^ 1u, abort_flag, status)) break;
+        const uint32_t fb = full0 + 8 * stage;
+        const uint32_t sw = smem_u32(smem + stage * STAGE_BYTES);
+        const uint32_t sx = sw + W_BYTES;
+        mbar_arrive_expect_tx(fb, STAGE_BYTES);
+        tma_load_2d_hint(sw, &tmW, fb, kb * BK, t * TR, pol_w);
+        tma_load_2d_hint(sx, &tmX, fb, kb * BK, 0, pol_x);
+        tma_load_2d_hint(sx + X_BYTES, &tmX2, fb, kb * BK, 0, pol_x);
+        issued |= 1u << stage;
+        issued_phase = (issued_phase & ~(1u << stage)) | (phase << stage);
+        if (++stage == STAGES) {
+          stage = 0;
+          phase ^= 1u;
         }
-        g += kb1 - kb0;
       }
       for (int s = 0; s < STAGES; ++s)
         if (issued & (1u << s)) wait_drain(full0 + 8 * s, (issued_phase >> s) & 1u);
     }
   } else if (warp == 1) {
     if (lane == 0) {
+      // ------------------------------------------------------------ MMA issuer
       int stage = 0;
       uint32_t phase = 0;
       int it = 0;
@@ -813,7 +722,6 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint32_t acc_phase = (it >> 1) & 1;
         if (!wait_bounded(tempty0 + 8 * acc, acc_phase ^ 1u, abort_flag, status)) break;
         tc_fence_after();
-        const uint32_t d_tmem = tmem_base + acc * BNX;
         for (int kb = kb0; kb < kb1; ++kb) {
           if (!wait_bounded(full0 + 8 * stage, phase, abort_flag, status)) {
             ok = false;
@@ -824,9 +732,15 @@ __global__ void __launch_bounds__(kThreads, 1)
           const uint32_t sx = sw + W_BYTES;
 #pragma unroll
           for (int k = 0; k < BK / 16; ++k) {
-            const uint64_t adesc = make_sdesc(sw + k * 32);
-            tc_mma(d_tmem, adesc, make_sdesc(sx + k * 32), IDESC, (kb > kb0 || k > 0) ? 1u : 0u);
-            tc_mma(d_tmem, adesc, make_sdesc(sx + X_BYTES + k * 32), IDESC, 1u);
+            const uint64_t xh = make_sdesc(sx + k * 32);
+            const uint64_t xl = make_sdesc(sx + X_BYTES + k * 32);
+#pragma unroll
+            for (int h = 0; h < NH; ++h) {
+              const uint32_t d_tmem = tmem_base + (acc * NH + h) * BNX;
+              const uint64_t adesc = make_sdesc(sw + h * W_HALF + k * 32);
+              tc_mma(d_tmem, adesc, xh, IDESC, (kb > kb0 || k > 0) ? 1u : 0u);
+              tc_mma(d_tmem, adesc, xl, IDESC, 1u);
+            }
           }
           tc_commit(empty0 + 8 * stage);
           if (++stage == STAGES) {
@@ -840,6 +754,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       wait_drain(drain_bar, 0);
     }
   } else {
+    // -------------------------------------------------------------- epilogue warps 2..5
     const int q = warp & 3;
     int it = 0;
     for (int g = g_begin; g < g_end; ++it) {
@@ -854,15 +769,18 @@ __global__ void __launch_bounds__(kThreads, 1)
       ok = __shfl_sync(0xffffffffu, ok, 0);
       if (!ok) break;
       tc_fence_after();
-      const int r = q * 32 + lane;
       const int slot = blockIdx.x * p.max_seg + (t - t_first);
-      float* dst = p.ws + (static_cast<size_t>(slot) * 128 + r) * BNX;
-      const uint32_t trow = tmem_base + (static_cast<uint32_t>(q * 32) << 16) + acc * BNX;
+#pragma unroll
+      for (int h = 0; h < NH; ++h) {
+        const int r = h * 128 + q * 32 + lane;
+        float* dst = p.ws + (static_cast<size_t>(slot) * TR + r) * BNX;
+        const uint32_t trow = tmem_base + (static_cast<uint32_t>(q * 32) << 16) + (acc * NH + h) * BNX;
 #pragma unroll 1
-      for (int c = 0; c < BNX; c += 16) {
-        float v[16];
-        ld16f(trow + c, v);
-        store_f32x16(dst + c, v);
+        for (int c = 0; c < BNX; c += 16) {
+          float v[16];
+          ld16f(trow + c, v);
+          store_f32x16(dst + c, v);
+        }
       }
       tc_fence_before();
       __syncwarp();
@@ -931,7 +849,7 @@ int launch_kernel(const Maps& m, const Params& p, int grid, cudaStream_t stream)
     VLA_CUDA_TRY(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem));
     attr_set = true;
   }
-  kern<<<grid, kThreads, smem, stream>>>(m.a, m.a2, m.b, m.b2, p);
+  VLA_CUDA_TRY(launch_pdl(kern, dim3(grid), dim3(kThreads), smem, stream, m.a, m.a2, m.b, m.b2, p));
   note_launch();
   VLA_CUDA_TRY(cudaGetLastError());
   return VLA_OK;
@@ -965,17 +883,17 @@ int launch_reduce(const Src& src, const GemmArgs& a, cudaStream_t stream) {
     case EPI_RESID: {
       float* out = (epi == EPI_F32) ? a.epi.out_f32 : a.epi.resid;
       const int ld = (epi == EPI_F32) ? a.epi.ldo : a.epi.ldr;
-      reduce_f32_kernel<Src><<<blocks_for(static_cast<int64_t>(a.M) * a.N), 256, 0, stream>>>(
-          src, a.M, a.N, out, ld, epi == EPI_RESID);
+      VLA_CUDA_TRY(launch_pdl(reduce_f32_kernel<Src>, dim3(blocks_for(static_cast<int64_t>(a.M) * a.N)),
+                              dim3(256), 0, stream, src, a.M, a.N, out, ld, epi == EPI_RESID ? 1 : 0));
       break;
     }
     case EPI_SWIGLU:
-      reduce_swiglu_kernel<Src><<<blocks_for(static_cast<int64_t>(a.M) * a.N / 2), 256, 0, stream>>>(
-          src, a.M, a.N / 2, a.epi.out_hi, a.epi.out_lo, a.epi.ldo);
+      VLA_CUDA_TRY(launch_pdl(reduce_swiglu_kernel<Src>, dim3(blocks_for(static_cast<int64_t>(a.M) * a.N / 2)),
+                              dim3(256), 0, stream, src, a.M, a.N / 2, a.epi.out_hi, a.epi.out_lo, a.epi.ldo));
       break;
     case EPI_QKV:
-      reduce_qkv_kernel<Src><<<blocks_for(static_cast<int64_t>(a.M) * a.N / 2), 256, 0, stream>>>(
-          src, a.M, a.epi);
+      VLA_CUDA_TRY(launch_pdl(reduce_qkv_kernel<Src>, dim3(blocks_for(static_cast<int64_t>(a.M) * a.N / 2)),
+                              dim3(256), 0, stream, src, a.M, a.epi));
       break;
     default:
       return VLA_ERR_ARG;
@@ -1010,21 +928,21 @@ struct GemvPlan {
 GemvPlan gemv_plan(int M, int N, int K, int num_sms) {
   GemvPlan g{};
   g.bnx = M <= 16 ? 16 : M <= 32 ? 32 : M <= 64 ? 64 : 128;
-  g.tiles = (N + 127) / 128;
+  g.tiles = (N + 255) / 256;
   g.kbt = (K + BK - 1) / BK;
   const int total = g.tiles * g.kbt;
   int grid = total < num_sms ? total : num_sms;
   g.per_cta = (total + grid - 1) / grid;
   g.grid = (total + g.per_cta - 1) / g.per_cta;
   g.max_seg = (g.per_cta - 1) / g.kbt + 2;
-  g.ws_bytes = static_cast<size_t>(g.grid) * g.max_seg * 128 * g.bnx * sizeof(float);
+  g.ws_bytes = static_cast<size_t>(g.grid) * g.max_seg * 256 * g.bnx * sizeof(float);
   return g;
 }
 
 template <int BNX>
 int launch_gemv(const CUtensorMap& w, const CUtensorMap& x, const CUtensorMap& x2,
                 const GemvParams& p, int grid, cudaStream_t stream) {
-  constexpr int STAGE = 128 * BK * 2 + 2 * BNX * BK * 2;
+  constexpr int STAGE = 256 * BK * 2 + 2 * BNX * BK * 2;
   constexpr int STAGES = (196608 / STAGE) < 8 ? (196608 / STAGE) : 8;
   constexpr int smem = STAGES * STAGE + 1024 + 256;
   static bool attr_set = false;
@@ -1033,7 +951,7 @@ int launch_gemv(const CUtensorMap& w, const CUtensorMap& x, const CUtensorMap& x
     VLA_CUDA_TRY(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem));
     attr_set = true;
   }
-  kern<<<grid, kThreads, smem, stream>>>(w, x, x2, p);
+  VLA_CUDA_TRY(launch_pdl(kern, dim3(grid), dim3(kThreads), smem, stream, w, x, x2, p));
   note_launch();
   VLA_CUDA_TRY(cudaGetLastError());
   return VLA_OK;
@@ -1141,11 +1059,11 @@ int gemv_launch(const GemmArgs& a, cudaStream_t stream, int num_sms, GemmCost* c
       (reinterpret_cast<uintptr_t>(a.A_lo) & 15))
     return VLA_ERR_ARG;
   if (a.epi.kind == EPI_SWIGLU && (a.N & 1)) return VLA_ERR_ARG;
-  if (a.epi.kind == EPI_QKV && (a.N != 3 * a.epi.d || 128 % a.epi.hd)) return VLA_ERR_ARG;
+  if (a.epi.kind == EPI_QKV && a.N != 3 * a.epi.d) return VLA_ERR_ARG;
   const GemvPlan pl = gemv_plan(a.M, a.N, a.K, num_sms);
   if (!a.workspace || a.workspace_bytes < pl.ws_bytes) return VLA_ERR_ARG;
   CUtensorMap mw, mx, mx2;
-  if (!make_map(&mw, a.B, a.N, a.K, a.ldb, 128) || !make_map(&mx, a.A, a.M, a.K, a.lda, pl.bnx) ||
+  if (!make_map(&mw, a.B, a.N, a.K, a.ldb, 256) || !make_map(&mx, a.A, a.M, a.K, a.lda, pl.bnx) ||
       !make_map(&mx2, a.A_lo, a.M, a.K, a.lda, pl.bnx))
     return cuda_fail(cudaErrorInvalidValue, "tensor maps (decode GEMM)");
   GemvParams p{};

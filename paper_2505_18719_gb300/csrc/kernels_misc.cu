@@ -17,6 +17,8 @@ __global__ void __launch_bounds__(256) assemble_kernel(const RowInfo* __restrict
                                                        const bf16* __restrict__ embed, int d,
                                                        int vocab, float* __restrict__ h,
                                                        uint32_t* status) {
+  pdl_launch_dependents();
+  pdl_wait();
   const RowInfo ri = rows[blockIdx.x];
   const bf16* src;
   if (ri.kind == ROW_VISUAL) {
@@ -43,6 +45,8 @@ __global__ void __launch_bounds__(256) rmsnorm_kernel(const float* __restrict__ 
                                                       const bf16* __restrict__ w, int d,
                                                       float eps, bf16* __restrict__ y_hi,
                                                       bf16* __restrict__ y_lo) {
+  pdl_launch_dependents();
+  pdl_wait();
   __shared__ float red[8];
   const float* row = h + static_cast<size_t>(blockIdx.x) * d;
   float ss = 0.f;
@@ -71,6 +75,8 @@ __global__ void __launch_bounds__(256) rmsnorm_kernel(const float* __restrict__ 
 
 __global__ void gather_rows_kernel(const float* __restrict__ src, const int* __restrict__ idx,
                                    int d, float* __restrict__ dst) {
+  pdl_launch_dependents();
+  pdl_wait();
   const float* s = src + static_cast<size_t>(idx[blockIdx.x]) * d;
   float* o = dst + static_cast<size_t>(blockIdx.x) * d;
   for (int c = threadIdx.x * 4; c < d; c += blockDim.x * 4)
@@ -79,6 +85,8 @@ __global__ void gather_rows_kernel(const float* __restrict__ src, const int* __r
 
 __global__ void scatter_rows_kernel(const float* __restrict__ src, const int* __restrict__ sidx,
                                     const int* __restrict__ didx, int d, float* __restrict__ dst) {
+  pdl_launch_dependents();
+  pdl_wait();
   const float* s = src + static_cast<size_t>(sidx[blockIdx.x]) * d;
   float* o = dst + static_cast<size_t>(didx[blockIdx.x]) * d;
   for (int c = threadIdx.x * 4; c < d; c += blockDim.x * 4)
@@ -91,7 +99,8 @@ int assemble_launch(const RowInfo* rows, int n_rows, const bf16* visual, const i
                     const int* tokens, const bf16* embed, int d, int vocab, float* h,
                     uint32_t* status, cudaStream_t s) {
   if (n_rows <= 0) return VLA_OK;
-  assemble_kernel<<<n_rows, 256, 0, s>>>(rows, visual, ids, tokens, embed, d, vocab, h, status);
+  VLA_CUDA_TRY(launch_pdl(assemble_kernel, dim3(n_rows), dim3(256), 0, s, rows, visual, ids, tokens,
+                          embed, d, vocab, h, status));
   note_launch();
   VLA_CUDA_TRY(cudaGetLastError());
   return VLA_OK;
@@ -100,7 +109,7 @@ int assemble_launch(const RowInfo* rows, int n_rows, const bf16* visual, const i
 int rmsnorm_launch(const float* h, const bf16* w, int M, int d, float eps, bf16* y_hi,
                    bf16* y_lo, cudaStream_t s) {
   if (M <= 0) return VLA_OK;
-  rmsnorm_kernel<<<M, 256, 0, s>>>(h, w, d, eps, y_hi, y_lo);
+  VLA_CUDA_TRY(launch_pdl(rmsnorm_kernel, dim3(M), dim3(256), 0, s, h, w, d, eps, y_hi, y_lo));
   note_launch();
   VLA_CUDA_TRY(cudaGetLastError());
   return VLA_OK;
@@ -108,7 +117,7 @@ int rmsnorm_launch(const float* h, const bf16* w, int M, int d, float eps, bf16*
 
 int gather_rows_launch(const float* src, const int* idx, int n, int d, float* dst, cudaStream_t s) {
   if (n <= 0) return VLA_OK;
-  gather_rows_kernel<<<n, 256, 0, s>>>(src, idx, d, dst);
+  VLA_CUDA_TRY(launch_pdl(gather_rows_kernel, dim3(n), dim3(256), 0, s, src, idx, d, dst));
   note_launch();
   VLA_CUDA_TRY(cudaGetLastError());
   return VLA_OK;
@@ -120,7 +129,7 @@ namespace vla {
 int scatter_rows_launch(const float* src, const int* sidx, const int* didx, int n, int d, float* dst,
                         cudaStream_t s) {
   if (n <= 0) return VLA_OK;
-  scatter_rows_kernel<<<n, 256, 0, s>>>(src, sidx, didx, d, dst);
+  VLA_CUDA_TRY(launch_pdl(scatter_rows_kernel, dim3(n), dim3(256), 0, s, src, sidx, didx, d, dst));
   note_launch();
   VLA_CUDA_TRY(cudaGetLastError());
   return VLA_OK;

@@ -89,6 +89,8 @@ def load(path: str = LIB_PATH):
         "vla_op_gemm_bf16_noalloc": (i32, [vp, vp, i32, vp, i32, vp, i32, i32, i32, i32, i32, i32, vp]),
         "vla_op_action_head": (i32, [vp, i32, i32, i32, vp, vp, f32, vp, f32, vp, vp, vp, vp, vp, vp, vp]),
         "vla_op_num_sms": (i32, []),
+        "vla_op_attn_decode": (i32, [vp, vp, i32, i32, i32, i32, vp, vp, i32, i32, i32, vp, vp, vp, ctypes.c_size_t, vp]),
+        "vla_op_attn_decode_workspace_bytes": (ctypes.c_size_t, [i32, i32, i32, i32, i32]),
     }
     for name, (res, args) in sig.items():
         f = getattr(lib, name)
@@ -207,6 +209,16 @@ def vla_op_action_head(h_ptr, ldh, B, d, final_norm_ptr, head_rows_ptr, eps, uni
 
 def vla_op_num_sms() -> int:
     return load().vla_op_num_sms()
+
+
+def vla_op_attn_decode(q_ptr, kv_ptr, max_env, H, hd, cap, env_ptr, pos_ptr, B, max_ctx, out_hi_ptr, out_lo_ptr,
+                       ws_ptr, ws_bytes, stream=0, max_keys_per_cta=0) -> int:
+    return load().vla_op_attn_decode(q_ptr, kv_ptr, max_env, H, hd, cap, env_ptr, pos_ptr, B, max_ctx,
+                                     max_keys_per_cta, out_hi_ptr, out_lo_ptr, ws_ptr, ws_bytes, stream or None)
+
+
+def vla_op_attn_decode_workspace_bytes(B, H, hd, max_ctx, max_keys_per_cta=0) -> int:
+    return load().vla_op_attn_decode_workspace_bytes(B, H, hd, max_ctx, max_keys_per_cta)
 
 
 # ---------------------------------------------------------------------------- convenience

@@ -129,3 +129,34 @@ def test_action_head_matches_fp64(T, forced):
             assert int(bins[b].item()) == k
             assert act[b].item() == O.bin_centre(k)
     assert checked >= B // 2
+
+
+@pytest.mark.parametrize("B,H,hd,cap,ctx", [(3, 2, 64, 64, [1, 7, 64]), (5, 4, 128, 1152, [1, 129, 300, 1116, 161]),
+                                          (64, 32, 128, 320, None)])
+def test_decode_attention_matches_fp64(B, H, hd, cap, ctx):
+    """Flash-decoding over the fp16 cache vs brute-force softmax attention in fp64."""
+    max_env = B + 1
+    kv = I.normal_bf16((max_env, 2, H, cap, hd), 77, B, 1.0).float().half()   # fp16 cache values
+    q = I.normal_bf16((B, H, hd), 77, 100 + B, 1.0).float()
+    if ctx is None:
+        ctx = I.randint_i32((B,), 77, 200, 272, 310).tolist()
+    env = torch.tensor([(b * 7 + 1) % max_env for b in range(B)], dtype=torch.int32)
+    pos = torch.tensor([c - 1 for c in ctx], dtype=torch.int32)
+    max_ctx = max(ctx)
+    nbytes = V.vla_op_attn_decode_workspace_bytes(B, H, hd, max_ctx, 0)
+    ws = torch.empty(nbytes // 4 + 64, dtype=torch.float32, device="cuda")
+    oh = torch.empty(B, H * hd, dtype=torch.bfloat16, device="cuda")
+    ol = torch.empty(B, H * hd, dtype=torch.bfloat16, device="cuda")
+    kvd, qd, envd, posd = kv.cuda(), q.cuda(), env.cuda(), pos.cuda()
+    rc = V.vla_op_attn_decode(qd.data_ptr(), kvd.data_ptr(), max_env, H, hd, cap, envd.data_ptr(), posd.data_ptr(),
+                              B, max_ctx, oh.data_ptr(), ol.data_ptr(), ws.data_ptr(), nbytes, 0)
+    assert rc == 0, V.vla_last_error()
+    torch.cuda.synchronize()
+    got = (oh.double() + ol.double()).cpu().reshape(B, H, hd)
+    kv64 = kv.double()
+    for b in range(B):
+        e, n = int(env[b]), ctx[b]
+        k, v = kv64[e, 0, :, :n], kv64[e, 1, :, :n]                  # [H, n, hd]
+        sc = torch.einsum("hd,hnd->hn", q[b].double(), k) / math.sqrt(hd)
+        o = torch.einsum("hn,hnd->hd", torch.softmax(sc, -1), v)
+        assert (got[b] - o).abs().max().item() < 1e-4, b
