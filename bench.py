@@ -171,6 +171,14 @@ CASES = {
     "gemv_decode_gate_up": (64, 22016, 4096, 0, 0, True),
     "gemv_decode_down": (64, 4096, 11008, 0, 0, True),
     "attn_decode": None,                                       # see run_attn_case
+    # the same prefill shapes on CTA pairs (2-SM MMAs, 256 x 256 tiles)
+    "pair_prefill_qkv": (4608, 12288, 4096, 256, 1, True),
+    "pair_prefill_down": (4608, 4096, 11008, 256, 1, True),
+    "pair_prefill_gate_up_18k": (18432, 22016, 4096, 256, 1, True),
+    "gemm_prefill_gate_up_18k": (18432, 22016, 4096, 256, 1, True),
+    # decode GEMM at 2x / 4x the weight bytes of the q|k|v step (fixed vs per-byte cost)
+    "gemv_decode_k8192": (64, 12288, 8192, 0, 0, True),
+    "gemv_decode_k16384": (64, 12288, 16384, 0, 0, True),
 }
 
 
@@ -181,10 +189,12 @@ def run_attn_case(args):
     __graft_entry__.build()
     from paper_2505_18719_gb300 import inputs as I
     from paper_2505_18719_gb300 import vla as V
-    B, H, hd, cap = 64, 32, 128, 320
+    B, H, hd = 64, 32, 128
+    scale = max(1, args.attn_ctx_scale)
+    cap = 320 * scale
     kv = I.normal_bf16((B, 2, H, cap, hd), 5, 1, 1.0).cuda().half()
     q = I.normal_bf16((B, H, hd), 5, 2, 1.0).cuda().float()
-    ctx = I.randint_i32((B,), 5, 3, 273, 311)
+    ctx = I.randint_i32((B,), 5, 3, 273, 311) * scale
     env = torch.arange(B, dtype=torch.int32, device="cuda")
     pos = (ctx - 1).cuda()
     max_ctx = int(ctx.max())
@@ -234,7 +244,14 @@ def run_case(args):
     W = I.normal_bf16((N, K), 1, 3, 0.02).cuda()
     C = torch.empty(M, N, dtype=torch.float32, device="cuda")
     stream = torch.cuda.current_stream()
-    if args.case.startswith("gemv"):
+    if args.case.startswith("pair"):
+        ws = None
+
+        def launch():
+            rc = V.vla_op_gemm_pair_bf16(A.data_ptr(), A_lo.data_ptr() if split_a else 0, K, W.data_ptr(), K,
+                                         C.data_ptr(), N, M, N, K, stream.cuda_stream)
+            assert rc == 0, V.vla_last_error()
+    elif args.case.startswith("gemv"):
         nbytes = V.vla_op_gemm_decode_workspace_bytes(M, N, K)
         ws = torch.empty(max(1, nbytes // 4), dtype=torch.float32, device="cuda")
 
@@ -280,6 +297,7 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--case", choices=sorted(CASES), help="time one kernel shape instead of the hot path")
     ap.add_argument("--attn-keys", type=int, default=0, help="attn_decode case: max keys per CTA (0 = default)")
+    ap.add_argument("--attn-ctx-scale", type=int, default=1, help="attn_decode case: context length multiplier")
     args = ap.parse_args()
     if args.impl == "reference":
         return run_reference(args)

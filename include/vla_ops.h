@@ -26,6 +26,13 @@ int vla_op_gemm_bf16(const void* A, const void* A_lo, int lda, const void* W, in
                      int ldc, int M, int N, int K, int block_n, int splits, float* workspace,
                      void* cuda_stream);
 
+/* vla_op_gemm_bf16 (C f32 = (A + A_lo) · W^T, A_lo may be NULL) on CTA pairs: each pair of
+ * SMs computes 256 x 256 output tiles with 2-SM tcgen05 MMAs (cta_group::2), each SM loading
+ * half of the A and B tiles.  Same arguments and results as vla_op_gemm_bf16 without
+ * split-K; the prefill projections run this way. */
+int vla_op_gemm_pair_bf16(const void* A, const void* A_lo, int lda, const void* W, int ldw,
+                          float* C, int ldc, int M, int N, int K, void* cuda_stream);
+
 /* The decode-step projection (§3.1 projections at decode batch sizes, Algorithm 1 rollout):
  * C[M, N] (f32) = (A + A_lo)[M, K] · W[N, K]^T for M <= 128 activation rows, bf16 operands,
  * A_lo required.  Streams W from HBM once: swap-AB tcgen05 MMAs (W rows are the MMA's M),

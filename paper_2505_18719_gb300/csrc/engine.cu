@@ -218,6 +218,13 @@ int run_gemm(vla_handle* h, int cls, const bf16* A, size_t a_plane, int lda, con
   if (!stream_k && gemm_workspace_bytes(g) > h->ws_bytes) {
     g.splits = 1;
   }
+  // Large tile GEMMs run on CTA pairs (256 x 256 tiles, 2-SM MMAs) when there are enough
+  // pair tiles to cover half the SMs.
+  if (!stream_k && g.splits == 1 && g.block_n == 256) {
+    const int64_t pair_tiles = static_cast<int64_t>((M + 255) / 256) *
+                               (epi.kind == EPI_SWIGLU ? (N / 2 + 127) / 128 : (N + 255) / 256);
+    g.pair = pair_tiles >= h->num_sms / 2;
+  }
   if (h->ev_used.size() > 8192) prof_harvest(h);
   int ev = prof_begin(h, cls);
   GemmCost cost{0, 0};
@@ -785,6 +792,30 @@ int vla_op_gemm_bf16(const void* A, const void* A_lo, int lda, const void* W, in
     return set_err(nullptr, VLA_ERR_ARG, "vla_op_gemm_bf16: splits > 1 needs a workspace");
   const int rc = gemm_launch(g, static_cast<cudaStream_t>(cuda_stream), query_num_sms(), nullptr);
   if (rc != VLA_OK && rc != VLA_ERR_CUDA) return set_err(nullptr, rc, "vla_op_gemm_bf16: unsupported arguments");
+  return rc;
+}
+
+int vla_op_gemm_pair_bf16(const void* A, const void* A_lo, int lda, const void* W, int ldw, float* C, int ldc,
+                          int M, int N, int K, void* cuda_stream) {
+  if (!A || !W || !C || M < 1 || N < 1 || K < 1 || ldc < N)
+    return set_err(nullptr, VLA_ERR_ARG, "vla_op_gemm_pair_bf16: bad argument");
+  GemmArgs g;
+  g.A = static_cast<const bf16*>(A);
+  g.A_lo = static_cast<const bf16*>(A_lo);
+  g.lda = lda;
+  g.B = static_cast<const bf16*>(W);
+  g.ldb = ldw;
+  g.M = M;
+  g.N = N;
+  g.K = K;
+  g.block_n = 256;
+  g.splits = 1;
+  g.pair = true;
+  g.epi.kind = EPI_F32;
+  g.epi.out_f32 = C;
+  g.epi.ldo = ldc;
+  const int rc = gemm_launch(g, static_cast<cudaStream_t>(cuda_stream), query_num_sms(), nullptr);
+  if (rc != VLA_OK && rc != VLA_ERR_CUDA) return set_err(nullptr, rc, "vla_op_gemm_pair_bf16: unsupported arguments");
   return rc;
 }
 

@@ -40,6 +40,7 @@ struct GemmArgs {
   int M = 0, N = 0, K = 0;
   int block_n = 256;        // 128 or 256
   int splits = 1;           // split-K factor (> 1 needs workspace)
+  bool pair = false;        // 2-SM tiles (256 x 256 per CTA pair); needs block_n 256, splits 1
   float* workspace = nullptr;
   size_t workspace_bytes = 0;
   EpiArgs epi;

@@ -444,6 +444,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   }
 
+  // Lanes 1..31 of the producer and MMA warps got here long before their lane 0: reconverge
+  // each warp first, since the CTA barrier counts whole converged warps.
+  __syncwarp();
   tc_fence_before();
   __syncthreads();
   if (warp == 1) {
@@ -454,12 +457,211 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 }
 
+// ----------------------------------------------------------------------------- 2-SM GEMM
+// The same GEMM on CTA pairs (clusters of 2 on one TPC): a pair computes a 256 x 256 output
+// tile with tcgen05.mma.cta_group::2 (M = 256, N = 256, K = 16).  Each CTA loads only its half
+// of A (128 rows, hi and lo) and its half of B (128 rows of W; SwiGLU: the even CTA the gate
+// rows, the odd CTA the matching up rows) into its own shared memory; the MMA of the pair reads
+// both halves, so each SM fills 48 KB of operands per 64-wide k-block instead of 64 KB, for the
+// same MMA work.  Each CTA's TMEM holds the pair's accumulator rows of that CTA (two 256-column
+// accumulators), and each CTA runs the same epilogue on its rows.
+//  * even CTA (leader): its producer posts the expected bytes of both CTAs on its full
+//    barrier; its MMA thread issues all MMAs and commits stage releases and accumulator
+//    readiness to the barriers of both CTAs (multicast commit);
+//  * odd CTA: its producer's TMA loads complete on the leader's full barrier;
+//  * both epilogues release an accumulator on the leader's tempty barrier (8 warp arrivals).
+// All waits are bounded; a cluster barrier closes the kernel before TMEM is freed, so no CTA
+// leaves while its partner's MMAs may still read its shared memory.
+template <int STAGES, int EPI, bool SPLIT>
+__global__ void __launch_bounds__(kThreads, 1)
+    gemm_tc2_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmA2,
+                    const __grid_constant__ CUtensorMap tmB, const __grid_constant__ CUtensorMap tmB2,
+                    const Params p) {
+  constexpr int BN = 256;
+  constexpr int A_BYTES = BM * BK * 2;            // 128 rows of A (one half of the pair's 256)
+  constexpr int A_TOTAL = SPLIT ? 2 * A_BYTES : A_BYTES;
+  constexpr int B_BYTES = (BN / 2) * BK * 2;      // this CTA's 128 rows of B
+  constexpr int STAGE_BYTES = A_TOTAL + B_BYTES;
+  constexpr uint32_t TMEM_COLS = 2 * BN;
+  constexpr uint32_t IDESC = (1u << 4) | (1u << 7) | (1u << 10) | (static_cast<uint32_t>(BN >> 3) << 17) |
+                             (static_cast<uint32_t>(256 >> 4) << 24);
+  constexpr bool SWIGLU = (EPI == EPI_SWIGLU);
+
+  pdl_launch_dependents();
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~static_cast<uintptr_t>(1023));
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + STAGES * STAGE_BYTES);
+  const uint32_t full0 = smem_u32(bars);
+  const uint32_t empty0 = full0 + 8 * STAGES;
+  const uint32_t tfull0 = empty0 + 8 * STAGES;
+  const uint32_t tempty0 = tfull0 + 16;
+  const uint32_t drain_bar = tempty0 + 16;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * STAGES + 5);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const uint32_t rank = cluster_ctarank();
+  const uint32_t leader = rank & ~1u;
+  const bool is_leader = rank == leader;
+  const uint16_t pair_mask = static_cast<uint16_t>(3u << leader);
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < STAGES; ++s) {
+      mbar_init(full0 + 8 * s, 1);
+      mbar_init(empty0 + 8 * s, 1);
+    }
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(tfull0 + 8 * a, 1);
+      mbar_init(tempty0 + 8 * a, 8);
+    }
+    mbar_init(drain_bar, 1);
+    *abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmA)) : "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmB)) : "memory");
+  }
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                     smem_u32(tmem_slot)),
+                 "r"(TMEM_COLS)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
+  }
+  tc_fence_before();
+  cluster_sync();  // both CTAs' barriers are initialised before either touches the other's
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+  const int units = p.tiles_m * p.tiles_n;
+  const int n_pairs = gridDim.x >> 1;
+  const int pair = blockIdx.x >> 1;
+  uint32_t* status = p.epi.status;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ------------------------------------------------------------ TMA producer (both CTAs)
+      pdl_wait();
+      int stage = 0;
+      uint32_t phase = 0;
+      uint32_t issued = 0, issued_phase = 0;
+      bool ok = true;
+      for (int u = pair; u < units && ok; u += n_pairs) {
+        int m_blk, n_blk, split;
+        unit_coords(p, u, m_blk, n_blk, split);
+        const int row_a = m_blk * 256 + static_cast<int>(rank - leader) * 128;
+        for (int kb = 0; kb < p.kb_total; ++kb) {
+          if (!wait_bounded(empty0 + 8 * stage, phase ^ 1u, abort_flag, status)) {
+            ok = false;
+            break;
+          }
+          const uint32_t fb = mapa_shared(full0 + 8 * stage, leader);
+          const uint32_t sa = smem_u32(smem + stage * STAGE_BYTES);
+          const uint32_t sb = sa + A_TOTAL;
+          if (is_leader) mbar_arrive_expect_tx(full0 + 8 * stage, 2 * STAGE_BYTES);
+          tma_load_2d_pair(sa, &tmA, fb, kb * BK, row_a);
+          if (SPLIT) tma_load_2d_pair(sa + A_BYTES, &tmA2, fb, kb * BK, row_a);
+          if (SWIGLU)
+            tma_load_2d_pair(sb, rank == leader ? &tmB : &tmB2, fb, kb * BK, n_blk * (BN / 2));
+          else
+            tma_load_2d_pair(sb, &tmB, fb, kb * BK, n_blk * BN + static_cast<int>(rank - leader) * (BN / 2));
+          issued |= 1u << stage;
+          issued_phase = (issued_phase & ~(1u << stage)) | (phase << stage);
+          if (++stage == STAGES) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+      }
+      // Drain (leader only: the pair's loads complete on the leader's barriers).
+      if (is_leader)
+        for (int s = 0; s < STAGES; ++s)
+          if (issued & (1u << s)) wait_drain(full0 + 8 * s, (issued_phase >> s) & 1u);
+    }
+  } else if (warp == 1) {
+    if (lane == 0 && is_leader) {
+      // ------------------------------------------------------------ MMA issuer (leader)
+      int stage = 0;
+      uint32_t phase = 0;
+      int it = 0;
+      bool ok = true;
+      for (int u = pair; u < units && ok; u += n_pairs, ++it) {
+        const int acc = it & 1;
+        const uint32_t acc_phase = (it >> 1) & 1;
+        if (!wait_bounded(tempty0 + 8 * acc, acc_phase ^ 1u, abort_flag, status)) break;
+        tc_fence_after();
+        const uint32_t d_tmem = tmem_base + acc * BN;
+        for (int kb = 0; kb < p.kb_total; ++kb) {
+          if (!wait_bounded(full0 + 8 * stage, phase, abort_flag, status)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t sa = smem_u32(smem + stage * STAGE_BYTES);
+          const uint32_t sb = sa + A_TOTAL;
+#pragma unroll
+          for (int k = 0; k < BK / 16; ++k) {
+            const uint64_t bdesc = make_sdesc(sb + k * 32);
+            tc_mma_pair(d_tmem, make_sdesc(sa + k * 32), bdesc, IDESC, (kb > 0 || k > 0) ? 1u : 0u);
+            if (SPLIT) tc_mma_pair(d_tmem, make_sdesc(sa + A_BYTES + k * 32), bdesc, IDESC, 1u);
+          }
+          tc_commit_pair(empty0 + 8 * stage, pair_mask);
+          if (++stage == STAGES) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+        if (ok) tc_commit_pair(tfull0 + 8 * acc, pair_mask);
+      }
+      tc_commit_pair(drain_bar, static_cast<uint16_t>(1u << leader));
+      wait_drain(drain_bar, 0);
+    }
+  } else {
+    // -------------------------------------------------------------- epilogue warps 2..5
+    const int q = warp & 3;
+    const uint32_t tempty_leader = mapa_shared(tempty0, leader);
+    int it = 0;
+    for (int u = pair; u < units; u += n_pairs, ++it) {
+      int m_blk, n_blk, split;
+      unit_coords(p, u, m_blk, n_blk, split);
+      const int acc = it & 1;
+      const uint32_t acc_phase = (it >> 1) & 1;
+      int ok = 1;
+      if (lane == 0) ok = wait_bounded(tfull0 + 8 * acc, acc_phase, abort_flag, status) ? 1 : 0;
+      ok = __shfl_sync(0xffffffffu, ok, 0);
+      if (!ok) break;
+      tc_fence_after();
+      const int m = m_blk * 256 + static_cast<int>(rank - leader) * 128 + q * 32 + lane;
+      const uint32_t trow = tmem_base + (static_cast<uint32_t>(q * 32) << 16) + acc * BN;
+      if (EPI == EPI_SWIGLU)
+        epilogue_swiglu<BN>(p, trow, m, n_blk * (BN / 2));
+      else if (EPI == EPI_QKV)
+        epilogue_qkv<BN>(p, trow, m, n_blk * BN);
+      else
+        epilogue_plain<BN, EPI>(p, trow, m, n_blk * BN, 0);
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive_cluster(tempty_leader + 8 * acc);
+    }
+  }
+
+  __syncwarp();  // reconverge the role warps before the CTA and cluster barriers
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync();  // the partner's MMAs have finished reading this CTA's shared memory
+  if (warp == 1) {
+    tc_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(tmem_base), "r"(TMEM_COLS)
+                 : "memory");
+  }
+}
+
 // ----------------------------------------------------------------------------- partial sums
 // Partials of a split GEMM are summed in a fixed order, so results do not depend on the
 // launch.  Two layouts:
 //  SplitSrc   split-K of the tile GEMM: ws[s][M][N], s = 0 .. S-1.
-//  StreamSrc  stream-K of the weight-streaming GEMM: ws[slot][256][BNX] (output row n of
-//             tile t = n / 256 at row n % 256, batch row m at column m); the CTAs whose
+//  StreamSrc  stream-K of the weight-streaming GEMM: ws[slot][BNX][256] (output row n of
+//             tile t = n / 256 at column n % 256, batch row m at row m); the CTAs whose
 //             iteration ranges cover tile t are c = t*KB / P .. ((t+1)*KB - 1) / P, and CTA c
 //             keeps tile t in slot c * max_seg + t - (c * P) / KB.
 struct SplitSrc {
@@ -475,14 +677,14 @@ struct SplitSrc {
 struct StreamSrc {
   const float* ws;
   int BNX, KB, P, max_seg;
-  static constexpr bool kBatchFastest = true;
+  static constexpr bool kBatchFastest = false;
   __device__ __forceinline__ float operator()(int m, int n) const {
     const int t = n >> 8, r = n & 255;
     const int c0 = (t * KB) / P, c1 = (t * KB + KB - 1) / P;
     float a = 0.f;
     for (int c = c0; c <= c1; ++c) {
       const int slot = c * max_seg + t - (c * P) / KB;
-      a += ws[(static_cast<size_t>(slot) * 256 + r) * BNX + m];
+      a += ws[(static_cast<size_t>(slot) * BNX + m) * 256 + r];
     }
     return a;
   }
@@ -770,16 +972,19 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (!ok) break;
       tc_fence_after();
       const int slot = blockIdx.x * p.max_seg + (t - t_first);
+      // partial layout [slot][batch column][tile row]: for each batch column the 32 lanes of a
+      // warp store 32 consecutive rows (coalesced), and the reduction reads rows contiguously
 #pragma unroll
       for (int h = 0; h < NH; ++h) {
         const int r = h * 128 + q * 32 + lane;
-        float* dst = p.ws + (static_cast<size_t>(slot) * TR + r) * BNX;
+        float* dst = p.ws + static_cast<size_t>(slot) * BNX * TR + r;
         const uint32_t trow = tmem_base + (static_cast<uint32_t>(q * 32) << 16) + (acc * NH + h) * BNX;
 #pragma unroll 1
         for (int c = 0; c < BNX; c += 16) {
           float v[16];
           ld16f(trow + c, v);
-          store_f32x16(dst + c, v);
+#pragma unroll
+          for (int i = 0; i < 16; ++i) dst[static_cast<size_t>(c + i) * TR] = v[i];
         }
       }
       tc_fence_before();
@@ -788,6 +993,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   }
 
+  // Lanes 1..31 of the producer and MMA warps got here long before their lane 0: reconverge
+  // each warp first, since the CTA barrier counts whole converged warps.
+  __syncwarp();
   tc_fence_before();
   __syncthreads();
   if (warp == 1) {
@@ -853,6 +1061,48 @@ int launch_kernel(const Maps& m, const Params& p, int grid, cudaStream_t stream)
   note_launch();
   VLA_CUDA_TRY(cudaGetLastError());
   return VLA_OK;
+}
+
+template <int EPI, bool SPLIT>
+int launch_pair_kernel(const Maps& m, const Params& p, int grid, cudaStream_t stream) {
+  constexpr int STAGE = (SPLIT ? 2 : 1) * BM * BK * 2 + 128 * BK * 2;
+  constexpr int STAGES = (196608 / STAGE) < 8 ? (196608 / STAGE) : 8;
+  constexpr int smem = STAGES * STAGE + 1024 + 256;
+  static bool attr_set = false;
+  auto kern = gemm_tc2_kernel<STAGES, EPI, SPLIT>;
+  if (!attr_set) {
+    VLA_CUDA_TRY(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem));
+    attr_set = true;
+  }
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(grid);
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 2;
+  VLA_CUDA_TRY(cudaLaunchKernelEx(&cfg, kern, m.a, m.a2, m.b, m.b2, p));
+  note_launch();
+  VLA_CUDA_TRY(cudaGetLastError());
+  return VLA_OK;
+}
+
+template <bool SPLIT>
+int dispatch_pair(int epi, const Maps& m, const Params& p, int grid, cudaStream_t s) {
+  switch (epi) {
+    case EPI_F32: return launch_pair_kernel<EPI_F32, SPLIT>(m, p, grid, s);
+    case EPI_RESID: return launch_pair_kernel<EPI_RESID, SPLIT>(m, p, grid, s);
+    case EPI_SWIGLU: return launch_pair_kernel<EPI_SWIGLU, SPLIT>(m, p, grid, s);
+    case EPI_QKV: return launch_pair_kernel<EPI_QKV, SPLIT>(m, p, grid, s);
+  }
+  return VLA_ERR_ARG;
 }
 
 template <int BN, bool SPLIT>
@@ -988,12 +1238,13 @@ int gemm_launch(const GemmArgs& a, cudaStream_t stream, int num_sms, GemmCost* c
   if (epi == EPI_QKV && (a.epi.d % BN || BN % a.epi.hd || a.N != 3 * a.epi.d)) return VLA_ERR_ARG;
 
   const int splits = gemm_effective_splits(a.K, a.splits);
+  if (a.pair && (BN != 256 || splits != 1)) return VLA_ERR_ARG;
   const int kbt = (a.K + BK - 1) / BK;
   Params p{};
   p.M = a.M;
   p.N = a.N;
   p.K = a.K;
-  p.tiles_m = (a.M + BM - 1) / BM;
+  p.tiles_m = a.pair ? (a.M + 255) / 256 : (a.M + BM - 1) / BM;
   p.splits = splits;
   p.kb_total = kbt;
   p.kb_per_split = (kbt + splits - 1) / splits;
@@ -1024,12 +1275,22 @@ int gemm_launch(const GemmArgs& a, cudaStream_t stream, int num_sms, GemmCost* c
       return cuda_fail(cudaErrorInvalidValue, "tensor map B (gate/up)");
   } else {
     p.tiles_n = (a.N + BN - 1) / BN;
-    if (!make_map(&mb, a.B, a.N, a.K, a.ldb, BN)) return cuda_fail(cudaErrorInvalidValue, "tensor map B");
+    // a pair's CTAs each load half of the 256-row B tile
+    if (!make_map(&mb, a.B, a.N, a.K, a.ldb, a.pair ? BN / 2 : BN))
+      return cuda_fail(cudaErrorInvalidValue, "tensor map B");
     mb2 = mb;
   }
   const int64_t units = static_cast<int64_t>(p.tiles_m) * p.tiles_n * p.splits;
-  const int grid = static_cast<int>(units < num_sms ? units : num_sms);
   int rc;
+  if (a.pair) {
+    const int pairs = static_cast<int>(units < num_sms / 2 ? units : num_sms / 2);
+    rc = split ? dispatch_pair<true>(epi, maps, p, 2 * pairs, stream)
+               : dispatch_pair<false>(epi, maps, p, 2 * pairs, stream);
+    if (rc != VLA_OK) return rc;
+    if (cost) *cost = gemm_cost(a);
+    return VLA_OK;
+  }
+  const int grid = static_cast<int>(units < num_sms ? units : num_sms);
   if (split)
     rc = (BN == 256) ? dispatch_epi<256, true>(run_epi, maps, p, grid, stream)
                      : dispatch_epi<128, true>(run_epi, maps, p, grid, stream);

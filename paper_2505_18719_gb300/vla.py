@@ -84,6 +84,7 @@ def load(path: str = LIB_PATH):
         "vla_profile_read": (i32, [vp, vp, vp, vp, vp]),
         "vla_launch_count": (i64, [vp]),
         "vla_op_gemm_bf16": (i32, [vp, vp, i32, vp, i32, vp, i32, i32, i32, i32, i32, i32, vp, vp]),
+        "vla_op_gemm_pair_bf16": (i32, [vp, vp, i32, vp, i32, vp, i32, i32, i32, i32, vp]),
         "vla_op_gemm_decode_bf16": (i32, [vp, vp, i32, vp, i32, vp, i32, i32, i32, i32, vp, ctypes.c_size_t, vp]),
         "vla_op_gemm_decode_workspace_bytes": (ctypes.c_size_t, [i32, i32, i32]),
         "vla_op_gemm_bf16_noalloc": (i32, [vp, vp, i32, vp, i32, vp, i32, i32, i32, i32, i32, i32, vp]),
@@ -179,6 +180,11 @@ def vla_op_gemm_bf16(A_ptr, A_lo_ptr, lda, W_ptr, ldw, C_ptr, ldc, M, N, K, bloc
                      ws_ptr=0, stream=0) -> int:
     return load().vla_op_gemm_bf16(A_ptr, A_lo_ptr or None, lda, W_ptr, ldw, C_ptr, ldc, M, N, K,
                                    block_n, splits, ws_ptr or None, stream or None)
+
+
+def vla_op_gemm_pair_bf16(A_ptr, A_lo_ptr, lda, W_ptr, ldw, C_ptr, ldc, M, N, K, stream=0) -> int:
+    return load().vla_op_gemm_pair_bf16(A_ptr, A_lo_ptr or None, lda, W_ptr, ldw, C_ptr, ldc, M, N, K,
+                                        stream or None)
 
 
 def vla_op_gemm_decode_bf16(A_ptr, A_lo_ptr, lda, W_ptr, ldw, C_ptr, ldc, M, N, K, ws_ptr, ws_bytes,

@@ -55,6 +55,32 @@ def test_gemm_matches_fp64(M, N, K, bn, splits, split_a):
     assert err < 2e-5 * math.sqrt(K) * 8, err
 
 
+PAIR_CASES = [
+    # M, N, K, split A
+    (1, 256, 64, False),
+    (200, 512, 688, True),      # one pair tile in M, ragged K
+    (300, 768, 1024, True),     # ragged M over two pair tiles
+    (4608, 1024, 512, True),    # many tiles, persistent pairs
+    (513, 300, 256, False),     # ragged N
+]
+
+
+@pytest.mark.parametrize("M,N,K,split_a", PAIR_CASES)
+def test_pair_gemm_matches_fp64(M, N, K, split_a):
+    A = I.normal_bf16((M, K), 97, 1000 + M, 1.0)
+    A_lo = I.normal_bf16((M, K), 97, 3000 + M, 2.0 ** -9)
+    W = I.normal_bf16((N, K), 97, 2000 + N, 1.0)
+    Ad, Ald, Wd = A.cuda(), A_lo.cuda(), W.cuda()
+    C = torch.full((M, N), float("nan"), dtype=torch.float32, device="cuda")
+    rc = V.vla_op_gemm_pair_bf16(Ad.data_ptr(), Ald.data_ptr() if split_a else 0, K, Wd.data_ptr(), K,
+                                 C.data_ptr(), N, M, N, K, 0)
+    assert rc == 0, V.vla_last_error()
+    torch.cuda.synchronize()
+    Aref = A.double() + A_lo.double() if split_a else A.double()
+    err = (C.cpu().double() - Aref @ W.double().T).abs().max().item()
+    assert err < 2e-5 * math.sqrt(K) * 8, err
+
+
 DECODE_CASES = [
     # M (<= 128 rows), N, K
     (1, 128, 64),
