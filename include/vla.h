@@ -53,6 +53,7 @@ typedef enum {
 
 /* Model and handle sizes.
  * Supported: head_dim in {64, 128}; n_heads * head_dim == d_model; d_model % 128 == 0;
+ *   d_model <= 6400;
  * d_ffn % 8 == 0; n_action_bins == 256; 1 <= action_dim <= 16; vocab >= n_action_bins. */
 typedef struct {
   int n_layers, d_model, n_heads, head_dim, d_ffn, vocab;

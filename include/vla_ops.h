@@ -66,8 +66,10 @@ int vla_op_gemm_bf16_noalloc(const void* A, const void* A_lo, int lda, const voi
  * sampler of vla_decode_actions with uniforms (f32 [B, 256]) at `temperature`.
  * forced (int32 [B] bin indices 0..255, or NULL) selects whose log-prob is returned.
  * Outputs (device, [B]): bins_out int32 (sampled bin k), logprobs_out f32, actions_out f32,
- * logits_out f32 [B, 256] (may be NULL).  status: device uint32 word, OR-ed with
- * VLA_STATUS_* bits. */
+ * logits_out f32 [B, 256] (required: the logits are formed there before sampling).  status:
+ * device uint32 word, OR-ed with VLA_STATUS_* bits.  h must be 16-byte aligned with ldh a
+ * multiple of 4, head_rows 16-byte aligned, final_norm 8-byte aligned, d a multiple of 8 and
+ * at most 6400 (else VLA_ERR_UNSUPPORTED). */
 int vla_op_action_head(const float* h, int ldh, int B, int d, const void* final_norm,
                        const void* head_rows, float eps, const float* uniforms,
                        float temperature, const int32_t* forced, int32_t* bins_out,
@@ -79,7 +81,7 @@ int vla_op_action_head(const float* h, int ldh, int B, int d, const void* final_
  *   q         f32 [B, H, hd] (already rotated);
  *   kv        fp16 cache laid out [env][K,V][H][cap][hd] (one layer, max_env envs);
  *   env, pos  int32 [B] each: query b reads env env[b], keys 0..pos[b] (pos[b] < cap);
- *   max_keys_per_cta  longest key range one CTA handles (0 = the library's default, 160);
+ *   max_keys_per_cta  longest key range one CTA handles (0 = the library's default, 320);
  *   out_hi / out_lo  bf16 [B, H*hd]: the output o as the pair hi + lo;
  *   workspace f32, at least vla_op_attn_decode_workspace_bytes(B, H, hd, max_ctx,
  *             max_keys_per_cta) bytes, max_ctx >= every pos[b] + 1.

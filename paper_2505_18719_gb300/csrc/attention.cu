@@ -9,9 +9,9 @@
 //    fp16 hi/lo pair; the output is written as the bf16 hi/lo pair the O-projection GEMM
 //    reads.
 //  * attn_decode: one query per env (the decode step) with the key range split across CTAs
-//    (flash-decoding); each CTA writes its partial (max, sum, unnormalised output) and a
-//    combine kernel merges the splits in a fixed order.  16 lanes x 16 bytes read one
-//    128-element key row, so each warp streams two rows per instruction.
+//    (flash-decoding); each CTA writes its partial (max, sum, unnormalised output) and the
+//    last CTA of the (env, head) to finish merges the splits in a fixed order.  16 lanes x
+//    16 bytes read one 128-element key row, so each warp streams two rows per instruction.
 //
 // Keys visible to a query at position p are positions 0..p (all of them are in the cache:
 // chunk rows write their K/V in the QKV epilogue before attention runs).
@@ -271,14 +271,19 @@ __global__ void __launch_bounds__(128) attn_chunk_mma_kernel(const float* __rest
 // each lane group loads 4 key rows (K and V) before using any (memory-level parallelism), the
 // dot products reduce with xor shuffles inside the group, online softmax per lane group; the
 // groups of the CTA merge through shared memory into one partial (max, sum, unnormalised
-// output) per range, which the combine kernel merges across ranges in a fixed order.
+// output) per range.  The last CTA of an (env, head) to finish (a ticket on counters[b * H +
+// head], no waiting) merges the S partials in range order and writes the normalised output as
+// the bf16 pair; with S == 1 the CTA writes it directly.
 template <int HD>
 __global__ void __launch_bounds__(128) attn_decode_kernel(const float* __restrict__ q,
                                                           const RowInfo* __restrict__ rows,
                                                           KVLayout kv, int layer, int H,
                                                           int chunk, int S, float scale_log2,
                                                           float* __restrict__ part_o,
-                                                          float2* __restrict__ part_ml) {
+                                                          float2* __restrict__ part_ml,
+                                                          int* __restrict__ counters,
+                                                          bf16* __restrict__ out_hi,
+                                                          bf16* __restrict__ out_lo) {
   constexpr int LPK = HD / 8;     // lanes per key row (8 fp16 = 16 bytes per lane)
   constexpr int KPI = 32 / LPK;   // key rows per warp instruction
   constexpr int U = 4;            // key rows per lane group loaded ahead
@@ -372,7 +377,26 @@ __global__ void __launch_bounds__(128) attn_decode_kernel(const float* __restric
   float M = -INFINITY;
   for (int w = 0; w < 4; ++w)
     for (int k = 0; k < KPI; ++k) M = fmaxf(M, s_m[w][k]);
-  const size_t slot = (static_cast<size_t>(b) * H + head) * S + split;
+  float L = 0.f;
+  for (int w = 0; w < 4; ++w)
+    for (int k = 0; k < KPI; ++k)
+      if (s_m[w][k] != -INFINITY) L += s_l[w][k] * exp2f(s_m[w][k] - M);
+  const size_t bh = static_cast<size_t>(b) * H + head;
+  const size_t out_off = static_cast<size_t>(b) * d + head * HD;
+  if (S == 1) {
+    for (int c = threadIdx.x; c < HD; c += blockDim.x) {
+      float acc = 0.f;
+      for (int w = 0; w < 4; ++w)
+        for (int k = 0; k < KPI; ++k)
+          if (s_m[w][k] != -INFINITY) acc += s_o[w][k][c] * exp2f(s_m[w][k] - M);
+      bf16 hi, lo;
+      split_bf16(acc / L, hi, lo);
+      out_hi[out_off + c] = hi;
+      out_lo[out_off + c] = lo;
+    }
+    return;
+  }
+  const size_t slot = bh * S + split;
   for (int c = threadIdx.x; c < HD; c += blockDim.x) {
     float acc = 0.f;
     for (int w = 0; w < 4; ++w)
@@ -380,38 +404,44 @@ __global__ void __launch_bounds__(128) attn_decode_kernel(const float* __restric
         if (s_m[w][k] != -INFINITY) acc += s_o[w][k][c] * exp2f(s_m[w][k] - M);
     part_o[slot * HD + c] = acc;
   }
-  if (threadIdx.x == 0) {
-    float L = 0.f;
-    for (int w = 0; w < 4; ++w)
-      for (int k = 0; k < KPI; ++k)
-        if (s_m[w][k] != -INFINITY) L += s_l[w][k] * exp2f(s_m[w][k] - M);
-    part_ml[slot] = make_float2(M, L);
-  }
-}
+  if (threadIdx.x == 0) part_ml[slot] = make_float2(M, L);
 
-template <int HD>
-__global__ void attn_combine_kernel(const float* __restrict__ part_o,
-                                    const float2* __restrict__ part_ml, int H, int S,
-                                    bf16* __restrict__ out_hi, bf16* __restrict__ out_lo) {
-  pdl_launch_dependents();
-  pdl_wait();
-  const int bh = blockIdx.x;  // b * H + head
-  const int c = threadIdx.x;
-  float M = -INFINITY;
-  for (int s = 0; s < S; ++s) M = fmaxf(M, part_ml[static_cast<size_t>(bh) * S + s].x);
-  float L = 0.f, acc = 0.f;
+  // ticket: the partial is published (fence) before the counter moves
+  __shared__ int s_last;
+  __threadfence();
+  __syncthreads();
+  if (threadIdx.x == 0) s_last = (atomicAdd(counters + bh, 1) == S - 1);
+  __syncthreads();
+  if (!s_last) return;
+  __threadfence();
+  float Mx = -INFINITY;
+  for (int s = 0; s < S; ++s) Mx = fmaxf(Mx, __ldcg(&part_ml[bh * S + s].x));
+  float Lt = 0.f;
+  float acc[(HD + 127) / 128];
+#pragma unroll
+  for (int i = 0; i < (HD + 127) / 128; ++i) acc[i] = 0.f;
   for (int s = 0; s < S; ++s) {
-    const float2 ml = part_ml[static_cast<size_t>(bh) * S + s];
+    const float2 ml = __ldcg(&part_ml[bh * S + s]);
     if (ml.x == -INFINITY) continue;
-    const float w = exp2f(ml.x - M);
-    L += ml.y * w;
-    acc += part_o[(static_cast<size_t>(bh) * S + s) * HD + c] * w;
+    const float w = exp2f(ml.x - Mx);
+    Lt += ml.y * w;
+#pragma unroll
+    for (int i = 0; i < (HD + 127) / 128; ++i) {
+      const int c = threadIdx.x + i * 128;
+      if (c < HD) acc[i] += __ldcg(&part_o[(bh * S + s) * HD + c]) * w;
+    }
   }
-  const int b = bh / H, head = bh - b * H;
-  bf16 hi, lo;
-  split_bf16(acc / L, hi, lo);
-  out_hi[static_cast<size_t>(b) * H * HD + head * HD + c] = hi;
-  out_lo[static_cast<size_t>(b) * H * HD + head * HD + c] = lo;
+#pragma unroll
+  for (int i = 0; i < (HD + 127) / 128; ++i) {
+    const int c = threadIdx.x + i * 128;
+    if (c < HD) {
+      bf16 hi, lo;
+      split_bf16(acc[i] / Lt, hi, lo);
+      out_hi[out_off + c] = hi;
+      out_lo[out_off + c] = lo;
+    }
+  }
+  if (threadIdx.x == 0) counters[bh] = 0;  // ready for the next launch
 }
 
 }  // namespace
@@ -451,7 +481,7 @@ int attn_chunk_launch(const float* q, bf16* out_hi, bf16* out_lo, const AttnTile
 
 int attn_decode_launch(const float* q, bf16* out_hi, bf16* out_lo, const RowInfo* rows, int B,
                        int max_ctx, KVLayout kv, int layer, int H, int hd, int chunk,
-                       float* part_o, float2* part_ml, cudaStream_t stream) {
+                       float* part_o, float2* part_ml, int* counters, cudaStream_t stream) {
   if (B <= 0) return VLA_OK;
   // equal key ranges (multiples of 16) no longer than `chunk`
   const int S = (max_ctx + chunk - 1) / chunk;
@@ -460,16 +490,10 @@ int attn_decode_launch(const float* q, bf16* out_hi, bf16* out_lo, const RowInfo
   dim3 grid(S, H, B);
   if (hd == 128) {
     VLA_CUDA_TRY(launch_pdl(attn_decode_kernel<128>, grid, dim3(128), 0, stream, q, rows, kv, layer, H,
-                            c, S, scale_log2, part_o, part_ml));
-    note_launch();
-    VLA_CUDA_TRY(launch_pdl(attn_combine_kernel<128>, dim3(B * H), dim3(128), 0, stream, part_o, part_ml,
-                            H, S, out_hi, out_lo));
+                            c, S, scale_log2, part_o, part_ml, counters, out_hi, out_lo));
   } else if (hd == 64) {
     VLA_CUDA_TRY(launch_pdl(attn_decode_kernel<64>, grid, dim3(128), 0, stream, q, rows, kv, layer, H,
-                            c, S, scale_log2, part_o, part_ml));
-    note_launch();
-    VLA_CUDA_TRY(launch_pdl(attn_combine_kernel<64>, dim3(B * H), dim3(64), 0, stream, part_o, part_ml,
-                            H, S, out_hi, out_lo));
+                            c, S, scale_log2, part_o, part_ml, counters, out_hi, out_lo));
   } else {
     return VLA_ERR_UNSUPPORTED;
   }

@@ -15,9 +15,11 @@ int attn_chunk_launch(const float* q, bf16* out_hi, bf16* out_lo, const AttnTile
                       int n_tiles, KVLayout kv, int layer, int H, int hd, cudaStream_t stream);
 
 // One query per env row b (rows[b] gives env and position); key range split into equal ranges
-// of at most `chunk` keys (chunk <= 256); partials in part_o [B*H*S*hd] f32 and part_ml [B*H*S] (S = ceil(max_ctx/chunk)).
+// of at most `chunk` keys (a multiple of 16 at least 16); partials in part_o [B*H*S*hd] f32 and part_ml [B*H*S]
+// (S = ceil(max_ctx/chunk)); counters [B*H] int must be zero at launch and are zero again
+// when the kernel completes.
 int attn_decode_launch(const float* q, bf16* out_hi, bf16* out_lo, const RowInfo* rows, int B,
                        int max_ctx, KVLayout kv, int layer, int H, int hd, int chunk,
-                       float* part_o, float2* part_ml, cudaStream_t stream);
+                       float* part_o, float2* part_ml, int* counters, cudaStream_t stream);
 
 }  // namespace vla

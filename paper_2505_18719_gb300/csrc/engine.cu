@@ -109,6 +109,7 @@ struct vla_handle {
   size_t ws_bytes = 0;
   float* h_last = nullptr;
   float* head_in = nullptr;
+  float* head_z = nullptr;  // action-bin logits [B * A, 256]
   float2* rope = nullptr;
   RowInfo* rows = nullptr;
   AttnTile* tiles = nullptr;
@@ -119,7 +120,8 @@ struct vla_handle {
   uint32_t* status = nullptr;
   float* part_o = nullptr;
   float2* part_ml = nullptr;
-  int attn_chunk = 160;  // max keys per decode-attention CTA
+  int* attn_tickets = nullptr;  // [B * H], zero between decode-attention launches
+  int attn_chunk = 320;  // max keys per decode-attention CTA
   int max_tiles = 0;
   // pinned host staging (ring of slots, each guarded by an event)
   static constexpr int kSlots = 4;
@@ -225,13 +227,23 @@ int run_gemm(vla_handle* h, int cls, const bf16* A, size_t a_plane, int lda, con
                                (epi.kind == EPI_SWIGLU ? (N / 2 + 127) / 128 : (N + 255) / 256);
     g.pair = pair_tiles >= h->num_sms / 2;
   }
+  // A following RMSNorm is fused into the weight-streaming GEMM's reduction; after a tile
+  // GEMM it is its own kernel.
+  const EpiArgs norm = epi;
+  if (!stream_k) g.epi.norm_w = nullptr;
   if (h->ev_used.size() > 8192) prof_harvest(h);
   int ev = prof_begin(h, cls);
   GemmCost cost{0, 0};
-  const int rc = stream_k ? gemv_launch(g, h->stream, h->num_sms, &cost)
-                          : gemm_launch(g, h->stream, h->num_sms, &cost);
+  int rc = stream_k ? gemv_launch(g, h->stream, h->num_sms, &cost)
+                    : gemm_launch(g, h->stream, h->num_sms, &cost);
   prof_end(h, ev, cls, cost.flops, cost.bytes);
   if (rc != VLA_OK) return fail(h, rc, t_err.empty() ? "gemm launch failed" : t_err);
+  if (!stream_k && norm.norm_w) {
+    ev = prof_begin(h, VLA_KCLASS_OTHER);
+    rc = rmsnorm_launch(norm.resid, norm.norm_w, M, N, norm.norm_eps, norm.norm_hi, norm.norm_lo, h->stream);
+    prof_end(h, ev, VLA_KCLASS_OTHER, 0, 6.0 * M * N);
+    if (rc) return fail(h, rc, t_err);
+  }
   return VLA_OK;
 }
 
@@ -245,10 +257,11 @@ int forward_layers(vla_handle* h, int M, const RowInfo* rows_dev, bool decode, i
   const size_t pd = static_cast<size_t>(h->max_tokens) * d;   // hi -> lo plane offsets
   const size_t pf = static_cast<size_t>(h->max_tokens) * F;
   int rc;
+  // the first layer's attention RMSNorm; every later RMSNorm follows a residual add
+  int ev = prof_begin(h, VLA_KCLASS_OTHER);
+  if ((rc = rmsnorm_launch(h->h, h->attn_norm[0], M, d, c.rms_eps, h->y, h->y + pd, h->stream))) return fail(h, rc, t_err);
+  prof_end(h, ev, VLA_KCLASS_OTHER, 0, 6.0 * M * d);
   for (int l = 0; l < c.n_layers; ++l) {
-    int ev = prof_begin(h, VLA_KCLASS_OTHER);
-    if ((rc = rmsnorm_launch(h->h, h->attn_norm[l], M, d, c.rms_eps, h->y, h->y + pd, h->stream))) return fail(h, rc, t_err);
-    prof_end(h, ev, VLA_KCLASS_OTHER, 0, 6.0 * M * d);
 
     EpiArgs e;
     e.kind = EPI_QKV;
@@ -264,7 +277,7 @@ int forward_layers(vla_handle* h, int M, const RowInfo* rows_dev, bool decode, i
     if (decode) {
       ev = prof_begin(h, VLA_KCLASS_ATTN_DECODE);
       rc = attn_decode_launch(h->q, h->ao, h->ao + pd, rows_dev, M, max_ctx, h->kvl, l, H, hd,
-                              h->attn_chunk, h->part_o, h->part_ml, h->stream);
+                              h->attn_chunk, h->part_o, h->part_ml, h->attn_tickets, h->stream);
       prof_end(h, ev, VLA_KCLASS_ATTN_DECODE, 0, 0);
     } else {
       ev = prof_begin(h, VLA_KCLASS_ATTN_PREFILL);
@@ -277,11 +290,12 @@ int forward_layers(vla_handle* h, int M, const RowInfo* rows_dev, bool decode, i
     eo.kind = EPI_RESID;
     eo.resid = h->h;
     eo.ldr = d;
+    eo.norm_w = h->ffn_norm[l];
+    eo.norm_eps = c.rms_eps;
+    eo.norm_hi = h->y;
+    eo.norm_lo = h->y + pd;
+    eo.ldn = d;
     if ((rc = run_gemm(h, gcls, h->ao, pd, d, h->wo[l], d, M, d, d, eo))) return rc;
-
-    ev = prof_begin(h, VLA_KCLASS_OTHER);
-    if ((rc = rmsnorm_launch(h->h, h->ffn_norm[l], M, d, c.rms_eps, h->y, h->y + pd, h->stream))) return fail(h, rc, t_err);
-    prof_end(h, ev, VLA_KCLASS_OTHER, 0, 6.0 * M * d);
 
     EpiArgs eg;
     eg.kind = EPI_SWIGLU;
@@ -294,6 +308,13 @@ int forward_layers(vla_handle* h, int M, const RowInfo* rows_dev, bool decode, i
     ed.kind = EPI_RESID;
     ed.resid = h->h;
     ed.ldr = d;
+    if (l + 1 < c.n_layers) {
+      ed.norm_w = h->attn_norm[l + 1];
+      ed.norm_eps = c.rms_eps;
+      ed.norm_hi = h->y;
+      ed.norm_lo = h->y + pd;
+      ed.ldn = d;
+    }
     if ((rc = run_gemm(h, gcls, h->u, pf, F, h->wdown[l], F, M, d, F, ed))) return rc;
   }
   return VLA_OK;
@@ -317,9 +338,10 @@ int vla_create(const vla_config* cfg, const vla_weights* w, void* cuda_stream, v
     return set_err(nullptr, VLA_ERR_ARG, "vla_create: non-positive size in config");
   if (c.head_dim != 64 && c.head_dim != 128)
     return set_err(nullptr, VLA_ERR_UNSUPPORTED, "vla_create: head_dim must be 64 or 128");
-  if (c.n_heads * c.head_dim != c.d_model || c.d_model % 128 || c.d_ffn % 8)
+  if (c.n_heads * c.head_dim != c.d_model || c.d_model % 128 || c.d_model > 6400 || c.d_ffn % 8)
     return set_err(nullptr, VLA_ERR_UNSUPPORTED,
-                   "vla_create: need n_heads*head_dim == d_model, d_model % 128 == 0, d_ffn % 8 == 0");
+                   "vla_create: need n_heads*head_dim == d_model, d_model % 128 == 0, d_model <= 6400, "
+                   "d_ffn % 8 == 0");
   if (c.n_action_bins != 256 || c.vocab < 256 || c.action_dim < 1 || c.action_dim > 16)
     return set_err(nullptr, VLA_ERR_UNSUPPORTED,
                    "vla_create: need n_action_bins == 256, vocab >= 256, 1 <= action_dim <= 16");
@@ -398,6 +420,7 @@ int vla_create(const vla_config* cfg, const vla_weights* w, void* cuda_stream, v
             alloc(reinterpret_cast<void**>(&h->ws), ws) &&
             alloc(reinterpret_cast<void**>(&h->h_last), static_cast<size_t>(B) * d * sizeof(float)) &&
             alloc(reinterpret_cast<void**>(&h->head_in), static_cast<size_t>(B) * A * d * sizeof(float)) &&
+            alloc(reinterpret_cast<void**>(&h->head_z), static_cast<size_t>(B) * A * 256 * sizeof(float)) &&
             alloc(reinterpret_cast<void**>(&h->rope), static_cast<size_t>(cap) * (c.head_dim / 2) * sizeof(float2)) &&
             alloc(reinterpret_cast<void**>(&h->rows), T * sizeof(RowInfo)) &&
             alloc(reinterpret_cast<void**>(&h->tiles), static_cast<size_t>(h->max_tiles) * sizeof(AttnTile)) &&
@@ -407,7 +430,9 @@ int vla_create(const vla_config* cfg, const vla_weights* w, void* cuda_stream, v
             alloc(reinterpret_cast<void**>(&h->pending), static_cast<size_t>(B) * sizeof(int)) &&
             alloc(reinterpret_cast<void**>(&h->status), sizeof(uint32_t)) &&
             alloc(reinterpret_cast<void**>(&h->part_o), static_cast<size_t>(B) * c.n_heads * max_S * c.head_dim * sizeof(float)) &&
-            alloc(reinterpret_cast<void**>(&h->part_ml), static_cast<size_t>(B) * c.n_heads * max_S * sizeof(float2));
+            alloc(reinterpret_cast<void**>(&h->part_ml), static_cast<size_t>(B) * c.n_heads * max_S * sizeof(float2)) &&
+            alloc(reinterpret_cast<void**>(&h->attn_tickets), static_cast<size_t>(B) * c.n_heads * sizeof(int)) &&
+            cudaMemset(h->attn_tickets, 0, static_cast<size_t>(B) * c.n_heads * sizeof(int)) == cudaSuccess;
   if (!ok) {
     cudaGetLastError();
     vla_destroy(h);
@@ -546,6 +571,7 @@ int vla_decode_actions(vla_handle* h, const float* uniforms, float temperature, 
   for (int b = 0; b < B; ++b) max_len_p = std::max(max_len_p, h->len_prefill[b]);
 
   HeadArgs ha;
+  ha.z = h->head_z;
   ha.B = B;
   ha.n_pos = 1;
   ha.A = A;
@@ -643,6 +669,7 @@ int vla_score_actions(vla_handle* h, const int32_t* tokens, float temperature, f
     return fail(h, rc, t_err);
 
   HeadArgs ha;
+  ha.z = h->head_z;
   ha.h = h->head_in;
   ha.ldh = d;
   ha.B = B;
@@ -720,9 +747,9 @@ void vla_destroy(vla_handle* h) {
   if (!h) return;
   cudaSetDevice(h->dev);
   cudaStreamSynchronize(h->stream);
-  void* bufs[] = {h->kv, h->h, h->y, h->q, h->ao, h->u, h->ws, h->h_last, h->head_in, h->rope,
+  void* bufs[] = {h->kv, h->h, h->y, h->q, h->ao, h->u, h->ws, h->h_last, h->head_in, h->head_z, h->rope,
                   h->rows, h->tiles, h->sidx, h->didx, h->fed, h->pending, h->status, h->part_o,
-                  h->part_ml};
+                  h->part_ml, h->attn_tickets};
   for (void* p : bufs)
     if (p) cudaFree(p);
   for (int s = 0; s < vla_handle::kSlots; ++s) {
@@ -852,10 +879,11 @@ int vla_op_action_head(const float* hs, int ldh, int B, int d, const void* final
                        float eps, const float* uniforms, float temperature, const int32_t* forced,
                        int32_t* bins_out, float* logprobs_out, float* actions_out, float* logits_out,
                        uint32_t* status, void* cuda_stream) {
-  if (!hs || B < 1 || d < 8 || ldh < d || !final_norm || !head_rows || !logprobs_out || !status ||
+  if (!hs || B < 1 || d < 8 || ldh < d || !final_norm || !head_rows || !logprobs_out || !logits_out || !status ||
       !finite_nonneg(temperature) || (temperature > 0.f && !uniforms))
     return set_err(nullptr, VLA_ERR_ARG, "vla_op_action_head: bad argument");
   HeadArgs ha;
+  ha.z = logits_out;
   ha.h = hs;
   ha.ldh = ldh;
   ha.B = B;
@@ -879,15 +907,16 @@ int vla_op_action_head(const float* hs, int ldh, int B, int d, const void* final
   return action_head_launch(ha, static_cast<cudaStream_t>(cuda_stream));
 }
 
-static const int kOpAttnChunk = 160;
+static const int kOpAttnChunk = 320;
 
 size_t vla_op_attn_decode_workspace_bytes(int B, int H, int hd, int max_ctx, int max_keys_per_cta) {
   if (B < 1 || H < 1 || hd < 1 || max_ctx < 1) return 0;
   const int chunk = max_keys_per_cta > 0 ? max_keys_per_cta : kOpAttnChunk;
   const size_t S = (static_cast<size_t>(max_ctx) + chunk - 1) / chunk;
-  // RowInfo table, then partial outputs and (max, sum) pairs
+  // RowInfo table, then partial outputs, (max, sum) pairs and the per-(env, head) tickets
   return static_cast<size_t>(B) * sizeof(RowInfo) + 256 + static_cast<size_t>(B) * H * S * hd * sizeof(float) +
-         256 + static_cast<size_t>(B) * H * S * sizeof(float2) + 256 + 256;
+         256 + static_cast<size_t>(B) * H * S * sizeof(float2) + 256 + static_cast<size_t>(B) * H * sizeof(int) +
+         256 + 256;
 }
 
 int vla_op_attn_decode(const float* q, const void* kv, int max_env, int H, int hd, int cap, const int32_t* env,
@@ -910,7 +939,11 @@ int vla_op_attn_decode(const float* q, const void* kv, int max_env, int H, int h
   char* base = reinterpret_cast<char*>(workspace) + ((static_cast<size_t>(B) * sizeof(RowInfo) + 255) / 256) * 256;
   const size_t S = (static_cast<size_t>(max_ctx) + chunk - 1) / chunk;
   float* part_o = reinterpret_cast<float*>(base);
-  float2* part_ml = reinterpret_cast<float2*>(base + ((static_cast<size_t>(B) * H * S * hd * sizeof(float) + 255) / 256) * 256);
+  char* ml_base = base + ((static_cast<size_t>(B) * H * S * hd * sizeof(float) + 255) / 256) * 256;
+  float2* part_ml = reinterpret_cast<float2*>(ml_base);
+  int* counters = reinterpret_cast<int*>(ml_base + ((static_cast<size_t>(B) * H * S * sizeof(float2) + 255) / 256) * 256);
+  if (cudaMemsetAsync(counters, 0, static_cast<size_t>(B) * H * sizeof(int), st) != cudaSuccess)
+    return cuda_fail(cudaGetLastError(), "vla_op_attn_decode: tickets");
   KVLayout L{};
   L.base = static_cast<f16*>(const_cast<void*>(kv));
   L.cap = cap;
@@ -919,7 +952,7 @@ int vla_op_attn_decode(const float* q, const void* kv, int max_env, int H, int h
   L.env_stride = 2 * L.kv_stride;
   L.layer_stride = static_cast<int64_t>(max_env) * L.env_stride;
   const int rc = attn_decode_launch(q, static_cast<bf16*>(out_hi), static_cast<bf16*>(out_lo), rows, B, max_ctx, L,
-                                    0, H, hd, chunk, part_o, part_ml, st);
+                                    0, H, hd, chunk, part_o, part_ml, counters, st);
   if (rc != VLA_OK && rc != VLA_ERR_CUDA) return set_err(nullptr, rc, "vla_op_attn_decode: unsupported arguments");
   return rc;
 }

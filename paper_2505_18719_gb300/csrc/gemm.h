@@ -28,6 +28,14 @@ struct EpiArgs {
   int layer = 0;
   const float2* rope = nullptr;   // EPI_QKV: [cap][hd/2] (cos, sin)
   int d = 0, hd = 0;
+  // EPI_RESID of the weight-streaming GEMM only: after the residual add, the row's RMSNorm
+  // with weight norm_w (N elements) is written as the bf16 pair norm_hi / norm_lo
+  // [m * ldn + n] in the same kernel.  The tile GEMM rejects it.
+  const bf16* norm_w = nullptr;
+  float norm_eps = 0.f;
+  bf16* norm_hi = nullptr;
+  bf16* norm_lo = nullptr;
+  int ldn = 0;
   uint32_t* status = nullptr;
 };
 
@@ -60,7 +68,8 @@ int gemm_launch(const GemmArgs& a, cudaStream_t stream, int num_sms, GemmCost* c
 
 // Weight-streaming (decode) GEMM for M <= 128 rows with a split A (A_lo required): swap-AB
 // tcgen05 MMAs, stream-K over the weight tiles, partials in `workspace`
-// (gemv_workspace_bytes), then the epilogue of `a.epi` in a fixed-order reduction.
+// (gemv_workspace_bytes), then the epilogue of `a.epi` in a fixed-order reduction (EPI_RESID
+// with norm_w set: fused with the following RMSNorm).
 size_t gemv_workspace_bytes(int M, int N, int K, int num_sms);
 int gemv_launch(const GemmArgs& a, cudaStream_t stream, int num_sms, GemmCost* cost);
 

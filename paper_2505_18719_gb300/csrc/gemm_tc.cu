@@ -20,7 +20,9 @@
 // Work units (m-tile, n-tile, k-split) are rastered in groups of 16 m-tiles so that the
 // tiles in flight share A and B in L2.  Every mbarrier wait is bounded (globaltimer): on
 // timeout the CTA records VLA_STATUS_TIMEOUT, drains its own copies and MMAs, frees TMEM and
-// exits.  No TMA multicast and no clusters are used.
+// exits.  No TMA multicast is used; the pair variant (gemm_tc2_kernel) runs on clusters of two
+// CTAs issuing cta_group::2 MMAs on 256 x 256 tiles.
+#include <algorithm>
 #include <cstdio>
 #include <cstring>
 #include <mutex>
@@ -781,6 +783,215 @@ __global__ void reduce_qkv_kernel(Src src, int M, EpiArgs e) {
   }
 }
 
+// Stream-K reductions of the weight-streaming GEMM, per work item (x: 256-column tile of the
+// product, y: chunk of kMR batch rows).  The CTAs whose ranges cover a tile are found once per
+// thread and four CTAs' partials are loaded before their adds, which run in ascending CTA
+// order as in StreamSrc.  One CTA per work item (a grid of at most two CTAs per SM, which
+// would leave room for the next GEMM's CTAs, measured slower: the reduction is bound by
+// the latency of its loads).
+constexpr int kMR = 4;
+
+struct TileSum {
+  const float* base;  // ws + column r of the tile
+  int c0, c1;
+  int t, KB, P, max_seg, BNX;
+  __device__ __forceinline__ TileSum(const StreamSrc& s, int n) {
+    t = n >> 8;
+    KB = s.KB;
+    P = s.P;
+    max_seg = s.max_seg;
+    BNX = s.BNX;
+    c0 = (t * KB) / P;
+    c1 = (t * KB + KB - 1) / P;
+    base = s.ws + (n & 255);
+  }
+  __device__ __forceinline__ const float* row(int c, int m) const {
+    const int slot = c * max_seg + t - (c * P) / KB;
+    return base + (static_cast<size_t>(slot) * BNX + m) * 256;
+  }
+  // acc[j] = sum over c of partial(c, row m0 + j), rows m0 + j < M only
+  __device__ __forceinline__ void sum(int m0, int M, float (&acc)[kMR]) const {
+#pragma unroll
+    for (int j = 0; j < kMR; ++j) acc[j] = 0.f;
+    for (int c = c0; c <= c1; c += 4) {
+      float v[4][kMR];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const float* src = row(c + u <= c1 ? c + u : c1, m0);
+#pragma unroll
+        for (int j = 0; j < kMR; ++j) v[u][j] = (c + u <= c1 && m0 + j < M) ? src[j * 256] : 0.f;
+      }
+#pragma unroll
+      for (int u = 0; u < 4; ++u)
+        if (c + u <= c1) {
+#pragma unroll
+          for (int j = 0; j < kMR; ++j) acc[j] += v[u][j];
+        }
+    }
+  }
+  // columns n .. n+3 (n % 4 == 0) of row m
+  __device__ __forceinline__ float4 sum4(int m) const {
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int c = c0; c <= c1; c += 4) {
+      float4 v[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u)
+        v[u] = (c + u <= c1) ? *reinterpret_cast<const float4*>(row(c + u, m)) : make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+      for (int u = 0; u < 4; ++u)
+        if (c + u <= c1) {
+          acc.x += v[u].x;
+          acc.y += v[u].y;
+          acc.z += v[u].z;
+          acc.w += v[u].w;
+        }
+    }
+    return acc;
+  }
+};
+
+__device__ __forceinline__ bool next_item(int& item, int nx, int ny, int& x, int& y) {
+  if (item >= nx * ny) return false;
+  y = item / nx;
+  x = item - y * nx;
+  item += gridDim.x;
+  return true;
+}
+
+// items (ceil(N / 256), ceil(M / kMR)), 256 threads: out[m][n] (+)= sum
+__global__ void stream_reduce_f32_kernel(StreamSrc src, int M, int N, float* out, int ldo,
+                                         int resid) {
+  pdl_launch_dependents();
+  pdl_wait();
+  const int nx = (N + 255) / 256, ny = (M + kMR - 1) / kMR;
+  int item = blockIdx.x, bx, by;
+  while (next_item(item, nx, ny, bx, by)) {
+    const int n = bx * 256 + threadIdx.x;
+    if (n >= N) continue;
+    const int m0 = by * kMR;
+    float acc[kMR];
+    TileSum(src, n).sum(m0, M, acc);
+#pragma unroll
+    for (int j = 0; j < kMR; ++j) {
+      if (m0 + j >= M) break;
+      float* o = out + static_cast<size_t>(m0 + j) * ldo + n;
+      *o = resid ? *o + acc[j] : acc[j];
+    }
+  }
+}
+
+// items (ceil(F / 256), ceil(M / kMR)), 256 threads: gate column f, up column f + F
+__global__ void stream_reduce_swiglu_kernel(StreamSrc src, int M, int F, bf16* out_hi,
+                                            bf16* out_lo, int ldo) {
+  pdl_launch_dependents();
+  pdl_wait();
+  const int nx = (F + 255) / 256, ny = (M + kMR - 1) / kMR;
+  int item = blockIdx.x, bx, by;
+  while (next_item(item, nx, ny, bx, by)) {
+    const int f = bx * 256 + threadIdx.x;
+    if (f >= F) continue;
+    const int m0 = by * kMR;
+    float g[kMR], u[kMR];
+    TileSum(src, f).sum(m0, M, g);
+    TileSum(src, f + F).sum(m0, M, u);
+#pragma unroll
+    for (int j = 0; j < kMR; ++j) {
+      if (m0 + j >= M) break;
+      bf16 hi, lo;
+      split_bf16(silu_f(g[j]) * u[j], hi, lo);
+      out_hi[static_cast<size_t>(m0 + j) * ldo + f] = hi;
+      out_lo[static_cast<size_t>(m0 + j) * ldo + f] = lo;
+    }
+  }
+}
+
+// items (3d / 256, ceil(M / kMR)), 128 threads; 256 % hd == 0 and d % 256 == 0, so both
+// halves of a rotary pair sit in one tile: thread p takes pair (i, i + hd/2) of local head
+// p / (hd/2).
+__global__ void stream_reduce_qkv_kernel(StreamSrc src, int M, EpiArgs e) {
+  pdl_launch_dependents();
+  pdl_wait();
+  const int d = e.d, hd = e.hd, half = hd >> 1;
+  const int p = threadIdx.x;
+  const int i = p % half;
+  const int nx = 3 * d / 256, ny = (M + kMR - 1) / kMR;
+  int item = blockIdx.x, bx, by;
+  while (next_item(item, nx, ny, bx, by)) {
+    const int c = bx * 256 + (p / half) * hd + i;
+    const int sec = c / d;
+    const int head = (c - sec * d) / hd;
+    const int m0 = by * kMR;
+    float a[kMR], b[kMR];
+    TileSum(src, c).sum(m0, M, a);
+    TileSum(src, c + half).sum(m0, M, b);
+#pragma unroll
+    for (int j = 0; j < kMR; ++j) {
+      const int m = m0 + j;
+      if (m >= M) break;
+      const RowInfo ri = e.rows[m];
+      float x = a[j], y = b[j];
+      if (sec < 2) {
+        const float2 cs = e.rope[static_cast<size_t>(ri.pos) * half + i];
+        const float rx = x * cs.x - y * cs.y;
+        const float ry = y * cs.x + x * cs.y;
+        x = rx;
+        y = ry;
+      }
+      if (sec == 0) {
+        float* dst = e.out_q + static_cast<size_t>(m) * d + head * hd;
+        dst[i] = x;
+        dst[i + half] = y;
+      } else {
+        f16* dst = e.kv.base + static_cast<int64_t>(e.layer) * e.kv.layer_stride +
+                   static_cast<int64_t>(ri.env) * e.kv.env_stride + (sec == 2 ? e.kv.kv_stride : 0) +
+                   static_cast<int64_t>(head) * e.kv.head_stride + static_cast<int64_t>(ri.pos) * hd;
+        dst[i] = __float2half_rn(x);
+        dst[i + half] = __float2half_rn(y);
+      }
+    }
+  }
+}
+
+// grid (M), 1024 threads (N % 4 == 0): h[m][n] += sum, then the RMSNorm of the updated row
+// times w as the bf16 pair y_hi / y_lo (the next GEMM's A).  The row sums are in the same
+// order as stream_reduce_f32_kernel's.
+__global__ void __launch_bounds__(1024) stream_reduce_resid_norm_kernel(StreamSrc src, int N, float* h,
+                                                                         int ldh, const bf16* w, float eps,
+                                                                         bf16* y_hi, bf16* y_lo, int ldy) {
+  pdl_launch_dependents();
+  pdl_wait();
+  __shared__ float red[32];
+  const int m = blockIdx.x;
+  float* hrow = h + static_cast<size_t>(m) * ldh;
+  float ss = 0.f;
+  for (int n = threadIdx.x * 4; n < N; n += blockDim.x * 4) {
+    const float4 acc = TileSum(src, n).sum4(m);
+    float4 v = *reinterpret_cast<const float4*>(hrow + n);
+    v.x += acc.x;
+    v.y += acc.y;
+    v.z += acc.z;
+    v.w += acc.w;
+    *reinterpret_cast<float4*>(hrow + n) = v;
+    ss += v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w;
+  }
+  ss = warp_sum(ss);
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = ss;
+  __syncthreads();
+  float tot = 0.f;
+  for (int i = 0; i < static_cast<int>(blockDim.x >> 5); ++i) tot += red[i];
+  const float r = rsqrtf(tot / static_cast<float>(N) + eps);
+  for (int n = threadIdx.x * 4; n < N; n += blockDim.x * 4) {
+    const float4 v = *reinterpret_cast<const float4*>(hrow + n);
+    const uint2 ww = *reinterpret_cast<const uint2*>(w + n);
+    const float2 w0 = unpack_bf16x2(ww.x), w1 = unpack_bf16x2(ww.y);
+    uint2 hi, lo;
+    split_pack2(v.x * r * w0.x, v.y * r * w0.y, hi.x, lo.x);
+    split_pack2(v.z * r * w1.x, v.w * r * w1.y, hi.y, lo.y);
+    *reinterpret_cast<uint2*>(y_hi + static_cast<size_t>(m) * ldy + n) = hi;
+    *reinterpret_cast<uint2*>(y_lo + static_cast<size_t>(m) * ldy + n) = lo;
+  }
+}
+
 // ----------------------------------------------------------------------------- decode GEMM
 // Weight-streaming GEMM for decode-sized batches (M <= 128 rows of activations), where the
 // projections are bound by reading the weights from HBM once.
@@ -1226,6 +1437,7 @@ size_t gemm_workspace_bytes(const GemmArgs& a) {
 int gemm_launch(const GemmArgs& a, cudaStream_t stream, int num_sms, GemmCost* cost) {
   if (a.M < 1 || a.N < 1 || a.K < 1 || !a.A || !a.B) return VLA_ERR_ARG;
   if (a.block_n != 128 && a.block_n != 256) return VLA_ERR_ARG;
+  if (a.epi.norm_w) return VLA_ERR_ARG;  // fused RMSNorm: weight-streaming GEMM only
   if ((a.lda % 8) || (a.ldb % 8) || a.lda < a.K || a.ldb < a.K) return VLA_ERR_ARG;
   if ((reinterpret_cast<uintptr_t>(a.A) & 15) || (reinterpret_cast<uintptr_t>(a.B) & 15) ||
       (reinterpret_cast<uintptr_t>(a.A_lo) & 15))
@@ -1321,8 +1533,16 @@ int gemv_launch(const GemmArgs& a, cudaStream_t stream, int num_sms, GemmCost* c
     return VLA_ERR_ARG;
   if (a.epi.kind == EPI_SWIGLU && (a.N & 1)) return VLA_ERR_ARG;
   if (a.epi.kind == EPI_QKV && a.N != 3 * a.epi.d) return VLA_ERR_ARG;
+  if (a.epi.norm_w) {
+    if (a.epi.kind != EPI_RESID || (a.N & 3) || (a.epi.ldr & 3) || (a.epi.ldn & 3) || !a.epi.norm_hi ||
+        !a.epi.norm_lo || (reinterpret_cast<uintptr_t>(a.epi.resid) & 15) ||
+        (reinterpret_cast<uintptr_t>(a.epi.norm_w) & 7) || (reinterpret_cast<uintptr_t>(a.epi.norm_hi) & 7) ||
+        (reinterpret_cast<uintptr_t>(a.epi.norm_lo) & 7))
+      return VLA_ERR_ARG;
+  }
   const GemvPlan pl = gemv_plan(a.M, a.N, a.K, num_sms);
-  if (!a.workspace || a.workspace_bytes < pl.ws_bytes) return VLA_ERR_ARG;
+  if (!a.workspace || a.workspace_bytes < pl.ws_bytes || (reinterpret_cast<uintptr_t>(a.workspace) & 15))
+    return VLA_ERR_ARG;
   CUtensorMap mw, mx, mx2;
   if (!make_map(&mw, a.B, a.N, a.K, a.ldb, 256) || !make_map(&mx, a.A, a.M, a.K, a.lda, pl.bnx) ||
       !make_map(&mx2, a.A_lo, a.M, a.K, a.lda, pl.bnx))
@@ -1345,7 +1565,43 @@ int gemv_launch(const GemmArgs& a, cudaStream_t stream, int num_sms, GemmCost* c
   }
   if (rc != VLA_OK) return rc;
   const StreamSrc src{a.workspace, pl.bnx, pl.kbt, pl.per_cta, pl.max_seg};
-  if ((rc = launch_reduce(src, a, stream)) != VLA_OK) return rc;
+  const int ny = (a.M + kMR - 1) / kMR;
+  auto grid_for = [&](int nx) { return dim3(nx * ny); };
+  switch (a.epi.kind) {
+    case EPI_F32:
+    case EPI_RESID: {
+      const bool resid = a.epi.kind == EPI_RESID;
+      if (resid && a.epi.norm_w) {
+        VLA_CUDA_TRY(launch_pdl(stream_reduce_resid_norm_kernel, dim3(a.M), dim3(1024), 0, stream, src, a.N,
+                                a.epi.resid, a.epi.ldr, a.epi.norm_w, a.epi.norm_eps, a.epi.norm_hi,
+                                a.epi.norm_lo, a.epi.ldn));
+        break;
+      }
+      VLA_CUDA_TRY(launch_pdl(stream_reduce_f32_kernel, grid_for((a.N + 255) / 256), dim3(256), 0, stream, src,
+                              a.M, a.N, resid ? a.epi.resid : a.epi.out_f32, resid ? a.epi.ldr : a.epi.ldo,
+                              resid ? 1 : 0));
+      break;
+    }
+    case EPI_SWIGLU:
+      VLA_CUDA_TRY(launch_pdl(stream_reduce_swiglu_kernel, grid_for((a.N / 2 + 255) / 256), dim3(256), 0,
+                              stream, src, a.M, a.N / 2, a.epi.out_hi, a.epi.out_lo, a.epi.ldo));
+      break;
+    case EPI_QKV:
+      if (256 % a.epi.hd == 0 && a.epi.d % 256 == 0) {
+        VLA_CUDA_TRY(launch_pdl(stream_reduce_qkv_kernel, grid_for(a.N / 256), dim3(128), 0, stream, src, a.M,
+                                a.epi));
+      } else {
+        // rotary pairs may straddle tiles: element-wise reduction
+        if ((rc = launch_reduce(src, a, stream)) != VLA_OK) return rc;
+        if (cost) *cost = gemm_cost(a);
+        return VLA_OK;
+      }
+      break;
+    default:
+      return VLA_ERR_ARG;
+  }
+  note_launch();
+  VLA_CUDA_TRY(cudaGetLastError());
   if (cost) *cost = gemm_cost(a);
   return VLA_OK;
 }

@@ -41,6 +41,8 @@ struct HeadArgs {
   float* lp_out = nullptr;          // [B, A]
   float* act_out = nullptr;         // [B, A]
   float* logits_out = nullptr;      // [B, A, 256]
+  float* z = nullptr;               // scratch [B * n_pos, 256] logits (may alias logits_out
+                                    // when A == n_pos and step == 0)
   int* fed_out = nullptr;           // [B, A] token fed to the next step (forced or sampled)
   uint32_t* status = nullptr;
 };
