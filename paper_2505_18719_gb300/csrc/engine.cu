@@ -110,6 +110,8 @@ struct vla_handle {
   float* h_last = nullptr;
   float* head_in = nullptr;
   float* head_z = nullptr;  // action-bin logits [B * A, 256]
+  float* q_last = nullptr;  // last layer of a prefill: queries of each env's final row [B, d]
+  RowInfo* last_rows = nullptr;  // and those rows' RowInfo [B]
   float2* rope = nullptr;
   RowInfo* rows = nullptr;
   AttnTile* tiles = nullptr;
@@ -247,10 +249,21 @@ int run_gemm(vla_handle* h, int cls, const bf16* A, size_t a_plane, int lda, con
   return VLA_OK;
 }
 
+// Rows whose last-layer output is needed (a prefill only feeds the head with each env's
+// final row): idx [n] into the chunk's rows, rows [n] their RowInfo, max_ctx = longest context.
+struct LastRows {
+  int n = 0;
+  const int* idx = nullptr;
+  const RowInfo* rows = nullptr;
+  int max_ctx = 0;
+};
+
 // All decoder layers over M rows already assembled in h->h (Llama-2 layer, §3.1).
 // decode == true: one query per env row (rows[b] gives env and position), split-K attention.
+// last != nullptr: the last layer computes q|k|v (the KV cache) for all M rows but attention,
+// O, SwiGLU FFN and the residual only for last->rows, whose output lands in h->h_last.
 int forward_layers(vla_handle* h, int M, const RowInfo* rows_dev, bool decode, int n_tiles,
-                   int max_ctx) {
+                   int max_ctx, const LastRows* last = nullptr) {
   const vla_config& c = h->cfg;
   const int d = c.d_model, F = c.d_ffn, H = c.n_heads, hd = c.head_dim;
   const int gcls = decode ? VLA_KCLASS_GEMM_DECODE : VLA_KCLASS_GEMM_PREFILL;
@@ -274,7 +287,22 @@ int forward_layers(vla_handle* h, int M, const RowInfo* rows_dev, bool decode, i
     e.hd = hd;
     if ((rc = run_gemm(h, gcls, h->y, pd, d, h->wqkv[l], d, M, 3 * d, d, e))) return rc;
 
-    if (decode) {
+    const bool pruned = last && last->n > 0 && l + 1 == c.n_layers;
+    int Mr = M;           // rows past the attention
+    float* resid = h->h;  // their residual stream
+    if (pruned) {
+      ev = prof_begin(h, VLA_KCLASS_OTHER);
+      if ((rc = gather_rows_launch(h->q, last->idx, last->n, d, h->q_last, h->stream)) ||
+          (rc = gather_rows_launch(h->h, last->idx, last->n, d, h->h_last, h->stream)))
+        return fail(h, rc, t_err);
+      prof_end(h, ev, VLA_KCLASS_OTHER, 0, 16.0 * last->n * d);
+      ev = prof_begin(h, VLA_KCLASS_ATTN_DECODE);
+      rc = attn_decode_launch(h->q_last, h->ao, h->ao + pd, last->rows, last->n, last->max_ctx, h->kvl, l, H, hd,
+                              h->attn_chunk, h->part_o, h->part_ml, h->attn_tickets, h->stream);
+      prof_end(h, ev, VLA_KCLASS_ATTN_DECODE, 0, 0);
+      Mr = last->n;
+      resid = h->h_last;
+    } else if (decode) {
       ev = prof_begin(h, VLA_KCLASS_ATTN_DECODE);
       rc = attn_decode_launch(h->q, h->ao, h->ao + pd, rows_dev, M, max_ctx, h->kvl, l, H, hd,
                               h->attn_chunk, h->part_o, h->part_ml, h->attn_tickets, h->stream);
@@ -288,25 +316,25 @@ int forward_layers(vla_handle* h, int M, const RowInfo* rows_dev, bool decode, i
 
     EpiArgs eo;
     eo.kind = EPI_RESID;
-    eo.resid = h->h;
+    eo.resid = resid;
     eo.ldr = d;
     eo.norm_w = h->ffn_norm[l];
     eo.norm_eps = c.rms_eps;
     eo.norm_hi = h->y;
     eo.norm_lo = h->y + pd;
     eo.ldn = d;
-    if ((rc = run_gemm(h, gcls, h->ao, pd, d, h->wo[l], d, M, d, d, eo))) return rc;
+    if ((rc = run_gemm(h, gcls, h->ao, pd, d, h->wo[l], d, Mr, d, d, eo))) return rc;
 
     EpiArgs eg;
     eg.kind = EPI_SWIGLU;
     eg.out_hi = h->u;
     eg.out_lo = h->u + pf;
     eg.ldo = F;
-    if ((rc = run_gemm(h, gcls, h->y, pd, d, h->wgu[l], d, M, 2 * F, d, eg))) return rc;
+    if ((rc = run_gemm(h, gcls, h->y, pd, d, h->wgu[l], d, Mr, 2 * F, d, eg))) return rc;
 
     EpiArgs ed;
     ed.kind = EPI_RESID;
-    ed.resid = h->h;
+    ed.resid = resid;
     ed.ldr = d;
     if (l + 1 < c.n_layers) {
       ed.norm_w = h->attn_norm[l + 1];
@@ -315,7 +343,7 @@ int forward_layers(vla_handle* h, int M, const RowInfo* rows_dev, bool decode, i
       ed.norm_lo = h->y + pd;
       ed.ldn = d;
     }
-    if ((rc = run_gemm(h, gcls, h->u, pf, F, h->wdown[l], F, M, d, F, ed))) return rc;
+    if ((rc = run_gemm(h, gcls, h->u, pf, F, h->wdown[l], F, Mr, d, F, ed))) return rc;
   }
   return VLA_OK;
 }
@@ -421,6 +449,8 @@ int vla_create(const vla_config* cfg, const vla_weights* w, void* cuda_stream, v
             alloc(reinterpret_cast<void**>(&h->h_last), static_cast<size_t>(B) * d * sizeof(float)) &&
             alloc(reinterpret_cast<void**>(&h->head_in), static_cast<size_t>(B) * A * d * sizeof(float)) &&
             alloc(reinterpret_cast<void**>(&h->head_z), static_cast<size_t>(B) * A * 256 * sizeof(float)) &&
+            alloc(reinterpret_cast<void**>(&h->q_last), static_cast<size_t>(B) * d * sizeof(float)) &&
+            alloc(reinterpret_cast<void**>(&h->last_rows), static_cast<size_t>(B) * sizeof(RowInfo)) &&
             alloc(reinterpret_cast<void**>(&h->rope), static_cast<size_t>(cap) * (c.head_dim / 2) * sizeof(float2)) &&
             alloc(reinterpret_cast<void**>(&h->rows), T * sizeof(RowInfo)) &&
             alloc(reinterpret_cast<void**>(&h->tiles), static_cast<size_t>(h->max_tiles) * sizeof(AttnTile)) &&
@@ -441,7 +471,8 @@ int vla_create(const vla_config* cfg, const vla_weights* w, void* cuda_stream, v
   h->kvl.base = h->kv;
   // pinned staging
   h->stage_bytes = T * sizeof(RowInfo) + static_cast<size_t>(h->max_tiles) * sizeof(AttnTile) +
-                   2 * std::max(T, static_cast<size_t>(B) * A) * sizeof(int) + 1024;
+                   2 * std::max(T, static_cast<size_t>(B) * A) * sizeof(int) + static_cast<size_t>(B) * sizeof(RowInfo) +
+                   1024;
   for (int s = 0; s < vla_handle::kSlots; ++s) {
     if (cudaMallocHost(&h->stage_host[s], h->stage_bytes) != cudaSuccess ||
         cudaEventCreateWithFlags(&h->stage_ev[s], cudaEventDisableTiming) != cudaSuccess) {
@@ -514,11 +545,21 @@ int vla_prefill(vla_handle* h, int batch, const void* visual, int n_visual, cons
     last[b] = r - 1;
   }
   int* sidx = reinterpret_cast<int*>(tiles + n_tiles);
-  for (int b = 0; b < batch; ++b) sidx[b] = last[b];
+  RowInfo* last_rows = reinterpret_cast<RowInfo*>(sidx + batch);
+  LastRows lr;
+  lr.n = batch;
+  lr.idx = h->sidx;
+  lr.rows = h->last_rows;
+  for (int b = 0; b < batch; ++b) {
+    sidx[b] = last[b];
+    last_rows[b] = rows[last[b]];
+    lr.max_ctx = std::max(lr.max_ctx, h->len[b] + chunk[b]);
+  }
   int rc;
   if ((rc = upload(h, h->rows, rows, total * sizeof(RowInfo))) ||
       (rc = upload(h, h->tiles, tiles, n_tiles * sizeof(AttnTile))) ||
-      (rc = upload(h, h->sidx, sidx, batch * sizeof(int))))
+      (rc = upload(h, h->sidx, sidx, batch * sizeof(int))) ||
+      (rc = upload(h, h->last_rows, last_rows, batch * sizeof(RowInfo))))
     return fail(h, rc, t_err);
   cudaEventRecord(h->stage_ev[slot], h->stream);
 
@@ -527,8 +568,8 @@ int vla_prefill(vla_handle* h, int batch, const void* visual, int n_visual, cons
                        h->pending, h->embed, c.d_model, c.vocab, h->h, h->status, h->stream);
   prof_end(h, ev, VLA_KCLASS_OTHER, 0, 6.0 * total * c.d_model);
   if (rc) return fail(h, rc, t_err);
-  if ((rc = forward_layers(h, static_cast<int>(total), h->rows, false, n_tiles, 0))) return rc;
-  if ((rc = gather_rows_launch(h->h, h->sidx, batch, c.d_model, h->h_last, h->stream))) return fail(h, rc, t_err);
+  // the last layer runs past q|k|v only for each env's final row, straight into h_last
+  if ((rc = forward_layers(h, static_cast<int>(total), h->rows, false, n_tiles, 0, &lr))) return rc;
 
   for (int b = 0; b < batch; ++b) {
     h->len[b] += chunk[b];
@@ -747,7 +788,7 @@ void vla_destroy(vla_handle* h) {
   if (!h) return;
   cudaSetDevice(h->dev);
   cudaStreamSynchronize(h->stream);
-  void* bufs[] = {h->kv, h->h, h->y, h->q, h->ao, h->u, h->ws, h->h_last, h->head_in, h->head_z, h->rope,
+  void* bufs[] = {h->kv, h->h, h->y, h->q, h->ao, h->u, h->ws, h->h_last, h->head_in, h->head_z, h->q_last, h->last_rows, h->rope,
                   h->rows, h->tiles, h->sidx, h->didx, h->fed, h->pending, h->status, h->part_o,
                   h->part_ml, h->attn_tickets};
   for (void* p : bufs)
