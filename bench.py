@@ -34,6 +34,15 @@ sys.path.insert(0, ROOT)
 WORKLOAD = "7b_b64_ragged_score"
 
 
+# DRAM bytes of one launch of the dominant kernel from an ncu capture (set to None whenever
+# that kernel changes): gemm_tc2_kernel, the q|k|v projection of this step's prefill
+# (18385 x 12288 x 4096, case pair_prefill_qkv_18385; fp32 output in the case).
+PROFILED_TRAFFIC = {"bytes": 2.975106e9 + 0.877365e9,
+                    "launch": "gemm_tc2_kernel q|k|v, M=18385 N=12288 K=4096",
+                    "algorithmic_bytes": 2.0 * 18385 * 4096 * 2 + 2.0 * 12288 * 4096 + 4.0 * 18385 * 12288,
+                    "profile": "profiles/gemm_tc2_prefill_qkv_18385x12288x4096.md"}
+
+
 def phase_work(sh, B, n_visual, lengths):
     """Algorithmic work of one step's phases (7B: 6.476e9 matrix parameters, 16 KB of fp16 K+V
     per token per layer).  Prefill FLOPs count what the method needs: every row through every
@@ -206,6 +215,8 @@ CASES = {
     "pair_prefill_qkv": (4608, 12288, 4096, 256, 1, True),
     "pair_prefill_down": (4608, 4096, 11008, 256, 1, True),
     "pair_prefill_gate_up_18k": (18432, 22016, 4096, 256, 1, True),
+    # the q|k|v launch of the bench step's prefill (64 envs, 18385 rows)
+    "pair_prefill_qkv_18385": (18385, 12288, 4096, 256, 1, True),
     "gemm_prefill_gate_up_18k": (18432, 22016, 4096, 256, 1, True),
     # score-pass shapes (64 envs x 6 teacher-forced rows): tile / split choices
     "gemm_score_qkv_bn256": (384, 12288, 4096, 256, 1, True),
@@ -472,7 +483,9 @@ def main():
         achieved = gp["flops"] / (gp["ms"] / 1e3) / 1e12
         roof = {"bound": "tensor", "kernel": "gemm_tc (prefill/score projections)",
                 "achieved": achieved, "peak": tf_sus, "unit": "TFLOP/s", "frac": achieved / tf_sus,
-                "peak_kind": f"{peak_kind} bf16 sustained", "traffic": None,
+                "peak_kind": f"{peak_kind} bf16 sustained",
+                "traffic": PROFILED_TRAFFIC["bytes"] if PROFILED_TRAFFIC else None,
+                "traffic_launch": PROFILED_TRAFFIC,
                 "launches": gp["launches"], "avg_launch_ms": gp["ms"] / max(1, gp["launches"])}
     roof_dec = None
     if gd["ms"] > 0:

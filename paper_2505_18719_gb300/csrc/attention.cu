@@ -274,8 +274,11 @@ __global__ void __launch_bounds__(128) attn_chunk_mma_kernel(const float* __rest
 // output) per range.  The last CTA of an (env, head) to finish (a ticket on counters[b * H +
 // head], no waiting) merges the S partials in range order and writes the normalised output as
 // the bf16 pair; with S == 1 the CTA writes it directly.
-template <int HD>
-__global__ void __launch_bounds__(128) attn_decode_kernel(const float* __restrict__ q,
+// NW = 2 warps per CTA at <= 64 registers: 16 CTAs fit on an SM, so the 2048 (env, head) CTAs
+// of a 64-env, 32-head step are all resident at once (one wave, no tail).
+constexpr int kDecodeWarps = 2;
+template <int HD, int NW = kDecodeWarps>
+__global__ void __launch_bounds__(NW * 32, 512 / NW) attn_decode_kernel(const float* __restrict__ q,
                                                           const RowInfo* __restrict__ rows,
                                                           KVLayout kv, int layer, int H,
                                                           int chunk, int S, float scale_log2,
@@ -287,8 +290,9 @@ __global__ void __launch_bounds__(128) attn_decode_kernel(const float* __restric
   constexpr int LPK = HD / 8;     // lanes per key row (8 fp16 = 16 bytes per lane)
   constexpr int KPI = 32 / LPK;   // key rows per warp instruction
   constexpr int U = 4;            // key rows per lane group loaded ahead
-  __shared__ float s_m[4][KPI], s_l[4][KPI];
-  __shared__ float s_o[4][KPI][HD];
+  constexpr int NT = NW * 32;      // threads
+  __shared__ float s_m[NW][KPI], s_l[NW][KPI];
+  __shared__ float s_o[NW][KPI][HD];
 
   pdl_launch_dependents();
   pdl_wait();
@@ -322,7 +326,7 @@ __global__ void __launch_bounds__(128) attn_decode_kernel(const float* __restric
 #pragma unroll
   for (int e = 0; e < 8; ++e) o[e] = 0.f;
 
-  for (int key0 = k_begin + warp * KPI * U; key0 < k_end; key0 += 4 * KPI * U) {
+  for (int key0 = k_begin + warp * KPI * U; key0 < k_end; key0 += NW * KPI * U) {
     uint4 kk[U], vv[U];
 #pragma unroll
     for (int u = 0; u < U; ++u) {
@@ -375,10 +379,10 @@ __global__ void __launch_bounds__(128) attn_decode_kernel(const float* __restric
   __syncthreads();
   // merge the 4 * KPI partial states in a fixed order
   float M = -INFINITY;
-  for (int w = 0; w < 4; ++w)
+  for (int w = 0; w < NW; ++w)
     for (int k = 0; k < KPI; ++k) M = fmaxf(M, s_m[w][k]);
   float L = 0.f;
-  for (int w = 0; w < 4; ++w)
+  for (int w = 0; w < NW; ++w)
     for (int k = 0; k < KPI; ++k)
       if (s_m[w][k] != -INFINITY) L += s_l[w][k] * exp2f(s_m[w][k] - M);
   const size_t bh = static_cast<size_t>(b) * H + head;
@@ -386,7 +390,7 @@ __global__ void __launch_bounds__(128) attn_decode_kernel(const float* __restric
   if (S == 1) {
     for (int c = threadIdx.x; c < HD; c += blockDim.x) {
       float acc = 0.f;
-      for (int w = 0; w < 4; ++w)
+      for (int w = 0; w < NW; ++w)
         for (int k = 0; k < KPI; ++k)
           if (s_m[w][k] != -INFINITY) acc += s_o[w][k][c] * exp2f(s_m[w][k] - M);
       bf16 hi, lo;
@@ -399,7 +403,7 @@ __global__ void __launch_bounds__(128) attn_decode_kernel(const float* __restric
   const size_t slot = bh * S + split;
   for (int c = threadIdx.x; c < HD; c += blockDim.x) {
     float acc = 0.f;
-    for (int w = 0; w < 4; ++w)
+    for (int w = 0; w < NW; ++w)
       for (int k = 0; k < KPI; ++k)
         if (s_m[w][k] != -INFINITY) acc += s_o[w][k][c] * exp2f(s_m[w][k] - M);
     part_o[slot * HD + c] = acc;
@@ -417,23 +421,23 @@ __global__ void __launch_bounds__(128) attn_decode_kernel(const float* __restric
   float Mx = -INFINITY;
   for (int s = 0; s < S; ++s) Mx = fmaxf(Mx, __ldcg(&part_ml[bh * S + s].x));
   float Lt = 0.f;
-  float acc[(HD + 127) / 128];
+  float acc[(HD + NT - 1) / NT];
 #pragma unroll
-  for (int i = 0; i < (HD + 127) / 128; ++i) acc[i] = 0.f;
+  for (int i = 0; i < (HD + NT - 1) / NT; ++i) acc[i] = 0.f;
   for (int s = 0; s < S; ++s) {
     const float2 ml = __ldcg(&part_ml[bh * S + s]);
     if (ml.x == -INFINITY) continue;
     const float w = exp2f(ml.x - Mx);
     Lt += ml.y * w;
 #pragma unroll
-    for (int i = 0; i < (HD + 127) / 128; ++i) {
-      const int c = threadIdx.x + i * 128;
+    for (int i = 0; i < (HD + NT - 1) / NT; ++i) {
+      const int c = threadIdx.x + i * NT;
       if (c < HD) acc[i] += __ldcg(&part_o[(bh * S + s) * HD + c]) * w;
     }
   }
 #pragma unroll
-  for (int i = 0; i < (HD + 127) / 128; ++i) {
-    const int c = threadIdx.x + i * 128;
+  for (int i = 0; i < (HD + NT - 1) / NT; ++i) {
+    const int c = threadIdx.x + i * NT;
     if (c < HD) {
       bf16 hi, lo;
       split_bf16(acc[i] / Lt, hi, lo);
@@ -489,10 +493,10 @@ int attn_decode_launch(const float* q, bf16* out_hi, bf16* out_lo, const RowInfo
   const float scale_log2 = 1.4426950408889634f / sqrtf(static_cast<float>(hd));
   dim3 grid(S, H, B);
   if (hd == 128) {
-    VLA_CUDA_TRY(launch_pdl(attn_decode_kernel<128>, grid, dim3(128), 0, stream, q, rows, kv, layer, H,
+    VLA_CUDA_TRY(launch_pdl(attn_decode_kernel<128>, grid, dim3(kDecodeWarps * 32), 0, stream, q, rows, kv, layer, H,
                             c, S, scale_log2, part_o, part_ml, counters, out_hi, out_lo));
   } else if (hd == 64) {
-    VLA_CUDA_TRY(launch_pdl(attn_decode_kernel<64>, grid, dim3(128), 0, stream, q, rows, kv, layer, H,
+    VLA_CUDA_TRY(launch_pdl(attn_decode_kernel<64>, grid, dim3(kDecodeWarps * 32), 0, stream, q, rows, kv, layer, H,
                             c, S, scale_log2, part_o, part_ml, counters, out_hi, out_lo));
   } else {
     return VLA_ERR_UNSUPPORTED;
