@@ -829,16 +829,16 @@ struct TileSum {
         }
     }
   }
-  // columns n .. n+3 (n % 4 == 0) of row m
+  // columns n .. n+3 (n % 4 == 0) of row m; six CTAs' partials in flight
   __device__ __forceinline__ float4 sum4(int m) const {
     float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-    for (int c = c0; c <= c1; c += 4) {
-      float4 v[4];
+    for (int c = c0; c <= c1; c += 6) {
+      float4 v[6];
 #pragma unroll
-      for (int u = 0; u < 4; ++u)
+      for (int u = 0; u < 6; ++u)
         v[u] = (c + u <= c1) ? *reinterpret_cast<const float4*>(row(c + u, m)) : make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll
-      for (int u = 0; u < 4; ++u)
+      for (int u = 0; u < 6; ++u)
         if (c + u <= c1) {
           acc.x += v[u].x;
           acc.y += v[u].y;
@@ -849,6 +849,40 @@ struct TileSum {
     return acc;
   }
 };
+
+// Two columns' sums (each as TileSum::sum) with both columns' loads in flight together.
+__device__ __forceinline__ void sum_pair(const TileSum& A, const TileSum& B, int m0, int M, float (&a)[kMR],
+                                         float (&b)[kMR]) {
+#pragma unroll
+  for (int j = 0; j < kMR; ++j) a[j] = b[j] = 0.f;
+  const int na = A.c1 - A.c0 + 1, nb = B.c1 - B.c0 + 1;
+  const int n = na > nb ? na : nb;
+  for (int i = 0; i < n; i += 4) {
+    float va[4][kMR], vb[4][kMR];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const bool ia = i + u < na, ib = i + u < nb;
+      const float* sa = A.row(ia ? A.c0 + i + u : A.c1, m0);
+      const float* sb = B.row(ib ? B.c0 + i + u : B.c1, m0);
+#pragma unroll
+      for (int j = 0; j < kMR; ++j) {
+        va[u][j] = (ia && m0 + j < M) ? sa[j * 256] : 0.f;
+        vb[u][j] = (ib && m0 + j < M) ? sb[j * 256] : 0.f;
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      if (i + u < na) {
+#pragma unroll
+        for (int j = 0; j < kMR; ++j) a[j] += va[u][j];
+      }
+      if (i + u < nb) {
+#pragma unroll
+        for (int j = 0; j < kMR; ++j) b[j] += vb[u][j];
+      }
+    }
+  }
+}
 
 __device__ __forceinline__ bool next_item(int& item, int nx, int ny, int& x, int& y) {
   if (item >= nx * ny) return false;
@@ -892,8 +926,7 @@ __global__ void stream_reduce_swiglu_kernel(StreamSrc src, int M, int F, bf16* o
     if (f >= F) continue;
     const int m0 = by * kMR;
     float g[kMR], u[kMR];
-    TileSum(src, f).sum(m0, M, g);
-    TileSum(src, f + F).sum(m0, M, u);
+    sum_pair(TileSum(src, f), TileSum(src, f + F), m0, M, g, u);
 #pragma unroll
     for (int j = 0; j < kMR; ++j) {
       if (m0 + j >= M) break;
@@ -922,8 +955,7 @@ __global__ void stream_reduce_qkv_kernel(StreamSrc src, int M, EpiArgs e) {
     const int head = (c - sec * d) / hd;
     const int m0 = by * kMR;
     float a[kMR], b[kMR];
-    TileSum(src, c).sum(m0, M, a);
-    TileSum(src, c + half).sum(m0, M, b);
+    sum_pair(TileSum(src, c), TileSum(src, c + half), m0, M, a, b);
 #pragma unroll
     for (int j = 0; j < kMR; ++j) {
       const int m = m0 + j;
@@ -954,8 +986,9 @@ __global__ void stream_reduce_qkv_kernel(StreamSrc src, int M, EpiArgs e) {
 
 // grid (M), 1024 threads (N % 4 == 0): h[m][n] += sum, then the RMSNorm of the updated row
 // times w as the bf16 pair y_hi / y_lo (the next GEMM's A).  The row sums are in the same
-// order as stream_reduce_f32_kernel's.
-__global__ void __launch_bounds__(1024) stream_reduce_resid_norm_kernel(StreamSrc src, int N, float* h,
+// order as stream_reduce_f32_kernel's.  At most 48 registers: with one 1024-thread CTA on an
+// SM, the next weight-streaming GEMM's CTA (192 threads x 40) still fits beside it.
+__global__ void __maxnreg__(48) stream_reduce_resid_norm_kernel(StreamSrc src, int N, float* h,
                                                                          int ldh, const bf16* w, float eps,
                                                                          bf16* y_hi, bf16* y_lo, int ldy) {
   pdl_launch_dependents();
