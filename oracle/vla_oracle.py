@@ -216,6 +216,7 @@ class HeadOut:
     action: float             # bin centre
     logprobs: torch.Tensor    # fp64 [256] log softmax(z / T)   (T = 0: T = 1 values)
     margin: float             # top-1 minus top-2 of the perturbed score s
+    entropy: float = 0.0      # -sum_k p_k log p_k of the same distribution
 
 
 def bin_centre(k: int, n_bins: int = 256) -> float:
@@ -256,12 +257,76 @@ def sample_bins(z: torch.Tensor, temperature: float, u: Optional[torch.Tensor]):
     return k, lp, margin
 
 
+def token_entropy(z: torch.Tensor, temperature: float) -> float:
+    """Entropy of one action token's distribution over the bins (the rollout entropy the
+    paper tracks in its training dynamics, §5): H = -sum_k p_k log p_k with p = softmax(z/T),
+    the distribution the sampler draws from; T = 0 uses T = 1, as the log-probs do."""
+    zt = z / temperature if temperature > 0.0 else z
+    lp = zt - torch.logsumexp(zt, dim=0)
+    return float(-(torch.exp(lp) * lp).sum())
+
+
 def action_head(shape: Shape, W: Weights, h_last: torch.Tensor, temperature: float,
                 u: Optional[torch.Tensor]) -> HeadOut:
     """Logits, sample, log-probs and the de-tokenised action for one hidden state."""
     z = head_logits(shape, W, h_last)
     k, lp, margin = sample_bins(z, temperature, u)
-    return HeadOut(z, k, shape.vocab - shape.n_bins + k, bin_centre(k, shape.n_bins), lp, margin)
+    return HeadOut(z, k, shape.vocab - shape.n_bins + k, bin_centre(k, shape.n_bins), lp, margin,
+                   token_entropy(z, temperature))
+
+
+# =========================================================================== value head
+def value_head(shape: Shape, W: Weights, h_last: torch.Tensor, w_value: torch.Tensor,
+               bias: float) -> float:
+    """V(o_t, v_t^in) of Algorithm 1 ("value model estimates") for a homogeneous value model
+    (§3.2 / the pipeline figure: the same decoder as the policy): the final RMSNorm of the
+    last prefix row, then one linear output, V = y . w_value + bias."""
+    y = rms_norm(h_last, W.final_norm, shape.rms_eps)
+    return float(y @ f64(w_value)) + float(bias)
+
+
+# =========================================================================== learning phase
+def gae(rewards, values, dones, gamma: float, lam: float):
+    """Generalised advantage estimation (Algorithm 1, "compute advantages"; §3.4 cites
+    Schulman et al. 2015) over M steps of B envs, walking t = M-1 .. 0:
+
+      delta_t = r_t + gamma * (1 - done_t) * V_{t+1} - V_t
+      A_t     = delta_t + gamma * lam * (1 - done_t) * A_{t+1},   A_M = 0
+      R_t     = A_t + V_t                        (the value model's regression target)
+
+    rewards [M, B]; values [M + 1, B] = V_0 .. V_M (V_M bootstraps the unfinished tail);
+    dones [M, B]: 1 where the episode ended with step t (then nothing past t is used).
+    Returns (A [M, B], R [M, B]) in fp64."""
+    r = torch.as_tensor(rewards, dtype=F64)
+    v = torch.as_tensor(values, dtype=F64)
+    d = torch.as_tensor(dones, dtype=F64)
+    M = r.shape[0]
+    adv = torch.zeros_like(r)
+    nxt = torch.zeros_like(r[0])
+    for t in range(M - 1, -1, -1):
+        live = 1.0 - d[t]
+        delta = r[t] + gamma * live * v[t + 1] - v[t]
+        nxt = delta + gamma * lam * live * nxt
+        adv[t] = nxt
+    return adv, adv + v[:M]
+
+
+def ppo_clip_objective(lp_new, lp_old, adv, eps: float):
+    """The clipped PPO objective of Eq. 2 over N samples (env-steps):
+
+      log pi(a_t | .) = sum_i log pi(v_out,t,i | .)        (Eq. 1: the 7 token log-probs)
+      rho_t = exp(log pi_theta(a_t | .) - log pi_theta_old(a_t | .))
+      L     = mean_t min(rho_t A_t, clip(rho_t, 1 - eps, 1 + eps) A_t)
+
+    lp_new, lp_old [N, A] token log-probs; adv [N].  Returns (L, rho [N], fraction of samples
+    with |rho - 1| > eps) in fp64.  L is the objective to maximise; a loss is -L."""
+    ln = torch.as_tensor(lp_new, dtype=F64).sum(dim=-1)
+    lo = torch.as_tensor(lp_old, dtype=F64).sum(dim=-1)
+    a = torch.as_tensor(adv, dtype=F64)
+    rho = torch.exp(ln - lo)
+    obj = torch.minimum(rho * a, torch.clamp(rho, 1.0 - eps, 1.0 + eps) * a)
+    clipped = ((rho - 1.0).abs() > eps).to(F64)
+    return float(obj.mean()), rho, float(clipped.mean())
 
 
 # =========================================================================== engine
@@ -369,7 +434,7 @@ class Oracle:
         out = {"tokens": np.zeros((n, A), np.int64), "bins": np.zeros((n, A), np.int64),
                "actions": np.zeros((n, A), np.float64), "logprobs": np.zeros((n, A)),
                "sampled_logprobs": np.zeros((n, A)), "logits": np.zeros((n, A, sh.n_bins)),
-               "margins": np.zeros((n, A))}
+               "margins": np.zeros((n, A)), "entropy": np.zeros((n, A))}
         for b in env_ids:
             self._truncate(b, self.envs[b].len_prefill)
         h_cur = [self.envs[b].h_last_prefill for b in env_ids]
@@ -386,6 +451,7 @@ class Oracle:
                 out["logprobs"][j, i] = float(ho.logprobs[kk])
                 out["logits"][j, i] = ho.logits.numpy()
                 out["margins"][j, i] = ho.margin
+                out["entropy"][j, i] = ho.entropy
                 fed[j] = tok
             if i == A - 1:
                 break
@@ -406,6 +472,7 @@ class Oracle:
         chunks = [self.W.embed_rows([int(t) for t in tokens[j, :A - 1]]) for j in range(n)]
         hs = self._forward(env_ids, chunks)
         lp = np.zeros((n, A))
+        ent = np.zeros((n, A))
         logits = np.zeros((n, A, sh.n_bins))
         base = sh.vocab - sh.n_bins
         for j, b in enumerate(env_ids):
@@ -413,9 +480,15 @@ class Oracle:
             for i in range(A):
                 ho = action_head(sh, self.W, hrow[i], temperature, None)
                 lp[j, i] = float(ho.logprobs[int(tokens[j, i]) - base])
+                ent[j, i] = ho.entropy
                 logits[j, i] = ho.logits.numpy()
             self.envs[b].pending = int(tokens[j, A - 1])
-        return {"logprobs": lp, "logits": logits}
+        return {"logprobs": lp, "logits": logits, "entropy": ent}
+
+    def value(self, env_ids: Sequence[int], w_value: torch.Tensor, bias: float) -> np.ndarray:
+        """Value-model estimates at each env's latest prefill (the state of the step)."""
+        return np.array([value_head(self.shape, self.W, self.envs[b].h_last_prefill, w_value, bias)
+                         for b in env_ids])
 
     # ------------------------------------------------------------------ full recompute
     def recompute_last_hidden(self, b: int, extra_ids: Sequence[int] = ()) -> torch.Tensor:

@@ -7,6 +7,7 @@ that a pin catches each of them.
 """
 import math
 import os
+import types
 
 import numpy as np
 import pytest
@@ -355,6 +356,126 @@ def test_head_token_and_action_mapping():
     assert ho.action == -1 + (2 * ho.k + 1) / 256
 
 
+# ============================================================================ entropy, value, GAE, PPO
+def test_entropy_closed_forms():
+    """Rollout entropy (§5): uniform logits give log 256 at any T; a two-level z has the closed
+    form -p1 log p1 - 255 p0 log p0; H(z, T) = H(z / T, 1); 0 <= H <= log 256."""
+    z0 = torch.zeros(256, dtype=torch.float64)
+    for T in (0.0, 0.5, 1.0, 1.5):
+        assert abs(O.token_entropy(z0, T) - math.log(256.0)) < 1e-12
+    a = 3.0
+    z = torch.zeros(256, dtype=torch.float64)
+    z[17] = a
+    p1 = math.exp(a) / (math.exp(a) + 255.0)
+    p0 = 1.0 / (math.exp(a) + 255.0)
+    want = -p1 * math.log(p1) - 255.0 * p0 * math.log(p0)
+    assert abs(O.token_entropy(z, 1.0) - want) < 1e-12
+    g = torch.Generator().manual_seed(5)
+    zr = torch.randn(256, generator=g, dtype=torch.float64) * 4.0
+    for T in (0.5, 1.5):
+        assert abs(O.token_entropy(zr, T) - O.token_entropy(zr / T, 1.0)) < 1e-12
+        h = O.token_entropy(zr, T)
+        assert 0.0 <= h <= math.log(256.0) + 1e-12
+    z[17] = 1e4
+    assert O.token_entropy(z, 1.0) < 1e-12
+
+
+def test_value_head_closed_form():
+    """V = RMSNorm(h_last) . w_value + b: a constant hidden row c normalises to sign(c) times
+    the final-norm gains, so V = sign(c) * sum(g * w) + b; V is affine in (w, b)."""
+    d = 8
+    sh = O.Shape(1, d, 2, 4, 16, 300)
+    g = torch.tensor([1.0, 0.5, 2.0, 1.0, 1.0, 0.25, 1.0, 1.0], dtype=torch.float64)
+    W = types.SimpleNamespace(final_norm=g)
+    w = torch.tensor([0.5, -1.0, 0.25, 2.0, 0.0, 4.0, -0.5, 1.0], dtype=torch.float64)
+    for c in (3.0, -0.75):
+        h = torch.full((d,), c, dtype=torch.float64)
+        want = math.copysign(1.0, c) * float((g * w).sum()) / math.sqrt(1.0 + sh.rms_eps / c ** 2) + 0.125
+        assert abs(O.value_head(sh, W, h, w, 0.125) - want) < 1e-12
+    h = torch.randn(d, generator=torch.Generator().manual_seed(3), dtype=torch.float64)
+    v1, v2 = O.value_head(sh, W, h, w, 0.0), O.value_head(sh, W, h, 2.0 * w, 0.0)
+    assert abs(v2 - 2.0 * v1) < 1e-12
+    assert abs(O.value_head(sh, W, h, w, 1.5) - v1 - 1.5) < 1e-12
+
+
+def _golden_rows(name):
+    rows = []
+    for line in open(os.path.join(GOLDEN, name)):
+        line = line.strip()
+        if line and not line.startswith("#"):
+            rows.append(line.split())
+    return rows
+
+
+def test_gae_golden_fixture():
+    rows = _golden_rows("gae_m3.txt")
+    r = [[float(x[1])] for x in rows[:3]]
+    v = [[float(x[2])] for x in rows[:4]]
+    dn = [[float(x[3])] for x in rows[:3]]
+    adv, ret = O.gae(r, v, dn, 0.5, 0.5)
+    for t in range(3):
+        assert float(adv[t, 0]) == float(rows[t][4])
+        assert float(ret[t, 0]) == float(rows[t][5])
+
+
+def test_gae_special_cases():
+    """lambda = 1, no terminal: A_t = sum_k gamma^k r_{t+k} + gamma^(M-t) V_M - V_t (discounted
+    return minus value); lambda = 0: A_t is the one-step TD error; a terminal at t makes
+    A_t = r_t - V_t; envs are independent columns."""
+    g = torch.Generator().manual_seed(11)
+    M, B, gam = 6, 3, 0.9
+    r = torch.randn(M, B, generator=g, dtype=torch.float64)
+    v = torch.randn(M + 1, B, generator=g, dtype=torch.float64)
+    zero = torch.zeros(M, B, dtype=torch.float64)
+    adv, _ = O.gae(r, v, zero, gam, 1.0)
+    for t in range(M):
+        ret = sum(gam ** k * r[t + k] for k in range(M - t)) + gam ** (M - t) * v[M]
+        assert torch.allclose(adv[t], ret - v[t], atol=1e-12)
+    adv0, _ = O.gae(r, v, zero, gam, 0.0)
+    assert torch.allclose(adv0, r + gam * v[1:] - v[:M], atol=1e-12)
+    dn = zero.clone()
+    dn[2, 1] = 1.0
+    adv2, _ = O.gae(r, v, dn, gam, 0.95)
+    assert abs(float(adv2[2, 1]) - float(r[2, 1] - v[2, 1])) < 1e-12
+    assert torch.allclose(adv2[:, 0], O.gae(r[:, :1], v[:, :1], zero[:, :1], gam, 0.95)[0][:, 0], atol=1e-12)
+
+
+def test_ppo_clip_golden_fixture():
+    rows = _golden_rows("ppo_clip_eps02.txt")
+    rho = [float(x[0]) for x in rows]
+    adv = [float(x[1]) for x in rows]
+    lp_old = torch.full((4, 7), -1.25, dtype=torch.float64)
+    lp_new = lp_old + torch.tensor([math.log(x) / 7.0 for x in rho], dtype=torch.float64)[:, None]
+    obj, rr, frac = O.ppo_clip_objective(lp_new, lp_old, adv, 0.2)
+    assert abs(obj - 0.725) < 1e-12
+    assert abs(frac - 0.75) < 1e-12
+    assert torch.allclose(rr, torch.tensor(rho, dtype=torch.float64), atol=1e-12)
+
+
+def test_ppo_clip_unclipped_equals_ratio_times_advantage():
+    """Inside the trust region the objective is the plain importance-weighted advantage, and at
+    rho = 1 it is mean(A)."""
+    g = torch.Generator().manual_seed(2)
+    lp_old = -torch.rand(10, 7, generator=g, dtype=torch.float64) * 3.0
+    adv = torch.randn(10, generator=g, dtype=torch.float64)
+    obj, _, frac = O.ppo_clip_objective(lp_old, lp_old, adv, 0.2)
+    assert abs(obj - float(adv.mean())) < 1e-12 and frac == 0.0
+    lp_new = lp_old + 0.01 / 7.0
+    obj2, rho, _ = O.ppo_clip_objective(lp_new, lp_old, adv, 0.2)
+    assert abs(obj2 - float((rho * adv).mean())) < 1e-12
+
+
+def test_decode_and_score_report_entropy_of_their_logits():
+    orc = _micro_oracle(1)
+    _prefill(orc, [0], 3, [2])
+    out = orc.decode([0], _uniforms(1), 1.5)
+    sc = orc.score([0], torch.tensor(out["tokens"]), 1.5)
+    for i in range(MICRO.action_dim):
+        z = torch.tensor(out["logits"][0, i], dtype=torch.float64)
+        assert abs(out["entropy"][0, i] - O.token_entropy(z, 1.5)) < 1e-12
+        assert abs(sc["entropy"][0, i] - out["entropy"][0, i]) < 1e-12
+
+
 # ============================================================================ mutations
 def _bruteforce_gap():
     w = micro_weights()
@@ -412,3 +533,26 @@ def test_mutation_untempered_sampling_is_caught():
     mask = p * n >= 5
     chi2 = float(np.sum((counts[mask] - p[mask] * n) ** 2 / (p[mask] * n)))
     assert scipy_stats.chi2.sf(chi2, int(mask.sum()) - 1) < 1e-6
+
+
+def test_mutation_gae_without_terminal_mask_is_caught(monkeypatch):
+    good = O.gae
+
+    def bad_gae(rewards, values, dones, gamma, lam):
+        return good(rewards, values, torch.zeros_like(torch.as_tensor(dones, dtype=torch.float64)), gamma, lam)
+    monkeypatch.setattr(O, "gae", bad_gae)
+    with pytest.raises(AssertionError):
+        test_gae_golden_fixture()
+
+
+def test_mutation_ppo_max_instead_of_min_is_caught(monkeypatch):
+    def bad(lp_new, lp_old, adv, eps):
+        ln = torch.as_tensor(lp_new, dtype=torch.float64).sum(-1)
+        lo = torch.as_tensor(lp_old, dtype=torch.float64).sum(-1)
+        a = torch.as_tensor(adv, dtype=torch.float64)
+        rho = torch.exp(ln - lo)
+        obj = torch.maximum(rho * a, torch.clamp(rho, 1 - eps, 1 + eps) * a)
+        return float(obj.mean()), rho, float(((rho - 1).abs() > eps).to(torch.float64).mean())
+    monkeypatch.setattr(O, "ppo_clip_objective", bad)
+    with pytest.raises(AssertionError):
+        test_ppo_clip_golden_fixture()
