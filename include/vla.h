@@ -130,6 +130,43 @@ int vla_decode_actions(vla_handle* h, const float* uniforms, float temperature,
 int vla_score_actions(vla_handle* h, const int32_t* tokens, float temperature,
                       float* logprobs_out, float* logits_out);
 
+/* Rollout entropy (the training-dynamics quantity of §5): H = -sum_k p_k log p_k of each
+ * action token's 256-bin distribution in the latest vla_decode_actions or vla_score_actions
+ * call on this handle, at that call's temperature (T == 0: the T = 1 distribution, as for
+ * the log-probs).  entropy_out device f32 [B, action_dim]; asynchronous on the handle's
+ * stream.  VLA_ERR_STATE if neither has run since the latest prefill. */
+int vla_action_entropy(vla_handle* h, float* entropy_out);
+
+/* Value-model estimate V_t of Algorithm 1 at each env's latest prefill (the step's state),
+ * for a handle whose decoder is a homogeneous value model (the policy's architecture with
+ * one scalar output): V_b = RMSNorm(h_b; final_norm) . w_value + bias, h_b the last
+ * prefix row's final hidden state.  w_value device bf16 [d_model] (read during the call);
+ * values_out device f32 [B].  VLA_ERR_STATE before any prefill. */
+int vla_value(vla_handle* h, const void* w_value, float bias, float* values_out);
+
+/* Generalised advantage estimation (Algorithm 1, "compute advantages"), all device f32:
+ *   rewards [M, B], values [M + 1, B] (V_0 .. V_M; V_M bootstraps the unfinished tail),
+ *   dones [M, B] (1 where the episode ended with step t, else 0);
+ *   delta_t = r_t + gamma (1 - done_t) V_{t+1} - V_t,
+ *   A_t = delta_t + gamma lam (1 - done_t) A_{t+1} (A_M = 0) -> adv_out [M, B];
+ *   returns_out [M, B] = A_t + V_t, or NULL.
+ * Needs M, B >= 1 and 0 <= gamma, lam <= 1 (else VLA_ERR_ARG).  Asynchronous on cuda_stream. */
+int vla_gae(const float* rewards, const float* values, const float* dones, int M, int B,
+            float gamma, float lam, float* adv_out, float* returns_out, void* cuda_stream);
+
+/* The clipped PPO objective of Eq. 2 over N samples (env-steps), all device f32:
+ *   lp_new, lp_old [N, A]: token log-probs under the current and the rollout policy; an
+ *   action's log-prob is their sum over the A tokens (Eq. 1); adv [N];
+ *   rho = exp(sum lp_new - sum lp_old);
+ *   objective_out [1] = mean over samples of min(rho A, clip(rho, 1 - eps, 1 + eps) A)
+ *   (to maximise; a loss is its negative); ratio_out [N] (rho) and clip_frac_out [1]
+ *   (share of samples with |rho - 1| > eps) may be NULL.
+ * One fixed-order reduction: repeated calls give identical results.  Needs N, A >= 1 and
+ * eps >= 0 (else VLA_ERR_ARG).  Asynchronous on cuda_stream. */
+int vla_ppo_clip(const float* lp_new, const float* lp_old, const float* adv, int N, int A,
+                 float eps, float* objective_out, float* ratio_out, float* clip_frac_out,
+                 void* cuda_stream);
+
 /* Reset environments (episode end, Algorithm 1 terminal flags): env_mask HOST uint8
  * [max_batch], nonzero = reset; NULL = all.  A reset env has an empty context. */
 int vla_reset(vla_handle* h, const uint8_t* env_mask);

@@ -160,13 +160,22 @@ __global__ void __launch_bounds__(256) head_sample_kernel(const HeadArgs a) {
   }
   const float e = expf(zt - zmax);
   float se = warp_sum(e);
+  float sez = warp_sum(e * (zt - zmax));  // for the entropy: sum_k p_k (zt_k - zmax) * sum_e
   __syncthreads();  // red_f reuse
-  if (lane == 0) red_f[warp] = se;
+  if (lane == 0) {
+    red_f[warp] = se;
+    red_m[warp] = sez;
+  }
   __syncthreads();
-  float sum_e = 0.f;
+  float sum_e = 0.f, sum_ez = 0.f;
 #pragma unroll
-  for (int w = 0; w < 8; ++w) sum_e += red_f[w];
+  for (int w = 0; w < 8; ++w) {
+    sum_e += red_f[w];
+    sum_ez += red_m[w];
+  }
   const float lse = zmax + logf(sum_e);
+  // rollout entropy of this token's bin distribution: H = lse - sum_k p_k zt_k
+  if (tid == 0 && a.entropy_out) a.entropy_out[out_i] = logf(sum_e) - sum_ez / sum_e;
 
   if (a.logits_out) a.logits_out[static_cast<size_t>(out_i) * 256 + k] = z;
   if (!isfinite(z)) atomicOr(a.status, VLA_STATUS_NONFINITE);

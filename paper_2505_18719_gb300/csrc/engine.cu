@@ -113,6 +113,8 @@ struct vla_handle {
   float* h_last = nullptr;
   float* head_in = nullptr;
   float* head_z = nullptr;  // action-bin logits [B * A, 256]
+  float* head_entropy = nullptr;  // entropy of each action token's distribution [B, A]
+  bool entropy_valid = false;     // set by decode / score, cleared by prefill / reset
   float* q_last = nullptr;  // last layer of a prefill: queries of each env's final row [B, d]
   RowInfo* last_rows = nullptr;  // and those rows' RowInfo [B]
   float2* rope = nullptr;
@@ -452,6 +454,7 @@ int vla_create(const vla_config* cfg, const vla_weights* w, void* cuda_stream, v
             alloc(reinterpret_cast<void**>(&h->h_last), static_cast<size_t>(B) * d * sizeof(float)) &&
             alloc(reinterpret_cast<void**>(&h->head_in), static_cast<size_t>(B) * A * d * sizeof(float)) &&
             alloc(reinterpret_cast<void**>(&h->head_z), static_cast<size_t>(B) * A * 256 * sizeof(float)) &&
+            alloc(reinterpret_cast<void**>(&h->head_entropy), static_cast<size_t>(B) * A * sizeof(float)) &&
             alloc(reinterpret_cast<void**>(&h->q_last), static_cast<size_t>(B) * d * sizeof(float)) &&
             alloc(reinterpret_cast<void**>(&h->last_rows), static_cast<size_t>(B) * sizeof(RowInfo)) &&
             alloc(reinterpret_cast<void**>(&h->rope), static_cast<size_t>(cap) * (c.head_dim / 2) * sizeof(float2)) &&
@@ -581,6 +584,7 @@ int vla_prefill(vla_handle* h, int batch, const void* visual, int n_visual, cons
     h->prefilled[b] = 1;
   }
   h->active_batch = batch;
+  h->entropy_valid = false;
   return VLA_OK;
 }
 
@@ -616,6 +620,7 @@ int vla_decode_actions(vla_handle* h, const float* uniforms, float temperature, 
 
   HeadArgs ha;
   ha.z = h->head_z;
+  ha.entropy_out = h->head_entropy;
   ha.B = B;
   ha.n_pos = 1;
   ha.A = A;
@@ -660,6 +665,7 @@ int vla_decode_actions(vla_handle* h, const float* uniforms, float temperature, 
     h->len[b] = h->len_prefill[b] + (A - 1);
     h->has_pending[b] = 1;
   }
+  h->entropy_valid = true;
   return VLA_OK;
 }
 
@@ -714,6 +720,7 @@ int vla_score_actions(vla_handle* h, const int32_t* tokens, float temperature, f
 
   HeadArgs ha;
   ha.z = h->head_z;
+  ha.entropy_out = h->head_entropy;
   ha.h = h->head_in;
   ha.ldh = d;
   ha.B = B;
@@ -743,6 +750,7 @@ int vla_score_actions(vla_handle* h, const int32_t* tokens, float temperature, f
     h->len[b] = h->len_prefill[b] + (A - 1);
     h->has_pending[b] = 1;
   }
+  h->entropy_valid = true;
   return VLA_OK;
 }
 
@@ -755,7 +763,53 @@ int vla_reset(vla_handle* h, const uint8_t* env_mask) {
     h->has_pending[b] = 0;
     h->prefilled[b] = 0;
   }
+  h->entropy_valid = false;
   return VLA_OK;
+}
+
+int vla_action_entropy(vla_handle* h, float* entropy_out) {
+  if (!h) return set_err(nullptr, VLA_ERR_ARG, "vla_action_entropy: NULL handle");
+  if (!entropy_out) return fail(h, VLA_ERR_ARG, "vla_action_entropy: NULL buffer");
+  int rc;
+  if ((rc = check_turn_state(h, "vla_action_entropy"))) return rc;
+  if (!h->entropy_valid) return fail(h, VLA_ERR_STATE, "vla_action_entropy: no decode or score since the prefill");
+  cudaSetDevice(h->dev);
+  const size_t n = static_cast<size_t>(h->active_batch) * h->cfg.action_dim;
+  if (cudaMemcpyAsync(entropy_out, h->head_entropy, n * sizeof(float), cudaMemcpyDeviceToDevice, h->stream) !=
+      cudaSuccess)
+    return fail(h, cuda_fail(cudaGetLastError(), "entropy copy"), t_err);
+  return VLA_OK;
+}
+
+int vla_value(vla_handle* h, const void* w_value, float bias, float* values_out) {
+  if (!h) return set_err(nullptr, VLA_ERR_ARG, "vla_value: NULL handle");
+  if (!w_value || !values_out || !std::isfinite(bias)) return fail(h, VLA_ERR_ARG, "vla_value: bad argument");
+  int rc;
+  if ((rc = check_turn_state(h, "vla_value"))) return rc;
+  cudaSetDevice(h->dev);
+  const vla_config& c = h->cfg;
+  rc = value_head_launch(h->h_last, c.d_model, h->active_batch, c.d_model, h->final_norm,
+                         static_cast<const bf16*>(w_value), c.rms_eps, bias, values_out, h->stream);
+  if (rc) return fail(h, rc, t_err);
+  return VLA_OK;
+}
+
+int vla_gae(const float* rewards, const float* values, const float* dones, int M, int B, float gamma, float lam,
+            float* adv_out, float* returns_out, void* cuda_stream) {
+  if (!rewards || !values || !dones || !adv_out || M < 1 || B < 1 || !(gamma >= 0.f && gamma <= 1.f) ||
+      !(lam >= 0.f && lam <= 1.f))
+    return set_err(nullptr, VLA_ERR_ARG, "vla_gae: bad argument");
+  const int rc = gae_launch(rewards, values, dones, M, B, gamma, lam, adv_out, returns_out,
+                            static_cast<cudaStream_t>(cuda_stream));
+  return rc;
+}
+
+int vla_ppo_clip(const float* lp_new, const float* lp_old, const float* adv, int N, int A, float eps,
+                 float* objective_out, float* ratio_out, float* clip_frac_out, void* cuda_stream) {
+  if (!lp_new || !lp_old || !adv || !objective_out || N < 1 || A < 1 || !(eps >= 0.f) || !std::isfinite(eps))
+    return set_err(nullptr, VLA_ERR_ARG, "vla_ppo_clip: bad argument");
+  return ppo_clip_launch(lp_new, lp_old, adv, N, A, eps, objective_out, ratio_out, clip_frac_out,
+                         static_cast<cudaStream_t>(cuda_stream));
 }
 
 int vla_sync(vla_handle* h) {
@@ -791,7 +845,7 @@ void vla_destroy(vla_handle* h) {
   if (!h) return;
   cudaSetDevice(h->dev);
   cudaStreamSynchronize(h->stream);
-  void* bufs[] = {h->kv, h->h, h->y, h->q, h->ao, h->u, h->ws, h->h_last, h->head_in, h->head_z, h->q_last, h->last_rows, h->rope,
+  void* bufs[] = {h->kv, h->h, h->y, h->q, h->ao, h->u, h->ws, h->h_last, h->head_in, h->head_z, h->head_entropy, h->q_last, h->last_rows, h->rope,
                   h->rows, h->tiles, h->sidx, h->didx, h->fed, h->pending, h->status, h->part_o,
                   h->part_ml, h->attn_tickets};
   for (void* p : bufs)

@@ -44,8 +44,17 @@ struct HeadArgs {
   float* z = nullptr;               // scratch [B * n_pos, 256] logits (may alias logits_out
                                     // when A == n_pos and step == 0)
   int* fed_out = nullptr;           // [B, A] token fed to the next step (forced or sampled)
+  float* entropy_out = nullptr;     // [B, A] entropy of each token's bin distribution
   uint32_t* status = nullptr;
 };
 int action_head_launch(const HeadArgs& a, cudaStream_t s);
+
+// learning.cu
+int value_head_launch(const float* h, int ldh, int B, int d, const bf16* gain, const bf16* w, float eps,
+                      float bias, float* out, cudaStream_t s);
+int gae_launch(const float* r, const float* v, const float* done, int M, int B, float gamma, float lam,
+               float* adv, float* ret, cudaStream_t s);
+int ppo_clip_launch(const float* lp_new, const float* lp_old, const float* adv, int N, int A, float eps,
+                    float* objective, float* ratio, float* clip_frac, cudaStream_t s);
 
 }  // namespace vla

@@ -83,6 +83,10 @@ def load(path: str = LIB_PATH):
         "vla_profile": (i32, [vp, u32]),
         "vla_profile_read": (i32, [vp, vp, vp, vp, vp]),
         "vla_launch_count": (i64, [vp]),
+        "vla_action_entropy": (i32, [vp, vp]),
+        "vla_value": (i32, [vp, vp, f32, vp]),
+        "vla_gae": (i32, [vp, vp, vp, i32, i32, f32, f32, vp, vp, vp]),
+        "vla_ppo_clip": (i32, [vp, vp, vp, i32, i32, f32, vp, vp, vp, vp]),
         "vla_op_gemm_bf16": (i32, [vp, vp, i32, vp, i32, vp, i32, i32, i32, i32, i32, i32, vp, vp]),
         "vla_op_gemm_pair_bf16": (i32, [vp, vp, i32, vp, i32, vp, i32, i32, i32, i32, vp]),
         "vla_op_gemm_decode_bf16": (i32, [vp, vp, i32, vp, i32, vp, i32, i32, i32, i32, vp, ctypes.c_size_t, vp]),
@@ -137,6 +141,26 @@ def vla_decode_actions(h, uniforms_ptr: int, temperature: float, forced_ptr: int
 def vla_score_actions(h, tokens_ptr: int, temperature: float, logprobs_ptr: int, logits_ptr: int = 0) -> int:
     return load().vla_score_actions(h, tokens_ptr or None, float(temperature), logprobs_ptr or None,
                                     logits_ptr or None)
+
+
+def vla_action_entropy(h, entropy_ptr: int) -> int:
+    return load().vla_action_entropy(h, entropy_ptr or None)
+
+
+def vla_value(h, w_value_ptr: int, bias: float, values_ptr: int) -> int:
+    return load().vla_value(h, w_value_ptr or None, float(bias), values_ptr or None)
+
+
+def vla_gae(rewards_ptr: int, values_ptr: int, dones_ptr: int, M: int, B: int, gamma: float, lam: float,
+            adv_ptr: int, returns_ptr: int = 0, stream: int = 0) -> int:
+    return load().vla_gae(rewards_ptr or None, values_ptr or None, dones_ptr or None, M, B, float(gamma),
+                          float(lam), adv_ptr or None, returns_ptr or None, stream or None)
+
+
+def vla_ppo_clip(lp_new_ptr: int, lp_old_ptr: int, adv_ptr: int, N: int, A: int, eps: float, objective_ptr: int,
+                 ratio_ptr: int = 0, clip_frac_ptr: int = 0, stream: int = 0) -> int:
+    return load().vla_ppo_clip(lp_new_ptr or None, lp_old_ptr or None, adv_ptr or None, N, A, float(eps),
+                               objective_ptr or None, ratio_ptr or None, clip_frac_ptr or None, stream or None)
 
 
 def vla_reset(h, env_mask: Optional[Sequence[int]] = None) -> int:
@@ -292,7 +316,22 @@ class Policy:
                                       forced.data_ptr() if forced is not None else 0, out["tokens"].data_ptr(),
                                       out["logprobs"].data_ptr(), out["actions"].data_ptr(),
                                       out["logits"].data_ptr() if want_logits else 0))
+        out["entropy"] = self.entropy(dev)
         return out
+
+    def entropy(self, device=None):
+        """Entropies [B, action_dim] of the latest decode / score (vla_action_entropy)."""
+        t = self.torch
+        e = t.empty(self.B, self.shape.action_dim, dtype=t.float32, device=device or t.device("cuda"))
+        self.check(vla_action_entropy(self.h, e.data_ptr()))
+        return e
+
+    def value(self, w_value, bias: float):
+        """Value-model estimates [B] at the latest prefill (vla_value); w_value bf16 [d] on the GPU."""
+        t = self.torch
+        v = t.empty(self.B, dtype=t.float32, device=w_value.device)
+        self.check(vla_value(self.h, w_value.data_ptr(), bias, v.data_ptr()))
+        return v
 
     def score(self, tokens, temperature: float, want_logits: bool = True):
         t = self.torch
@@ -301,6 +340,7 @@ class Policy:
                "logits": t.empty(B, A, 256, dtype=t.float32, device=tokens.device) if want_logits else None}
         self.check(vla_score_actions(self.h, tokens.data_ptr(), temperature, out["logprobs"].data_ptr(),
                                      out["logits"].data_ptr() if want_logits else 0))
+        out["entropy"] = self.entropy(tokens.device)
         return out
 
     def reset(self, mask=None):

@@ -4,7 +4,7 @@ Tolerances (fixed by the method's bf16 weights / fp32 accumulation):
   * action tokens bit-exact in teacher-forced mode wherever the oracle's top-2 margin of the
     perturbed score exceeds 0.05;
   * actions bit-exact wherever the tokens match;
-  * logits and log-probs within 2e-2 absolute.
+  * logits, log-probs and the rollout entropy within 2e-2 absolute.
 The GPU decodes with forced_tokens = the oracle's tokens, so both sides condition on the
 same trajectory.
 """
@@ -39,10 +39,13 @@ class TurnReport:
     logit_err_by_step: Optional[list] = None
     emul_logit_err: Optional[float] = None      # vs the GPU-rounding oracle (attribution)
     emul_lp_err: Optional[float] = None
+    entropy_err: Optional[float] = None         # rollout entropy of decode (and score)
+    value_err: Optional[float] = None           # value head at the turn's prefill
 
     def ok(self) -> bool:
         errs = [self.max_lp_err, self.max_logit_err]
-        errs += [e for e in (self.score_lp_err, self.score_vs_decode_err, self.score_logit_err) if e is not None]
+        errs += [e for e in (self.score_lp_err, self.score_vs_decode_err, self.score_logit_err,
+                             self.entropy_err, self.value_err) if e is not None]
         return self.token_mismatch == 0 and self.action_mismatch == 0 and max(errs) <= TOL
 
 
@@ -87,6 +90,11 @@ def run_parity(wl: I.Workload, weights_cpu=None, weights_dev=None, n_check: Opti
                 if o_ is not None:
                     o_.prefill(envs, [inp.visual[b] for b in envs],
                                [inp.ids[b, :int(inp.lengths[b])].tolist() for b in envs])
+            # value head (Algorithm 1: V_t) at the prefill, same decoder weights
+            wv = I.normal_bf16((sh.d_model,), 2025, 77, 0.02)
+            gv = pol.value(wv.to(device), 0.25).cpu().numpy()
+            ov = orc.value(envs, wv, 0.25)
+            value_err = float(np.max(np.abs(gv[envs] - ov)))
             u_cpu = inp.uniforms
             od = orc.decode(envs, u_cpu[envs], T)
             forced = torch.full((wl.batch, sh.action_dim), base, dtype=torch.int32)
@@ -100,6 +108,8 @@ def run_parity(wl: I.Workload, weights_cpu=None, weights_dev=None, n_check: Opti
             pol.sync()
             g = {k: v.cpu().numpy() for k, v in gd.items() if v is not None}
             rep = compare_decode(t, envs, od, g)
+            rep.entropy_err = float(np.max(np.abs(g["entropy"][envs] - od["entropy"])))
+            rep.value_err = value_err
             if emu is not None:
                 ed = emu.decode(envs, u_cpu[envs], T, forced=forced[envs])
                 rep.emul_logit_err = float(np.max(np.abs(g["logits"][envs] - ed["logits"])))
@@ -115,6 +125,8 @@ def run_parity(wl: I.Workload, weights_cpu=None, weights_dev=None, n_check: Opti
                 rep.score_lp_err = float(np.max(np.abs(glp[envs] - os_["logprobs"])))
                 rep.score_logit_err = float(np.max(np.abs(glg[envs] - os_["logits"])))
                 rep.score_vs_decode_err = float(np.max(np.abs(glp - g["logprobs"])))
+                rep.entropy_err = max(rep.entropy_err,
+                                      float(np.max(np.abs(sc["entropy"].cpu().numpy()[envs] - os_["entropy"]))))
             reports.append(rep)
     finally:
         pol.close()
