@@ -43,23 +43,25 @@ PROFILED_TRAFFIC = {"bytes": 2.975106e9 + 0.877365e9,
                     "profile": "profiles/gemm_tc2_prefill_qkv_18385x12288x4096.md"}
 
 
-def phase_work(sh, B, n_visual, lengths):
-    """Algorithmic work of one step's phases (7B: 6.476e9 matrix parameters, 16 KB of fp16 K+V
-    per token per layer).  Prefill FLOPs count what the method needs: every row through every
-    layer except that the last layer only needs q|k|v for all rows (KV cache) and the rest for
-    each env's final row; attention FLOPs are the causal ones.  Decode bytes are, per forward,
-    all weights + the K/V each env reads (positions 0..pos) and writes + the 256 head rows.
+def phase_work(sh, past, chunk):
+    """Algorithmic work of one turn's phases for envs whose chunk of chunk[b] rows lands after
+    past[b] cached positions (7B: 6.476e9 matrix parameters, 16 KB of fp16 K+V per position
+    and layer).  Prefill FLOPs count what the method needs: every row through every layer,
+    except that the last layer only needs q|k|v for all rows (KV cache) and the rest for each
+    env's final row; attention FLOPs are the causal ones.  Decode bytes are, per forward, all
+    weights + the K/V each env reads (positions 0..pos) and writes + the 256 head rows.
     Score: one weight stream, K/V reads of the 6 teacher-forced rows, 2 P flops per row."""
-    d, F, L, hd = sh.d_model, sh.d_ffn, sh.n_layers, sh.head_dim
+    d, F, L = sh.d_model, sh.d_ffn, sh.n_layers
     per_layer = 4 * d * d + 3 * F * d
     qkv_params = 3 * d * d
     params = L * per_layer
     w_bytes = 2.0 * params
     kv_tok = 2.0 * 2 * d * L                    # fp16 K and V, all layers
     A = sh.action_dim
-    P = [n_visual + int(x) for x in lengths]   # prefix lengths (first turn)
-    T = sum(P)
-    attn = sum(2.0 * d * (p * (p + 1)) for p in P)          # per layer, causal, n = p, past = 0
+    B = len(chunk)
+    T = sum(chunk)
+    P = [p + n for p, n in zip(past, chunk)]    # context after the prefill
+    attn = sum(2.0 * d * (2 * n * p + n * (n + 1)) for p, n in zip(past, chunk))  # per layer
     flops_pre = (L - 1) * (2.0 * T * per_layer + attn) \
         + 2.0 * T * qkv_params + 2.0 * B * (per_layer - qkv_params) + sum(4.0 * d * p for p in P)
     flops_pre_formula = 2.0 * params * T + L * attn
@@ -71,7 +73,7 @@ def phase_work(sh, B, n_visual, lengths):
     sc_bytes = w_bytes + sum((p + n) * kv_tok for p in P) + B * n * kv_tok + 2.0 * 256 * d
     sc_flops = 2.0 * params * B * n + L * sum(2.0 * d * (2 * n * p + n * (n + 1)) for p in P)
     return {"prefill_flops": flops_pre, "prefill_flops_all_rows": flops_pre_formula,
-            "decode_bytes": dec_bytes, "score_bytes": sc_bytes, "score_flops": sc_flops}
+            "decode_bytes": dec_bytes, "score_bytes": sc_bytes, "score_flops": sc_flops, "rows": T}
 
 
 def peaks():
@@ -374,25 +376,46 @@ def main():
     w_dev = {k: v.cuda() for k, v in w_cpu.items()}
     # each rank: its own batch of envs (weak scaling); rank 0 = the workload's own inputs
     wl_r = wl if rank == 0 else I.dataclasses.replace(wl, index=wl.index + 1000 * rank)
-    inp = I.make_turn_inputs(wl_r, 0)
-    lengths = inp.lengths.tolist()
-    max_tokens = B * (wl.n_visual + max(lengths) + 8)
+    turns = [I.make_turn_inputs(wl_r, t) for t in range(wl.turns)]
+    lens = [tin.lengths.tolist() for tin in turns]
+    max_tokens = B * max(tin.visual.shape[1] + max(l) + 8 for tin, l in zip(turns, lens))
     stream = torch.cuda.current_stream()
     pol = V.Policy(sh, w_dev, B, wl.kv_capacity, max_tokens, stream=stream)
 
-    vis_d, ids_d, u_d = inp.visual.cuda(), inp.ids.cuda(), inp.uniforms.cuda()
+    dev_in = [(tin.visual.cuda(), tin.ids.cuda(), tin.uniforms.cuda()) for tin in turns]
     tok = torch.empty(B, A, dtype=torch.int32, device="cuda")
     lp = torch.empty(B, A, dtype=torch.float32, device="cuda")
     act = torch.empty(B, A, dtype=torch.float32, device="cuda")
     slp = torch.empty(B, A, dtype=torch.float32, device="cuda")
     T = wl.temperature
     h = pol.h
+    reset_masks = {t: [1 if b in ended else 0 for b in range(B)] for t, ended in wl.resets}
 
-    def step(vis, ids, u):
+    def step(inputs, ev=None, before_turn=None, after_turn=None):
+        """reset, then per turn: episode ends, prefill (append), 7-token decode; then the score
+        pass of the last turn.  ev: events [turn][3] + [2] for the score, for phase times."""
         pol.check(V.vla_reset(h, None))
-        pol.check(V.vla_prefill(h, B, vis.data_ptr(), vis.shape[1], ids.data_ptr(), lengths, ids.shape[1]))
-        pol.check(V.vla_decode_actions(h, u.data_ptr(), T, 0, tok.data_ptr(), lp.data_ptr(), act.data_ptr(), 0))
-        pol.check(V.vla_score_actions(h, tok.data_ptr(), T, slp.data_ptr(), 0))
+        for t, (vis, ids, u) in enumerate(inputs):
+            if before_turn:
+                before_turn(t)
+            if t in reset_masks:
+                pol.check(V.vla_reset(h, reset_masks[t]))
+            if ev:
+                ev[t][0].record(stream)
+            pol.check(V.vla_prefill(h, B, vis.data_ptr(), vis.shape[1], ids.data_ptr(), lens[t], ids.shape[1]))
+            if ev:
+                ev[t][1].record(stream)
+            pol.check(V.vla_decode_actions(h, u.data_ptr(), T, 0, tok.data_ptr(), lp.data_ptr(), act.data_ptr(), 0))
+            if ev:
+                ev[t][2].record(stream)
+            if after_turn:
+                after_turn(t)
+        if wl.score:
+            if ev:
+                ev[-1][0].record(stream)
+            pol.check(V.vla_score_actions(h, tok.data_ptr(), T, slp.data_ptr(), 0))
+            if ev:
+                ev[-1][1].record(stream)
 
     def barrier():
         if dist is not None:
@@ -400,7 +423,7 @@ def main():
 
     # ---- warm-up
     for _ in range(args.warmup):
-        step(vis_d, ids_d, u_d)
+        step(dev_in)
     pol.sync()
 
     # ---- timed region (device-resident inputs); GEMM classes timed with events
@@ -412,7 +435,7 @@ def main():
     with ClockSampler(local) as clk:
         ev0.record(stream)
         for _ in range(args.steps):
-            step(vis_d, ids_d, u_d)
+            step(dev_in)
         ev1.record(stream)
         torch.cuda.synchronize()
     barrier()
@@ -424,43 +447,60 @@ def main():
     ms_step = ms_total / args.steps
 
     # ---- phase breakdown (separate, untimed for the headline)
-    phase = {}
-    e = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
-    pol.check(V.vla_reset(h, None))
-    e[0].record(stream)
-    pol.check(V.vla_prefill(h, B, vis_d.data_ptr(), vis_d.shape[1], ids_d.data_ptr(), lengths, ids_d.shape[1]))
-    e[1].record(stream)
-    pol.check(V.vla_decode_actions(h, u_d.data_ptr(), T, 0, tok.data_ptr(), lp.data_ptr(), act.data_ptr(), 0))
-    e[2].record(stream)
-    pol.check(V.vla_score_actions(h, tok.data_ptr(), T, slp.data_ptr(), 0))
-    e[3].record(stream)
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(wl.turns)]
+    evs.append([torch.cuda.Event(enable_timing=True) for _ in range(2)])
+    step(dev_in, ev=evs)
     pol.sync()
-    t_pre, t_dec, t_sc = e[0].elapsed_time(e[1]), e[1].elapsed_time(e[2]), e[2].elapsed_time(e[3])
+    t_pre_t = [evs[t][0].elapsed_time(evs[t][1]) for t in range(wl.turns)]
+    t_dec_t = [evs[t][1].elapsed_time(evs[t][2]) for t in range(wl.turns)]
+    t_pre, t_dec = sum(t_pre_t), sum(t_dec_t)
+    t_sc = evs[-1][0].elapsed_time(evs[-1][1]) if wl.score else 0.0
     # one more step with every kernel class bracketed by events (outside the timed region)
     V.vla_profile(h, (1 << len(V.KCLASS)) - 1)
-    step(vis_d, ids_d, u_d)
+    step(dev_in)
     per_class = V.vla_profile_read(h)
     V.vla_profile(h, 0)
-    prefill_tokens = sum(lengths) + B * wl.n_visual
+
+    # algorithmic work per turn (context lengths tracked as the handle does)
+    ctx, pending = [0] * B, [0] * B
+    works = []
+    for t in range(wl.turns):
+        for b in (wl.resets and dict(wl.resets).get(t, ()) or ()):
+            ctx[b], pending[b] = 0, 0
+        chunk = [pending[b] + turns[t].visual.shape[1] + int(lens[t][b]) for b in range(B)]
+        works.append(phase_work(sh, ctx, chunk))
+        ctx = [ctx[b] + chunk[b] + A - 1 for b in range(B)]
+        pending = [1] * B
+    prefill_rows = sum(w_["rows"] for w_ in works)
     phase = {"prefill_ms": t_pre, "decode_ms": t_dec, "score_ms": t_sc,
-             "prefill_tok_s": prefill_tokens / (t_pre / 1e3), "decode_action_tok_s": B * A / (t_dec / 1e3),
+             "prefill_tok_s": prefill_rows / (t_pre / 1e3), "decode_action_tok_s": wl.turns * B * A / (t_dec / 1e3),
              "kernel_classes_ms": {k: round(v["ms"], 3) for k, v in per_class.items()},
              "kernel_classes_launches": {k: v["launches"] for k, v in per_class.items()}}
+    if wl.turns > 1:
+        phase["prefill_ms_per_turn"] = [round(x, 3) for x in t_pre_t]
+        phase["decode_ms_per_turn"] = [round(x, 3) for x in t_dec_t]
+        phase["decode_action_tok_s_per_turn"] = [round(B * A / (x / 1e3), 1) for x in t_dec_t]
 
-    # ---- e2e through the C ABI with host buffers
-    vis_h = inp.visual.pin_memory()
-    ids_h = inp.ids.pin_memory()
-    u_h = inp.uniforms.pin_memory()
-    out_h = [torch.empty(B, A, dtype=t).pin_memory() for t in (torch.int32, torch.float32, torch.float32, torch.float32)]
-    vis_e, ids_e, u_e = torch.empty_like(vis_d), torch.empty_like(ids_d), torch.empty_like(u_d)
+    # ---- e2e through the C ABI with host buffers: each turn's inputs are copied in before
+    # its prefill and its tokens / log-probs / actions copied out after its decode
+    host_in = [(tin.visual.pin_memory(), tin.ids.pin_memory(), tin.uniforms.pin_memory()) for tin in turns]
+    e2e_in = [tuple(torch.empty_like(x) for x in di) for di in dev_in]
+    out_h = [[torch.empty(B, A, dtype=t_).pin_memory() for t_ in (torch.int32, torch.float32, torch.float32)]
+             for _ in range(wl.turns)]
+    score_h = torch.empty(B, A, dtype=torch.float32).pin_memory()
+
+    def copy_in(t):
+        for dst, src in zip(e2e_in[t], host_in[t]):
+            dst.copy_(src, non_blocking=True)
+
+    def copy_out(t):
+        for dst, src in zip(out_h[t], (tok, lp, act)):
+            dst.copy_(src, non_blocking=True)
 
     def e2e_step():
-        vis_e.copy_(vis_h, non_blocking=True)
-        ids_e.copy_(ids_h, non_blocking=True)
-        u_e.copy_(u_h, non_blocking=True)
-        step(vis_e, ids_e, u_e)
-        for dst, src in zip(out_h, (tok, lp, act, slp)):
-            dst.copy_(src, non_blocking=True)
+        step(e2e_in, before_turn=copy_in, after_turn=copy_out)
+        if wl.score:
+            score_h.copy_(slp, non_blocking=True)
 
     e2e_step()
     pol.sync()
@@ -472,8 +512,8 @@ def main():
     ev1.record(stream)
     torch.cuda.synchronize()
     e2e_ms = max_over_ranks(ev0.elapsed_time(ev1), dist) / args.steps
-    h2d = vis_h.numel() * 2 + ids_h.numel() * 4 + u_h.numel() * 4
-    d2h = sum(t.numel() * 4 for t in out_h)
+    h2d = sum(v_.numel() * 2 + i_.numel() * 4 + u_.numel() * 4 for v_, i_, u_ in host_in)
+    d2h = sum(x.numel() * 4 for o in out_h for x in o) + (score_h.numel() * 4 if wl.score else 0)
 
     hbm, tf_burst, tf_sus, peak_kind = peaks()
     gp = prof["gemm_prefill"]
@@ -487,6 +527,9 @@ def main():
                 "traffic": PROFILED_TRAFFIC["bytes"] if PROFILED_TRAFFIC else None,
                 "traffic_launch": PROFILED_TRAFFIC,
                 "launches": gp["launches"], "avg_launch_ms": gp["ms"] / max(1, gp["launches"])}
+        # every prefill GEMM carries the activation as a bf16 pair: the MMAs issued are twice
+        # the algorithmic product
+        roof["issued_mma_frac"] = 2.0 * achieved / tf_sus
     roof_dec = None
     if gd["ms"] > 0:
         gbs = gd["bytes"] / (gd["ms"] / 1e3) / 1e9
@@ -495,41 +538,48 @@ def main():
                     "peak_kind": f"{peak_kind} HBM copy",
                     "note": "each launch bracketed by events, which also stops it overlapping its neighbours",
                     "launches": gd["launches"], "avg_launch_ms": gd["ms"] / max(1, gd["launches"])}
-    if roof is not None:
-        # every prefill GEMM carries the activation as a bf16 pair: the MMAs issued are twice the
-        # algorithmic product
-        roof["issued_mma_frac"] = 2.0 * roof["achieved"] / tf_sus
-    pw = phase_work(sh, B, wl.n_visual, lengths)
+    pre_fl = sum(w_["prefill_flops"] for w_ in works)
+    dec_by = sum(w_["decode_bytes"] for w_ in works)
     phase_roof = {
-        "prefill": {"bound": "tensor", "tflop": pw["prefill_flops"] / 1e12, "ms": t_pre,
-                    "achieved": pw["prefill_flops"] / (t_pre / 1e3) / 1e12, "peak": tf_burst, "unit": "TFLOP/s",
-                    "frac": pw["prefill_flops"] / (t_pre / 1e3) / 1e12 / tf_burst,
-                    "peak_kind": f"{peak_kind} bf16 burst",
-                    "tflop_if_every_row_ran_every_layer": pw["prefill_flops_all_rows"] / 1e12},
-        "decode": {"bound": "hbm", "gb": pw["decode_bytes"] / 1e9, "ms": t_dec,
-                   "achieved": pw["decode_bytes"] / (t_dec / 1e3) / 1e9, "peak": hbm, "unit": "GB/s",
-                   "frac": pw["decode_bytes"] / (t_dec / 1e3) / 1e9 / hbm, "peak_kind": f"{peak_kind} HBM copy"},
-        "score": {"bound": "hbm", "gb": pw["score_bytes"] / 1e9, "tflop": pw["score_flops"] / 1e12, "ms": t_sc,
-                  "achieved": pw["score_bytes"] / (t_sc / 1e3) / 1e9, "peak": hbm, "unit": "GB/s",
-                  "frac": pw["score_bytes"] / (t_sc / 1e3) / 1e9 / hbm,
-                  "tflops": pw["score_flops"] / (t_sc / 1e3) / 1e12, "peak_kind": f"{peak_kind} HBM copy"},
+        "prefill": {"bound": "tensor", "tflop": pre_fl / 1e12, "ms": t_pre,
+                    "achieved": pre_fl / (t_pre / 1e3) / 1e12, "peak": tf_burst, "unit": "TFLOP/s",
+                    "frac": pre_fl / (t_pre / 1e3) / 1e12 / tf_burst, "peak_kind": f"{peak_kind} bf16 burst",
+                    "tflop_if_every_row_ran_every_layer": sum(w_["prefill_flops_all_rows"] for w_ in works) / 1e12},
+        "decode": {"bound": "hbm", "gb": dec_by / 1e9, "ms": t_dec,
+                   "achieved": dec_by / (t_dec / 1e3) / 1e9, "peak": hbm, "unit": "GB/s",
+                   "frac": dec_by / (t_dec / 1e3) / 1e9 / hbm, "peak_kind": f"{peak_kind} HBM copy"},
     }
+    if wl.turns > 1:
+        phase_roof["decode"]["frac_per_turn"] = [round(w_["decode_bytes"] / (x / 1e3) / 1e9 / hbm, 3)
+                                                 for w_, x in zip(works, t_dec_t)]
+    if wl.score:
+        sw = works[-1]
+        phase_roof["score"] = {"bound": "hbm", "gb": sw["score_bytes"] / 1e9, "tflop": sw["score_flops"] / 1e12,
+                               "ms": t_sc, "achieved": sw["score_bytes"] / (t_sc / 1e3) / 1e9, "peak": hbm,
+                               "unit": "GB/s", "frac": sw["score_bytes"] / (t_sc / 1e3) / 1e9 / hbm,
+                               "tflops": sw["score_flops"] / (t_sc / 1e3) / 1e12,
+                               "peak_kind": f"{peak_kind} HBM copy"}
 
     n_gpus = world
-    value = n_gpus * B * A / (ms_step / 1e3)
+    acts = wl.turns * B * A                     # action tokens per step
+    value = n_gpus * acts / (ms_step / 1e3)
+    text = f"U{{{wl.text_len_range[0]}..{wl.text_len_range[1]}}}" if wl.text_len is None else str(wl.text_len)
+    step_desc = ("reset + prefill + 7-token decode" if wl.turns == 1 else
+                 f"reset + {wl.turns} turns x (prefill/append + 7-token decode)") + (" + score" if wl.score else "")
     line = {
         "metric": METRIC, "value": value, "unit": "action tokens/s", "n_gpus": n_gpus,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16 weights, fp32 accumulate",
         "data": "synthetic (seeded; random-init weights)",
         "config": {"workload": wl.name, "model": sh.name, "batch_per_gpu": B, "n_visual": wl.n_visual,
-                   "text_len": "U{16..48}", "action_tokens": A, "temperature": T,
-                   "step": "reset + prefill + 7-token decode + score",
+                   "text_len": text, "turns": wl.turns, "append_visual": wl.append_visual if wl.turns > 1 else 0,
+                   "append_text": wl.append_text if wl.turns > 1 else 0, "action_tokens": A, "temperature": T,
+                   "step": step_desc,
                    "l2": "no flush: 13 GB of weights streamed per forward (> 129 MB L2)",
                    "parallelism": f"replicas x{n_gpus}"},
         "phases": phase,
         "roofline": roof, "roofline_decode": roof_dec, "phase_roofline": phase_roof,
-        "e2e": {"value": n_gpus * B * A / (e2e_ms / 1e3), "unit": "action tokens/s",
+        "e2e": {"value": n_gpus * acts / (e2e_ms / 1e3), "unit": "action tokens/s",
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms},
         "gpu_launches": launches,
         "clocks": clk.summary(),

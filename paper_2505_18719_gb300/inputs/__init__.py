@@ -143,6 +143,9 @@ class Workload:
     score: bool = False
     kv_capacity: int = 0
     index: int = 0
+    # episode ends: (turn, env ids) = these envs are reset before that turn's prefill and
+    # start a new episode whose first prefix is that turn's chunk (Algorithm 1 terminal flags)
+    resets: tuple = ()
 
     @property
     def input_seed(self) -> int:
@@ -161,6 +164,10 @@ WORKLOADS: Dict[str, Workload] = {w.name: w for w in (
              kv_capacity=320, index=4),
     Workload("7b_b256_multiturn", LLAMA7B, 256, 256, 64, turns=4, append_visual=256,
              append_text=0, kv_capacity=1152, index=5),
+    # the same trajectory with the instruction's 64 ids re-sent every turn (up to 1307 positions),
+    # the paper's sampling temperature 1.5, and three envs whose episode ends after turn 1
+    Workload("7b_b256_multiturn_t15", LLAMA7B, 256, 256, 64, turns=4, append_visual=256,
+             append_text=64, temperature=1.5, kv_capacity=1344, index=6, resets=((2, (0, 5, 131)),)),
 )}
 
 

@@ -85,6 +85,12 @@ def run_parity(wl: I.Workload, weights_cpu=None, weights_dev=None, n_check: Opti
             inp = I.make_turn_inputs(wl, t)
             if envs is None:
                 envs = check_envs(wl, inp.lengths, n_check)
+            for t_r, ended in wl.resets:
+                if t_r == t:
+                    pol.reset([1 if b in ended else 0 for b in range(wl.batch)])
+                    for o_ in (orc, emu):
+                        if o_ is not None and any(b in envs for b in ended):
+                            o_.reset([b for b in ended if b in envs])
             pol.prefill(inp.visual.to(device), inp.ids.to(device), inp.lengths.tolist())
             for o_ in (orc, emu):
                 if o_ is not None:

@@ -58,3 +58,12 @@ def test_7b_b64_ragged_score_parity(llama_weights):
 def test_7b_b256_multiturn_parity(llama_weights):
     w, wd = llama_weights
     _assert_ok(P.run_parity(I.WORKLOADS["7b_b256_multiturn"], w, wd, n_check=2, cache_f64=False))
+
+
+@pytest.mark.slow
+def test_7b_b256_multiturn_t15_with_resets_parity(llama_weights):
+    """Four turns with 64 text ids re-sent per turn (up to 1307 positions), T = 1.5, and three
+    envs (one of them compared) whose episode ends after turn 1: their turn-2 prefill starts a
+    fresh context in the same batch as the others' appends."""
+    w, wd = llama_weights
+    _assert_ok(P.run_parity(I.WORKLOADS["7b_b256_multiturn_t15"], w, wd, n_check=2, cache_f64=False))

@@ -356,6 +356,21 @@ def test_head_token_and_action_mapping():
     assert ho.action == -1 + (2 * ho.k + 1) / 256
 
 
+def test_reset_env_restarts_like_a_fresh_env():
+    """An env reset at an episode end (Algorithm 1 terminal flags) and prefilled again gives the
+    same decode, bit for bit, as a never-used env given the same prefix."""
+    orc = _micro_oracle(2)
+    _prefill(orc, [0, 1], 3, [2, 4])
+    orc.decode([0, 1], _uniforms(2), 1.0)
+    orc.reset([0])
+    fresh = _micro_oracle(1)
+    _prefill(orc, [0], 5, [3])
+    _prefill(fresh, [0], 5, [3])
+    a = orc.decode([0], _uniforms(1), 1.5)
+    b = fresh.decode([0], _uniforms(1), 1.5)
+    assert np.array_equal(a["logits"], b["logits"]) and np.array_equal(a["tokens"], b["tokens"])
+
+
 # ============================================================================ entropy, value, GAE, PPO
 def test_entropy_closed_forms():
     """Rollout entropy (§5): uniform logits give log 256 at any T; a two-level z has the closed
