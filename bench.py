@@ -213,6 +213,7 @@ CASES = {
     "gemv_decode_gate_up": (64, 22016, 4096, 0, 0, True),
     "gemv_decode_down": (64, 4096, 11008, 0, 0, True),
     "attn_decode": None,                                       # see run_attn_case
+    "learning": None,                                          # see run_learning_case
     # the same prefill shapes on CTA pairs (2-SM MMAs, 256 x 256 tiles)
     "pair_prefill_qkv": (4608, 12288, 4096, 256, 1, True),
     "pair_prefill_down": (4608, 4096, 11008, 256, 1, True),
@@ -227,6 +228,12 @@ CASES = {
     "gemm_score_o_s2": (384, 4096, 4096, 128, 2, True),
     "gemm_score_down_s1": (384, 4096, 11008, 128, 1, True),
     "gemm_score_down_s2": (384, 4096, 11008, 128, 2, True),
+    "gemm_score_gate_up_bn256": (384, 22016, 4096, 256, 1, True),
+    "gemm_score_gate_up_bn128": (384, 22016, 4096, 128, 1, True),
+    "pair_score_gate_up": (384, 22016, 4096, 256, 1, True),
+    "pair_score_qkv": (384, 12288, 4096, 256, 1, True),
+    "pair_score_down": (384, 4096, 11008, 256, 1, True),
+    "gemm_score_down_bn256": (384, 4096, 11008, 256, 1, True),
     "gemv_score_o_m128": (128, 4096, 4096, 0, 0, True),
     "gemv_score_down_m128": (128, 4096, 11008, 0, 0, True),
     # decode GEMM at 2x / 4x the weight bytes of the q|k|v step (fixed vs per-byte cost)
@@ -282,6 +289,44 @@ def run_attn_case(args):
     return 0
 
 
+def run_learning_case(args):
+    """GAE over 128 steps x 256 envs and the clipped PPO objective over those 32768 samples
+    (7 token log-probs each): the learning-phase quantities of one rollout batch."""
+    import torch
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2505_18719_gb300 import inputs as I
+    from paper_2505_18719_gb300 import vla as V
+    M, B, A = 128, 256, 7
+    r = I.normal_bf16((M, B), 9, 1, 1.0).float().cuda()
+    v = I.normal_bf16((M + 1, B), 9, 2, 1.0).float().cuda()
+    dn = (I.uniform_f32((M, B), 9, 3) < 0.05).float().cuda()
+    adv = torch.empty(M, B, device="cuda")
+    ret = torch.empty(M, B, device="cuda")
+    lp_old = (-I.uniform_f32((M * B, A), 9, 4) * 6.0).cuda()
+    lp_new = lp_old + 0.01
+    obj = torch.empty(1, device="cuda")
+    out = {"case": "learning", "M": M, "B": B, "A": A}
+    for name, fn, nbytes in (
+            ("gae", lambda: V.vla_gae(r.data_ptr(), v.data_ptr(), dn.data_ptr(), M, B, 0.99, 0.95, adv.data_ptr(),
+                                      ret.data_ptr(), 0), 4.0 * (M * B * 5 + B)),
+            ("ppo_clip", lambda: V.vla_ppo_clip(lp_new.data_ptr(), lp_old.data_ptr(), adv.data_ptr(), M * B, A, 0.2,
+                                                obj.data_ptr(), 0, 0, 0), 4.0 * M * B * (2 * A + 1))):
+        for _ in range(args.warmup):
+            assert fn() == 0
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for _ in range(args.steps):
+            assert fn() == 0
+        e1.record()
+        torch.cuda.synchronize()
+        us = e0.elapsed_time(e1) / args.steps * 1e3
+        out[name] = {"us": round(us, 2), "bytes": nbytes, "gbs": round(nbytes / us / 1e3, 1)}
+    print(json.dumps(out))
+    return 0
+
+
 def run_case(args):
     """Time one GEMM shape through vla_op_gemm_bf16 (CUDA events, device-resident operands)."""
     import torch
@@ -291,6 +336,8 @@ def run_case(args):
     from paper_2505_18719_gb300 import vla as V
     if args.case == "attn_decode":
         return run_attn_case(args)
+    if args.case == "learning":
+        return run_learning_case(args)
     M, N, K, bn, splits, split_a = CASES[args.case]
     A = I.normal_bf16((M, K), 1, 1, 1.0).cuda()
     A_lo = I.normal_bf16((M, K), 1, 2, 2.0 ** -9).cuda()
