@@ -214,6 +214,7 @@ CASES = {
     "gemv_decode_down": (64, 4096, 11008, 0, 0, True),
     "attn_decode": None,                                       # see run_attn_case
     "learning": None,                                          # see run_learning_case
+    "attn_chunk": None,                                        # see run_attn_chunk_case
     # the same prefill shapes on CTA pairs (2-SM MMAs, 256 x 256 tiles)
     "pair_prefill_qkv": (4608, 12288, 4096, 256, 1, True),
     "pair_prefill_down": (4608, 4096, 11008, 256, 1, True),
@@ -289,6 +290,51 @@ def run_attn_case(args):
     return 0
 
 
+def run_attn_chunk_case(args):
+    """Prefill chunk attention of one layer of the bench step: 64 envs, 256 visual + U{16..48}
+    text rows each, 32 heads x 128, in tiles of <= 64 query rows."""
+    import torch
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2505_18719_gb300 import inputs as I
+    from paper_2505_18719_gb300 import vla as V
+    B, H, hd, cap = 64, 32, 128, 320
+    lens = (256 + I.randint_i32((B,), 5, 7, 16, 48)).tolist()
+    rows = sum(lens)
+    kv = I.normal_bf16((B, 2, H, cap, hd), 5, 1, 1.0).cuda().half()
+    q = I.normal_bf16((rows, H * hd), 5, 2, 1.0).cuda().float()
+    tiles, r = [], 0
+    for b, n in enumerate(lens):
+        for t0 in range(0, n, 64):
+            tiles.append((b, r + t0, min(64, n - t0), t0))
+        r += n
+    tiles_dev = torch.zeros(len(tiles) * 4, dtype=torch.int32, device="cuda")
+    oh = torch.empty(rows, H * hd, dtype=torch.bfloat16, device="cuda")
+    ol = torch.empty_like(oh)
+
+    def launch():
+        rc = V.vla_op_attn_chunk(q.data_ptr(), kv.data_ptr(), B, H, hd, cap, tiles, rows, tiles_dev.data_ptr(),
+                                 oh.data_ptr(), ol.data_ptr())
+        assert rc == 0, V.vla_last_error(None)
+
+    for _ in range(args.warmup):
+        launch()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(args.steps):
+        launch()
+    e1.record()
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1) / args.steps
+    flops = sum(2.0 * H * hd * n * (n + 1) for n in lens)   # causal QK^T + PV
+    _, tf_burst, _, kind = peaks()
+    print(json.dumps({"case": args.case, "B": B, "H": H, "hd": hd, "rows": rows, "tiles": len(tiles), "ms": ms,
+                      "tflops": flops / ms / 1e9, "tc_frac_of_burst": flops / ms / 1e9 / tf_burst,
+                      "issued_mma_tflops": 2 * flops / ms / 1e9, "peaks": kind}))
+    return 0
+
+
 def run_learning_case(args):
     """GAE over 128 steps x 256 envs and the clipped PPO objective over those 32768 samples
     (7 token log-probs each): the learning-phase quantities of one rollout batch."""
@@ -338,6 +384,8 @@ def run_case(args):
         return run_attn_case(args)
     if args.case == "learning":
         return run_learning_case(args)
+    if args.case == "attn_chunk":
+        return run_attn_chunk_case(args)
     M, N, K, bn, splits, split_a = CASES[args.case]
     A = I.normal_bf16((M, K), 1, 1, 1.0).cuda()
     A_lo = I.normal_bf16((M, K), 1, 2, 2.0 ** -9).cuda()

@@ -92,6 +92,22 @@ int vla_op_attn_decode(const float* q, const void* kv, int max_env, int H, int h
                        size_t workspace_bytes, void* cuda_stream);
 size_t vla_op_attn_decode_workspace_bytes(int B, int H, int hd, int max_ctx, int max_keys_per_cta);
 
+/* Chunk causal attention (§3.1 self-attention; a prefill or appended chunk of each env attends
+ * to its whole cached context, §3.3), the prefill / score kernel on its own:
+ *   q          f32 [rows, H*hd] (already rotated), rows packed chunk after chunk;
+ *   kv         fp16 cache [env][K,V][H][cap][hd] (one layer, max_env envs), already holding
+ *              the chunk's own K/V;
+ *   tiles_host HOST int32 [n_tiles][4] = (env, row0, nrows, pos0): query rows row0 ..
+ *              row0+nrows-1 at positions pos0 .. pos0+nrows-1 of env, keys 0 .. position;
+ *              1 <= nrows <= 64, env < max_env, pos0 >= 0, pos0 + nrows <= cap,
+ *              row0 + nrows <= rows (checked on the host: VLA_ERR_ARG, nothing runs);
+ *   tiles_dev  device int32 [n_tiles][4] the tiles are copied to (the caller's scratch);
+ *   out_hi / out_lo  bf16 [rows, H*hd]: the output as the pair hi + lo.
+ * hd in {64, 128}. */
+int vla_op_attn_chunk(const float* q, const void* kv, int max_env, int H, int hd, int cap,
+                      const int32_t* tiles_host, int n_tiles, int rows, int32_t* tiles_dev,
+                      void* out_hi, void* out_lo, void* cuda_stream);
+
 /* Number of SMs the kernels size their persistent grids for (device property). */
 int vla_op_num_sms(void);
 

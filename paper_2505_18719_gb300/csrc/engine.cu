@@ -1056,6 +1056,35 @@ int vla_op_attn_decode(const float* q, const void* kv, int max_env, int H, int h
   return rc;
 }
 
+int vla_op_attn_chunk(const float* q, const void* kv, int max_env, int H, int hd, int cap,
+                      const int32_t* tiles_host, int n_tiles, int rows, int32_t* tiles_dev, void* out_hi,
+                      void* out_lo, void* cuda_stream) {
+  if (!q || !kv || !tiles_host || !tiles_dev || !out_hi || !out_lo || max_env < 1 || H < 1 || cap < 1 ||
+      n_tiles < 1 || rows < 1 || (hd != 64 && hd != 128))
+    return set_err(nullptr, VLA_ERR_ARG, "vla_op_attn_chunk: bad argument");
+  for (int i = 0; i < n_tiles; ++i) {
+    const int32_t* t = tiles_host + 4 * i;
+    if (t[0] < 0 || t[0] >= max_env || t[2] < 1 || t[2] > 64 || t[3] < 0 || t[3] + t[2] > cap || t[1] < 0 ||
+        t[1] + t[2] > rows)
+      return set_err(nullptr, VLA_ERR_ARG, "vla_op_attn_chunk: tile outside the buffers");
+  }
+  cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
+  if (cudaMemcpyAsync(tiles_dev, tiles_host, static_cast<size_t>(n_tiles) * 4 * sizeof(int32_t),
+                      cudaMemcpyHostToDevice, st) != cudaSuccess)
+    return cuda_fail(cudaGetLastError(), "vla_op_attn_chunk: tile copy");
+  KVLayout L{};
+  L.base = static_cast<f16*>(const_cast<void*>(kv));
+  L.cap = cap;
+  L.head_stride = static_cast<int64_t>(cap) * hd;
+  L.kv_stride = static_cast<int64_t>(H) * L.head_stride;
+  L.env_stride = 2 * L.kv_stride;
+  L.layer_stride = static_cast<int64_t>(max_env) * L.env_stride;
+  const int rc = attn_chunk_launch(q, static_cast<bf16*>(out_hi), static_cast<bf16*>(out_lo),
+                                   reinterpret_cast<const AttnTile*>(tiles_dev), n_tiles, L, 0, H, hd, st);
+  if (rc != VLA_OK && rc != VLA_ERR_CUDA) return set_err(nullptr, rc, "vla_op_attn_chunk: unsupported arguments");
+  return rc;
+}
+
 int vla_op_num_sms(void) { return query_num_sms(); }
 
 }  // extern "C"

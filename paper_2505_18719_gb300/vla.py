@@ -96,6 +96,7 @@ def load(path: str = LIB_PATH):
         "vla_op_num_sms": (i32, []),
         "vla_op_attn_decode": (i32, [vp, vp, i32, i32, i32, i32, vp, vp, i32, i32, i32, vp, vp, vp, ctypes.c_size_t, vp]),
         "vla_op_attn_decode_workspace_bytes": (ctypes.c_size_t, [i32, i32, i32, i32, i32]),
+        "vla_op_attn_chunk": (i32, [vp, vp, i32, i32, i32, i32, vp, i32, i32, vp, vp, vp, vp]),
     }
     for name, (res, args) in sig.items():
         f = getattr(lib, name)
@@ -235,6 +236,15 @@ def vla_op_action_head(h_ptr, ldh, B, d, final_norm_ptr, head_rows_ptr, eps, uni
                                      uniforms_ptr or None, float(temperature), forced_ptr or None,
                                      bins_ptr or None, lp_ptr, act_ptr or None, logits_ptr or None,
                                      status_ptr, stream or None)
+
+
+def vla_op_attn_chunk(q_ptr, kv_ptr, max_env, H, hd, cap, tiles, rows, tiles_dev_ptr, out_hi_ptr, out_lo_ptr,
+                      stream=0) -> int:
+    """tiles: host sequence of (env, row0, nrows, pos0)."""
+    flat = [int(x) for t in tiles for x in t]
+    arr = (ctypes.c_int32 * len(flat))(*flat)
+    return load().vla_op_attn_chunk(q_ptr or None, kv_ptr or None, max_env, H, hd, cap, arr, len(tiles), rows,
+                                    tiles_dev_ptr or None, out_hi_ptr or None, out_lo_ptr or None, stream or None)
 
 
 def vla_op_num_sms() -> int:

@@ -186,3 +186,46 @@ def test_decode_attention_matches_fp64(B, H, hd, cap, ctx):
         sc = torch.einsum("hd,hnd->hn", q[b].double(), k) / math.sqrt(hd)
         o = torch.einsum("hn,hnd->hd", torch.softmax(sc, -1), v)
         assert (got[b] - o).abs().max().item() < 1e-4, b
+
+
+@pytest.mark.parametrize("hd", [64, 128])
+def test_chunk_attention_matches_fp64(hd):
+    """Prefill / score chunk attention vs brute-force causal softmax attention in fp64: chunks of
+    1..130 rows appended after 0..200 cached positions, split into tiles of <= 64 rows."""
+    H, cap, max_env = 3, 384, 6
+    chunks = [(0, 0, 1), (1, 0, 63), (2, 0, 64), (3, 7, 130), (4, 200, 17), (5, 100, 64)]  # (env, past, n)
+    rows = sum(n for _, _, n in chunks)
+    kv = I.normal_bf16((max_env, 2, H, cap, hd), 91, hd, 1.0).float().half()
+    q = I.normal_bf16((rows, H * hd), 91, 1000 + hd, 1.0).float()
+    tiles, qpos, qenv = [], [], []
+    r = 0
+    for env, past, n in chunks:
+        for t0 in range(0, n, 64):
+            tiles.append((env, r + t0, min(64, n - t0), past + t0))
+        qpos += [past + i for i in range(n)]
+        qenv += [env] * n
+        r += n
+    tiles_dev = torch.zeros(len(tiles) * 4, dtype=torch.int32, device="cuda")
+    oh = torch.empty(rows, H * hd, dtype=torch.bfloat16, device="cuda")
+    ol = torch.empty_like(oh)
+    qd, kvd = q.cuda(), kv.cuda()
+    rc = V.vla_op_attn_chunk(qd.data_ptr(), kvd.data_ptr(), max_env, H, hd, cap, tiles, rows,
+                             tiles_dev.data_ptr(), oh.data_ptr(), ol.data_ptr())
+    assert rc == 0, V.vla_last_error(None)
+    torch.cuda.synchronize()
+    out = oh.cpu().double() + ol.cpu().double()
+    kv64 = kv.double()
+    err = 0.0
+    for i in range(rows):
+        env, p = qenv[i], qpos[i]
+        for hh in range(H):
+            qi = q[i, hh * hd:(hh + 1) * hd].double()
+            K = kv64[env, 0, hh, :p + 1]
+            Vv = kv64[env, 1, hh, :p + 1]
+            w = torch.softmax(K @ qi / math.sqrt(hd), dim=0)
+            err = max(err, float((out[i, hh * hd:(hh + 1) * hd] - w @ Vv).abs().max()))
+    assert err < 3e-3, err
+    # a tile outside the buffers is refused on the host
+    bad = [(0, 0, 65, 0)]
+    assert V.vla_op_attn_chunk(qd.data_ptr(), kvd.data_ptr(), max_env, H, hd, cap, bad, rows,
+                               tiles_dev.data_ptr(), oh.data_ptr(), ol.data_ptr()) == V.VLA_ERR_ARG
