@@ -87,6 +87,7 @@ DECODE_CASES = [
     (4, 768, 256),
     (16, 3072, 1024),
     (24, 200, 688),        # ragged N and K, score-sized M
+    (64, 512, 192),        # 1.5 k-steps of 128
     (64, 12288, 4096),     # 7B q|k|v decode step
     (64, 4096, 11008),     # 7B down-projection decode step
     (100, 1376, 256),
