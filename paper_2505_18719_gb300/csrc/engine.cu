@@ -116,6 +116,11 @@ struct vla_handle {
   float* head_entropy = nullptr;  // entropy of each action token's distribution [B, A]
   bool entropy_valid = false;     // set by decode / score, cleared by prefill / reset
   float* q_last = nullptr;  // last layer of a prefill: queries of each env's final row [B, d]
+  // deferred RMSNorm between tile GEMMs: per-tile row sums of squares [d / 128 + 1][T], and
+  // whether y currently holds an unnormalised row (h * w) whose scale the next GEMM applies
+  float* ss_part = nullptr;
+  bool y_deferred = false;
+  int y_ss_tiles = 0;
   RowInfo* last_rows = nullptr;  // and those rows' RowInfo [B]
   float2* rope = nullptr;
   RowInfo* rows = nullptr;
@@ -205,8 +210,17 @@ void prof_harvest(vla_handle* h) {
 }
 
 // A is the bf16 hi/lo pair: hi at A, lo at A + a_plane.
+// The GEMM that will consume h->y after a residual GEMM's RMSNorm (its N, K and epilogue).
+struct NextGemm {
+  int N, K, epi;
+};
+
+// epi.norm_w set (a residual GEMM followed by an RMSNorm into h->y): when this GEMM and `next`
+// both run as unsplit tile GEMMs, y is written unnormalised with per-tile sums of squares and
+// `next` applies the row scale in its epilogue; otherwise the norm is exact here (fused into
+// the weight-streaming reduction, or its own kernel).
 int run_gemm(vla_handle* h, int cls, const bf16* A, size_t a_plane, int lda, const bf16* W, int ldw,
-             int M, int N, int K, EpiArgs epi) {
+             int M, int N, int K, EpiArgs epi, const NextGemm* next = nullptr) {
   const Plan pl = plan_gemm(M, N, K, epi.kind, h->cfg.d_model, h->num_sms);
   GemmArgs g;
   g.A = A;
@@ -235,10 +249,29 @@ int run_gemm(vla_handle* h, int cls, const bf16* A, size_t a_plane, int lda, con
                                (epi.kind == EPI_SWIGLU ? (N / 2 + 127) / 128 : (N + 255) / 256);
     g.pair = pair_tiles >= h->num_sms / 2;
   }
-  // A following RMSNorm is fused into the weight-streaming GEMM's reduction; after a tile
-  // GEMM it is its own kernel.
+  // A following RMSNorm is fused into the weight-streaming GEMM's reduction; after a tile GEMM
+  // it is deferred to the consuming tile GEMM when both run unsplit, else its own kernel.
   const EpiArgs norm = epi;
-  if (!stream_k) g.epi.norm_w = nullptr;
+  bool defer_norm = false;
+  if (!stream_k && norm.norm_w && next && g.splits == 1 && M > 128 && N % 128 == 0) {
+    const Plan pn = plan_gemm(M, next->N, next->K, next->epi, h->cfg.d_model, h->num_sms);
+    defer_norm = pn.splits == 1;
+  }
+  if (!stream_k) {
+    if (defer_norm)
+      g.epi.ss_out = h->ss_part;
+    else
+      g.epi.norm_w = nullptr;
+  }
+  // the consumer of a deferred norm: y is unnormalised, scale its rows here
+  const bool consume = (A == h->y) && h->y_deferred && (epi.kind == EPI_QKV || epi.kind == EPI_SWIGLU);
+  if (consume) {
+    if (stream_k || g.splits != 1) return fail(h, VLA_ERR_ARG, "deferred RMSNorm reached a split GEMM");
+    g.epi.row_ss = h->ss_part;
+    g.epi.row_ss_n = h->y_ss_tiles;
+    g.epi.row_d = K;
+    g.epi.row_eps = h->cfg.rms_eps;
+  }
   if (h->ev_used.size() > 8192) prof_harvest(h);
   int ev = prof_begin(h, cls);
   GemmCost cost{0, 0};
@@ -246,7 +279,12 @@ int run_gemm(vla_handle* h, int cls, const bf16* A, size_t a_plane, int lda, con
                     : gemm_launch(g, h->stream, h->num_sms, &cost);
   prof_end(h, ev, cls, cost.flops, cost.bytes);
   if (rc != VLA_OK) return fail(h, rc, t_err.empty() ? "gemm launch failed" : t_err);
-  if (!stream_k && norm.norm_w) {
+  if (consume) h->y_deferred = false;
+  if (defer_norm) {
+    h->y_deferred = true;
+    h->y_ss_tiles = (N + g.block_n - 1) / g.block_n;
+  }
+  if (!stream_k && norm.norm_w && !defer_norm) {
     ev = prof_begin(h, VLA_KCLASS_OTHER);
     rc = rmsnorm_launch(norm.resid, norm.norm_w, M, N, norm.norm_eps, norm.norm_hi, norm.norm_lo, h->stream);
     prof_end(h, ev, VLA_KCLASS_OTHER, 0, 6.0 * M * N);
@@ -277,6 +315,7 @@ int forward_layers(vla_handle* h, int M, const RowInfo* rows_dev, bool decode, i
   const size_t pf = static_cast<size_t>(h->max_tokens) * F;
   int rc;
   // the first layer's attention RMSNorm; every later RMSNorm follows a residual add
+  h->y_deferred = false;
   int ev = prof_begin(h, VLA_KCLASS_OTHER);
   if ((rc = rmsnorm_launch(h->h, h->attn_norm[0], M, d, c.rms_eps, h->y, h->y + pd, h->stream))) return fail(h, rc, t_err);
   prof_end(h, ev, VLA_KCLASS_OTHER, 0, 6.0 * M * d);
@@ -329,7 +368,8 @@ int forward_layers(vla_handle* h, int M, const RowInfo* rows_dev, bool decode, i
     eo.norm_hi = h->y;
     eo.norm_lo = h->y + pd;
     eo.ldn = d;
-    if ((rc = run_gemm(h, gcls, h->ao, pd, d, h->wo[l], d, Mr, d, d, eo))) return rc;
+    const NextGemm gate_up{2 * F, d, EPI_SWIGLU};
+    if ((rc = run_gemm(h, gcls, h->ao, pd, d, h->wo[l], d, Mr, d, d, eo, &gate_up))) return rc;
 
     EpiArgs eg;
     eg.kind = EPI_SWIGLU;
@@ -349,7 +389,8 @@ int forward_layers(vla_handle* h, int M, const RowInfo* rows_dev, bool decode, i
       ed.norm_lo = h->y + pd;
       ed.ldn = d;
     }
-    if ((rc = run_gemm(h, gcls, h->u, pf, F, h->wdown[l], F, Mr, d, F, ed))) return rc;
+    const NextGemm qkv_next{3 * d, d, EPI_QKV};
+    if ((rc = run_gemm(h, gcls, h->u, pf, F, h->wdown[l], F, Mr, d, F, ed, &qkv_next))) return rc;
   }
   return VLA_OK;
 }
@@ -457,6 +498,7 @@ int vla_create(const vla_config* cfg, const vla_weights* w, void* cuda_stream, v
             alloc(reinterpret_cast<void**>(&h->head_z), static_cast<size_t>(B) * A * 256 * sizeof(float)) &&
             alloc(reinterpret_cast<void**>(&h->head_entropy), static_cast<size_t>(B) * A * sizeof(float)) &&
             alloc(reinterpret_cast<void**>(&h->q_last), static_cast<size_t>(B) * d * sizeof(float)) &&
+            alloc(reinterpret_cast<void**>(&h->ss_part), static_cast<size_t>(d / 128 + 1) * T * sizeof(float)) &&
             alloc(reinterpret_cast<void**>(&h->last_rows), static_cast<size_t>(B) * sizeof(RowInfo)) &&
             alloc(reinterpret_cast<void**>(&h->rope), static_cast<size_t>(cap) * (c.head_dim / 2) * sizeof(float2)) &&
             alloc(reinterpret_cast<void**>(&h->rows), T * sizeof(RowInfo)) &&
@@ -846,7 +888,7 @@ void vla_destroy(vla_handle* h) {
   if (!h) return;
   cudaSetDevice(h->dev);
   cudaStreamSynchronize(h->stream);
-  void* bufs[] = {h->kv, h->h, h->y, h->q, h->ao, h->u, h->ws, h->h_last, h->head_in, h->head_z, h->head_entropy, h->q_last, h->last_rows, h->rope,
+  void* bufs[] = {h->kv, h->h, h->y, h->q, h->ao, h->u, h->ws, h->h_last, h->head_in, h->head_z, h->head_entropy, h->q_last, h->ss_part, h->last_rows, h->rope,
                   h->rows, h->tiles, h->sidx, h->didx, h->fed, h->pending, h->status, h->part_o,
                   h->part_ml, h->attn_tickets};
   for (void* p : bufs)

@@ -36,6 +36,17 @@ struct EpiArgs {
   bf16* norm_hi = nullptr;
   bf16* norm_lo = nullptr;
   int ldn = 0;
+  // EPI_RESID of the tile GEMMs with norm_w set and ss_out != nullptr: the row of the updated
+  // residual times norm_w goes to norm_hi / norm_lo NOT normalised, and the sum of squares of
+  // the row's columns in each BN-wide tile to ss_out[n_tile * M + m]; the consuming GEMM
+  // applies the normalisation (row_ss).
+  float* ss_out = nullptr;
+  // EPI_QKV / EPI_SWIGLU of the tile GEMMs: row_ss != nullptr scales each output row by
+  // rsqrt(sum_{t < row_ss_n} row_ss[t * M + m] / row_d + row_eps) first (the RMSNorm of an
+  // input given unnormalised: the norm is a per-row scale, so it commutes with the product).
+  const float* row_ss = nullptr;
+  int row_ss_n = 0, row_d = 0;
+  float row_eps = 0.f;
   uint32_t* status = nullptr;
 };
 

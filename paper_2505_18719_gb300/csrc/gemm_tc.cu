@@ -130,11 +130,22 @@ __device__ __forceinline__ void ld16f(uint32_t taddr, float (&v)[16]) {
   for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
 }
 
+// 1 / RMS of row m from the per-tile sums of squares (fixed order), or 1 without them.
+__device__ __forceinline__ float row_scale(const Params& p, int m) {
+  if (!p.epi.row_ss || m >= p.M) return 1.f;
+  float ss = 0.f;
+  for (int t = 0; t < p.epi.row_ss_n; ++t) ss += p.epi.row_ss[static_cast<size_t>(t) * p.M + m];
+  return rsqrtf(ss / static_cast<float>(p.epi.row_d) + p.epi.row_eps);
+}
+
 // Plain epilogues: F32 / RESID / PARTIAL, 16 columns at a time.
 template <int BN, int EPI>
 __device__ __forceinline__ void epilogue_plain(const Params& p, uint32_t trow, int m, int n0,
                                                int split) {
   const bool row_ok = m < p.M;
+  // residual + the next RMSNorm's numerator (h * w) and this tile's sum of squares of h
+  const bool norm_next = (EPI == EPI_RESID) && p.epi.ss_out != nullptr;
+  float ss = 0.f;
 #pragma unroll 1
   for (int c = 0; c < BN; c += 16) {
     float v[16];
@@ -170,16 +181,50 @@ __device__ __forceinline__ void epilogue_plain(const Params& p, uint32_t trow, i
           o = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
         }
         d4[i] = o;
+        if (norm_next) {
+          v[4 * i] = o.x;
+          v[4 * i + 1] = o.y;
+          v[4 * i + 2] = o.z;
+          v[4 * i + 3] = o.w;
+        }
       }
     } else {
-      for (int i = 0; i < 16 && n + i < p.N; ++i) {
-        if (EPI == EPI_RESID)
+#pragma unroll
+      for (int i = 0; i < 16; ++i) {
+        if (n + i >= p.N) continue;
+        if (EPI == EPI_RESID) {
           dst[i] += v[i];
-        else
+          v[i] = dst[i];
+        } else {
           dst[i] = v[i];
+        }
+      }
+    }
+    if (norm_next) {
+      const int cnt = n + 16 <= p.N ? 16 : p.N - n;
+      float y[16];
+#pragma unroll
+      for (int i = 0; i < 16; ++i) {
+        const float hv = i < cnt ? v[i] : 0.f;
+        ss += hv * hv;
+        y[i] = i < cnt ? hv * bf2f(p.epi.norm_w[n + i]) : 0.f;
+      }
+      const size_t off = static_cast<size_t>(m) * p.epi.ldn + n;
+      if (cnt == 16 && (p.epi.ldn & 7) == 0) {
+        store_split16(p.epi.norm_hi + off, p.epi.norm_lo + off, y);
+      } else {
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+          if (i >= cnt) continue;
+          bf16 hi, lo;
+          split_bf16(y[i], hi, lo);
+          p.epi.norm_hi[off + i] = hi;
+          p.epi.norm_lo[off + i] = lo;
+        }
       }
     }
   }
+  if (norm_next && row_ok) p.epi.ss_out[static_cast<size_t>(n0 / BN) * p.M + m] = ss;
 }
 
 // SwiGLU: tile columns [0, BN/2) are gate features f0.., [BN/2, BN) the matching up features.
@@ -187,6 +232,7 @@ template <int BN>
 __device__ __forceinline__ void epilogue_swiglu(const Params& p, uint32_t trow, int m, int f0) {
   const int F = p.N >> 1;
   const bool row_ok = m < p.M;
+  const float rs = row_scale(p, m);
 #pragma unroll 1
   for (int j = 0; j < BN / 2; j += 16) {
     float g[16], u[16];
@@ -196,12 +242,14 @@ __device__ __forceinline__ void epilogue_swiglu(const Params& p, uint32_t trow, 
     if (!row_ok || f >= F) continue;
     float o[16];
 #pragma unroll
-    for (int i = 0; i < 16; ++i) o[i] = silu_f(g[i]) * u[i];
+    for (int i = 0; i < 16; ++i) o[i] = silu_f(g[i] * rs) * (u[i] * rs);
     const size_t off = static_cast<size_t>(m) * p.epi.ldo + f;
     if (f + 16 <= F && ((p.epi.ldo & 7) == 0)) {
       store_split16(p.epi.out_hi + off, p.epi.out_lo + off, o);
     } else {
-      for (int i = 0; i < 16 && f + i < F; ++i) {
+#pragma unroll
+      for (int i = 0; i < 16; ++i) {
+        if (f + i >= F) continue;
         bf16 hi, lo;
         split_bf16(o[i], hi, lo);
         p.epi.out_hi[off + i] = hi;
@@ -220,6 +268,7 @@ __device__ __forceinline__ void epilogue_qkv(const Params& p, uint32_t trow, int
   const int sec = n0 / d;              // 0 q, 1 k, 2 v
   const int head0 = (n0 - sec * d) / hd;
   const bool row_ok = m < p.M;
+  const float rs = row_scale(p, m);
   RowInfo ri{0, 0, 0, 0};
   if (row_ok) ri = p.epi.rows[m];
   const KVLayout& kv = p.epi.kv;
@@ -240,6 +289,8 @@ __device__ __forceinline__ void epilogue_qkv(const Params& p, uint32_t trow, int
       for (int j = 0; j < hd; j += 16) {
         float v[16];
         ld16f(tcol + j, v);
+#pragma unroll
+        for (int i = 0; i < 16; ++i) v[i] *= rs;
         if (row_ok) store_f16x16(dst + j, v);
       }
     } else {
@@ -254,8 +305,9 @@ __device__ __forceinline__ void epilogue_qkv(const Params& p, uint32_t trow, int
 #pragma unroll
         for (int i = 0; i < 16; ++i) {
           const float2 t = cs[i];
-          ra[i] = a[i] * t.x - b[i] * t.y;
-          rb[i] = b[i] * t.x + a[i] * t.y;
+          const float ai = a[i] * rs, bi = b[i] * rs;
+          ra[i] = ai * t.x - bi * t.y;
+          rb[i] = bi * t.x + ai * t.y;
         }
         if (sec == 0) {
           float* dst = p.epi.out_q + static_cast<size_t>(m) * d + head * hd;
@@ -1470,7 +1522,10 @@ size_t gemm_workspace_bytes(const GemmArgs& a) {
 int gemm_launch(const GemmArgs& a, cudaStream_t stream, int num_sms, GemmCost* cost) {
   if (a.M < 1 || a.N < 1 || a.K < 1 || !a.A || !a.B) return VLA_ERR_ARG;
   if (a.block_n != 128 && a.block_n != 256) return VLA_ERR_ARG;
-  if (a.epi.norm_w) return VLA_ERR_ARG;  // fused RMSNorm: weight-streaming GEMM only
+  // a following RMSNorm: only as the deferred form (ss_out), on an unsplit residual GEMM
+  if (a.epi.norm_w && (!a.epi.ss_out || a.epi.kind != EPI_RESID || !a.epi.norm_hi || !a.epi.norm_lo))
+    return VLA_ERR_ARG;
+  if (a.epi.row_ss && a.epi.kind != EPI_QKV && a.epi.kind != EPI_SWIGLU) return VLA_ERR_ARG;
   if ((a.lda % 8) || (a.ldb % 8) || a.lda < a.K || a.ldb < a.K) return VLA_ERR_ARG;
   if ((reinterpret_cast<uintptr_t>(a.A) & 15) || (reinterpret_cast<uintptr_t>(a.B) & 15) ||
       (reinterpret_cast<uintptr_t>(a.A_lo) & 15))
@@ -1484,6 +1539,7 @@ int gemm_launch(const GemmArgs& a, cudaStream_t stream, int num_sms, GemmCost* c
 
   const int splits = gemm_effective_splits(a.K, a.splits);
   if (a.pair && (BN != 256 || splits != 1)) return VLA_ERR_ARG;
+  if ((a.epi.ss_out || a.epi.row_ss) && splits != 1) return VLA_ERR_ARG;
   const int kbt = (a.K + BK - 1) / BK;
   Params p{};
   p.M = a.M;
