@@ -37,7 +37,8 @@ namespace {
 constexpr int BM = 128;
 constexpr int BK = 64;  // 64 bf16 = 128 bytes = one swizzle atom row
 constexpr int kThreads = 192;
-constexpr int kGroupM = 16;
+constexpr int kGroupM = 16;      // 128-row m-tiles per raster group (2048 rows)
+constexpr int kGroupMPair = 8;   // 256-row m-tiles per raster group of the pair kernel
 
 // Shared-memory matrix descriptor: K-major operand, 128-byte swizzle, rows of 128 bytes,
 // 8-row core-matrix groups 1024 bytes apart (SBO); LBO unused for this layout.
@@ -61,17 +62,18 @@ __device__ __forceinline__ constexpr uint32_t make_idesc() {
 struct Params {
   int M, N, K;          // N: columns of B used (SwiGLU: 2F)
   int tiles_m, tiles_n, splits, kb_total, kb_per_split;
+  int group_m;          // m-tiles per raster group
   EpiArgs epi;
 };
 
 __device__ __forceinline__ void unit_coords(const Params& p, int u, int& m_blk, int& n_blk,
                                             int& split) {
   const int ncols = p.tiles_n * p.splits;        // (n-tile, split) pairs
-  const int per_group = kGroupM * ncols;
+  const int per_group = p.group_m * ncols;
   const int g = u / per_group;
   const int r = u - g * per_group;
-  const int first_m = g * kGroupM;
-  const int gsize = min(kGroupM, p.tiles_m - first_m);
+  const int first_m = g * p.group_m;
+  const int gsize = min(p.group_m, p.tiles_m - first_m);
   m_blk = first_m + r % gsize;
   const int col = r / gsize;
   n_blk = col / p.splits;
@@ -1546,6 +1548,7 @@ int gemm_launch(const GemmArgs& a, cudaStream_t stream, int num_sms, GemmCost* c
   p.N = a.N;
   p.K = a.K;
   p.tiles_m = a.pair ? (a.M + 255) / 256 : (a.M + BM - 1) / BM;
+  p.group_m = a.pair ? kGroupMPair : kGroupM;
   p.splits = splits;
   p.kb_total = kbt;
   p.kb_per_split = (kbt + splits - 1) / splits;
