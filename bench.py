@@ -43,6 +43,19 @@ PROFILED_TRAFFIC = {"bytes": 3.094091e9 + 0.879448e9,
                     "profile": "profiles/gemm_tc2_prefill_qkv_18385x12288x4096.md"}
 
 
+def workload_config(wl, n_gpus):
+    """The `config` object of the JSON line (both arms)."""
+    text = f"U{{{wl.text_len_range[0]}..{wl.text_len_range[1]}}}" if wl.text_len is None else str(wl.text_len)
+    step = ("reset + prefill + 7-token decode" if wl.turns == 1 else
+            f"reset + {wl.turns} turns x (prefill/append + 7-token decode)") + (" + score" if wl.score else "")
+    return {"workload": wl.name, "model": wl.shape.name, "batch_per_gpu": wl.batch, "n_visual": wl.n_visual,
+            "text_len": text, "turns": wl.turns, "append_visual": wl.append_visual if wl.turns > 1 else 0,
+            "append_text": wl.append_text if wl.turns > 1 else 0, "action_tokens": wl.shape.action_dim,
+            "temperature": wl.temperature, "step": step,
+            "l2": "no flush: 13 GB of weights streamed per forward (> 129 MB L2)",
+            "parallelism": f"replicas x{n_gpus}"}
+
+
 def phase_work(sh, past, chunk):
     """Algorithmic work of one turn's phases for envs whose chunk of chunk[b] rows lands after
     past[b] cached positions (7B: 6.476e9 matrix parameters, 16 KB of fp16 K+V per position
@@ -189,8 +202,7 @@ def run_reference(args):
         "n_gpus": world, "steps": args.steps, "warmup": args.warmup, "ms_per_step": per_step * 1e3,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
         "data": "synthetic (seeded; random-init weights)",
-        "config": {"workload": wl.name, "model": wl.shape.name, "batch": wl.batch,
-                   "sample": "1 env per step (prefill + 7 tokens + score)"},
+        "config": dict(workload_config(wl, world), sample="1 env per step (prefill + 7 tokens + score)"),
         "cpu_baseline": {"value": value, "unit": "action tokens/s", "cores": threads, "kind": "oracle",
                          "sample": f"1 of {wl.batch} envs, prefix {prefix} tokens, prefill+decode+score, fp64"},
         "e2e": {"value": value, "unit": "action tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
@@ -663,20 +675,12 @@ def main():
     n_gpus = world
     acts = wl.turns * B * A                     # action tokens per step
     value = n_gpus * acts / (ms_step / 1e3)
-    text = f"U{{{wl.text_len_range[0]}..{wl.text_len_range[1]}}}" if wl.text_len is None else str(wl.text_len)
-    step_desc = ("reset + prefill + 7-token decode" if wl.turns == 1 else
-                 f"reset + {wl.turns} turns x (prefill/append + 7-token decode)") + (" + score" if wl.score else "")
     line = {
         "metric": METRIC, "value": value, "unit": "action tokens/s", "n_gpus": n_gpus,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16 weights, fp32 accumulate",
         "data": "synthetic (seeded; random-init weights)",
-        "config": {"workload": wl.name, "model": sh.name, "batch_per_gpu": B, "n_visual": wl.n_visual,
-                   "text_len": text, "turns": wl.turns, "append_visual": wl.append_visual if wl.turns > 1 else 0,
-                   "append_text": wl.append_text if wl.turns > 1 else 0, "action_tokens": A, "temperature": T,
-                   "step": step_desc,
-                   "l2": "no flush: 13 GB of weights streamed per forward (> 129 MB L2)",
-                   "parallelism": f"replicas x{n_gpus}"},
+        "config": workload_config(wl, n_gpus),
         "phases": phase,
         "roofline": roof, "roofline_decode": roof_dec, "phase_roofline": phase_roof,
         "e2e": {"value": n_gpus * acts / (e2e_ms / 1e3), "unit": "action tokens/s",
