@@ -227,6 +227,7 @@ CASES = {
     "attn_decode": None,                                       # see run_attn_case
     "learning": None,                                          # see run_learning_case
     "attn_chunk": None,                                        # see run_attn_chunk_case
+    "attn_score": None,                                        # 6 rows per env after the prefix
     # the same prefill shapes on CTA pairs (2-SM MMAs, 256 x 256 tiles)
     "pair_prefill_qkv": (4608, 12288, 4096, 256, 1, True),
     "pair_prefill_down": (4608, 4096, 11008, 256, 1, True),
@@ -311,14 +312,17 @@ def run_attn_chunk_case(args):
     from paper_2505_18719_gb300 import inputs as I
     from paper_2505_18719_gb300 import vla as V
     B, H, hd, cap = 64, 32, 128, 320
-    lens = (256 + I.randint_i32((B,), 5, 7, 16, 48)).tolist()
+    prefix = (256 + I.randint_i32((B,), 5, 7, 16, 48)).tolist()
+    score = args.case == "attn_score"       # the score pass: 6 rows per env after its prefix
+    lens = [6] * B if score else prefix
+    past = prefix if score else [0] * B
     rows = sum(lens)
     kv = I.normal_bf16((B, 2, H, cap, hd), 5, 1, 1.0).cuda().half()
     q = I.normal_bf16((rows, H * hd), 5, 2, 1.0).cuda().float()
     tiles, r = [], 0
     for b, n in enumerate(lens):
         for t0 in range(0, n, 64):
-            tiles.append((b, r + t0, min(64, n - t0), t0))
+            tiles.append((b, r + t0, min(64, n - t0), past[b] + t0))
         r += n
     tiles_dev = torch.zeros(len(tiles) * 4, dtype=torch.int32, device="cuda")
     oh = torch.empty(rows, H * hd, dtype=torch.bfloat16, device="cuda")
@@ -339,11 +343,12 @@ def run_attn_chunk_case(args):
     e1.record()
     torch.cuda.synchronize()
     ms = e0.elapsed_time(e1) / args.steps
-    flops = sum(2.0 * H * hd * n * (n + 1) for n in lens)   # causal QK^T + PV
+    flops = sum(2.0 * H * hd * n * (n + 1 + 2 * p) for n, p in zip(lens, past))   # causal QK^T + PV
+    kv_bytes = sum((p + n) * 2.0 * H * hd * 2 for n, p in zip(lens, past))
     _, tf_burst, _, kind = peaks()
     print(json.dumps({"case": args.case, "B": B, "H": H, "hd": hd, "rows": rows, "tiles": len(tiles), "ms": ms,
                       "tflops": flops / ms / 1e9, "tc_frac_of_burst": flops / ms / 1e9 / tf_burst,
-                      "issued_mma_tflops": 2 * flops / ms / 1e9, "peaks": kind}))
+                      "issued_mma_tflops": 2 * flops / ms / 1e9, "kv_gbs": kv_bytes / ms / 1e6, "peaks": kind}))
     return 0
 
 
@@ -396,7 +401,7 @@ def run_case(args):
         return run_attn_case(args)
     if args.case == "learning":
         return run_learning_case(args)
-    if args.case == "attn_chunk":
+    if args.case in ("attn_chunk", "attn_score"):
         return run_attn_chunk_case(args)
     M, N, K, bn, splits, split_a = CASES[args.case]
     A = I.normal_bf16((M, K), 1, 1, 1.0).cuda()

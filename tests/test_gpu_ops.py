@@ -230,3 +230,4 @@ def test_chunk_attention_matches_fp64(hd):
     bad = [(0, 0, 65, 0)]
     assert V.vla_op_attn_chunk(qd.data_ptr(), kvd.data_ptr(), max_env, H, hd, cap, bad, rows,
                                tiles_dev.data_ptr(), oh.data_ptr(), ol.data_ptr()) == V.VLA_ERR_ARG
+
