@@ -130,7 +130,7 @@ int vla_decode_actions(vla_handle* h, const float* uniforms, float temperature,
 int vla_score_actions(vla_handle* h, const int32_t* tokens, float temperature,
                       float* logprobs_out, float* logits_out);
 
-/* Rollout entropy (the training-dynamics quantity of §5): H = -sum_k p_k log p_k of each
+/* Rollout entropy (the training-dynamics quantity of §4.2): H = -sum_k p_k log p_k of each
  * action token's 256-bin distribution in the latest vla_decode_actions or vla_score_actions
  * call on this handle, at that call's temperature (T == 0: the T = 1 distribution, as for
  * the log-probs).  entropy_out device f32 [B, action_dim]; asynchronous on the handle's

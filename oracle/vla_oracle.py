@@ -259,7 +259,7 @@ def sample_bins(z: torch.Tensor, temperature: float, u: Optional[torch.Tensor]):
 
 def token_entropy(z: torch.Tensor, temperature: float) -> float:
     """Entropy of one action token's distribution over the bins (the rollout entropy the
-    paper tracks in its training dynamics, §5): H = -sum_k p_k log p_k with p = softmax(z/T),
+    paper tracks in its training dynamics, §4.2): H = -sum_k p_k log p_k with p = softmax(z/T),
     the distribution the sampler draws from; T = 0 uses T = 1, as the log-probs do."""
     zt = z / temperature if temperature > 0.0 else z
     lp = zt - torch.logsumexp(zt, dim=0)
@@ -287,7 +287,7 @@ def value_head(shape: Shape, W: Weights, h_last: torch.Tensor, w_value: torch.Te
 
 # =========================================================================== learning phase
 def gae(rewards, values, dones, gamma: float, lam: float):
-    """Generalised advantage estimation (Algorithm 1, "compute advantages"; §3.4 cites
+    """Generalised advantage estimation (Algorithm 1, "compute advantages"; §3.3 cites
     Schulman et al. 2015) over M steps of B envs, walking t = M-1 .. 0:
 
       delta_t = r_t + gamma * (1 - done_t) * V_{t+1} - V_t

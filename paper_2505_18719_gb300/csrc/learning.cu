@@ -1,7 +1,7 @@
 // The value model's output and the learning-phase quantities of the method, on the device:
 //  * value head: V(o_t, v_t^in) of Algorithm 1 for a homogeneous value model (the same decoder
 //    as the policy): the final RMSNorm of each env's last prefix row, then one linear output;
-//  * GAE (Algorithm 1, "compute advantages"; §3.4): the reverse recursion over M steps,
+//  * GAE (Algorithm 1, "compute advantages"; §3.3): the reverse recursion over M steps,
 //    one thread per env;
 //  * the clipped PPO objective of Eq. 2 with action log-probs as the sum of the 7 token
 //    log-probs (Eq. 1): one CTA, a fixed-order reduction, so the result is deterministic.

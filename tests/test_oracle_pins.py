@@ -373,7 +373,7 @@ def test_reset_env_restarts_like_a_fresh_env():
 
 # ============================================================================ entropy, value, GAE, PPO
 def test_entropy_closed_forms():
-    """Rollout entropy (§5): uniform logits give log 256 at any T; a two-level z has the closed
+    """Rollout entropy (§4.2): uniform logits give log 256 at any T; a two-level z has the closed
     form -p1 log p1 - 255 p0 log p0; H(z, T) = H(z / T, 1); 0 <= H <= log 256."""
     z0 = torch.zeros(256, dtype=torch.float64)
     for T in (0.0, 0.5, 1.0, 1.5):
