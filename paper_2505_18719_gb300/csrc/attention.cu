@@ -274,11 +274,13 @@ __global__ void __launch_bounds__(128) attn_chunk_mma_kernel(const float* __rest
 // output) per range.  The last CTA of an (env, head) to finish (a ticket on counters[b * H +
 // head], no waiting) merges the S partials in range order and writes the normalised output as
 // the bf16 pair; with S == 1 the CTA writes it directly.
-// NW = 2 warps per CTA at <= 64 registers: 16 CTAs fit on an SM, so the 2048 (env, head) CTAs
-// of a 64-env, 32-head step are all resident at once (one wave, no tail).
+// NW = 2 warps per CTA; ptxas allocates 64 registers for both head dims with no spill, so 16
+// CTAs fit on an SM and the 2048 (env, head) CTAs of a 64-env, 32-head step are all resident
+// at once (one wave, no tail).  No minimum-blocks bound is given: capping at 64 forces a small
+// spill in the 64-dim variant.
 constexpr int kDecodeWarps = 2;
 template <int HD, int NW = kDecodeWarps>
-__global__ void __launch_bounds__(NW * 32, 512 / NW) attn_decode_kernel(const float* __restrict__ q,
+__global__ void __launch_bounds__(NW * 32) attn_decode_kernel(const float* __restrict__ q,
                                                           const RowInfo* __restrict__ rows,
                                                           KVLayout kv, int layer, int H,
                                                           int chunk, int S, float scale_log2,

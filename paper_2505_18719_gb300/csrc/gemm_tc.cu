@@ -81,20 +81,6 @@ __device__ __forceinline__ void unit_coords(const Params& p, int u, int& m_blk, 
 }
 
 // ----------------------------------------------------------------------------- epilogues
-__device__ __forceinline__ void store_bf16x16(bf16* dst, const float (&v)[16]) {
-  uint4 a, b;
-  a.x = pack_bf16x2(v[0], v[1]);
-  a.y = pack_bf16x2(v[2], v[3]);
-  a.z = pack_bf16x2(v[4], v[5]);
-  a.w = pack_bf16x2(v[6], v[7]);
-  b.x = pack_bf16x2(v[8], v[9]);
-  b.y = pack_bf16x2(v[10], v[11]);
-  b.z = pack_bf16x2(v[12], v[13]);
-  b.w = pack_bf16x2(v[14], v[15]);
-  reinterpret_cast<uint4*>(dst)[0] = a;
-  reinterpret_cast<uint4*>(dst)[1] = b;
-}
-
 // 16 values as bf16 hi/lo pairs (two 32-byte stores each).
 __device__ __forceinline__ void store_split16(bf16* hi_dst, bf16* lo_dst, const float (&v)[16]) {
   uint32_t h[8], l[8];
