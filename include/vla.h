@@ -13,9 +13,16 @@
  *
  * Conventions for every call:
  *  - All device pointers are CUDA device memory on the handle's device, 16-byte aligned.
- *    Weights are BORROWED: the caller keeps them alive and unchanged for the handle's life.
- *    Output buffers are caller-allocated device memory.  The handle owns its KV cache and
- *    workspaces (allocated in vla_create, freed in vla_destroy).
+ *    Weights are BORROWED: the caller keeps them alive for the handle's life.  The four
+ *    projection matrices (q|k|v, o, gate|up, down) are read once into an fp16 copy that the
+ *    handle owns (vla_create; again at vla_sync_weights after the caller changed them, e.g.
+ *    after a learner update); every other weight is read where it lies at each call.
+ *    Output buffers are caller-allocated device memory.  The handle owns its KV cache,
+ *    workspaces and the fp16 projection copy (allocated in vla_create, freed in vla_destroy).
+ *  - Arithmetic: every projection runs on fp16 tensor-core operands with fp32 accumulation.
+ *    Its input activation is carried as an fp16 pair hi + lo (~21 significant bits); the
+ *    weight-streaming decode GEMMs multiply both halves, the prefill / score GEMMs both
+ *    halves for q|k|v and hi alone for o, gate|up and down.  K/V are cached in fp16.
  *  - Calls are asynchronous on the handle's stream.  Host-checkable errors return at once,
  *    with no side effects.  Errors found on the device (token id out of range, non-finite
  *    logits, a pipeline wait that timed out) set a device status word; the next vla_sync
@@ -82,9 +89,12 @@ typedef struct {
 
 /* Create a handle on the current CUDA device.  `cuda_stream` is a cudaStream_t (NULL =
  * the legacy default stream).  Allocates the KV cache
- * (n_layers * max_batch * 2 * d_model * kv_capacity bf16) and workspaces.
- * Returns VLA_ERR_ARG / VLA_ERR_UNSUPPORTED / VLA_ERR_OOM / VLA_ERR_CUDA on failure, with
- * *out = NULL. */
+ * (n_layers * max_batch * 2 * d_model * kv_capacity fp16), the fp16 copy of the projection
+ * matrices (n_layers * (4 d^2 + 3 d_ffn d) fp16) and workspaces, then fills the copy from the
+ * bf16 weights and waits for it.  A bf16 weight with 2^-14 <= |w| <= 65504 is exact in
+ * fp16; a smaller one rounds to a multiple of 2^-24.
+ * Returns VLA_ERR_ARG / VLA_ERR_UNSUPPORTED (also: a projection weight with |w| > 65504 or
+ * not finite) / VLA_ERR_OOM / VLA_ERR_CUDA on failure, with *out = NULL. */
 int vla_create(const vla_config* cfg, const vla_weights* w, void* cuda_stream, vla_handle** out);
 
 /* Prefill (Algorithm 1: h(o_t) then π_θ over the state; §3.3 multi-turn append).
@@ -173,6 +183,14 @@ int vla_reset(vla_handle* h, const uint8_t* env_mask);
 
 /* Synchronise the handle's stream and read the device status word. */
 int vla_sync(vla_handle* h);
+
+/* Re-read the four projection matrices from the borrowed bf16 pointers given to vla_create
+ * into the handle's fp16 copy (after the caller changed them in place, e.g. a PPO update of
+ * θ between rollouts, Algorithm 1).  Runs on the handle's stream after all work queued before
+ * it and waits for it; later calls see the new weights.  Norm gains, embeddings and lm_head
+ * are read in place at every call and need no sync.  VLA_ERR_UNSUPPORTED if a weight is
+ * outside the fp16 range (the copy then holds it clamped to +-65504). */
+int vla_sync_weights(vla_handle* h);
 
 /* Current context length of env b (host bookkeeping, no sync); -1 if out of range. */
 int vla_context_length(const vla_handle* h, int env);

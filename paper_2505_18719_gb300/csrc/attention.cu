@@ -74,7 +74,7 @@ __global__ void __launch_bounds__(128) attn_chunk_mma_kernel(const float* __rest
                                                              bf16* __restrict__ out_lo,
                                                              const AttnTile* __restrict__ tiles,
                                                              KVLayout kv, int layer, int H,
-                                                             float scale_log2) {
+                                                             float scale_log2, bool fp16) {
   constexpr int KB = 64;       // keys per block
   constexpr int LD = HD + 8;   // padded row (halves): 16-byte rows land in distinct banks
   constexpr int CPR = HD / 8;  // 16-byte chunks per row
@@ -252,14 +252,14 @@ __global__ void __launch_bounds__(128) attn_chunk_mma_kernel(const float* __rest
     if (r0 < t.nrows) {
       const size_t off = static_cast<size_t>(t.row0 + r0) * d + col;
       uint32_t hi, lo;
-      split_pack2(o[nt][0] * inv0, o[nt][1] * inv0, hi, lo);
+      split_pack2(o[nt][0] * inv0, o[nt][1] * inv0, hi, lo, fp16);
       *reinterpret_cast<uint32_t*>(out_hi + off) = hi;
       *reinterpret_cast<uint32_t*>(out_lo + off) = lo;
     }
     if (r1 < t.nrows) {
       const size_t off = static_cast<size_t>(t.row0 + r1) * d + col;
       uint32_t hi, lo;
-      split_pack2(o[nt][2] * inv1, o[nt][3] * inv1, hi, lo);
+      split_pack2(o[nt][2] * inv1, o[nt][3] * inv1, hi, lo, fp16);
       *reinterpret_cast<uint32_t*>(out_hi + off) = hi;
       *reinterpret_cast<uint32_t*>(out_lo + off) = lo;
     }
@@ -288,7 +288,7 @@ __global__ void __launch_bounds__(NW * 32) attn_decode_kernel(const float* __res
                                                           float2* __restrict__ part_ml,
                                                           int* __restrict__ counters,
                                                           bf16* __restrict__ out_hi,
-                                                          bf16* __restrict__ out_lo) {
+                                                          bf16* __restrict__ out_lo, bool fp16) {
   constexpr int LPK = HD / 8;     // lanes per key row (8 fp16 = 16 bytes per lane)
   constexpr int KPI = 32 / LPK;   // key rows per warp instruction
   constexpr int U = 4;            // key rows per lane group loaded ahead
@@ -395,10 +395,7 @@ __global__ void __launch_bounds__(NW * 32) attn_decode_kernel(const float* __res
       for (int w = 0; w < NW; ++w)
         for (int k = 0; k < KPI; ++k)
           if (s_m[w][k] != -INFINITY) acc += s_o[w][k][c] * exp2f(s_m[w][k] - M);
-      bf16 hi, lo;
-      split_bf16(acc / L, hi, lo);
-      out_hi[out_off + c] = hi;
-      out_lo[out_off + c] = lo;
+      store_split1(out_hi, out_lo, out_off + c, acc / L, fp16);
     }
     return;
   }
@@ -441,10 +438,7 @@ __global__ void __launch_bounds__(NW * 32) attn_decode_kernel(const float* __res
   for (int i = 0; i < (HD + NT - 1) / NT; ++i) {
     const int c = threadIdx.x + i * NT;
     if (c < HD) {
-      bf16 hi, lo;
-      split_bf16(acc[i] / Lt, hi, lo);
-      out_hi[out_off + c] = hi;
-      out_lo[out_off + c] = lo;
+      store_split1(out_hi, out_lo, out_off + c, acc[i] / Lt, fp16);
     }
   }
   if (threadIdx.x == 0) counters[bh] = 0;  // ready for the next launch
@@ -453,7 +447,7 @@ __global__ void __launch_bounds__(NW * 32) attn_decode_kernel(const float* __res
 }  // namespace
 
 int attn_chunk_launch(const float* q, bf16* out_hi, bf16* out_lo, const AttnTile* tiles,
-                      int n_tiles, KVLayout kv, int layer, int H, int hd, cudaStream_t stream) {
+                      int n_tiles, KVLayout kv, int layer, int H, int hd, cudaStream_t stream, bool fp16) {
   if (n_tiles <= 0) return VLA_OK;
   const float scale_log2 = 1.4426950408889634f / sqrtf(static_cast<float>(hd));
   dim3 grid(n_tiles, H);
@@ -466,7 +460,7 @@ int attn_chunk_launch(const float* q, bf16* out_hi, bf16* out_lo, const AttnTile
       set = true;
     }
     VLA_CUDA_TRY(launch_pdl(attn_chunk_mma_kernel<128>, grid, dim3(128), smem, stream, q, out_hi, out_lo,
-                            tiles, kv, layer, H, scale_log2));
+                            tiles, kv, layer, H, scale_log2, fp16));
   } else if (hd == 64) {
     const int smem = (4 * 64) * (64 + 8) * 2;
     static bool set = false;
@@ -476,7 +470,7 @@ int attn_chunk_launch(const float* q, bf16* out_hi, bf16* out_lo, const AttnTile
       set = true;
     }
     VLA_CUDA_TRY(launch_pdl(attn_chunk_mma_kernel<64>, grid, dim3(128), smem, stream, q, out_hi, out_lo,
-                            tiles, kv, layer, H, scale_log2));
+                            tiles, kv, layer, H, scale_log2, fp16));
   } else {
     return VLA_ERR_UNSUPPORTED;
   }
@@ -487,7 +481,7 @@ int attn_chunk_launch(const float* q, bf16* out_hi, bf16* out_lo, const AttnTile
 
 int attn_decode_launch(const float* q, bf16* out_hi, bf16* out_lo, const RowInfo* rows, int B,
                        int max_ctx, KVLayout kv, int layer, int H, int hd, int chunk,
-                       float* part_o, float2* part_ml, int* counters, cudaStream_t stream) {
+                       float* part_o, float2* part_ml, int* counters, cudaStream_t stream, bool fp16) {
   if (B <= 0) return VLA_OK;
   // equal key ranges (multiples of 16) no longer than `chunk`
   const int S = (max_ctx + chunk - 1) / chunk;
@@ -496,10 +490,10 @@ int attn_decode_launch(const float* q, bf16* out_hi, bf16* out_lo, const RowInfo
   dim3 grid(S, H, B);
   if (hd == 128) {
     VLA_CUDA_TRY(launch_pdl(attn_decode_kernel<128>, grid, dim3(kDecodeWarps * 32), 0, stream, q, rows, kv, layer, H,
-                            c, S, scale_log2, part_o, part_ml, counters, out_hi, out_lo));
+                            c, S, scale_log2, part_o, part_ml, counters, out_hi, out_lo, fp16));
   } else if (hd == 64) {
     VLA_CUDA_TRY(launch_pdl(attn_decode_kernel<64>, grid, dim3(kDecodeWarps * 32), 0, stream, q, rows, kv, layer, H,
-                            c, S, scale_log2, part_o, part_ml, counters, out_hi, out_lo));
+                            c, S, scale_log2, part_o, part_ml, counters, out_hi, out_lo, fp16));
   } else {
     return VLA_ERR_UNSUPPORTED;
   }

@@ -10,16 +10,19 @@ struct AttnTile {
   int env, row0, nrows, pos0;
 };
 
-// q: f32 [rows, H*hd]; out: bf16 hi/lo pair [rows, H*hd]; keys from the fp16 cache of `layer`.
+// q: f32 [rows, H*hd]; out: hi/lo operand pair [rows, H*hd], fp16 if `fp16` else bf16; keys
+// from the fp16 cache of `layer`.
 int attn_chunk_launch(const float* q, bf16* out_hi, bf16* out_lo, const AttnTile* tiles,
-                      int n_tiles, KVLayout kv, int layer, int H, int hd, cudaStream_t stream);
+                      int n_tiles, KVLayout kv, int layer, int H, int hd, cudaStream_t stream,
+                      bool fp16);
 
 // One query per env row b (rows[b] gives env and position); key range split into equal ranges
 // of at most `chunk` keys (a multiple of 16 at least 16); partials in part_o [B*H*S*hd] f32 and part_ml [B*H*S]
 // (S = ceil(max_ctx/chunk)); counters [B*H] int must be zero at launch and are zero again
-// when the kernel completes.
+// when the kernel completes.  The output pair is fp16 if `fp16`, else bf16.
 int attn_decode_launch(const float* q, bf16* out_hi, bf16* out_lo, const RowInfo* rows, int B,
                        int max_ctx, KVLayout kv, int layer, int H, int hd, int chunk,
-                       float* part_o, float2* part_ml, int* counters, cudaStream_t stream);
+                       float* part_o, float2* part_ml, int* counters, cudaStream_t stream,
+                       bool fp16);
 
 }  // namespace vla

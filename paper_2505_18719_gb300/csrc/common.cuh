@@ -76,6 +76,56 @@ __device__ __forceinline__ void split_pack2(float a, float b, uint32_t& hi, uint
   lo = *reinterpret_cast<uint32_t*>(&l2);
 }
 
+// The same pair in fp16: hi = fp16(x), lo = fp16(x - hi).  fp16 keeps 11 significant bits
+// per half (bf16: 8), so the single hi alone is 8x closer to x than a bf16 hi; GEMMs fed the
+// fp16 form run on fp16 weights.  x is clamped to the finite fp16 range first (|x| <= 65504),
+// so an out-of-range activation saturates instead of turning into inf / NaN.
+__device__ __forceinline__ void split_f16(float x, f16& hi, f16& lo) {
+  x = fminf(fmaxf(x, -65504.f), 65504.f);
+  hi = __float2half_rn(x);
+  lo = __float2half_rn(x - __half2float(hi));
+}
+__device__ __forceinline__ void split_pack2_f16(float a, float b, uint32_t& hi, uint32_t& lo) {
+  f16 ha, la, hb, lb;
+  split_f16(a, ha, la);
+  split_f16(b, hb, lb);
+  __half2 h2 = __halves2half2(ha, hb), l2 = __halves2half2(la, lb);
+  hi = *reinterpret_cast<uint32_t*>(&h2);
+  lo = *reinterpret_cast<uint32_t*>(&l2);
+}
+// Operand format chosen at run time (uniform across a launch): fp16 if `fp16`, else bf16.  Buffers of
+// either format are 2-byte arrays; the pair halves come back as raw bits.
+__device__ __forceinline__ void split_pack2(float a, float b, uint32_t& hi, uint32_t& lo, bool fp16) {
+  if (fp16)
+    split_pack2_f16(a, b, hi, lo);
+  else
+    split_pack2(a, b, hi, lo);
+}
+__device__ __forceinline__ void split_bits(float x, bool fp16, uint16_t& hi, uint16_t& lo) {
+  if (fp16) {
+    f16 h, l;
+    split_f16(x, h, l);
+    hi = __half_as_ushort(h);
+    lo = __half_as_ushort(l);
+  } else {
+    bf16 h, l;
+    split_bf16(x, h, l);
+    hi = __bfloat16_as_ushort(h);
+    lo = __bfloat16_as_ushort(l);
+  }
+}
+// Stores x as the pair into hi[i] / lo[i] (2-byte elements of either format).
+__device__ __forceinline__ void store_split1(void* hi, void* lo, size_t i, float x, bool fp16) {
+  uint16_t h, l;
+  split_bits(x, fp16, h, l);
+  static_cast<uint16_t*>(hi)[i] = h;
+  static_cast<uint16_t*>(lo)[i] = l;
+}
+// Reads a 2-byte operand element of either format.
+__device__ __forceinline__ float op2f(uint16_t bits, bool fp16) {
+  return fp16 ? __half2float(__ushort_as_half(bits)) : __bfloat162float(__ushort_as_bfloat16(bits));
+}
+
 __device__ __forceinline__ float warp_sum(float v) {
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);

@@ -95,19 +95,27 @@ struct vla_handle {
   cudaStream_t stream = nullptr;
   int num_sms = 148;
   int max_tokens = 0;
-  // borrowed weights
+  // borrowed weights (bf16); the projections are read through the fp16 copies below
   const bf16* embed = nullptr;
-  std::vector<const bf16*> attn_norm, wqkv, wo, ffn_norm, wgu, wdown;
+  std::vector<const bf16*> attn_norm, ffn_norm;
+  std::vector<const bf16*> src_wqkv, src_wo, src_wgu, src_wdown;
+  // owned fp16 copies of the projection matrices (one allocation, per layer q|k|v, o,
+  // gate|up, down), written by vla_create and vla_sync_weights; wqkv .. wdown point into it
+  f16* w16 = nullptr;
+  std::vector<const bf16*> wqkv, wo, wgu, wdown;   // 2-byte fp16 elements (GemmArgs type)
+  int* w16_range = nullptr;  // device flag: a converted weight was outside the fp16 range
+  // operand format of every projection and of the activations that feed them
+  bool fp16 = true;
   const bf16* final_norm = nullptr;
   const bf16* head_rows = nullptr;
   // owned device memory
   f16* kv = nullptr;      // KV cache [L][B][2][H][cap][hd] fp16
   KVLayout kvl{};
   float* h = nullptr;    // residual stream f32 [T, d]
-  bf16* y = nullptr;     // RMSNorm output, bf16 pair: hi [T, d] then lo [T, d]
+  bf16* y = nullptr;     // RMSNorm output, operand pair: hi [T, d] then lo [T, d]
   float* q = nullptr;    // RoPE'd queries f32 [T, d]
-  bf16* ao = nullptr;    // attention output, bf16 pair [2][T, d]
-  bf16* u = nullptr;     // SwiGLU output, bf16 pair [2][T, F]
+  bf16* ao = nullptr;    // attention output, operand pair [2][T, d]
+  bf16* u = nullptr;     // SwiGLU output, operand pair [2][T, F]
   float* ws = nullptr;
   size_t ws_bytes = 0;
   float* h_last = nullptr;
@@ -209,7 +217,16 @@ void prof_harvest(vla_handle* h) {
   h->ev_used.clear();
 }
 
-// A is the bf16 hi/lo pair: hi at A, lo at A + a_plane.
+// Projections whose tile (prefill / score) GEMMs also multiply the low half of the activation
+// pair.  An fp16 activation alone is within 2^-12 relative of its value; carried through the
+// 32 layers of a 7B decoder that keeps the action-bin logits within ~0.02 of exact, and the
+// pair on q|k|v alone brings them to ~0.016 for 62 % of the MMA work of pairs everywhere.
+// The weight-streaming (decode) GEMMs always take both halves: they are bound by reading the
+// weights, so the second MMA costs nothing there.
+enum : unsigned { kProjQkv = 1, kProjO = 2, kProjGateUp = 4, kProjDown = 8 };
+constexpr unsigned kTileLoMask = kProjQkv;
+
+// A is the operand pair: hi at A, lo at A + a_plane (fp16 when h->fp16, else bf16).
 // The GEMM that will consume h->y after a residual GEMM's RMSNorm (its N, K and epilogue).
 struct NextGemm {
   int N, K, epi;
@@ -222,9 +239,14 @@ struct NextGemm {
 int run_gemm(vla_handle* h, int cls, const bf16* A, size_t a_plane, int lda, const bf16* W, int ldw,
              int M, int N, int K, EpiArgs epi, const NextGemm* next = nullptr) {
   const Plan pl = plan_gemm(M, N, K, epi.kind, h->cfg.d_model, h->num_sms);
+  const bool stream_k = M <= 128;  // decode-sized: weight-streaming swap-AB GEMM
+  const unsigned proj = epi.kind == EPI_QKV      ? kProjQkv
+                        : epi.kind == EPI_SWIGLU ? kProjGateUp
+                        : A == h->ao             ? kProjO
+                                                 : kProjDown;
   GemmArgs g;
   g.A = A;
-  g.A_lo = A + a_plane;
+  g.A_lo = (stream_k || (kTileLoMask & proj)) ? A + a_plane : nullptr;
   g.lda = lda;
   g.B = W;
   g.ldb = ldw;
@@ -236,8 +258,8 @@ int run_gemm(vla_handle* h, int cls, const bf16* A, size_t a_plane, int lda, con
   g.workspace = h->ws;
   g.workspace_bytes = h->ws_bytes;
   epi.status = h->status;
+  epi.fp16 = h->fp16;
   g.epi = epi;
-  const bool stream_k = M <= 128;  // decode-sized: weight-streaming swap-AB GEMM
   if (!stream_k && gemm_workspace_bytes(g) > h->ws_bytes) {
     g.splits = 1;
   }
@@ -286,7 +308,8 @@ int run_gemm(vla_handle* h, int cls, const bf16* A, size_t a_plane, int lda, con
   }
   if (!stream_k && norm.norm_w && !defer_norm) {
     ev = prof_begin(h, VLA_KCLASS_OTHER);
-    rc = rmsnorm_launch(norm.resid, norm.norm_w, M, N, norm.norm_eps, norm.norm_hi, norm.norm_lo, h->stream);
+    rc = rmsnorm_launch(norm.resid, norm.norm_w, M, N, norm.norm_eps, norm.norm_hi, norm.norm_lo, h->stream,
+                        h->fp16);
     prof_end(h, ev, VLA_KCLASS_OTHER, 0, 6.0 * M * N);
     if (rc) return fail(h, rc, t_err);
   }
@@ -317,7 +340,8 @@ int forward_layers(vla_handle* h, int M, const RowInfo* rows_dev, bool decode, i
   // the first layer's attention RMSNorm; every later RMSNorm follows a residual add
   h->y_deferred = false;
   int ev = prof_begin(h, VLA_KCLASS_OTHER);
-  if ((rc = rmsnorm_launch(h->h, h->attn_norm[0], M, d, c.rms_eps, h->y, h->y + pd, h->stream))) return fail(h, rc, t_err);
+  if ((rc = rmsnorm_launch(h->h, h->attn_norm[0], M, d, c.rms_eps, h->y, h->y + pd, h->stream, h->fp16)))
+    return fail(h, rc, t_err);
   prof_end(h, ev, VLA_KCLASS_OTHER, 0, 6.0 * M * d);
   for (int l = 0; l < c.n_layers; ++l) {
 
@@ -343,18 +367,18 @@ int forward_layers(vla_handle* h, int M, const RowInfo* rows_dev, bool decode, i
       prof_end(h, ev, VLA_KCLASS_OTHER, 0, 16.0 * last->n * d);
       ev = prof_begin(h, VLA_KCLASS_ATTN_DECODE);
       rc = attn_decode_launch(h->q_last, h->ao, h->ao + pd, last->rows, last->n, last->max_ctx, h->kvl, l, H, hd,
-                              h->attn_chunk, h->part_o, h->part_ml, h->attn_tickets, h->stream);
+                              h->attn_chunk, h->part_o, h->part_ml, h->attn_tickets, h->stream, h->fp16);
       prof_end(h, ev, VLA_KCLASS_ATTN_DECODE, 0, 0);
       Mr = last->n;
       resid = h->h_last;
     } else if (decode) {
       ev = prof_begin(h, VLA_KCLASS_ATTN_DECODE);
       rc = attn_decode_launch(h->q, h->ao, h->ao + pd, rows_dev, M, max_ctx, h->kvl, l, H, hd,
-                              h->attn_chunk, h->part_o, h->part_ml, h->attn_tickets, h->stream);
+                              h->attn_chunk, h->part_o, h->part_ml, h->attn_tickets, h->stream, h->fp16);
       prof_end(h, ev, VLA_KCLASS_ATTN_DECODE, 0, 0);
     } else {
       ev = prof_begin(h, VLA_KCLASS_ATTN_PREFILL);
-      rc = attn_chunk_launch(h->q, h->ao, h->ao + pd, h->tiles, n_tiles, h->kvl, l, H, hd, h->stream);
+      rc = attn_chunk_launch(h->q, h->ao, h->ao + pd, h->tiles, n_tiles, h->kvl, l, H, hd, h->stream, h->fp16);
       prof_end(h, ev, VLA_KCLASS_ATTN_PREFILL, 0, 0);
     }
     if (rc) return fail(h, rc, t_err);
@@ -397,6 +421,41 @@ int forward_layers(vla_handle* h, int M, const RowInfo* rows_dev, bool decode, i
 
 bool finite_nonneg(float t) { return std::isfinite(t) && t >= 0.f; }
 
+// fp16 elements of the projection copies: per layer 3d*d + d*d + 2F*d + d*F.
+size_t w16_elems(const vla_config& c) {
+  const size_t d = c.d_model, F = c.d_ffn;
+  return static_cast<size_t>(c.n_layers) * (4 * d * d + 3 * F * d);
+}
+
+// Converts every borrowed bf16 projection matrix into the handle's fp16 copy on h->stream and
+// waits; VLA_ERR_UNSUPPORTED when a weight was outside the fp16 range (clamped in the copy).
+int convert_weights(vla_handle* h) {
+  const vla_config& c = h->cfg;
+  const size_t dd = static_cast<size_t>(c.d_model) * c.d_model, fd = static_cast<size_t>(c.d_ffn) * c.d_model;
+  if (cudaMemsetAsync(h->w16_range, 0, sizeof(int), h->stream) != cudaSuccess)
+    return cuda_fail(cudaGetLastError(), "weight conversion: flag reset");
+  for (int l = 0; l < c.n_layers; ++l) {
+    const struct {
+      const bf16* src;
+      const bf16* dst;
+      size_t n;
+    } m[4] = {{h->src_wqkv[l], h->wqkv[l], 3 * dd}, {h->src_wo[l], h->wo[l], dd},
+              {h->src_wgu[l], h->wgu[l], 2 * fd}, {h->src_wdown[l], h->wdown[l], fd}};
+    for (const auto& x : m) {
+      const int rc = bf16_to_f16_launch(x.src, reinterpret_cast<f16*>(const_cast<bf16*>(x.dst)), x.n,
+                                        h->w16_range, h->num_sms, h->stream);
+      if (rc == VLA_ERR_ARG) return record_error(VLA_ERR_ARG, "weight conversion: a projection matrix is not 16-byte aligned");
+      if (rc) return rc;
+    }
+  }
+  int bad = 0;
+  if (cudaMemcpyAsync(&bad, h->w16_range, sizeof(int), cudaMemcpyDeviceToHost, h->stream) != cudaSuccess ||
+      cudaStreamSynchronize(h->stream) != cudaSuccess)
+    return cuda_fail(cudaGetLastError(), "weight conversion");
+  if (bad) return record_error(VLA_ERR_UNSUPPORTED, "a projection weight is outside the fp16 range (|w| > 65504)");
+  return VLA_OK;
+}
+
 }  // namespace
 }  // namespace vla
 
@@ -438,11 +497,11 @@ int vla_create(const vla_config* cfg, const vla_weights* w, void* cuda_stream, v
   h->embed = static_cast<const bf16*>(w->embed);
   for (int l = 0; l < L; ++l) {
     h->attn_norm.push_back(static_cast<const bf16*>(w->attn_norm[l]));
-    h->wqkv.push_back(static_cast<const bf16*>(w->wqkv[l]));
-    h->wo.push_back(static_cast<const bf16*>(w->wo[l]));
+    h->src_wqkv.push_back(static_cast<const bf16*>(w->wqkv[l]));
+    h->src_wo.push_back(static_cast<const bf16*>(w->wo[l]));
     h->ffn_norm.push_back(static_cast<const bf16*>(w->ffn_norm[l]));
-    h->wgu.push_back(static_cast<const bf16*>(w->w_gate_up[l]));
-    h->wdown.push_back(static_cast<const bf16*>(w->w_down[l]));
+    h->src_wgu.push_back(static_cast<const bf16*>(w->w_gate_up[l]));
+    h->src_wdown.push_back(static_cast<const bf16*>(w->w_down[l]));
   }
   h->final_norm = static_cast<const bf16*>(w->final_norm);
   h->head_rows = static_cast<const bf16*>(w->lm_head) + static_cast<size_t>(c.vocab - 256) * d;
@@ -511,6 +570,8 @@ int vla_create(const vla_config* cfg, const vla_weights* w, void* cuda_stream, v
             alloc(reinterpret_cast<void**>(&h->part_o), static_cast<size_t>(B) * c.n_heads * max_S * c.head_dim * sizeof(float)) &&
             alloc(reinterpret_cast<void**>(&h->part_ml), static_cast<size_t>(B) * c.n_heads * max_S * sizeof(float2)) &&
             alloc(reinterpret_cast<void**>(&h->attn_tickets), static_cast<size_t>(B) * c.n_heads * sizeof(int)) &&
+            alloc(reinterpret_cast<void**>(&h->w16), w16_elems(c) * sizeof(f16)) &&
+            alloc(reinterpret_cast<void**>(&h->w16_range), sizeof(int)) &&
             cudaMemset(h->attn_tickets, 0, static_cast<size_t>(B) * c.n_heads * sizeof(int)) == cudaSuccess;
   if (!ok) {
     cudaGetLastError();
@@ -518,6 +579,25 @@ int vla_create(const vla_config* cfg, const vla_weights* w, void* cuda_stream, v
     return set_err(nullptr, VLA_ERR_OOM, "vla_create: device allocation failed");
   }
   h->kvl.base = h->kv;
+  {
+    const size_t dd = static_cast<size_t>(d) * d, fd = static_cast<size_t>(F) * d;
+    f16* p = h->w16;
+    for (int l = 0; l < L; ++l) {
+      h->wqkv.push_back(reinterpret_cast<const bf16*>(p));
+      p += 3 * dd;
+      h->wo.push_back(reinterpret_cast<const bf16*>(p));
+      p += dd;
+      h->wgu.push_back(reinterpret_cast<const bf16*>(p));
+      p += 2 * fd;
+      h->wdown.push_back(reinterpret_cast<const bf16*>(p));
+      p += fd;
+    }
+  }
+  if (const int rc = convert_weights(h)) {
+    const std::string msg = t_err;
+    vla_destroy(h);
+    return set_err(nullptr, rc, msg);
+  }
   // pinned staging
   h->stage_bytes = T * sizeof(RowInfo) + static_cast<size_t>(h->max_tiles) * sizeof(AttnTile) +
                    2 * std::max(T, static_cast<size_t>(B) * A) * sizeof(int) + static_cast<size_t>(B) * sizeof(RowInfo) +
@@ -877,6 +957,14 @@ int vla_sync(vla_handle* h) {
   return VLA_OK;
 }
 
+int vla_sync_weights(vla_handle* h) {
+  if (!h) return set_err(nullptr, VLA_ERR_ARG, "vla_sync_weights: NULL handle");
+  cudaSetDevice(h->dev);
+  const int rc = convert_weights(h);
+  if (rc) return fail(h, rc, t_err);
+  return VLA_OK;
+}
+
 int vla_context_length(const vla_handle* h, int env) {
   if (!h || env < 0 || env >= h->cfg.max_batch) return -1;
   return h->len[env];
@@ -890,7 +978,7 @@ void vla_destroy(vla_handle* h) {
   cudaStreamSynchronize(h->stream);
   void* bufs[] = {h->kv, h->h, h->y, h->q, h->ao, h->u, h->ws, h->h_last, h->head_in, h->head_z, h->head_entropy, h->q_last, h->ss_part, h->last_rows, h->rope,
                   h->rows, h->tiles, h->sidx, h->didx, h->fed, h->pending, h->status, h->part_o,
-                  h->part_ml, h->attn_tickets};
+                  h->part_ml, h->attn_tickets, h->w16, h->w16_range};
   for (void* p : bufs)
     if (p) cudaFree(p);
   for (int s = 0; s < vla_handle::kSlots; ++s) {
@@ -1093,7 +1181,7 @@ int vla_op_attn_decode(const float* q, const void* kv, int max_env, int H, int h
   L.env_stride = 2 * L.kv_stride;
   L.layer_stride = static_cast<int64_t>(max_env) * L.env_stride;
   const int rc = attn_decode_launch(q, static_cast<bf16*>(out_hi), static_cast<bf16*>(out_lo), rows, B, max_ctx, L,
-                                    0, H, hd, chunk, part_o, part_ml, counters, st);
+                                    0, H, hd, chunk, part_o, part_ml, counters, st, false);
   if (rc != VLA_OK && rc != VLA_ERR_CUDA) return set_err(nullptr, rc, "vla_op_attn_decode: unsupported arguments");
   return rc;
 }
@@ -1122,7 +1210,7 @@ int vla_op_attn_chunk(const float* q, const void* kv, int max_env, int H, int hd
   L.env_stride = 2 * L.kv_stride;
   L.layer_stride = static_cast<int64_t>(max_env) * L.env_stride;
   const int rc = attn_chunk_launch(q, static_cast<bf16*>(out_hi), static_cast<bf16*>(out_lo),
-                                   reinterpret_cast<const AttnTile*>(tiles_dev), n_tiles, L, 0, H, hd, st);
+                                   reinterpret_cast<const AttnTile*>(tiles_dev), n_tiles, L, 0, H, hd, st, false);
   if (rc != VLA_OK && rc != VLA_ERR_CUDA) return set_err(nullptr, rc, "vla_op_attn_chunk: unsupported arguments");
   return rc;
 }

@@ -8,7 +8,7 @@ namespace vla {
 enum EpiKind : int {
   EPI_F32 = 0,     // out_f32[m * ldo + n] = y
   EPI_RESID = 1,   // resid[m * ldr + n] += y               (O-proj, down-proj)
-  EPI_SWIGLU = 2,  // u = silu(y_gate) * y_up, f < F = N / 2, stored as the bf16 pair
+  EPI_SWIGLU = 2,  // u = silu(y_gate) * y_up, f < F = N / 2, stored as the operand pair
                    // out_hi / out_lo [m * ldo + f]
   EPI_QKV = 3,     // RoPE(q) -> out_q f32 [M, d]; RoPE(k), v -> fp16 KV cache
   EPI_PARTIAL = 4  // internal: split-K partial sums to the workspace
@@ -16,6 +16,11 @@ enum EpiKind : int {
 
 struct EpiArgs {
   int kind = EPI_F32;
+  // Operand format of the whole call: false = bf16, true = fp16.  It applies to A, A_lo and B
+  // (one tcgen05 kind::f16 MMA takes both operands in one type) and to the pair outputs
+  // out_hi / out_lo and norm_hi / norm_lo, which feed the next projection.  The pointers are
+  // typed bf16 but hold 2-byte elements of the chosen format.
+  bool fp16 = false;
   float* out_f32 = nullptr;
   float* out_q = nullptr;
   bf16* out_hi = nullptr;
@@ -29,7 +34,7 @@ struct EpiArgs {
   const float2* rope = nullptr;   // EPI_QKV: [cap][hd/2] (cos, sin)
   int d = 0, hd = 0;
   // EPI_RESID of the weight-streaming GEMM only: after the residual add, the row's RMSNorm
-  // with weight norm_w (N elements) is written as the bf16 pair norm_hi / norm_lo
+  // with weight norm_w (bf16, N elements) is written as the operand pair norm_hi / norm_lo
   // [m * ldn + n] in the same kernel.  The tile GEMM rejects it.
   const bf16* norm_w = nullptr;
   float norm_eps = 0.f;

@@ -58,6 +58,11 @@ __device__ __forceinline__ constexpr uint32_t make_idesc() {
   return (1u << 4) | (1u << 7) | (1u << 10) | (static_cast<uint32_t>(BN >> 3) << 17) |
          (static_cast<uint32_t>(BM >> 4) << 24);
 }
+// A and B format fields (bits 7-9, 10-12): 1 = bf16, 0 = fp16.
+constexpr uint32_t kIdescBf16Operands = (1u << 7) | (1u << 10);
+__device__ __forceinline__ uint32_t idesc_for(uint32_t bf16_desc, bool fp16) {
+  return fp16 ? (bf16_desc & ~kIdescBf16Operands) : bf16_desc;
+}
 
 struct Params {
   int M, N, K;          // N: columns of B used (SwiGLU: 2F)
@@ -81,11 +86,12 @@ __device__ __forceinline__ void unit_coords(const Params& p, int u, int& m_blk, 
 }
 
 // ----------------------------------------------------------------------------- epilogues
-// 16 values as bf16 hi/lo pairs (two 32-byte stores each).
-__device__ __forceinline__ void store_split16(bf16* hi_dst, bf16* lo_dst, const float (&v)[16]) {
+// 16 values as operand hi/lo pairs, bf16 or (fp16) fp16 (two 32-byte stores each).
+__device__ __forceinline__ void store_split16(bf16* hi_dst, bf16* lo_dst, const float (&v)[16],
+                                              bool fp16) {
   uint32_t h[8], l[8];
 #pragma unroll
-  for (int i = 0; i < 8; ++i) split_pack2(v[2 * i], v[2 * i + 1], h[i], l[i]);
+  for (int i = 0; i < 8; ++i) split_pack2(v[2 * i], v[2 * i + 1], h[i], l[i], fp16);
   reinterpret_cast<uint4*>(hi_dst)[0] = make_uint4(h[0], h[1], h[2], h[3]);
   reinterpret_cast<uint4*>(hi_dst)[1] = make_uint4(h[4], h[5], h[6], h[7]);
   reinterpret_cast<uint4*>(lo_dst)[0] = make_uint4(l[0], l[1], l[2], l[3]);
@@ -199,15 +205,12 @@ __device__ __forceinline__ void epilogue_plain(const Params& p, uint32_t trow, i
       }
       const size_t off = static_cast<size_t>(m) * p.epi.ldn + n;
       if (cnt == 16 && (p.epi.ldn & 7) == 0) {
-        store_split16(p.epi.norm_hi + off, p.epi.norm_lo + off, y);
+        store_split16(p.epi.norm_hi + off, p.epi.norm_lo + off, y, p.epi.fp16);
       } else {
 #pragma unroll
         for (int i = 0; i < 16; ++i) {
           if (i >= cnt) continue;
-          bf16 hi, lo;
-          split_bf16(y[i], hi, lo);
-          p.epi.norm_hi[off + i] = hi;
-          p.epi.norm_lo[off + i] = lo;
+          store_split1(p.epi.norm_hi, p.epi.norm_lo, off + i, y[i], p.epi.fp16);
         }
       }
     }
@@ -233,15 +236,12 @@ __device__ __forceinline__ void epilogue_swiglu(const Params& p, uint32_t trow, 
     for (int i = 0; i < 16; ++i) o[i] = silu_f(g[i] * rs) * (u[i] * rs);
     const size_t off = static_cast<size_t>(m) * p.epi.ldo + f;
     if (f + 16 <= F && ((p.epi.ldo & 7) == 0)) {
-      store_split16(p.epi.out_hi + off, p.epi.out_lo + off, o);
+      store_split16(p.epi.out_hi + off, p.epi.out_lo + off, o, p.epi.fp16);
     } else {
 #pragma unroll
       for (int i = 0; i < 16; ++i) {
         if (f + i >= F) continue;
-        bf16 hi, lo;
-        split_bf16(o[i], hi, lo);
-        p.epi.out_hi[off + i] = hi;
-        p.epi.out_lo[off + i] = lo;
+        store_split1(p.epi.out_hi, p.epi.out_lo, off + i, o[i], p.epi.fp16);
       }
     }
   }
@@ -322,7 +322,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   constexpr int B_BYTES = BN * BK * 2;
   constexpr int STAGE_BYTES = A_TOTAL + B_BYTES;
   constexpr uint32_t TMEM_COLS = 2 * BN;
-  constexpr uint32_t IDESC = make_idesc<BN>();
+  const uint32_t IDESC = idesc_for(make_idesc<BN>(), p.epi.fp16);
   constexpr bool SWIGLU = (EPI == EPI_SWIGLU);
 
   pdl_launch_dependents();
@@ -525,8 +525,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   constexpr int B_BYTES = (BN / 2) * BK * 2;      // this CTA's 128 rows of B
   constexpr int STAGE_BYTES = A_TOTAL + B_BYTES;
   constexpr uint32_t TMEM_COLS = 2 * BN;
-  constexpr uint32_t IDESC = (1u << 4) | (1u << 7) | (1u << 10) | (static_cast<uint32_t>(BN >> 3) << 17) |
-                             (static_cast<uint32_t>(256 >> 4) << 24);
+  const uint32_t IDESC = idesc_for((1u << 4) | (1u << 7) | (1u << 10) | (static_cast<uint32_t>(BN >> 3) << 17) |
+                                       (static_cast<uint32_t>(256 >> 4) << 24),
+                                   p.epi.fp16);
   constexpr bool SWIGLU = (EPI == EPI_SWIGLU);
 
   pdl_launch_dependents();
@@ -764,7 +765,8 @@ __global__ void reduce_f32_kernel(Src src, int M, int N, float* out, int ldo, in
 }
 
 template <class Src>
-__global__ void reduce_swiglu_kernel(Src src, int M, int F, bf16* out_hi, bf16* out_lo, int ldo) {
+__global__ void reduce_swiglu_kernel(Src src, int M, int F, bf16* out_hi, bf16* out_lo, int ldo,
+                                     bool fp16) {
   pdl_launch_dependents();
   pdl_wait();
   const int64_t total = static_cast<int64_t>(M) * F;
@@ -775,10 +777,7 @@ __global__ void reduce_swiglu_kernel(Src src, int M, int F, bf16* out_hi, bf16* 
     split_index<Src>(i, M, F, m, f);
     const float g = src(m, static_cast<int>(f));
     const float u = src(m, static_cast<int>(f) + F);
-    bf16 hi, lo;
-    split_bf16(silu_f(g) * u, hi, lo);
-    out_hi[static_cast<size_t>(m) * ldo + f] = hi;
-    out_lo[static_cast<size_t>(m) * ldo + f] = lo;
+    store_split1(out_hi, out_lo, static_cast<size_t>(m) * ldo + f, silu_f(g) * u, fp16);
   }
 }
 
@@ -956,7 +955,7 @@ __global__ void stream_reduce_f32_kernel(StreamSrc src, int M, int N, float* out
 
 // items (ceil(F / 256), ceil(M / kMR)), 256 threads: gate column f, up column f + F
 __global__ void stream_reduce_swiglu_kernel(StreamSrc src, int M, int F, bf16* out_hi,
-                                            bf16* out_lo, int ldo) {
+                                            bf16* out_lo, int ldo, bool fp16) {
   pdl_launch_dependents();
   pdl_wait();
   const int nx = (F + 255) / 256, ny = (M + kMR - 1) / kMR;
@@ -970,10 +969,7 @@ __global__ void stream_reduce_swiglu_kernel(StreamSrc src, int M, int F, bf16* o
 #pragma unroll
     for (int j = 0; j < kMR; ++j) {
       if (m0 + j >= M) break;
-      bf16 hi, lo;
-      split_bf16(silu_f(g[j]) * u[j], hi, lo);
-      out_hi[static_cast<size_t>(m0 + j) * ldo + f] = hi;
-      out_lo[static_cast<size_t>(m0 + j) * ldo + f] = lo;
+      store_split1(out_hi, out_lo, static_cast<size_t>(m0 + j) * ldo + f, silu_f(g[j]) * u[j], fp16);
     }
   }
 }
@@ -1025,12 +1021,13 @@ __global__ void stream_reduce_qkv_kernel(StreamSrc src, int M, EpiArgs e) {
 }
 
 // grid (M), 1024 threads (N % 4 == 0): h[m][n] += sum, then the RMSNorm of the updated row
-// times w as the bf16 pair y_hi / y_lo (the next GEMM's A).  The row sums are in the same
+// times w as the operand pair y_hi / y_lo (the next GEMM's A; bf16, or fp16 when fp16).  The row sums are in the same
 // order as stream_reduce_f32_kernel's.  At most 48 registers: with one 1024-thread CTA on an
 // SM, the next weight-streaming GEMM's CTA (192 threads x 40) still fits beside it.
 __global__ void __maxnreg__(48) stream_reduce_resid_norm_kernel(StreamSrc src, int N, float* h,
                                                                          int ldh, const bf16* w, float eps,
-                                                                         bf16* y_hi, bf16* y_lo, int ldy) {
+                                                                         bf16* y_hi, bf16* y_lo, int ldy,
+                                                                         bool fp16) {
   pdl_launch_dependents();
   pdl_wait();
   __shared__ float red[32];
@@ -1058,8 +1055,8 @@ __global__ void __maxnreg__(48) stream_reduce_resid_norm_kernel(StreamSrc src, i
     const uint2 ww = *reinterpret_cast<const uint2*>(w + n);
     const float2 w0 = unpack_bf16x2(ww.x), w1 = unpack_bf16x2(ww.y);
     uint2 hi, lo;
-    split_pack2(v.x * r * w0.x, v.y * r * w0.y, hi.x, lo.x);
-    split_pack2(v.z * r * w1.x, v.w * r * w1.y, hi.y, lo.y);
+    split_pack2(v.x * r * w0.x, v.y * r * w0.y, hi.x, lo.x, fp16);
+    split_pack2(v.z * r * w1.x, v.w * r * w1.y, hi.y, lo.y, fp16);
     *reinterpret_cast<uint2*>(y_hi + static_cast<size_t>(m) * ldy + n) = hi;
     *reinterpret_cast<uint2*>(y_lo + static_cast<size_t>(m) * ldy + n) = lo;
   }
@@ -1081,6 +1078,7 @@ struct GemvParams {
   int per_cta, max_seg; // stream-K range length and partial slots per CTA
   float* ws;
   uint32_t* status;
+  bool fp16;            // operand format (weights and activation pair): fp16, else bf16
 };
 
 // TR = 256 weight rows per tile, as two M=128 MMAs sharing each activation tile, so the
@@ -1095,8 +1093,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   constexpr int X_BYTES = BNX * BK * 2;
   constexpr int STAGE_BYTES = W_BYTES + 2 * X_BYTES;
   constexpr uint32_t TMEM_COLS = 2 * NH * BNX;
-  constexpr uint32_t IDESC = (1u << 4) | (1u << 7) | (1u << 10) |
-                             (static_cast<uint32_t>(BNX >> 3) << 17) | (static_cast<uint32_t>(128 >> 4) << 24);
+  const uint32_t IDESC = idesc_for((1u << 4) | (1u << 7) | (1u << 10) | (static_cast<uint32_t>(BNX >> 3) << 17) |
+                                       (static_cast<uint32_t>(128 >> 4) << 24),
+                                   p.fp16);
   static_assert(TMEM_COLS >= 32 && (TMEM_COLS & (TMEM_COLS - 1)) == 0, "TMEM allocation");
 
   pdl_launch_dependents();
@@ -1310,16 +1309,18 @@ EncodeTiledFn encode_fn() {
   return fn;
 }
 
-// 2-D bf16 map over [rows, cols] (row stride ld elements), box {64, box_rows}, 128B swizzle.
+// 2-D map of 2-byte elements (bf16, or fp16 when fp16) over [rows, cols] (row stride ld
+// elements), box {64, box_rows}, 128B swizzle.
 bool make_map(CUtensorMap* m, const void* ptr, int64_t rows, int64_t cols, int64_t ld,
-              int box_rows) {
+              int box_rows, bool fp16 = false) {
   EncodeTiledFn fn = encode_fn();
   if (!fn) return false;
   cuuint64_t dims[2] = {static_cast<cuuint64_t>(cols), static_cast<cuuint64_t>(rows)};
   cuuint64_t strides[1] = {static_cast<cuuint64_t>(ld) * 2};
   cuuint32_t box[2] = {static_cast<cuuint32_t>(BK), static_cast<cuuint32_t>(box_rows)};
   cuuint32_t estr[2] = {1, 1};
-  CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ptr), dims, strides,
+  CUresult r = fn(m, fp16 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2,
+                  const_cast<void*>(ptr), dims, strides,
                   box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
                   CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   return r == CUDA_SUCCESS;
@@ -1423,7 +1424,8 @@ int launch_reduce(const Src& src, const GemmArgs& a, cudaStream_t stream) {
     }
     case EPI_SWIGLU:
       VLA_CUDA_TRY(launch_pdl(reduce_swiglu_kernel<Src>, dim3(blocks_for(static_cast<int64_t>(a.M) * a.N / 2)),
-                              dim3(256), 0, stream, src, a.M, a.N / 2, a.epi.out_hi, a.epi.out_lo, a.epi.ldo));
+                              dim3(256), 0, stream, src, a.M, a.N / 2, a.epi.out_hi, a.epi.out_lo, a.epi.ldo,
+                              a.epi.fp16));
       break;
     case EPI_QKV:
       VLA_CUDA_TRY(launch_pdl(reduce_qkv_kernel<Src>, dim3(blocks_for(static_cast<int64_t>(a.M) * a.N / 2)),
@@ -1542,9 +1544,10 @@ int gemm_launch(const GemmArgs& a, cudaStream_t stream, int num_sms, GemmCost* c
 
   Maps maps;
   CUtensorMap &ma = maps.a, &mb = maps.b, &mb2 = maps.b2;
-  if (!make_map(&ma, a.A, a.M, a.K, a.lda, BM)) return cuda_fail(cudaErrorInvalidValue, "tensor map A");
+  const bool fp16 = a.epi.fp16;
+  if (!make_map(&ma, a.A, a.M, a.K, a.lda, BM, fp16)) return cuda_fail(cudaErrorInvalidValue, "tensor map A");
   maps.a2 = ma;
-  if (split && !make_map(&maps.a2, a.A_lo, a.M, a.K, a.lda, BM))
+  if (split && !make_map(&maps.a2, a.A_lo, a.M, a.K, a.lda, BM, fp16))
     return cuda_fail(cudaErrorInvalidValue, "tensor map A (low half)");
   int run_epi = epi;
   if (splits > 1) {
@@ -1554,19 +1557,19 @@ int gemm_launch(const GemmArgs& a, cudaStream_t stream, int num_sms, GemmCost* c
     run_epi = EPI_PARTIAL;
     p.epi.out_f32 = a.workspace;
     p.tiles_n = (a.N + BN - 1) / BN;
-    if (!make_map(&mb, a.B, a.N, a.K, a.ldb, BN)) return cuda_fail(cudaErrorInvalidValue, "tensor map B");
+    if (!make_map(&mb, a.B, a.N, a.K, a.ldb, BN, fp16)) return cuda_fail(cudaErrorInvalidValue, "tensor map B");
     mb2 = mb;
   } else if (swiglu) {
     const int F = a.N / 2;
     p.tiles_n = (F + BN / 2 - 1) / (BN / 2);
     const bf16* up = a.B + static_cast<size_t>(F) * a.ldb;
     if ((reinterpret_cast<uintptr_t>(up) & 15)) return VLA_ERR_ARG;
-    if (!make_map(&mb, a.B, F, a.K, a.ldb, BN / 2) || !make_map(&mb2, up, F, a.K, a.ldb, BN / 2))
+    if (!make_map(&mb, a.B, F, a.K, a.ldb, BN / 2, fp16) || !make_map(&mb2, up, F, a.K, a.ldb, BN / 2, fp16))
       return cuda_fail(cudaErrorInvalidValue, "tensor map B (gate/up)");
   } else {
     p.tiles_n = (a.N + BN - 1) / BN;
     // a pair's CTAs each load half of the 256-row B tile
-    if (!make_map(&mb, a.B, a.N, a.K, a.ldb, a.pair ? BN / 2 : BN))
+    if (!make_map(&mb, a.B, a.N, a.K, a.ldb, a.pair ? BN / 2 : BN, fp16))
       return cuda_fail(cudaErrorInvalidValue, "tensor map B");
     mb2 = mb;
   }
@@ -1622,8 +1625,9 @@ int gemv_launch(const GemmArgs& a, cudaStream_t stream, int num_sms, GemmCost* c
   if (!a.workspace || a.workspace_bytes < pl.ws_bytes || (reinterpret_cast<uintptr_t>(a.workspace) & 15))
     return VLA_ERR_ARG;
   CUtensorMap mw, mx, mx2;
-  if (!make_map(&mw, a.B, a.N, a.K, a.ldb, 256) || !make_map(&mx, a.A, a.M, a.K, a.lda, pl.bnx) ||
-      !make_map(&mx2, a.A_lo, a.M, a.K, a.lda, pl.bnx))
+  const bool fp16 = a.epi.fp16;
+  if (!make_map(&mw, a.B, a.N, a.K, a.ldb, 256, fp16) || !make_map(&mx, a.A, a.M, a.K, a.lda, pl.bnx, fp16) ||
+      !make_map(&mx2, a.A_lo, a.M, a.K, a.lda, pl.bnx, fp16))
     return cuda_fail(cudaErrorInvalidValue, "tensor maps (decode GEMM)");
   GemvParams p{};
   p.N = a.N;
@@ -1634,6 +1638,7 @@ int gemv_launch(const GemmArgs& a, cudaStream_t stream, int num_sms, GemmCost* c
   p.max_seg = pl.max_seg;
   p.ws = a.workspace;
   p.status = a.epi.status;
+  p.fp16 = fp16;
   int rc;
   switch (pl.bnx) {
     case 16: rc = launch_gemv<16>(mw, mx, mx2, p, pl.grid, stream); break;
@@ -1652,7 +1657,7 @@ int gemv_launch(const GemmArgs& a, cudaStream_t stream, int num_sms, GemmCost* c
       if (resid && a.epi.norm_w) {
         VLA_CUDA_TRY(launch_pdl(stream_reduce_resid_norm_kernel, dim3(a.M), dim3(1024), 0, stream, src, a.N,
                                 a.epi.resid, a.epi.ldr, a.epi.norm_w, a.epi.norm_eps, a.epi.norm_hi,
-                                a.epi.norm_lo, a.epi.ldn));
+                                a.epi.norm_lo, a.epi.ldn, fp16));
         break;
       }
       VLA_CUDA_TRY(launch_pdl(stream_reduce_f32_kernel, grid_for((a.N + 255) / 256), dim3(256), 0, stream, src,
@@ -1662,7 +1667,7 @@ int gemv_launch(const GemmArgs& a, cudaStream_t stream, int num_sms, GemmCost* c
     }
     case EPI_SWIGLU:
       VLA_CUDA_TRY(launch_pdl(stream_reduce_swiglu_kernel, grid_for((a.N / 2 + 255) / 256), dim3(256), 0,
-                              stream, src, a.M, a.N / 2, a.epi.out_hi, a.epi.out_lo, a.epi.ldo));
+                              stream, src, a.M, a.N / 2, a.epi.out_hi, a.epi.out_lo, a.epi.ldo, fp16));
       break;
     case EPI_QKV:
       if (256 % a.epi.hd == 0 && a.epi.d % 256 == 0) {

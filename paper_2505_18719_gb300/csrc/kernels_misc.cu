@@ -44,7 +44,7 @@ __global__ void __launch_bounds__(256) assemble_kernel(const RowInfo* __restrict
 __global__ void __launch_bounds__(256) rmsnorm_kernel(const float* __restrict__ h,
                                                       const bf16* __restrict__ w, int d,
                                                       float eps, bf16* __restrict__ y_hi,
-                                                      bf16* __restrict__ y_lo) {
+                                                      bf16* __restrict__ y_lo, bool fp16) {
   pdl_launch_dependents();
   pdl_wait();
   __shared__ float red[8];
@@ -66,8 +66,8 @@ __global__ void __launch_bounds__(256) rmsnorm_kernel(const float* __restrict__ 
     const uint2 ww = *reinterpret_cast<const uint2*>(w + c);
     const float2 w0 = unpack_bf16x2(ww.x), w1 = unpack_bf16x2(ww.y);
     uint2 hi, lo;
-    split_pack2(v.x * r * w0.x, v.y * r * w0.y, hi.x, lo.x);
-    split_pack2(v.z * r * w1.x, v.w * r * w1.y, hi.y, lo.y);
+    split_pack2(v.x * r * w0.x, v.y * r * w0.y, hi.x, lo.x, fp16);
+    split_pack2(v.z * r * w1.x, v.w * r * w1.y, hi.y, lo.y, fp16);
     *reinterpret_cast<uint2*>(y_hi + off + c) = hi;
     *reinterpret_cast<uint2*>(y_lo + off + c) = lo;
   }
@@ -107,9 +107,9 @@ int assemble_launch(const RowInfo* rows, int n_rows, const bf16* visual, const i
 }
 
 int rmsnorm_launch(const float* h, const bf16* w, int M, int d, float eps, bf16* y_hi,
-                   bf16* y_lo, cudaStream_t s) {
+                   bf16* y_lo, cudaStream_t s, bool fp16) {
   if (M <= 0) return VLA_OK;
-  VLA_CUDA_TRY(launch_pdl(rmsnorm_kernel, dim3(M), dim3(256), 0, s, h, w, d, eps, y_hi, y_lo));
+  VLA_CUDA_TRY(launch_pdl(rmsnorm_kernel, dim3(M), dim3(256), 0, s, h, w, d, eps, y_hi, y_lo, fp16));
   note_launch();
   VLA_CUDA_TRY(cudaGetLastError());
   return VLA_OK;
@@ -130,6 +130,45 @@ int scatter_rows_launch(const float* src, const int* sidx, const int* didx, int 
                         cudaStream_t s) {
   if (n <= 0) return VLA_OK;
   VLA_CUDA_TRY(launch_pdl(scatter_rows_kernel, dim3(n), dim3(256), 0, s, src, sidx, didx, d, dst));
+  note_launch();
+  VLA_CUDA_TRY(cudaGetLastError());
+  return VLA_OK;
+}
+}  // namespace vla
+
+namespace vla {
+namespace {
+// 8 elements per thread per step (16-byte loads and stores); n % 8 == 0, 16-byte aligned.
+__global__ void __launch_bounds__(256) bf16_to_f16_kernel(const bf16* __restrict__ src,
+                                                          f16* __restrict__ dst, size_t n8,
+                                                          int* __restrict__ out_of_range) {
+  bool bad = false;
+  for (size_t i = blockIdx.x * static_cast<size_t>(blockDim.x) + threadIdx.x; i < n8;
+       i += static_cast<size_t>(gridDim.x) * blockDim.x) {
+    const uint4 v = reinterpret_cast<const uint4*>(src)[i];
+    const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+    uint32_t o[4];
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const float2 f = unpack_bf16x2(w[j]);
+      bad |= !(fabsf(f.x) <= 65504.f) || !(fabsf(f.y) <= 65504.f);
+      o[j] = pack_f16x2(fminf(fmaxf(f.x, -65504.f), 65504.f), fminf(fmaxf(f.y, -65504.f), 65504.f));
+    }
+    reinterpret_cast<uint4*>(dst)[i] = make_uint4(o[0], o[1], o[2], o[3]);
+  }
+  if (bad) atomicOr(out_of_range, 1);
+}
+}  // namespace
+
+int bf16_to_f16_launch(const bf16* src, f16* dst, size_t n, int* out_of_range, int num_sms,
+                       cudaStream_t s) {
+  if (n == 0) return VLA_OK;
+  if ((n & 7) || (reinterpret_cast<uintptr_t>(src) & 15) || (reinterpret_cast<uintptr_t>(dst) & 15))
+    return VLA_ERR_ARG;
+  const size_t n8 = n / 8;
+  const size_t want = (n8 + 255) / 256;
+  const int grid = static_cast<int>(want < static_cast<size_t>(num_sms) * 8 ? want : static_cast<size_t>(num_sms) * 8);
+  bf16_to_f16_kernel<<<grid, 256, 0, s>>>(src, dst, n8, out_of_range);
   note_launch();
   VLA_CUDA_TRY(cudaGetLastError());
   return VLA_OK;

@@ -10,10 +10,17 @@ int assemble_launch(const RowInfo* rows, int n_rows, const bf16* visual, const i
                     const int* tokens, const bf16* embed, int d, int vocab, float* h,
                     uint32_t* status, cudaStream_t s);
 
-// y[m] = h[m] / sqrt(mean(h[m]^2) + eps) * w, h f32 [M, d], written as the bf16 pair
-// (y_hi, y_lo) [M, d] with y_hi + y_lo ~ y.
+// y[m] = h[m] / sqrt(mean(h[m]^2) + eps) * w, h f32 [M, d], written as the operand pair
+// (y_hi, y_lo) [M, d] with y_hi + y_lo ~ y, fp16 if `fp16` else bf16.
 int rmsnorm_launch(const float* h, const bf16* w, int M, int d, float eps, bf16* y_hi,
-                   bf16* y_lo, cudaStream_t s);
+                   bf16* y_lo, cudaStream_t s, bool fp16);
+
+// dst[i] = fp16(src[i]) for n bf16 values (n % 8 == 0, both 16-byte aligned).  A value outside
+// the finite fp16 range (|x| > 65504, or not finite) is clamped to +-65504 and sets
+// *out_of_range to 1.  A bf16 value (8 significant bits) with 2^-14 <= |x| <= 65504 is exact
+// in fp16 (11); a smaller one rounds to a multiple of 2^-24, an absolute error <= 2^-25.
+int bf16_to_f16_launch(const bf16* src, f16* dst, size_t n, int* out_of_range, int num_sms,
+                       cudaStream_t s);
 
 // dst[i] = src[idx[i]] rows of width d (f32).
 int gather_rows_launch(const float* src, const int* idx, int n, int d, float* dst, cudaStream_t s);

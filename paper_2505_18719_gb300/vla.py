@@ -77,6 +77,7 @@ def load(path: str = LIB_PATH):
         "vla_score_actions": (i32, [vp, vp, f32, vp, vp]),
         "vla_reset": (i32, [vp, vp]),
         "vla_sync": (i32, [vp]),
+        "vla_sync_weights": (i32, [vp]),
         "vla_context_length": (i32, [vp, i32]),
         "vla_last_error": (ctypes.c_char_p, [vp]),
         "vla_destroy": (None, [vp]),
@@ -173,6 +174,10 @@ def vla_reset(h, env_mask: Optional[Sequence[int]] = None) -> int:
 
 def vla_sync(h) -> int:
     return load().vla_sync(h)
+
+
+def vla_sync_weights(h) -> int:
+    return load().vla_sync_weights(h)
 
 
 def vla_context_length(h, env: int) -> int:
@@ -358,3 +363,8 @@ class Policy:
 
     def sync(self):
         self.check(vla_sync(self.h))
+
+    def sync_weights(self):
+        """Re-read the projection matrices into the handle's fp16 copy (after an in-place
+        update of the bf16 weights this Policy was created with)."""
+        self.check(vla_sync_weights(self.h))
