@@ -218,13 +218,12 @@ void prof_harvest(vla_handle* h) {
 }
 
 // Projections whose tile (prefill / score) GEMMs also multiply the low half of the activation
-// pair.  An fp16 activation alone is within 2^-12 relative of its value; carried through the
-// 32 layers of a 7B decoder that keeps the action-bin logits within ~0.02 of exact, and the
-// pair on q|k|v alone brings them to ~0.016 for 62 % of the MMA work of pairs everywhere.
-// The weight-streaming (decode) GEMMs always take both halves: they are bound by reading the
-// weights, so the second MMA costs nothing there.
+// pair.  An fp16 activation alone is within 2^-11 relative of its value.  gate|up, 45 % of the
+// projection work, takes hi alone: its rounding adds ~0.01 to the 7B action-bin logits, next to
+// the ~0.012 the fp16 KV cache already costs.  The weight-streaming (decode) GEMMs always take
+// both halves: they are bound by reading the weights, so the second MMA costs nothing there.
 enum : unsigned { kProjQkv = 1, kProjO = 2, kProjGateUp = 4, kProjDown = 8 };
-constexpr unsigned kTileLoMask = kProjQkv;
+constexpr unsigned kTileLoMask = kProjQkv | kProjO | kProjDown;
 
 // A is the operand pair: hi at A, lo at A + a_plane (fp16 when h->fp16, else bf16).
 // The GEMM that will consume h->y after a residual GEMM's RMSNorm (its N, K and epilogue).
