@@ -255,6 +255,9 @@ CASES = {
     "gemv_decode_k16384": (64, 12288, 16384, 0, 0, True),
 }
 
+# every GEMM case also with fp16 operands (the engine's form): NAME_f16
+CASES.update({k + "_f16": v for k, v in list(CASES.items()) if v is not None})
+
 
 def run_attn_case(args):
     """Decode attention for 64 envs x 32 heads at ~290 cached positions (one layer)."""
@@ -391,7 +394,8 @@ def run_learning_case(args):
 
 
 def run_case(args):
-    """Time one GEMM shape through vla_op_gemm_bf16 (CUDA events, device-resident operands)."""
+    """Time one GEMM shape through the GEMM op entry points (CUDA events, device-resident
+    operands); bf16 operands, or fp16 for the NAME_f16 cases."""
     import torch
     import __graft_entry__
     __graft_entry__.build()
@@ -404,32 +408,37 @@ def run_case(args):
     if args.case in ("attn_chunk", "attn_score"):
         return run_attn_chunk_case(args)
     M, N, K, bn, splits, split_a = CASES[args.case]
+    fp16 = args.case.endswith("_f16")
     A = I.normal_bf16((M, K), 1, 1, 1.0).cuda()
     A_lo = I.normal_bf16((M, K), 1, 2, 2.0 ** -9).cuda()
     W = I.normal_bf16((N, K), 1, 3, 0.02).cuda()
+    if fp16:
+        A, A_lo, W = A.half(), (A_lo * 2.0 ** -3).half(), W.half()
+    op_gemm, op_pair, op_decode = ((V.vla_op_gemm_f16, V.vla_op_gemm_pair_f16, V.vla_op_gemm_decode_f16) if fp16
+                                   else (V.vla_op_gemm_bf16, V.vla_op_gemm_pair_bf16, V.vla_op_gemm_decode_bf16))
     C = torch.empty(M, N, dtype=torch.float32, device="cuda")
     stream = torch.cuda.current_stream()
     if args.case.startswith("pair"):
         ws = None
 
         def launch():
-            rc = V.vla_op_gemm_pair_bf16(A.data_ptr(), A_lo.data_ptr() if split_a else 0, K, W.data_ptr(), K,
-                                         C.data_ptr(), N, M, N, K, stream.cuda_stream)
+            rc = op_pair(A.data_ptr(), A_lo.data_ptr() if split_a else 0, K, W.data_ptr(), K,
+                         C.data_ptr(), N, M, N, K, stream.cuda_stream)
             assert rc == 0, V.vla_last_error()
     elif args.case.startswith("gemv"):
         nbytes = V.vla_op_gemm_decode_workspace_bytes(M, N, K)
         ws = torch.empty(max(1, nbytes // 4), dtype=torch.float32, device="cuda")
 
         def launch():
-            rc = V.vla_op_gemm_decode_bf16(A.data_ptr(), A_lo.data_ptr(), K, W.data_ptr(), K, C.data_ptr(), N,
-                                           M, N, K, ws.data_ptr(), nbytes, stream.cuda_stream)
+            rc = op_decode(A.data_ptr(), A_lo.data_ptr(), K, W.data_ptr(), K, C.data_ptr(), N,
+                           M, N, K, ws.data_ptr(), nbytes, stream.cuda_stream)
             assert rc == 0, V.vla_last_error()
     else:
         ws = torch.empty(max(1, splits * M * N), dtype=torch.float32, device="cuda")
 
         def launch():
-            rc = V.vla_op_gemm_bf16(A.data_ptr(), A_lo.data_ptr() if split_a else 0, K, W.data_ptr(), K,
-                                    C.data_ptr(), N, M, N, K, bn, splits, ws.data_ptr(), stream.cuda_stream)
+            rc = op_gemm(A.data_ptr(), A_lo.data_ptr() if split_a else 0, K, W.data_ptr(), K,
+                         C.data_ptr(), N, M, N, K, bn, splits, ws.data_ptr(), stream.cuda_stream)
             assert rc == 0, V.vla_last_error()
 
     for _ in range(args.warmup):
@@ -446,7 +455,7 @@ def run_case(args):
     flops = 2.0 * M * N * K
     bytes_ = 2.0 * (M * K * (2 if split_a else 1) + N * K) + 4.0 * M * N
     print(json.dumps({"case": args.case, "M": M, "N": N, "K": K, "block_n": bn, "splits": splits,
-                      "split_a": split_a, "ms": ms, "tflops": flops / ms / 1e9,
+                      "split_a": split_a, "operands": "fp16" if fp16 else "bf16", "ms": ms, "tflops": flops / ms / 1e9,
                       "tc_frac_of_burst": flops / ms / 1e9 / tf_burst, "gbs": bytes_ / ms / 1e6,
                       "hbm_frac": bytes_ / ms / 1e6 / hbm, "peaks": kind}))
     return 0

@@ -16,7 +16,7 @@ extern "C" {
 /* C[M, N] (f32, row stride ldc) = (A + A_lo)[M, K] · W[N, K]^T with A, A_lo, W bf16
  * row-major (row strides lda, ldw elements, multiples of 8), fp32 accumulation on the tcgen05
  * tensor cores.  A_lo may be NULL (then C = A · W^T); otherwise the activation is the
- * unevaluated bf16 pair A + A_lo, the form in which the hot path feeds every projection.
+ * unevaluated bf16 pair A + A_lo (the engine itself runs the fp16 form below).
  * This is the contraction of every projection of the decoder layer (§3.1: the Llama-2
  * backbone's q/k/v, o, gate/up and down projections).  `block_n` in {128, 256} is the output
  * tile width; `splits` >= 1 splits K across CTAs (partials in `workspace`, f32
@@ -43,6 +43,20 @@ int vla_op_gemm_decode_bf16(const void* A, const void* A_lo, int lda, const void
                             float* C, int ldc, int M, int N, int K, float* workspace,
                             size_t workspace_bytes, void* cuda_stream);
 size_t vla_op_gemm_decode_workspace_bytes(int M, int N, int K);
+
+/* The same three contractions with fp16 operands: A, A_lo and W hold IEEE binary16 bits, the
+ * form in which the engine runs every projection (each fp16 half keeps 11 significant bits,
+ * so hi alone is 8x closer to the activation than a bf16 hi; the pair hi + lo keeps ~21).
+ * Arguments, layouts, workspaces, errors and the fp32 accumulation are those of the bf16
+ * entry points above. */
+int vla_op_gemm_f16(const void* A, const void* A_lo, int lda, const void* W, int ldw, float* C,
+                    int ldc, int M, int N, int K, int block_n, int splits, float* workspace,
+                    void* cuda_stream);
+int vla_op_gemm_pair_f16(const void* A, const void* A_lo, int lda, const void* W, int ldw,
+                         float* C, int ldc, int M, int N, int K, void* cuda_stream);
+int vla_op_gemm_decode_f16(const void* A, const void* A_lo, int lda, const void* W, int ldw,
+                           float* C, int ldc, int M, int N, int K, float* workspace,
+                           size_t workspace_bytes, void* cuda_stream);
 
 /* vla_op_gemm_bf16 without a caller workspace: the paper has no counterpart; this entry
  * point exists for callers that cannot allocate device memory (all device memory owned by

@@ -1023,10 +1023,15 @@ int64_t vla_launch_count(const vla_handle* h) {
 }
 
 // ---------------------------------------------------------------------------------- ops
-int vla_op_gemm_bf16(const void* A, const void* A_lo, int lda, const void* W, int ldw, float* C, int ldc,
-                     int M, int N, int K, int block_n, int splits, float* workspace, void* cuda_stream) {
+}  // extern "C"
+
+namespace {
+// The GEMM op entry points, bf16 (fp16 == false) or fp16 operands.
+int op_gemm(const std::string& name, bool fp16, const void* A, const void* A_lo, int lda, const void* W,
+            int ldw, float* C, int ldc, int M, int N, int K, int block_n, int splits, float* workspace,
+            void* cuda_stream) {
   if (!A || !W || !C || M < 1 || N < 1 || K < 1 || ldc < N)
-    return set_err(nullptr, VLA_ERR_ARG, "vla_op_gemm_bf16: bad argument");
+    return set_err(nullptr, VLA_ERR_ARG, name + ": bad argument");
   GemmArgs g;
   g.A = static_cast<const bf16*>(A);
   g.A_lo = static_cast<const bf16*>(A_lo);
@@ -1043,17 +1048,18 @@ int vla_op_gemm_bf16(const void* A, const void* A_lo, int lda, const void* W, in
   g.epi.kind = EPI_F32;
   g.epi.out_f32 = C;
   g.epi.ldo = ldc;
+  g.epi.fp16 = fp16;
   if (splits > 1 && gemm_effective_splits(K, splits) > 1 && !workspace)
-    return set_err(nullptr, VLA_ERR_ARG, "vla_op_gemm_bf16: splits > 1 needs a workspace");
+    return set_err(nullptr, VLA_ERR_ARG, name + ": splits > 1 needs a workspace");
   const int rc = gemm_launch(g, static_cast<cudaStream_t>(cuda_stream), query_num_sms(), nullptr);
-  if (rc != VLA_OK && rc != VLA_ERR_CUDA) return set_err(nullptr, rc, "vla_op_gemm_bf16: unsupported arguments");
+  if (rc != VLA_OK && rc != VLA_ERR_CUDA) return set_err(nullptr, rc, name + ": unsupported arguments");
   return rc;
 }
 
-int vla_op_gemm_pair_bf16(const void* A, const void* A_lo, int lda, const void* W, int ldw, float* C, int ldc,
-                          int M, int N, int K, void* cuda_stream) {
+int op_gemm_pair(const std::string& name, bool fp16, const void* A, const void* A_lo, int lda, const void* W,
+                 int ldw, float* C, int ldc, int M, int N, int K, void* cuda_stream) {
   if (!A || !W || !C || M < 1 || N < 1 || K < 1 || ldc < N)
-    return set_err(nullptr, VLA_ERR_ARG, "vla_op_gemm_pair_bf16: bad argument");
+    return set_err(nullptr, VLA_ERR_ARG, name + ": bad argument");
   GemmArgs g;
   g.A = static_cast<const bf16*>(A);
   g.A_lo = static_cast<const bf16*>(A_lo);
@@ -1069,16 +1075,17 @@ int vla_op_gemm_pair_bf16(const void* A, const void* A_lo, int lda, const void* 
   g.epi.kind = EPI_F32;
   g.epi.out_f32 = C;
   g.epi.ldo = ldc;
+  g.epi.fp16 = fp16;
   const int rc = gemm_launch(g, static_cast<cudaStream_t>(cuda_stream), query_num_sms(), nullptr);
-  if (rc != VLA_OK && rc != VLA_ERR_CUDA) return set_err(nullptr, rc, "vla_op_gemm_pair_bf16: unsupported arguments");
+  if (rc != VLA_OK && rc != VLA_ERR_CUDA) return set_err(nullptr, rc, name + ": unsupported arguments");
   return rc;
 }
 
-int vla_op_gemm_decode_bf16(const void* A, const void* A_lo, int lda, const void* W, int ldw, float* C,
-                            int ldc, int M, int N, int K, float* workspace, size_t workspace_bytes,
-                            void* cuda_stream) {
+int op_gemm_decode(const std::string& name, bool fp16, const void* A, const void* A_lo, int lda, const void* W,
+                   int ldw, float* C, int ldc, int M, int N, int K, float* workspace, size_t workspace_bytes,
+                   void* cuda_stream) {
   if (!A || !A_lo || !W || !C || M < 1 || M > 128 || N < 1 || K < 1 || ldc < N || !workspace)
-    return set_err(nullptr, VLA_ERR_ARG, "vla_op_gemm_decode_bf16: bad argument");
+    return set_err(nullptr, VLA_ERR_ARG, name + ": bad argument");
   GemmArgs g;
   g.A = static_cast<const bf16*>(A);
   g.A_lo = static_cast<const bf16*>(A_lo);
@@ -1093,10 +1100,50 @@ int vla_op_gemm_decode_bf16(const void* A, const void* A_lo, int lda, const void
   g.epi.kind = EPI_F32;
   g.epi.out_f32 = C;
   g.epi.ldo = ldc;
+  g.epi.fp16 = fp16;
   const int rc = gemv_launch(g, static_cast<cudaStream_t>(cuda_stream), query_num_sms(), nullptr);
   if (rc != VLA_OK && rc != VLA_ERR_CUDA)
-    return set_err(nullptr, rc, "vla_op_gemm_decode_bf16: unsupported arguments or workspace too small");
+    return set_err(nullptr, rc, name + ": unsupported arguments or workspace too small");
   return rc;
+}
+}  // namespace
+
+extern "C" {
+
+int vla_op_gemm_bf16(const void* A, const void* A_lo, int lda, const void* W, int ldw, float* C, int ldc,
+                     int M, int N, int K, int block_n, int splits, float* workspace, void* cuda_stream) {
+  return op_gemm("vla_op_gemm_bf16", false, A, A_lo, lda, W, ldw, C, ldc, M, N, K, block_n, splits, workspace,
+                 cuda_stream);
+}
+
+int vla_op_gemm_f16(const void* A, const void* A_lo, int lda, const void* W, int ldw, float* C, int ldc,
+                    int M, int N, int K, int block_n, int splits, float* workspace, void* cuda_stream) {
+  return op_gemm("vla_op_gemm_f16", true, A, A_lo, lda, W, ldw, C, ldc, M, N, K, block_n, splits, workspace,
+                 cuda_stream);
+}
+
+int vla_op_gemm_pair_bf16(const void* A, const void* A_lo, int lda, const void* W, int ldw, float* C, int ldc,
+                          int M, int N, int K, void* cuda_stream) {
+  return op_gemm_pair("vla_op_gemm_pair_bf16", false, A, A_lo, lda, W, ldw, C, ldc, M, N, K, cuda_stream);
+}
+
+int vla_op_gemm_pair_f16(const void* A, const void* A_lo, int lda, const void* W, int ldw, float* C, int ldc,
+                         int M, int N, int K, void* cuda_stream) {
+  return op_gemm_pair("vla_op_gemm_pair_f16", true, A, A_lo, lda, W, ldw, C, ldc, M, N, K, cuda_stream);
+}
+
+int vla_op_gemm_decode_bf16(const void* A, const void* A_lo, int lda, const void* W, int ldw, float* C,
+                            int ldc, int M, int N, int K, float* workspace, size_t workspace_bytes,
+                            void* cuda_stream) {
+  return op_gemm_decode("vla_op_gemm_decode_bf16", false, A, A_lo, lda, W, ldw, C, ldc, M, N, K, workspace,
+                        workspace_bytes, cuda_stream);
+}
+
+int vla_op_gemm_decode_f16(const void* A, const void* A_lo, int lda, const void* W, int ldw, float* C,
+                           int ldc, int M, int N, int K, float* workspace, size_t workspace_bytes,
+                           void* cuda_stream) {
+  return op_gemm_decode("vla_op_gemm_decode_f16", true, A, A_lo, lda, W, ldw, C, ldc, M, N, K, workspace,
+                        workspace_bytes, cuda_stream);
 }
 
 size_t vla_op_gemm_decode_workspace_bytes(int M, int N, int K) {

@@ -92,6 +92,9 @@ def load(path: str = LIB_PATH):
         "vla_op_gemm_pair_bf16": (i32, [vp, vp, i32, vp, i32, vp, i32, i32, i32, i32, vp]),
         "vla_op_gemm_decode_bf16": (i32, [vp, vp, i32, vp, i32, vp, i32, i32, i32, i32, vp, ctypes.c_size_t, vp]),
         "vla_op_gemm_decode_workspace_bytes": (ctypes.c_size_t, [i32, i32, i32]),
+        "vla_op_gemm_f16": (i32, [vp, vp, i32, vp, i32, vp, i32, i32, i32, i32, i32, i32, vp, vp]),
+        "vla_op_gemm_pair_f16": (i32, [vp, vp, i32, vp, i32, vp, i32, i32, i32, i32, vp]),
+        "vla_op_gemm_decode_f16": (i32, [vp, vp, i32, vp, i32, vp, i32, i32, i32, i32, vp, ctypes.c_size_t, vp]),
         "vla_op_gemm_bf16_noalloc": (i32, [vp, vp, i32, vp, i32, vp, i32, i32, i32, i32, i32, i32, vp]),
         "vla_op_action_head": (i32, [vp, i32, i32, i32, vp, vp, f32, vp, f32, vp, vp, vp, vp, vp, vp, vp]),
         "vla_op_num_sms": (i32, []),
@@ -225,6 +228,23 @@ def vla_op_gemm_decode_bf16(A_ptr, A_lo_ptr, lda, W_ptr, ldw, C_ptr, ldc, M, N, 
 
 def vla_op_gemm_decode_workspace_bytes(M, N, K) -> int:
     return load().vla_op_gemm_decode_workspace_bytes(M, N, K)
+
+
+def vla_op_gemm_f16(A_ptr, A_lo_ptr, lda, W_ptr, ldw, C_ptr, ldc, M, N, K, block_n=256, splits=1,
+                    ws_ptr=0, stream=0) -> int:
+    return load().vla_op_gemm_f16(A_ptr, A_lo_ptr or None, lda, W_ptr, ldw, C_ptr, ldc, M, N, K,
+                                  block_n, splits, ws_ptr or None, stream or None)
+
+
+def vla_op_gemm_pair_f16(A_ptr, A_lo_ptr, lda, W_ptr, ldw, C_ptr, ldc, M, N, K, stream=0) -> int:
+    return load().vla_op_gemm_pair_f16(A_ptr, A_lo_ptr or None, lda, W_ptr, ldw, C_ptr, ldc, M, N, K,
+                                       stream or None)
+
+
+def vla_op_gemm_decode_f16(A_ptr, A_lo_ptr, lda, W_ptr, ldw, C_ptr, ldc, M, N, K, ws_ptr, ws_bytes,
+                           stream=0) -> int:
+    return load().vla_op_gemm_decode_f16(A_ptr, A_lo_ptr, lda, W_ptr, ldw, C_ptr, ldc, M, N, K, ws_ptr,
+                                         ws_bytes, stream or None)
 
 
 def vla_op_gemm_bf16_noalloc(A_ptr, A_lo_ptr, lda, W_ptr, ldw, C_ptr, ldc, M, N, K, block_n=256,

@@ -231,3 +231,60 @@ def test_chunk_attention_matches_fp64(hd):
     assert V.vla_op_attn_chunk(qd.data_ptr(), kvd.data_ptr(), max_env, H, hd, cap, bad, rows,
                                tiles_dev.data_ptr(), oh.data_ptr(), ol.data_ptr()) == V.VLA_ERR_ARG
 
+
+
+# ------------------------------------------------------------------ fp16 operands (engine form)
+def _f16_operands(M, N, K, seed):
+    """fp16 A (11 significant bits used), its low half, and fp16 W, built from the seeded bf16
+    generators: bf16 values plus a finer bf16 term, rounded once to fp16."""
+    A = (I.normal_bf16((M, K), seed, 1000 + M, 1.0).float()
+         + I.normal_bf16((M, K), seed, 5000 + M, 2.0 ** -8).float()).half()
+    A_lo = I.normal_bf16((M, K), seed, 3000 + M, 2.0 ** -12).half()
+    W = (I.normal_bf16((N, K), seed, 2000 + N, 1.0).float()
+         + I.normal_bf16((N, K), seed, 6000 + N, 2.0 ** -8).float()).half()
+    return A, A_lo, W
+
+
+@pytest.mark.parametrize("M,N,K,bn,splits,split_a", GEMM_CASES[1::2] + [GEMM_CASES[0]])
+def test_gemm_f16_matches_fp64(M, N, K, bn, splits, split_a):
+    A, A_lo, W = _f16_operands(M, N, K, 91)
+    Ad, Ald, Wd = A.cuda(), A_lo.cuda(), W.cuda()
+    C = torch.full((M, N), float("nan"), dtype=torch.float32, device="cuda")
+    ws = torch.empty(max(1, splits * M * N), dtype=torch.float32, device="cuda")
+    rc = V.vla_op_gemm_f16(Ad.data_ptr(), Ald.data_ptr() if split_a else 0, K, Wd.data_ptr(), K,
+                           C.data_ptr(), N, M, N, K, bn, splits, ws.data_ptr(), 0)
+    assert rc == 0, V.vla_last_error()
+    torch.cuda.synchronize()
+    Aref = A.double() + A_lo.double() if split_a else A.double()
+    err = (C.cpu().double() - Aref @ W.double().T).abs().max().item()
+    # fp16 x fp16 products are exact in fp32; the error is the fp32 sums'
+    assert err < 2e-5 * math.sqrt(K) * 8, err
+
+
+@pytest.mark.parametrize("M,N,K,split_a", PAIR_CASES)
+def test_pair_gemm_f16_matches_fp64(M, N, K, split_a):
+    A, A_lo, W = _f16_operands(M, N, K, 92)
+    Ad, Ald, Wd = A.cuda(), A_lo.cuda(), W.cuda()
+    C = torch.full((M, N), float("nan"), dtype=torch.float32, device="cuda")
+    rc = V.vla_op_gemm_pair_f16(Ad.data_ptr(), Ald.data_ptr() if split_a else 0, K, Wd.data_ptr(), K,
+                                C.data_ptr(), N, M, N, K, 0)
+    assert rc == 0, V.vla_last_error()
+    torch.cuda.synchronize()
+    Aref = A.double() + A_lo.double() if split_a else A.double()
+    err = (C.cpu().double() - Aref @ W.double().T).abs().max().item()
+    assert err < 2e-5 * math.sqrt(K) * 8, err
+
+
+@pytest.mark.parametrize("M,N,K", DECODE_CASES[::2])
+def test_decode_gemm_f16_matches_fp64(M, N, K):
+    A, A_lo, W = _f16_operands(M, N, K, 93)
+    C = torch.full((M, N), float("nan"), dtype=torch.float32, device="cuda")
+    nbytes = V.vla_op_gemm_decode_workspace_bytes(M, N, K)
+    ws = torch.empty(max(1, nbytes // 4), dtype=torch.float32, device="cuda")
+    Ad, Ald, Wd = A.cuda(), A_lo.cuda(), W.cuda()
+    rc = V.vla_op_gemm_decode_f16(Ad.data_ptr(), Ald.data_ptr(), K, Wd.data_ptr(), K, C.data_ptr(), N,
+                                  M, N, K, ws.data_ptr(), nbytes, 0)
+    assert rc == 0, V.vla_last_error()
+    torch.cuda.synchronize()
+    err = (C.cpu().double() - (A.double() + A_lo.double()) @ W.double().T).abs().max().item()
+    assert err < 2e-5 * math.sqrt(K) * 8, err
