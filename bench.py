@@ -36,9 +36,10 @@ WORKLOAD = "7b_b64_ragged_score"
 
 # DRAM bytes of one launch of the dominant kernel from an ncu capture (set to None whenever
 # that kernel changes): gemm_tc2_kernel, the q|k|v projection of this step's prefill
-# (18385 x 12288 x 4096, case pair_prefill_qkv_18385; fp32 output in the case).
-PROFILED_TRAFFIC = {"bytes": 3.094091e9 + 0.879448e9,
-                    "launch": "gemm_tc2_kernel q|k|v, M=18385 N=12288 K=4096",
+# (18385 x 12288 x 4096, fp16 operand pair, case pair_prefill_qkv_18385_f16; fp32 output in
+# the case).
+PROFILED_TRAFFIC = {"bytes": 2.113555e9 + 0.879153e9,
+                    "launch": "gemm_tc2_kernel q|k|v (fp16 operands), M=18385 N=12288 K=4096",
                     "algorithmic_bytes": 2.0 * 18385 * 4096 * 2 + 2.0 * 12288 * 4096 + 4.0 * 18385 * 12288,
                     "profile": "profiles/gemm_tc2_prefill_qkv_18385x12288x4096.md"}
 
