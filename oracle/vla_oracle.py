@@ -146,20 +146,15 @@ class Weights:
         return lw
 
 
-def round_bf16(x: torch.Tensor) -> torch.Tensor:
-    """Round to the nearest bf16 value (attribution mode only)."""
-    return x.to(torch.float32).to(torch.bfloat16).to(F64)
-
-
-def round_bf16_pair(x: torch.Tensor) -> torch.Tensor:
-    """x -> hi + lo with hi = bf16(x), lo = bf16(x - hi) (attribution mode only)."""
-    hi = round_bf16(x)
-    return hi + round_bf16(x - hi)
-
-
 def round_f16(x: torch.Tensor) -> torch.Tensor:
     """Round to the nearest fp16 value (attribution mode only)."""
     return x.to(torch.float32).to(torch.float16).to(F64)
+
+
+def round_f16_pair(x: torch.Tensor) -> torch.Tensor:
+    """x -> hi + lo with hi = fp16(x), lo = fp16(x - hi) (attribution mode only)."""
+    hi = round_f16(x)
+    return hi + round_f16(x - hi)
 
 
 def _same(x):
@@ -174,10 +169,18 @@ class Rounding:
     act: object = _same   # GEMM input activations (norm outputs, attention output, SwiGLU)
     q: object = _same     # queries after RoPE
     kv: object = _same    # keys (after RoPE) and values as cached
+    # per-projection override of `act` for chunks of more than one row (prefill, score):
+    # {"qkv" | "o" | "gate_up" | "down": rounding}; None = `act` everywhere
+    act_chunk: Optional[dict] = None
 
 
 EXACT = Rounding()
-GPU_PATH = Rounding(act=round_bf16_pair, q=lambda x: x.to(torch.float32).to(F64), kv=round_f16)
+# The GPU path: fp16 activation pairs (fp16 weights hold the bf16 ones exactly above 2^-14),
+# fp32 queries, fp16 K/V; the multi-row projections use hi alone for gate|up.  Approximate
+# where the GPU's choice follows the whole call's rows rather than one env's chunk (the
+# last prefill layer runs gate|up on each env's final row through the two-half GEMM).
+GPU_PATH = Rounding(act=round_f16_pair, q=lambda x: x.to(torch.float32).to(F64), kv=round_f16,
+                    act_chunk={"gate_up": round_f16})
 
 
 def layer_forward(shape: Shape, lw: dict, h, pos, k_cache, v_cache, rnd: Rounding = EXACT):
@@ -189,7 +192,12 @@ def layer_forward(shape: Shape, lw: dict, h, pos, k_cache, v_cache, rnd: Roundin
     """
     n = h.shape[0]
     d, H, hd, F = shape.d_model, shape.n_heads, shape.head_dim, shape.d_ffn
-    y = rnd.act(rms_norm(h, lw["attn_norm"], shape.rms_eps))
+
+    def act(site, x):
+        f = rnd.act_chunk.get(site) if (rnd.act_chunk and n > 1) else None
+        return (f or rnd.act)(x)
+
+    y = act("qkv", rms_norm(h, lw["attn_norm"], shape.rms_eps))
     qkv = y @ lw["wqkv"].T
     q = qkv[:, 0:d].reshape(n, H, hd)
     k = qkv[:, d:2 * d].reshape(n, H, hd)
@@ -199,11 +207,11 @@ def layer_forward(shape: Shape, lw: dict, h, pos, k_cache, v_cache, rnd: Roundin
     k_all = torch.cat([k_cache, k], dim=0)
     v_all = torch.cat([v_cache, v], dim=0)
     k_pos = torch.arange(k_all.shape[0], dtype=torch.long)
-    o = rnd.act(causal_attention(q, k_all, v_all, pos, k_pos))
+    o = act("o", causal_attention(q, k_all, v_all, pos, k_pos))
     h = h + o.reshape(n, d) @ lw["wo"].T
-    y = rnd.act(rms_norm(h, lw["ffn_norm"], shape.rms_eps))
+    y = act("gate_up", rms_norm(h, lw["ffn_norm"], shape.rms_eps))
     gu = y @ lw["w_gate_up"].T
-    h = h + rnd.act(silu(gu[:, :F]) * gu[:, F:]) @ lw["w_down"].T
+    h = h + act("down", silu(gu[:, :F]) * gu[:, F:]) @ lw["w_down"].T
     return h, k_all, v_all
 
 
