@@ -21,8 +21,9 @@
  *    workspaces and the fp16 projection copy (allocated in vla_create, freed in vla_destroy).
  *  - Arithmetic: every projection runs on fp16 tensor-core operands with fp32 accumulation.
  *    Its input activation is carried as an fp16 pair hi + lo (~21 significant bits); the
- *    weight-streaming decode GEMMs multiply both halves, the prefill / score GEMMs both
- *    halves for q|k|v and hi alone for o, gate|up and down.  K/V are cached in fp16.
+ *    weight-streaming GEMMs (calls of at most 128 rows: decode steps of up to 128 envs)
+ *    multiply both halves, the tile GEMMs (prefill, score, larger decode batches) both halves
+ *    for q|k|v, o and down and hi alone for gate|up.  K/V are cached in fp16.
  *  - Calls are asynchronous on the handle's stream.  Host-checkable errors return at once,
  *    with no side effects.  Errors found on the device (token id out of range, non-finite
  *    logits, a pipeline wait that timed out) set a device status word; the next vla_sync

@@ -178,7 +178,8 @@ EXACT = Rounding()
 # The GPU path: fp16 activation pairs (fp16 weights hold the bf16 ones exactly above 2^-14),
 # fp32 queries, fp16 K/V; the multi-row projections use hi alone for gate|up.  Approximate
 # where the GPU's choice follows the whole call's rows rather than one env's chunk (the
-# last prefill layer runs gate|up on each env's final row through the two-half GEMM).
+# last prefill layer runs gate|up on each env's final row through the two-half GEMM; decode
+# of more than 128 envs runs gate|up on hi alone).
 GPU_PATH = Rounding(act=round_f16_pair, q=lambda x: x.to(torch.float32).to(F64), kv=round_f16,
                     act_chunk={"gate_up": round_f16})
 

@@ -217,11 +217,12 @@ void prof_harvest(vla_handle* h) {
   h->ev_used.clear();
 }
 
-// Projections whose tile (prefill / score) GEMMs also multiply the low half of the activation
-// pair.  An fp16 activation alone is within 2^-11 relative of its value.  gate|up, 45 % of the
-// projection work, takes hi alone: its rounding adds ~0.01 to the 7B action-bin logits, next to
-// the ~0.012 the fp16 KV cache already costs.  The weight-streaming (decode) GEMMs always take
-// both halves: they are bound by reading the weights, so the second MMA costs nothing there.
+// Projections whose tile GEMMs (M > 128 rows: prefill, score, decode of more than 128 envs)
+// also multiply the low half of the activation pair.  An fp16 activation alone is within 2^-11
+// relative of its value.  gate|up, 45 % of the projection work, takes hi alone: its rounding
+// adds ~0.01 to the 7B action-bin logits, next to the ~0.012 the fp16 KV cache already costs.
+// The weight-streaming GEMMs (M <= 128) always take both halves: they are bound by reading the
+// weights, so the second MMA costs nothing there.
 enum : unsigned { kProjQkv = 1, kProjO = 2, kProjGateUp = 4, kProjDown = 8 };
 constexpr unsigned kTileLoMask = kProjQkv | kProjO | kProjDown;
 
