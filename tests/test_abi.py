@@ -55,5 +55,11 @@ def test_host_argument_errors_without_gpu(lib):
     assert lib.vla_context_length(None, 0) == -1
     lib.vla_destroy(None)  # no-op
     assert lib.vla_op_gemm_bf16(None, None, 0, None, 0, None, 0, 0, 0, 0, 256, 1, None, None) == V.VLA_ERR_ARG
+    assert lib.vla_sync_weights(None) == V.VLA_ERR_ARG
+    assert lib.vla_op_gemm_f16(None, None, 0, None, 0, None, 0, 0, 0, 0, 256, 1, None, None) == V.VLA_ERR_ARG
+    assert "vla_op_gemm_f16" in V.vla_last_error(None)
+    assert lib.vla_op_gemm_pair_f16(None, None, 0, None, 0, None, 0, 0, 0, 0, None) == V.VLA_ERR_ARG
+    assert lib.vla_op_gemm_decode_f16(None, None, 0, None, 0, None, 0, 0, 0, 0, None, 0, None) == V.VLA_ERR_ARG
+    assert "vla_op_gemm_decode_f16" in V.vla_last_error(None)
     assert lib.vla_op_action_head(None, 0, 0, 0, None, None, 1e-6, None, 1.0, None, None, None, None,
                                   None, None, None) == V.VLA_ERR_ARG
