@@ -6,8 +6,8 @@
 //    6 teacher-forced action rows of the score pass) against keys 0..pos of that env.
 //    One CTA per (64-row tile, head); mma.sync tensor-core flash attention with fp32
 //    accumulation on fp16 K/V, the fp32 queries and the softmax weights each taken as an
-//    fp16 hi/lo pair; the output is written as the bf16 hi/lo pair the O-projection GEMM
-//    reads.
+//    fp16 hi/lo pair; the output is written as the operand hi/lo pair the O-projection GEMM
+//    reads (fp16 for the engine, bf16 for the op entry points).
 //  * attn_decode: one query per env (the decode step) with the key range split across CTAs
 //    (flash-decoding); each CTA writes its partial (max, sum, unnormalised output) and the
 //    last CTA of the (env, head) to finish merges the splits in a fixed order.  16 lanes x
@@ -273,7 +273,7 @@ __global__ void __launch_bounds__(128) attn_chunk_mma_kernel(const float* __rest
 // groups of the CTA merge through shared memory into one partial (max, sum, unnormalised
 // output) per range.  The last CTA of an (env, head) to finish (a ticket on counters[b * H +
 // head], no waiting) merges the S partials in range order and writes the normalised output as
-// the bf16 pair; with S == 1 the CTA writes it directly.
+// the operand pair; with S == 1 the CTA writes it directly.
 // NW = 2 warps per CTA; ptxas allocates 64 registers for both head dims with no spill, so 16
 // CTAs fit on an SM and the 2048 (env, head) CTAs of a 64-env, 32-head step are all resident
 // at once (one wave, no tail).  No minimum-blocks bound is given: capping at 64 forces a small

@@ -82,10 +82,10 @@ size_t gemm_workspace_bytes(const GemmArgs& a);
 // Launch; returns VLA_OK or an error code (host checks only; kernels report via status).
 int gemm_launch(const GemmArgs& a, cudaStream_t stream, int num_sms, GemmCost* cost);
 
-// Weight-streaming (decode) GEMM for M <= 128 rows with a split A (A_lo required): swap-AB
-// tcgen05 MMAs, stream-K over the weight tiles, partials in `workspace`
-// (gemv_workspace_bytes), then the epilogue of `a.epi` in a fixed-order reduction (EPI_RESID
-// with norm_w set: fused with the following RMSNorm).
+// Weight-streaming (decode) GEMM for M <= 128 rows with a split A (A_lo required; operand
+// format epi.fp16): swap-AB tcgen05 MMAs, stream-K over the weight tiles, partials in
+// `workspace` (gemv_workspace_bytes), then the epilogue of `a.epi` in a fixed-order reduction
+// (EPI_RESID with norm_w set: fused with the following RMSNorm).
 size_t gemv_workspace_bytes(int M, int N, int K, int num_sms);
 int gemv_launch(const GemmArgs& a, cudaStream_t stream, int num_sms, GemmCost* cost);
 

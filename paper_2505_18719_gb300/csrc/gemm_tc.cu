@@ -1,9 +1,10 @@
 // tcgen05 / TMEM / TMA GEMM for sm_103a with the decoder layer's fused epilogues.
 //
-// Y[M, N] = A[M, K] · B[N, K]^T, bf16 operands (both K-major), fp32 accumulation in TMEM.
-// With a split A (the activation carried as a bf16 pair hi + lo), each K step issues two
-// MMAs, hi·B and lo·B, into the same accumulator, so the product sees ~16 mantissa bits of
-// the activation while the weights stay bf16.
+// Y[M, N] = A[M, K] · B[N, K]^T, fp16 or bf16 operands (one format per launch, both K-major),
+// fp32 accumulation in TMEM.  With a split A (the activation carried as a pair hi + lo), each
+// K step issues two MMAs, hi·B and lo·B, into the same accumulator, so the product sees ~21
+// (fp16) or ~16 (bf16) significant bits of the activation; the weights are one 2-byte value
+// each.  The engine runs fp16 operands; the bf16 form serves the bf16 op entry points.
 // This is every projection of the Llama-2 backbone of the policy (paper §3.1): q|k|v, o,
 // gate|up and down.  Epilogues fuse what follows each projection in the layer: RoPE and
 // the KV-cache write after q|k|v, the residual add after o and down, SwiGLU after gate|up.
@@ -86,7 +87,7 @@ __device__ __forceinline__ void unit_coords(const Params& p, int u, int& m_blk, 
 }
 
 // ----------------------------------------------------------------------------- epilogues
-// 16 values as operand hi/lo pairs, bf16 or (fp16) fp16 (two 32-byte stores each).
+// 16 values as operand hi/lo pairs, fp16 if `fp16` else bf16 (two 32-byte stores each).
 __device__ __forceinline__ void store_split16(bf16* hi_dst, bf16* lo_dst, const float (&v)[16],
                                               bool fp16) {
   uint32_t h[8], l[8];

@@ -1,7 +1,8 @@
 // Row kernels of the hot path: chunk assembly (Algorithm 1: the state h(o_t) ‖ v_t^in, plus
 // the pending action token of the previous turn in a multi-turn trajectory, §3.3), RMSNorm
-// of the Llama-2 backbone (§3.1; fp32 math, output as the bf16 hi/lo pair the GEMM reads)
-// and row gathers.  All HBM-bound; one CTA per row, vector accesses.
+// of the Llama-2 backbone (§3.1; fp32 math, output as the operand hi/lo pair the GEMM reads),
+// row gathers and the bf16 -> fp16 conversion of the projection weights.  All HBM-bound; one
+// CTA per row, vector accesses.
 #include "misc.h"
 
 namespace vla {
