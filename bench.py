@@ -672,9 +672,13 @@ def main():
     pre_fl = sum(w_["prefill_flops"] for w_ in works)
     dec_by = sum(w_["decode_bytes"] for w_ in works)
     phase_roof = {
+        # the prefill runs ~0.2 s of back-to-back GEMMs every step under the power cap: its peak
+        # is the sustained one; the fraction of the burst peak is given beside it
         "prefill": {"bound": "tensor", "tflop": pre_fl / 1e12, "ms": t_pre,
-                    "achieved": pre_fl / (t_pre / 1e3) / 1e12, "peak": tf_burst, "unit": "TFLOP/s",
-                    "frac": pre_fl / (t_pre / 1e3) / 1e12 / tf_burst, "peak_kind": f"{peak_kind} bf16 burst",
+                    "achieved": pre_fl / (t_pre / 1e3) / 1e12, "peak": tf_sus, "unit": "TFLOP/s",
+                    "frac": pre_fl / (t_pre / 1e3) / 1e12 / tf_sus,
+                    "frac_of_burst": pre_fl / (t_pre / 1e3) / 1e12 / tf_burst,
+                    "peak_kind": f"{peak_kind} bf16 sustained (fp16 operands: same nominal dense rate)",
                     "tflop_if_every_row_ran_every_layer": sum(w_["prefill_flops_all_rows"] for w_ in works) / 1e12},
         "decode": {"bound": "hbm", "gb": dec_by / 1e9, "ms": t_dec,
                    "achieved": dec_by / (t_dec / 1e3) / 1e9, "peak": hbm, "unit": "GB/s",
