@@ -78,10 +78,11 @@ __device__ __forceinline__ void split_pack2(float a, float b, uint32_t& hi, uint
 
 // The same pair in fp16: hi = fp16(x), lo = fp16(x - hi).  fp16 keeps 11 significant bits
 // per half (bf16: 8), so the single hi alone is 8x closer to x than a bf16 hi; GEMMs fed the
-// fp16 form run on fp16 weights.  x is clamped to the finite fp16 range first (|x| <= 65504),
-// so an out-of-range activation saturates instead of turning into inf / NaN.
+// fp16 form run on fp16 weights.  A finite x beyond the fp16 range (|x| > 65504) saturates to
+// +-65504 instead of turning into inf; NaN and +-inf pass through unchanged, so a non-finite
+// activation still reaches the action head's non-finite check.
 __device__ __forceinline__ void split_f16(float x, f16& hi, f16& lo) {
-  x = fminf(fmaxf(x, -65504.f), 65504.f);
+  if (fabsf(x) > 65504.f && fabsf(x) != INFINITY) x = copysignf(65504.f, x);
   hi = __float2half_rn(x);
   lo = __float2half_rn(x - __half2float(hi));
 }
