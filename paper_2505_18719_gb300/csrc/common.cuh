@@ -122,10 +122,6 @@ __device__ __forceinline__ void store_split1(void* hi, void* lo, size_t i, float
   static_cast<uint16_t*>(hi)[i] = h;
   static_cast<uint16_t*>(lo)[i] = l;
 }
-// Reads a 2-byte operand element of either format.
-__device__ __forceinline__ float op2f(uint16_t bits, bool fp16) {
-  return fp16 ? __half2float(__ushort_as_half(bits)) : __bfloat162float(__ushort_as_bfloat16(bits));
-}
 
 __device__ __forceinline__ float warp_sum(float v) {
 #pragma unroll
