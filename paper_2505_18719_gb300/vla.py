@@ -290,8 +290,9 @@ def vla_op_attn_decode_workspace_bytes(B, H, hd, max_ctx, max_keys_per_cta=0) ->
 class Policy:
     """A handle plus the torch device tensors it borrows (weights) or fills (outputs).
 
-    torch is used only to hold device memory and to name the stream; all compute is in
-    libvla.so.
+    The four projection matrices are read into the handle's fp16 copy when it is created;
+    after changing them in place (a learner update), call ``sync_weights()``.  torch is used
+    only to hold device memory and to name the stream; all compute is in libvla.so.
     """
 
     def __init__(self, shape, weights_dev: Dict, max_batch: int, kv_capacity: int, max_tokens: int,
