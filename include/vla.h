@@ -23,7 +23,9 @@
  *    Its input activation is carried as an fp16 pair hi + lo (~21 significant bits); the
  *    weight-streaming GEMMs (calls of at most 128 rows: decode steps of up to 128 envs)
  *    multiply both halves, the tile GEMMs (prefill, score, larger decode batches) both halves
- *    for q|k|v, o and down and hi alone for gate|up.  K/V are cached in fp16.
+ *    for q|k|v, o and down and hi alone for gate|up.  K/V are cached in fp16.  A finite
+ *    activation beyond the fp16 range (|x| > 65504) is stored as +-65504 and raises
+ *    VLA_STATUS_SATURATED in the status word (reported by the next vla_sync).
  *  - Calls are asynchronous on the handle's stream.  Host-checkable errors return at once,
  *    with no side effects.  Errors found on the device (token id out of range, non-finite
  *    logits, a pipeline wait that timed out) set a device status word; the next vla_sync
@@ -58,6 +60,9 @@ typedef enum {
 #define VLA_STATUS_NONFINITE 0x2u     /* a logit was NaN or infinite                       */
 #define VLA_STATUS_TIMEOUT 0x4u       /* a pipeline wait in the GEMM exceeded its limit    */
 #define VLA_STATUS_BAD_FORCED 0x8u    /* forced / scored token not an action-bin id        */
+#define VLA_STATUS_SATURATED 0x10u    /* a finite GEMM input activation beyond the fp16 range
+                                         (|x| > 65504) was stored as +-65504 (results of that
+                                         call are not those of the model)                  */
 
 /* Model and handle sizes.
  * Supported: head_dim in {64, 128}; n_heads * head_dim == d_model; d_model % 128 == 0;

@@ -2,6 +2,11 @@
  * vla_ops.h — single-kernel entry points of libvla.so, for checking one operation of the
  * hot path at a time.  Same conventions as vla.h (device pointers, asynchronous on
  * `cuda_stream`, host-checkable errors returned at once); each returns a vla_status.
+ *
+ * Errors found on the device by the GEMM and RMSNorm entry points (VLA_STATUS_TIMEOUT: a
+ * pipeline wait ran out and that CTA's output tile was not written; VLA_STATUS_SATURATED)
+ * are OR-ed into one status word per device that the library owns; vla_op_read_status
+ * returns and clears it.
  */
 #ifndef VLA_OPS_H_
 #define VLA_OPS_H_
@@ -69,10 +74,24 @@ int vla_op_gemm_decode_f16(const void* A, const void* A_lo, int lda, const void*
  *    current); make that first call before any stream capture.
  *  - All calls share the one array: calls that overlap on the GPU (other streams, other
  *    threads) race on it.  Serialise them, e.g. on one stream.
- *  - Nothing carries over between calls: every partial is rewritten before it is read. */
+ *  - Nothing carries over between calls: every partial is rewritten before it is read.
+ *  - A pipeline timeout is reported in the op status word (vla_op_read_status). */
 int vla_op_gemm_bf16_noalloc(const void* A, const void* A_lo, int lda, const void* W, int ldw,
                              float* C, int ldc, int M, int N, int K, int block_n, int splits,
                              void* cuda_stream);
+
+/* RMSNorm of the decoder layer (§3.1, the Llama-2 backbone) on M rows: y = h / sqrt(mean(h^2)
+ * + eps) * w, h f32 [M, d] (row stride ldh, 16-byte aligned, ldh % 4 == 0), w bf16 [d], written
+ * as the operand pair the projections read: y_hi / y_lo [M, d] (row stride d, 8-byte aligned),
+ * fp16 halves when fp16 != 0 (the engine's form), else bf16.  d % 4 == 0.  In the fp16 form a
+ * finite value beyond +-65504 is stored as +-65504 and sets VLA_STATUS_SATURATED in the op
+ * status word (NaN and infinities pass through unchanged). */
+int vla_op_rmsnorm(const float* h, int ldh, int M, int d, const void* w, float eps, void* y_hi,
+                   void* y_lo, int fp16, void* cuda_stream);
+
+/* Reads the op entry points' status word of the current device into *status_out (VLA_STATUS_*
+ * bits) after all work queued on cuda_stream, then clears it; synchronises the stream. */
+int vla_op_read_status(void* cuda_stream, uint32_t* status_out);
 
 /* The fused action head (§3.1 action bins; Eq. 1 log-probs; Algorithm 1 f) on B given
  * hidden states h (f32 [B, d], row stride ldh): RMSNorm with final_norm (bf16 [d], eps),
@@ -124,6 +143,22 @@ int vla_op_attn_chunk(const float* q, const void* kv, int max_env, int H, int hd
 
 /* Number of SMs the kernels size their persistent grids for (device property). */
 int vla_op_num_sms(void);
+
+/* ---- failure injection, for tests of the error paths (no GPU fault is involved) ----------
+ * vla_test_inject_launch_error: the nth_launch-th kernel launch of the library from now on
+ *   (counting every kernel of every entry point) returns cuda_error (a cudaError_t value,
+ *   non-zero) without launching, as a failed launch would; the entry point then returns
+ *   VLA_ERR_CUDA.  nth_launch == 0 disarms.  Process-wide; not for concurrent use.
+ * vla_test_set_wait_limit_ns: limit of each bounded pipeline wait of the tcgen05 GEMMs
+ *   launched from now on (0 restores the default, 1 s).  A wait that runs out sets
+ *   VLA_STATUS_TIMEOUT, the CTA waits (within the same limit) for its own copies and MMAs,
+ *   frees its tensor memory and exits without writing its output tile.
+ * vla_test_stall_next_gemm: in the next single-CTA tile GEMM launch, CTA 0 leaves its first
+ *   pipeline stage unfilled, so its MMA thread waits on a barrier that nothing completes until
+ *   the limit runs out (then as above).  The other CTAs run normally. */
+int vla_test_inject_launch_error(int64_t nth_launch, int cuda_error);
+int vla_test_set_wait_limit_ns(uint64_t limit_ns);
+int vla_test_stall_next_gemm(void);
 
 #ifdef __cplusplus
 }

@@ -146,73 +146,29 @@ class Weights:
         return lw
 
 
-def round_f16(x: torch.Tensor) -> torch.Tensor:
-    """Round to the nearest fp16 value (attribution mode only)."""
-    return x.to(torch.float32).to(torch.float16).to(F64)
-
-
-def round_f16_pair(x: torch.Tensor) -> torch.Tensor:
-    """x -> hi + lo with hi = fp16(x), lo = fp16(x - hi) (attribution mode only)."""
-    hi = round_f16(x)
-    return hi + round_f16(x - hi)
-
-
-def _same(x):
-    return x
-
-
-@dataclass(frozen=True)
-class Rounding:
-    """Where an implementation stores activations at reduced precision.  The oracle proper
-    uses EXACT (no rounding); the attribution mode mirrors the GPU path so that rounding
-    error can be told apart from bugs."""
-    act: object = _same   # GEMM input activations (norm outputs, attention output, SwiGLU)
-    q: object = _same     # queries after RoPE
-    kv: object = _same    # keys (after RoPE) and values as cached
-    # per-projection override of `act` for chunks of more than one row (prefill, score):
-    # {"qkv" | "o" | "gate_up" | "down": rounding}; None = `act` everywhere
-    act_chunk: Optional[dict] = None
-
-
-EXACT = Rounding()
-# The GPU path: fp16 activation pairs (fp16 weights hold the bf16 ones exactly above 2^-14),
-# fp32 queries, fp16 K/V; the multi-row projections use hi alone for gate|up.  Approximate
-# where the GPU's choice follows the whole call's rows rather than one env's chunk (the
-# last prefill layer runs gate|up on each env's final row through the two-half GEMM; decode
-# of more than 128 envs runs gate|up on hi alone).
-GPU_PATH = Rounding(act=round_f16_pair, q=lambda x: x.to(torch.float32).to(F64), kv=round_f16,
-                    act_chunk={"gate_up": round_f16})
-
-
-def layer_forward(shape: Shape, lw: dict, h, pos, k_cache, v_cache, rnd: Rounding = EXACT):
+def layer_forward(shape: Shape, lw: dict, h, pos, k_cache, v_cache):
     """One decoder layer over the chunk rows h [n, d] at positions pos [n].
 
     k_cache / v_cache: [m, H, hd] post-RoPE keys / values already in the context
     (positions 0 .. m-1); returns (h_out, k_all, v_all) with the chunk appended.
-    `rnd` is EXACT for the oracle proper (attribution runs pass GPU_PATH).
     """
     n = h.shape[0]
     d, H, hd, F = shape.d_model, shape.n_heads, shape.head_dim, shape.d_ffn
-
-    def act(site, x):
-        f = rnd.act_chunk.get(site) if (rnd.act_chunk and n > 1) else None
-        return (f or rnd.act)(x)
-
-    y = act("qkv", rms_norm(h, lw["attn_norm"], shape.rms_eps))
+    y = rms_norm(h, lw["attn_norm"], shape.rms_eps)
     qkv = y @ lw["wqkv"].T
     q = qkv[:, 0:d].reshape(n, H, hd)
     k = qkv[:, d:2 * d].reshape(n, H, hd)
-    v = rnd.kv(qkv[:, 2 * d:3 * d].reshape(n, H, hd))
-    q = rnd.q(apply_rope(q, pos, shape.rope_theta))
-    k = rnd.kv(apply_rope(k, pos, shape.rope_theta))
+    v = qkv[:, 2 * d:3 * d].reshape(n, H, hd)
+    q = apply_rope(q, pos, shape.rope_theta)
+    k = apply_rope(k, pos, shape.rope_theta)
     k_all = torch.cat([k_cache, k], dim=0)
     v_all = torch.cat([v_cache, v], dim=0)
     k_pos = torch.arange(k_all.shape[0], dtype=torch.long)
-    o = act("o", causal_attention(q, k_all, v_all, pos, k_pos))
+    o = causal_attention(q, k_all, v_all, pos, k_pos)
     h = h + o.reshape(n, d) @ lw["wo"].T
-    y = act("gate_up", rms_norm(h, lw["ffn_norm"], shape.rms_eps))
+    y = rms_norm(h, lw["ffn_norm"], shape.rms_eps)
     gu = y @ lw["w_gate_up"].T
-    h = h + act("down", silu(gu[:, :F]) * gu[:, F:]) @ lw["w_down"].T
+    h = h + (silu(gu[:, :F]) * gu[:, F:]) @ lw["w_down"].T
     return h, k_all, v_all
 
 
@@ -361,11 +317,8 @@ class Oracle:
     """
 
     def __init__(self, shape: Shape, weights: Dict[str, torch.Tensor], n_envs: int,
-                 cache_f64: bool = True, rounding: Rounding = EXACT):
-        """rounding: EXACT for the oracle proper; attribution runs pass GPU_PATH (not the
-        parity gate) to separate rounding error from bugs."""
+                 cache_f64: bool = True):
         self.shape = shape
-        self.rnd = rounding
         self.W = Weights(shape, weights, cache_f64)
         self.envs = [self._fresh() for _ in range(n_envs)]
 
@@ -381,6 +334,10 @@ class Oracle:
             self.envs[b] = self._fresh()
 
     # ------------------------------------------------------------------ forward
+    def _layer(self, lw: dict, h, pos, k_cache, v_cache):
+        """One decoder layer (layer_forward); the single place the engine calls it."""
+        return layer_forward(self.shape, lw, h, pos, k_cache, v_cache)
+
     def _forward(self, env_ids: Sequence[int], chunks: Sequence[torch.Tensor]):
         """Run chunk rows [n_b, d] of each env through all layers; append KV; return h."""
         sh = self.shape
@@ -393,8 +350,7 @@ class Oracle:
             lw = self.W.layer(l)
             for j, b in enumerate(env_ids):
                 e = self.envs[b]
-                hs[j], e.k[l], e.v[l] = layer_forward(sh, lw, hs[j], poss[j], e.k[l], e.v[l],
-                                                      self.rnd)
+                hs[j], e.k[l], e.v[l] = self._layer(lw, hs[j], poss[j], e.k[l], e.v[l])
         for b, x in zip(env_ids, chunks):
             e = self.envs[b]
             e.rows.extend(list(x))

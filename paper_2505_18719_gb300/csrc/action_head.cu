@@ -20,8 +20,9 @@ struct ArgMax {
   float v;
   int i;
 };
+// Larger value wins; equal values -> lower index.  Callers map NaN scores to -inf first (a NaN
+// held in `a` would otherwise never be replaced, since no comparison with NaN is true).
 __device__ __forceinline__ ArgMax better(ArgMax a, ArgMax b) {
-  // larger value wins; equal values -> lower index (NaN never wins)
   if (b.v > a.v || (b.v == a.v && b.i < a.i)) return b;
   return a;
 }
@@ -138,7 +139,8 @@ __global__ void __launch_bounds__(256) head_sample_kernel(const HeadArgs a) {
     u = fminf(fmaxf(u, 5.9604644775390625e-8f), 0.99999994039535522f);  // [2^-24, 1-2^-24]
     s = zt - logf(-logf(u));
   }
-  ArgMax am{s, k};
+  // A NaN score (from a NaN logit, which raises VLA_STATUS_NONFINITE below) loses to every bin.
+  ArgMax am{isnan(s) ? -INFINITY : s, k};
   float mx = zt;
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) {
@@ -211,12 +213,8 @@ int action_head_launch(const HeadArgs& a, cudaStream_t s) {
   const size_t smem = static_cast<size_t>(kHeadRows) * a.d * sizeof(float);
   if (smem > 200 * 1024) return VLA_ERR_UNSUPPORTED;
   if (smem > 48 * 1024) {
-    static bool set = false;
-    if (!set) {
-      VLA_CUDA_TRY(cudaFuncSetAttribute(head_logits_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                        200 * 1024));
-      set = true;
-    }
+    static std::atomic<uint64_t> attr_done{0};
+    VLA_CUDA_TRY(set_smem_limit(head_logits_kernel, 200 * 1024, attr_done));
   }
   const int R = a.B * a.n_pos;
   VLA_CUDA_TRY(launch_pdl(head_logits_kernel, dim3(256 / kHeadBins, (R + kHeadRows - 1) / kHeadRows),

@@ -246,20 +246,22 @@ __global__ void __launch_bounds__(128) attn_chunk_mma_kernel(const float* __rest
   l1 += __shfl_xor_sync(0xffffffffu, l1, 1);
   l1 += __shfl_xor_sync(0xffffffffu, l1, 2);
   const float inv0 = 1.f / l0, inv1 = 1.f / l1;
+  // outputs are convex combinations of fp16 values, so the fp16 split never saturates here
+  uint32_t sat = 0;
 #pragma unroll
   for (int nt = 0; nt < NT_D; ++nt) {
     const int col = head * HD + nt * 8 + 2 * tq;
     if (r0 < t.nrows) {
       const size_t off = static_cast<size_t>(t.row0 + r0) * d + col;
       uint32_t hi, lo;
-      split_pack2(o[nt][0] * inv0, o[nt][1] * inv0, hi, lo, fp16);
+      split_pack2(o[nt][0] * inv0, o[nt][1] * inv0, hi, lo, fp16, sat);
       *reinterpret_cast<uint32_t*>(out_hi + off) = hi;
       *reinterpret_cast<uint32_t*>(out_lo + off) = lo;
     }
     if (r1 < t.nrows) {
       const size_t off = static_cast<size_t>(t.row0 + r1) * d + col;
       uint32_t hi, lo;
-      split_pack2(o[nt][2] * inv1, o[nt][3] * inv1, hi, lo, fp16);
+      split_pack2(o[nt][2] * inv1, o[nt][3] * inv1, hi, lo, fp16, sat);
       *reinterpret_cast<uint32_t*>(out_hi + off) = hi;
       *reinterpret_cast<uint32_t*>(out_lo + off) = lo;
     }
@@ -389,13 +391,14 @@ __global__ void __launch_bounds__(NW * 32) attn_decode_kernel(const float* __res
       if (s_m[w][k] != -INFINITY) L += s_l[w][k] * exp2f(s_m[w][k] - M);
   const size_t bh = static_cast<size_t>(b) * H + head;
   const size_t out_off = static_cast<size_t>(b) * d + head * HD;
+  uint32_t sat = 0;  // convex combinations of fp16 values: the fp16 split never saturates
   if (S == 1) {
     for (int c = threadIdx.x; c < HD; c += blockDim.x) {
       float acc = 0.f;
       for (int w = 0; w < NW; ++w)
         for (int k = 0; k < KPI; ++k)
           if (s_m[w][k] != -INFINITY) acc += s_o[w][k][c] * exp2f(s_m[w][k] - M);
-      store_split1(out_hi, out_lo, out_off + c, acc / L, fp16);
+      store_split1(out_hi, out_lo, out_off + c, acc / L, fp16, sat);
     }
     return;
   }
@@ -438,7 +441,7 @@ __global__ void __launch_bounds__(NW * 32) attn_decode_kernel(const float* __res
   for (int i = 0; i < (HD + NT - 1) / NT; ++i) {
     const int c = threadIdx.x + i * NT;
     if (c < HD) {
-      store_split1(out_hi, out_lo, out_off + c, acc[i] / Lt, fp16);
+      store_split1(out_hi, out_lo, out_off + c, acc[i] / Lt, fp16, sat);
     }
   }
   if (threadIdx.x == 0) counters[bh] = 0;  // ready for the next launch
@@ -453,22 +456,14 @@ int attn_chunk_launch(const float* q, bf16* out_hi, bf16* out_lo, const AttnTile
   dim3 grid(n_tiles, H);
   if (hd == 128) {
     const int smem = (4 * 64) * (128 + 8) * 2;
-    static bool set = false;
-    if (!set) {
-      VLA_CUDA_TRY(cudaFuncSetAttribute(attn_chunk_mma_kernel<128>,
-                                        cudaFuncAttributeMaxDynamicSharedMemorySize, smem));
-      set = true;
-    }
+    static std::atomic<uint64_t> attr_done{0};
+    VLA_CUDA_TRY(set_smem_limit(attn_chunk_mma_kernel<128>, smem, attr_done));
     VLA_CUDA_TRY(launch_pdl(attn_chunk_mma_kernel<128>, grid, dim3(128), smem, stream, q, out_hi, out_lo,
                             tiles, kv, layer, H, scale_log2, fp16));
   } else if (hd == 64) {
     const int smem = (4 * 64) * (64 + 8) * 2;
-    static bool set = false;
-    if (!set) {
-      VLA_CUDA_TRY(cudaFuncSetAttribute(attn_chunk_mma_kernel<64>,
-                                        cudaFuncAttributeMaxDynamicSharedMemorySize, smem));
-      set = true;
-    }
+    static std::atomic<uint64_t> attr_done{0};
+    VLA_CUDA_TRY(set_smem_limit(attn_chunk_mma_kernel<64>, smem, attr_done));
     VLA_CUDA_TRY(launch_pdl(attn_chunk_mma_kernel<64>, grid, dim3(128), smem, stream, q, out_hi, out_lo,
                             tiles, kv, layer, H, scale_log2, fp16));
   } else {

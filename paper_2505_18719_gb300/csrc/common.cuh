@@ -7,6 +7,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <atomic>
+
 #include "../../include/vla.h"
 
 namespace vla {
@@ -79,33 +81,38 @@ __device__ __forceinline__ void split_pack2(float a, float b, uint32_t& hi, uint
 // The same pair in fp16: hi = fp16(x), lo = fp16(x - hi).  fp16 keeps 11 significant bits
 // per half (bf16: 8), so the single hi alone is 8x closer to x than a bf16 hi; GEMMs fed the
 // fp16 form run on fp16 weights.  A finite x beyond the fp16 range (|x| > 65504) saturates to
-// +-65504 instead of turning into inf; NaN and +-inf pass through unchanged, so a non-finite
-// activation still reaches the action head's non-finite check.
-__device__ __forceinline__ void split_f16(float x, f16& hi, f16& lo) {
-  if (fabsf(x) > 65504.f && fabsf(x) != INFINITY) x = copysignf(65504.f, x);
+// +-65504 instead of turning into inf and sets `sat` (the kernel then raises
+// VLA_STATUS_SATURATED); NaN and +-inf pass through unchanged, so a non-finite activation still
+// reaches the action head's non-finite check.  The bf16 pair never saturates (fp32 range).
+__device__ __forceinline__ void split_f16(float x, f16& hi, f16& lo, uint32_t& sat) {
+  if (fabsf(x) > 65504.f && fabsf(x) != INFINITY) {
+    x = copysignf(65504.f, x);
+    sat = 1u;
+  }
   hi = __float2half_rn(x);
   lo = __float2half_rn(x - __half2float(hi));
 }
-__device__ __forceinline__ void split_pack2_f16(float a, float b, uint32_t& hi, uint32_t& lo) {
+__device__ __forceinline__ void split_pack2_f16(float a, float b, uint32_t& hi, uint32_t& lo, uint32_t& sat) {
   f16 ha, la, hb, lb;
-  split_f16(a, ha, la);
-  split_f16(b, hb, lb);
+  split_f16(a, ha, la, sat);
+  split_f16(b, hb, lb, sat);
   __half2 h2 = __halves2half2(ha, hb), l2 = __halves2half2(la, lb);
   hi = *reinterpret_cast<uint32_t*>(&h2);
   lo = *reinterpret_cast<uint32_t*>(&l2);
 }
 // Operand format chosen at run time (uniform across a launch): fp16 if `fp16`, else bf16.  Buffers of
 // either format are 2-byte arrays; the pair halves come back as raw bits.
-__device__ __forceinline__ void split_pack2(float a, float b, uint32_t& hi, uint32_t& lo, bool fp16) {
+__device__ __forceinline__ void split_pack2(float a, float b, uint32_t& hi, uint32_t& lo, bool fp16,
+                                            uint32_t& sat) {
   if (fp16)
-    split_pack2_f16(a, b, hi, lo);
+    split_pack2_f16(a, b, hi, lo, sat);
   else
     split_pack2(a, b, hi, lo);
 }
-__device__ __forceinline__ void split_bits(float x, bool fp16, uint16_t& hi, uint16_t& lo) {
+__device__ __forceinline__ void split_bits(float x, bool fp16, uint16_t& hi, uint16_t& lo, uint32_t& sat) {
   if (fp16) {
     f16 h, l;
-    split_f16(x, h, l);
+    split_f16(x, h, l, sat);
     hi = __half_as_ushort(h);
     lo = __half_as_ushort(l);
   } else {
@@ -116,11 +123,15 @@ __device__ __forceinline__ void split_bits(float x, bool fp16, uint16_t& hi, uin
   }
 }
 // Stores x as the pair into hi[i] / lo[i] (2-byte elements of either format).
-__device__ __forceinline__ void store_split1(void* hi, void* lo, size_t i, float x, bool fp16) {
+__device__ __forceinline__ void store_split1(void* hi, void* lo, size_t i, float x, bool fp16, uint32_t& sat) {
   uint16_t h, l;
-  split_bits(x, fp16, h, l);
+  split_bits(x, fp16, h, l, sat);
   static_cast<uint16_t*>(hi)[i] = h;
   static_cast<uint16_t*>(lo)[i] = l;
+}
+// Raises VLA_STATUS_SATURATED when this thread clamped a value (rare: one atomic per thread that did).
+__device__ __forceinline__ void report_saturation(uint32_t* status, uint32_t sat) {
+  if (sat && status) atomicOr(status, VLA_STATUS_SATURATED);
 }
 
 __device__ __forceinline__ float warp_sum(float v) {
@@ -146,9 +157,26 @@ __device__ __forceinline__ void pdl_launch_dependents() {
 }
 __device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 
+// ----------------------------------------------------------------------------- test hooks
+// Failure injection for the tests (set through vla_test_inject_launch_error): when armed with
+// n >= 1, the n-th kernel launch from then on returns `g_inject_error` without launching, as a
+// failed launch would; every launch site checks it first.  Nothing on the device is touched.
+extern std::atomic<int64_t> g_inject_countdown;
+extern std::atomic<int> g_inject_error;
+inline cudaError_t injected_launch_error() {
+  if (g_inject_countdown.load(std::memory_order_relaxed) <= 0) return cudaSuccess;
+  if (g_inject_countdown.fetch_sub(1) == 1) return static_cast<cudaError_t>(g_inject_error.load());
+  return cudaSuccess;
+}
+// Limit of every bounded mbarrier wait in the tcgen05 kernels, passed to each launch (1 s; a test
+// hook lowers it so that a wait that nothing completes runs out quickly).
+extern std::atomic<uint64_t> g_wait_limit_ns;
+constexpr uint64_t kDefaultWaitLimitNs = 1000000000ull;
+
 template <typename... KArgs, typename... Args>
 inline cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem,
                               cudaStream_t stream, Args... args) {
+  if (const cudaError_t inj = injected_launch_error()) return inj;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = grid;
   cfg.blockDim = block;
@@ -162,6 +190,42 @@ inline cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, siz
   return cudaLaunchKernelEx(&cfg, kern, static_cast<KArgs>(args)...);
 }
 
+// Raises a kernel's dynamic shared-memory limit on the current device.  Function attributes
+// belong to each device's context, so the call is made once per (kernel, device): `done` holds
+// one bit per device index < 64 (beyond that the call is repeated every time).  Host threads
+// racing here at worst both make the call.
+template <typename Kern>
+inline cudaError_t set_smem_limit(Kern kern, int bytes, std::atomic<uint64_t>& done) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  const uint64_t bit = (dev >= 0 && dev < 64) ? (1ull << dev) : 0ull;
+  if (bit && (done.load(std::memory_order_acquire) & bit)) return cudaSuccess;
+  e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+  if (e == cudaSuccess && bit) done.fetch_or(bit, std::memory_order_release);
+  return e;
+}
+
+// Makes `dev` current for the scope of one API call and gives the caller's device back on exit
+// (the library must not change the current device of the calling thread).
+struct DeviceGuard {
+  int prev = -1;
+  bool restore = false;
+  cudaError_t err = cudaSuccess;
+  explicit DeviceGuard(int dev) {
+    err = cudaGetDevice(&prev);
+    if (err == cudaSuccess && prev != dev) {
+      err = cudaSetDevice(dev);
+      restore = err == cudaSuccess;
+    }
+  }
+  ~DeviceGuard() {
+    if (restore) cudaSetDevice(prev);
+  }
+  DeviceGuard(const DeviceGuard&) = delete;
+  DeviceGuard& operator=(const DeviceGuard&) = delete;
+};
+
 }  // namespace vla
 
 // ----------------------------------------------------------------------------- host macros
@@ -174,4 +238,7 @@ inline cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, siz
 namespace vla {
 int cuda_fail(cudaError_t e, const char* what);  // records the message, returns VLA_ERR_CUDA
 int record_error(int code, const char* msg);      // records the message, returns `code`
+// Device address of the op entry points' status word on the current device (a file-scope
+// device variable: looking it up allocates nothing).  VLA_OK or an error code.
+int op_status_word(uint32_t** out);
 }

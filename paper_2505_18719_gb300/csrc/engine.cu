@@ -9,6 +9,7 @@
 #include <cmath>
 #include <cstdio>
 #include <cstring>
+#include <mutex>
 #include <string>
 #include <vector>
 
@@ -35,6 +36,30 @@ int cuda_fail(cudaError_t e, const char* what) {
 int record_error(int code, const char* msg) {
   t_err = msg;
   return code;
+}
+
+namespace {
+// Status word of the op entry points (vla_ops.h): a file-scope device variable, one per device
+// that loads the library, so that reporting a timeout or a saturation needs no allocation.
+__device__ uint32_t g_op_status_word;
+constexpr int kMaxOpDevices = 64;
+std::mutex g_op_status_mu;
+uint32_t* g_op_status_ptr[kMaxOpDevices] = {};
+}  // namespace
+
+int op_status_word(uint32_t** out) {
+  int dev = 0;
+  VLA_CUDA_TRY(cudaGetDevice(&dev));
+  if (dev < 0 || dev >= kMaxOpDevices) return record_error(VLA_ERR_UNSUPPORTED, "op status: device index >= 64");
+  std::lock_guard<std::mutex> lock(g_op_status_mu);
+  if (!g_op_status_ptr[dev]) {
+    // the variable's name is only a host-side stand-in: ask for its address on this device
+    void* p = nullptr;
+    VLA_CUDA_TRY(cudaGetSymbolAddress(&p, g_op_status_word));
+    g_op_status_ptr[dev] = static_cast<uint32_t*>(p);
+  }
+  *out = g_op_status_ptr[dev];
+  return VLA_OK;
 }
 
 static int set_err(std::string* dst, int code, const std::string& msg) {
@@ -308,8 +333,8 @@ int run_gemm(vla_handle* h, int cls, const bf16* A, size_t a_plane, int lda, con
   }
   if (!stream_k && norm.norm_w && !defer_norm) {
     ev = prof_begin(h, VLA_KCLASS_OTHER);
-    rc = rmsnorm_launch(norm.resid, norm.norm_w, M, N, norm.norm_eps, norm.norm_hi, norm.norm_lo, h->stream,
-                        h->fp16);
+    rc = rmsnorm_launch(norm.resid, norm.ldr, norm.norm_w, M, N, norm.norm_eps, norm.norm_hi, norm.norm_lo,
+                        h->stream, h->fp16, h->status);
     prof_end(h, ev, VLA_KCLASS_OTHER, 0, 6.0 * M * N);
     if (rc) return fail(h, rc, t_err);
   }
@@ -340,7 +365,8 @@ int forward_layers(vla_handle* h, int M, const RowInfo* rows_dev, bool decode, i
   // the first layer's attention RMSNorm; every later RMSNorm follows a residual add
   h->y_deferred = false;
   int ev = prof_begin(h, VLA_KCLASS_OTHER);
-  if ((rc = rmsnorm_launch(h->h, h->attn_norm[0], M, d, c.rms_eps, h->y, h->y + pd, h->stream, h->fp16)))
+  if ((rc = rmsnorm_launch(h->h, d, h->attn_norm[0], M, d, c.rms_eps, h->y, h->y + pd, h->stream, h->fp16,
+                           h->status)))
     return fail(h, rc, t_err);
   prof_end(h, ev, VLA_KCLASS_OTHER, 0, 6.0 * M * d);
   for (int l = 0; l < c.n_layers; ++l) {
@@ -487,10 +513,12 @@ int vla_create(const vla_config* cfg, const vla_weights* w, void* cuda_stream, v
         !w->w_down[l])
       return set_err(nullptr, VLA_ERR_ARG, "vla_create: NULL per-layer weight pointer");
 
+  int dev = 0;
+  if (const cudaError_t e = cudaGetDevice(&dev)) return cuda_fail(e, "vla_create: current device");
   vla_handle* h = new vla_handle();
   h->cfg = c;
   h->stream = static_cast<cudaStream_t>(cuda_stream);
-  cudaGetDevice(&h->dev);
+  h->dev = dev;
   h->num_sms = query_num_sms();
   const int A = c.action_dim, B = c.max_batch, d = c.d_model, F = c.d_ffn, L = c.n_layers;
   h->max_tokens = std::max(c.max_tokens, std::max(B, (A - 1) * B));
@@ -653,7 +681,8 @@ int vla_prefill(vla_handle* h, int batch, const void* visual, int n_visual, cons
   }
   if (any_text && !token_ids) return fail(h, VLA_ERR_ARG, "vla_prefill: NULL token_ids");
   if (total > h->max_tokens) return fail(h, VLA_ERR_CAPACITY, "vla_prefill: more rows than max_tokens");
-  cudaSetDevice(h->dev);
+  DeviceGuard dev_guard(h->dev);
+  if (dev_guard.err != cudaSuccess) return fail(h, cuda_fail(dev_guard.err, "vla_prefill: set device"), t_err);
 
   // host-side row table, attention tiles and last-row indices
   int slot;
@@ -726,7 +755,8 @@ int vla_decode_actions(vla_handle* h, const float* uniforms, float temperature, 
     return fail(h, VLA_ERR_ARG, "vla_decode_actions: NULL buffer");
   int rc;
   if ((rc = check_turn_state(h, "vla_decode_actions"))) return rc;
-  cudaSetDevice(h->dev);
+  DeviceGuard dev_guard(h->dev);
+  if (dev_guard.err != cudaSuccess) return fail(h, cuda_fail(dev_guard.err, "vla_decode_actions: set device"), t_err);
   const vla_config& c = h->cfg;
   const int B = h->active_batch, A = c.action_dim, d = c.d_model;
 
@@ -799,7 +829,8 @@ int vla_score_actions(vla_handle* h, const int32_t* tokens, float temperature, f
   if (!tokens || !logprobs_out) return fail(h, VLA_ERR_ARG, "vla_score_actions: NULL buffer");
   int rc;
   if ((rc = check_turn_state(h, "vla_score_actions"))) return rc;
-  cudaSetDevice(h->dev);
+  DeviceGuard dev_guard(h->dev);
+  if (dev_guard.err != cudaSuccess) return fail(h, cuda_fail(dev_guard.err, "vla_score_actions: set device"), t_err);
   const vla_config& c = h->cfg;
   const int B = h->active_batch, A = c.action_dim, d = c.d_model;
   const int n = A - 1;  // teacher-forced rows per env
@@ -896,7 +927,8 @@ int vla_action_entropy(vla_handle* h, float* entropy_out) {
   int rc;
   if ((rc = check_turn_state(h, "vla_action_entropy"))) return rc;
   if (!h->entropy_valid) return fail(h, VLA_ERR_STATE, "vla_action_entropy: no decode or score since the prefill");
-  cudaSetDevice(h->dev);
+  DeviceGuard dev_guard(h->dev);
+  if (dev_guard.err != cudaSuccess) return fail(h, cuda_fail(dev_guard.err, "vla_action_entropy: set device"), t_err);
   const size_t n = static_cast<size_t>(h->active_batch) * h->cfg.action_dim;
   if (cudaMemcpyAsync(entropy_out, h->head_entropy, n * sizeof(float), cudaMemcpyDeviceToDevice, h->stream) !=
       cudaSuccess)
@@ -909,7 +941,8 @@ int vla_value(vla_handle* h, const void* w_value, float bias, float* values_out)
   if (!w_value || !values_out || !std::isfinite(bias)) return fail(h, VLA_ERR_ARG, "vla_value: bad argument");
   int rc;
   if ((rc = check_turn_state(h, "vla_value"))) return rc;
-  cudaSetDevice(h->dev);
+  DeviceGuard dev_guard(h->dev);
+  if (dev_guard.err != cudaSuccess) return fail(h, cuda_fail(dev_guard.err, "vla_value: set device"), t_err);
   const vla_config& c = h->cfg;
   rc = value_head_launch(h->h_last, c.d_model, h->active_batch, c.d_model, h->final_norm,
                          static_cast<const bf16*>(w_value), c.rms_eps, bias, values_out, h->stream);
@@ -937,7 +970,8 @@ int vla_ppo_clip(const float* lp_new, const float* lp_old, const float* adv, int
 
 int vla_sync(vla_handle* h) {
   if (!h) return set_err(nullptr, VLA_ERR_ARG, "vla_sync: NULL handle");
-  cudaSetDevice(h->dev);
+  DeviceGuard dev_guard(h->dev);
+  if (dev_guard.err != cudaSuccess) return fail(h, cuda_fail(dev_guard.err, "vla_sync: set device"), t_err);
   cudaError_t e = cudaStreamSynchronize(h->stream);
   if (e != cudaSuccess) return fail(h, cuda_fail(e, "vla_sync: stream"), t_err);
   uint32_t st = 0;
@@ -950,6 +984,7 @@ int vla_sync(vla_handle* h) {
     if (st & VLA_STATUS_NONFINITE) msg += " non-finite logit;";
     if (st & VLA_STATUS_TIMEOUT) msg += " GEMM pipeline wait timed out;";
     if (st & VLA_STATUS_BAD_FORCED) msg += " forced/scored token is not an action-bin id;";
+    if (st & VLA_STATUS_SATURATED) msg += " an activation beyond the fp16 range was saturated;";
     char buf[32];
     snprintf(buf, sizeof(buf), " (0x%x)", st);
     return fail(h, VLA_ERR_DEVICE_STATUS, msg + buf);
@@ -959,7 +994,8 @@ int vla_sync(vla_handle* h) {
 
 int vla_sync_weights(vla_handle* h) {
   if (!h) return set_err(nullptr, VLA_ERR_ARG, "vla_sync_weights: NULL handle");
-  cudaSetDevice(h->dev);
+  DeviceGuard dev_guard(h->dev);
+  if (dev_guard.err != cudaSuccess) return fail(h, cuda_fail(dev_guard.err, "vla_sync_weights: set device"), t_err);
   const int rc = convert_weights(h);
   if (rc) return fail(h, rc, t_err);
   return VLA_OK;
@@ -974,7 +1010,7 @@ const char* vla_last_error(const vla_handle* h) { return h ? h->err.c_str() : t_
 
 void vla_destroy(vla_handle* h) {
   if (!h) return;
-  cudaSetDevice(h->dev);
+  DeviceGuard dev_guard(h->dev);  // best effort: the handle is freed whatever happens
   cudaStreamSynchronize(h->stream);
   void* bufs[] = {h->kv, h->h, h->y, h->q, h->ao, h->u, h->ws, h->h_last, h->head_in, h->head_z, h->head_entropy, h->q_last, h->ss_part, h->last_rows, h->rope,
                   h->rows, h->tiles, h->sidx, h->didx, h->fed, h->pending, h->status, h->part_o,
@@ -1052,6 +1088,7 @@ int op_gemm(const std::string& name, bool fp16, const void* A, const void* A_lo,
   g.epi.fp16 = fp16;
   if (splits > 1 && gemm_effective_splits(K, splits) > 1 && !workspace)
     return set_err(nullptr, VLA_ERR_ARG, name + ": splits > 1 needs a workspace");
+  if (const int rs = op_status_word(&g.epi.status)) return rs;
   const int rc = gemm_launch(g, static_cast<cudaStream_t>(cuda_stream), query_num_sms(), nullptr);
   if (rc != VLA_OK && rc != VLA_ERR_CUDA) return set_err(nullptr, rc, name + ": unsupported arguments");
   return rc;
@@ -1077,6 +1114,7 @@ int op_gemm_pair(const std::string& name, bool fp16, const void* A, const void* 
   g.epi.out_f32 = C;
   g.epi.ldo = ldc;
   g.epi.fp16 = fp16;
+  if (const int rs = op_status_word(&g.epi.status)) return rs;
   const int rc = gemm_launch(g, static_cast<cudaStream_t>(cuda_stream), query_num_sms(), nullptr);
   if (rc != VLA_OK && rc != VLA_ERR_CUDA) return set_err(nullptr, rc, name + ": unsupported arguments");
   return rc;
@@ -1102,6 +1140,7 @@ int op_gemm_decode(const std::string& name, bool fp16, const void* A, const void
   g.epi.out_f32 = C;
   g.epi.ldo = ldc;
   g.epi.fp16 = fp16;
+  if (const int rs = op_status_word(&g.epi.status)) return rs;
   const int rc = gemv_launch(g, static_cast<cudaStream_t>(cuda_stream), query_num_sms(), nullptr);
   if (rc != VLA_OK && rc != VLA_ERR_CUDA)
     return set_err(nullptr, rc, name + ": unsupported arguments or workspace too small");
@@ -1263,5 +1302,47 @@ int vla_op_attn_chunk(const float* q, const void* kv, int max_env, int H, int hd
 }
 
 int vla_op_num_sms(void) { return query_num_sms(); }
+
+int vla_op_rmsnorm(const float* hs, int ldh, int M, int d, const void* w, float eps, void* y_hi, void* y_lo,
+                   int fp16, void* cuda_stream) {
+  if (!hs || !w || !y_hi || !y_lo || M < 1 || d < 4 || (d & 3) || ldh < d || (ldh & 3) || !(eps >= 0.f) ||
+      (reinterpret_cast<uintptr_t>(hs) & 15) || (reinterpret_cast<uintptr_t>(w) & 7) ||
+      (reinterpret_cast<uintptr_t>(y_hi) & 7) || (reinterpret_cast<uintptr_t>(y_lo) & 7))
+    return set_err(nullptr, VLA_ERR_ARG, "vla_op_rmsnorm: bad argument");
+  uint32_t* status = nullptr;
+  if (const int rs = op_status_word(&status)) return rs;
+  return rmsnorm_launch(hs, ldh, static_cast<const bf16*>(w), M, d, eps, static_cast<bf16*>(y_hi),
+                        static_cast<bf16*>(y_lo), static_cast<cudaStream_t>(cuda_stream), fp16 != 0, status);
+}
+
+int vla_op_read_status(void* cuda_stream, uint32_t* status_out) {
+  if (!status_out) return set_err(nullptr, VLA_ERR_ARG, "vla_op_read_status: NULL status_out");
+  uint32_t* word = nullptr;
+  if (const int rs = op_status_word(&word)) return rs;
+  cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
+  VLA_CUDA_TRY(cudaMemcpyAsync(status_out, word, sizeof(uint32_t), cudaMemcpyDeviceToHost, st));
+  VLA_CUDA_TRY(cudaMemsetAsync(word, 0, sizeof(uint32_t), st));
+  VLA_CUDA_TRY(cudaStreamSynchronize(st));
+  return VLA_OK;
+}
+
+// ------------------------------------------------------------------- failure injection (tests)
+int vla_test_inject_launch_error(int64_t nth_launch, int cuda_error) {
+  if (nth_launch < 0 || (nth_launch > 0 && cuda_error == 0))
+    return set_err(nullptr, VLA_ERR_ARG, "vla_test_inject_launch_error: bad argument");
+  g_inject_error.store(cuda_error);
+  g_inject_countdown.store(nth_launch);
+  return VLA_OK;
+}
+
+int vla_test_set_wait_limit_ns(uint64_t limit_ns) {
+  g_wait_limit_ns.store(limit_ns ? limit_ns : kDefaultWaitLimitNs);
+  return VLA_OK;
+}
+
+int vla_test_stall_next_gemm(void) {
+  gemm_stall_next_launch();
+  return VLA_OK;
+}
 
 }  // extern "C"

@@ -87,6 +87,10 @@ int gemm_launch(const GemmArgs& a, cudaStream_t stream, int num_sms, GemmCost* c
 // `workspace` (gemv_workspace_bytes), then the epilogue of `a.epi` in a fixed-order reduction
 // (EPI_RESID with norm_w set: fused with the following RMSNorm).
 size_t gemv_workspace_bytes(int M, int N, int K, int num_sms);
+
+// Failure injection (test hook): in the next single-CTA tile GEMM launch, CTA 0 leaves its first
+// pipeline stage unfilled; its bounded wait on that stage runs out (VLA_STATUS_TIMEOUT).
+void gemm_stall_next_launch();
 int gemv_launch(const GemmArgs& a, cudaStream_t stream, int num_sms, GemmCost* cost);
 
 }  // namespace vla

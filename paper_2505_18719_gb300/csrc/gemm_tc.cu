@@ -70,6 +70,8 @@ struct Params {
   int tiles_m, tiles_n, splits, kb_total, kb_per_split;
   int group_m;          // m-tiles per raster group
   EpiArgs epi;
+  uint64_t wait_limit;  // ns per bounded mbarrier wait
+  int stall;            // failure injection (test hook): CTA 0 never fills its first stage
 };
 
 __device__ __forceinline__ void unit_coords(const Params& p, int u, int& m_blk, int& n_blk,
@@ -89,10 +91,10 @@ __device__ __forceinline__ void unit_coords(const Params& p, int u, int& m_blk, 
 // ----------------------------------------------------------------------------- epilogues
 // 16 values as operand hi/lo pairs, fp16 if `fp16` else bf16 (two 32-byte stores each).
 __device__ __forceinline__ void store_split16(bf16* hi_dst, bf16* lo_dst, const float (&v)[16],
-                                              bool fp16) {
+                                              bool fp16, uint32_t& sat) {
   uint32_t h[8], l[8];
 #pragma unroll
-  for (int i = 0; i < 8; ++i) split_pack2(v[2 * i], v[2 * i + 1], h[i], l[i], fp16);
+  for (int i = 0; i < 8; ++i) split_pack2(v[2 * i], v[2 * i + 1], h[i], l[i], fp16, sat);
   reinterpret_cast<uint4*>(hi_dst)[0] = make_uint4(h[0], h[1], h[2], h[3]);
   reinterpret_cast<uint4*>(hi_dst)[1] = make_uint4(h[4], h[5], h[6], h[7]);
   reinterpret_cast<uint4*>(lo_dst)[0] = make_uint4(l[0], l[1], l[2], l[3]);
@@ -136,7 +138,7 @@ __device__ __forceinline__ float row_scale(const Params& p, int m) {
 // Plain epilogues: F32 / RESID / PARTIAL, 16 columns at a time.
 template <int BN, int EPI>
 __device__ __forceinline__ void epilogue_plain(const Params& p, uint32_t trow, int m, int n0,
-                                               int split) {
+                                               int split, uint32_t& sat) {
   const bool row_ok = m < p.M;
   // residual + the next RMSNorm's numerator (h * w) and this tile's sum of squares of h
   const bool norm_next = (EPI == EPI_RESID) && p.epi.ss_out != nullptr;
@@ -206,12 +208,12 @@ __device__ __forceinline__ void epilogue_plain(const Params& p, uint32_t trow, i
       }
       const size_t off = static_cast<size_t>(m) * p.epi.ldn + n;
       if (cnt == 16 && (p.epi.ldn & 7) == 0) {
-        store_split16(p.epi.norm_hi + off, p.epi.norm_lo + off, y, p.epi.fp16);
+        store_split16(p.epi.norm_hi + off, p.epi.norm_lo + off, y, p.epi.fp16, sat);
       } else {
 #pragma unroll
         for (int i = 0; i < 16; ++i) {
           if (i >= cnt) continue;
-          store_split1(p.epi.norm_hi, p.epi.norm_lo, off + i, y[i], p.epi.fp16);
+          store_split1(p.epi.norm_hi, p.epi.norm_lo, off + i, y[i], p.epi.fp16, sat);
         }
       }
     }
@@ -221,7 +223,8 @@ __device__ __forceinline__ void epilogue_plain(const Params& p, uint32_t trow, i
 
 // SwiGLU: tile columns [0, BN/2) are gate features f0.., [BN/2, BN) the matching up features.
 template <int BN>
-__device__ __forceinline__ void epilogue_swiglu(const Params& p, uint32_t trow, int m, int f0) {
+__device__ __forceinline__ void epilogue_swiglu(const Params& p, uint32_t trow, int m, int f0,
+                                                uint32_t& sat) {
   const int F = p.N >> 1;
   const bool row_ok = m < p.M;
   const float rs = row_scale(p, m);
@@ -237,12 +240,12 @@ __device__ __forceinline__ void epilogue_swiglu(const Params& p, uint32_t trow, 
     for (int i = 0; i < 16; ++i) o[i] = silu_f(g[i] * rs) * (u[i] * rs);
     const size_t off = static_cast<size_t>(m) * p.epi.ldo + f;
     if (f + 16 <= F && ((p.epi.ldo & 7) == 0)) {
-      store_split16(p.epi.out_hi + off, p.epi.out_lo + off, o, p.epi.fp16);
+      store_split16(p.epi.out_hi + off, p.epi.out_lo + off, o, p.epi.fp16, sat);
     } else {
 #pragma unroll
       for (int i = 0; i < 16; ++i) {
         if (f + i >= F) continue;
-        store_split1(p.epi.out_hi, p.epi.out_lo, off + i, o[i], p.epi.fp16);
+        store_split1(p.epi.out_hi, p.epi.out_lo, off + i, o[i], p.epi.fp16, sat);
       }
     }
   }
@@ -373,6 +376,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t tmem_base = *tmem_slot;
   const int units = p.tiles_m * p.tiles_n * p.splits;
   uint32_t* status = p.epi.status;
+  const uint64_t limit = p.wait_limit;
 
   if (warp == 0) {
     if (lane == 0) {
@@ -382,15 +386,26 @@ __global__ void __launch_bounds__(kThreads, 1)
       uint32_t phase = 0;
       uint32_t issued = 0, issued_phase = 0;
       bool ok = true;
+      // Failure injection (test hook): CTA 0 leaves its first stage unfilled, so the MMA
+      // thread's bounded wait on that stage is one that nothing completes.
+      bool skip_stage = p.stall != 0 && blockIdx.x == 0;
       for (int u = blockIdx.x; u < units && ok; u += gridDim.x) {
         int m_blk, n_blk, split;
         unit_coords(p, u, m_blk, n_blk, split);
         const int kb0 = split * p.kb_per_split;
         const int kb1 = min(kb0 + p.kb_per_split, p.kb_total);
         for (int kb = kb0; kb < kb1; ++kb) {
-          if (!wait_bounded(empty0 + 8 * stage, phase ^ 1u, abort_flag, status)) {
+          if (!wait_bounded(empty0 + 8 * stage, phase ^ 1u, abort_flag, status, limit)) {
             ok = false;
             break;
+          }
+          if (skip_stage) {
+            skip_stage = false;
+            if (++stage == STAGES) {
+              stage = 0;
+              phase ^= 1u;
+            }
+            continue;
           }
           const uint32_t fb = full0 + 8 * stage;
           const uint32_t sa = smem_u32(smem + stage * STAGE_BYTES);
@@ -414,7 +429,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       // Drain: every stage's last issued copy has landed before the CTA may exit.
       for (int s = 0; s < STAGES; ++s)
-        if (issued & (1u << s)) wait_drain(full0 + 8 * s, (issued_phase >> s) & 1u);
+        if (issued & (1u << s)) wait_drain(full0 + 8 * s, (issued_phase >> s) & 1u, limit);
     }
   } else if (warp == 1) {
     if (lane == 0) {
@@ -430,11 +445,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int kb1 = min(kb0 + p.kb_per_split, p.kb_total);
         const int acc = it & 1;
         const uint32_t acc_phase = (it >> 1) & 1;
-        if (!wait_bounded(tempty0 + 8 * acc, acc_phase ^ 1u, abort_flag, status)) break;
+        if (!wait_bounded(tempty0 + 8 * acc, acc_phase ^ 1u, abort_flag, status, limit)) break;
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + acc * BN;
         for (int kb = kb0; kb < kb1; ++kb) {
-          if (!wait_bounded(full0 + 8 * stage, phase, abort_flag, status)) {
+          if (!wait_bounded(full0 + 8 * stage, phase, abort_flag, status, limit)) {
             ok = false;
             break;
           }
@@ -457,11 +472,12 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       // Drain: all MMAs issued by this thread have completed before TMEM is freed.
       tc_commit(drain_bar);
-      wait_drain(drain_bar, 0);
+      wait_drain(drain_bar, 0, limit);
     }
   } else {
     // -------------------------------------------------------------- epilogue warps 2..5
     const int q = warp & 3;  // TMEM lane quarter this warp may access
+    uint32_t sat = 0;
     int it = 0;
     for (int u = blockIdx.x; u < units; u += gridDim.x, ++it) {
       int m_blk, n_blk, split;
@@ -469,22 +485,23 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int acc = it & 1;
       const uint32_t acc_phase = (it >> 1) & 1;
       int ok = 1;
-      if (lane == 0) ok = wait_bounded(tfull0 + 8 * acc, acc_phase, abort_flag, status) ? 1 : 0;
+      if (lane == 0) ok = wait_bounded(tfull0 + 8 * acc, acc_phase, abort_flag, status, limit) ? 1 : 0;
       ok = __shfl_sync(0xffffffffu, ok, 0);
       if (!ok) break;
       tc_fence_after();
       const int m = m_blk * BM + q * 32 + lane;
       const uint32_t trow = tmem_base + (static_cast<uint32_t>(q * 32) << 16) + acc * BN;
       if (EPI == EPI_SWIGLU)
-        epilogue_swiglu<BN>(p, trow, m, n_blk * (BN / 2));
+        epilogue_swiglu<BN>(p, trow, m, n_blk * (BN / 2), sat);
       else if (EPI == EPI_QKV)
         epilogue_qkv<BN>(p, trow, m, n_blk * BN);
       else
-        epilogue_plain<BN, EPI>(p, trow, m, n_blk * BN, split);
+        epilogue_plain<BN, EPI>(p, trow, m, n_blk * BN, split, sat);
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(tempty0 + 8 * acc);
     }
+    report_saturation(status, sat);
   }
 
   // Lanes 1..31 of the producer and MMA warps got here long before their lane 0: reconverge
@@ -581,6 +598,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int n_pairs = gridDim.x >> 1;
   const int pair = blockIdx.x >> 1;
   uint32_t* status = p.epi.status;
+  const uint64_t limit = p.wait_limit;
 
   if (warp == 0) {
     if (lane == 0) {
@@ -595,7 +613,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         unit_coords(p, u, m_blk, n_blk, split);
         const int row_a = m_blk * 256 + static_cast<int>(rank - leader) * 128;
         for (int kb = 0; kb < p.kb_total; ++kb) {
-          if (!wait_bounded(empty0 + 8 * stage, phase ^ 1u, abort_flag, status)) {
+          if (!wait_bounded(empty0 + 8 * stage, phase ^ 1u, abort_flag, status, limit)) {
             ok = false;
             break;
           }
@@ -620,7 +638,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       // Drain (leader only: the pair's loads complete on the leader's barriers).
       if (is_leader)
         for (int s = 0; s < STAGES; ++s)
-          if (issued & (1u << s)) wait_drain(full0 + 8 * s, (issued_phase >> s) & 1u);
+          if (issued & (1u << s)) wait_drain(full0 + 8 * s, (issued_phase >> s) & 1u, limit);
     }
   } else if (warp == 1) {
     if (lane == 0 && is_leader) {
@@ -632,11 +650,11 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int u = pair; u < units && ok; u += n_pairs, ++it) {
         const int acc = it & 1;
         const uint32_t acc_phase = (it >> 1) & 1;
-        if (!wait_bounded(tempty0 + 8 * acc, acc_phase ^ 1u, abort_flag, status)) break;
+        if (!wait_bounded(tempty0 + 8 * acc, acc_phase ^ 1u, abort_flag, status, limit)) break;
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + acc * BN;
         for (int kb = 0; kb < p.kb_total; ++kb) {
-          if (!wait_bounded(full0 + 8 * stage, phase, abort_flag, status)) {
+          if (!wait_bounded(full0 + 8 * stage, phase, abort_flag, status, limit)) {
             ok = false;
             break;
           }
@@ -658,12 +676,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (ok) tc_commit_pair(tfull0 + 8 * acc, pair_mask);
       }
       tc_commit_pair(drain_bar, static_cast<uint16_t>(1u << leader));
-      wait_drain(drain_bar, 0);
+      wait_drain(drain_bar, 0, limit);
     }
   } else {
     // -------------------------------------------------------------- epilogue warps 2..5
     const int q = warp & 3;
     const uint32_t tempty_leader = mapa_shared(tempty0, leader);
+    uint32_t sat = 0;
     int it = 0;
     for (int u = pair; u < units; u += n_pairs, ++it) {
       int m_blk, n_blk, split;
@@ -671,22 +690,23 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int acc = it & 1;
       const uint32_t acc_phase = (it >> 1) & 1;
       int ok = 1;
-      if (lane == 0) ok = wait_bounded(tfull0 + 8 * acc, acc_phase, abort_flag, status) ? 1 : 0;
+      if (lane == 0) ok = wait_bounded(tfull0 + 8 * acc, acc_phase, abort_flag, status, limit) ? 1 : 0;
       ok = __shfl_sync(0xffffffffu, ok, 0);
       if (!ok) break;
       tc_fence_after();
       const int m = m_blk * 256 + static_cast<int>(rank - leader) * 128 + q * 32 + lane;
       const uint32_t trow = tmem_base + (static_cast<uint32_t>(q * 32) << 16) + acc * BN;
       if (EPI == EPI_SWIGLU)
-        epilogue_swiglu<BN>(p, trow, m, n_blk * (BN / 2));
+        epilogue_swiglu<BN>(p, trow, m, n_blk * (BN / 2), sat);
       else if (EPI == EPI_QKV)
         epilogue_qkv<BN>(p, trow, m, n_blk * BN);
       else
-        epilogue_plain<BN, EPI>(p, trow, m, n_blk * BN, 0);
+        epilogue_plain<BN, EPI>(p, trow, m, n_blk * BN, 0, sat);
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive_cluster(tempty_leader + 8 * acc);
     }
+    report_saturation(status, sat);
   }
 
   __syncwarp();  // reconverge the role warps before the CTA and cluster barriers
@@ -767,9 +787,10 @@ __global__ void reduce_f32_kernel(Src src, int M, int N, float* out, int ldo, in
 
 template <class Src>
 __global__ void reduce_swiglu_kernel(Src src, int M, int F, bf16* out_hi, bf16* out_lo, int ldo,
-                                     bool fp16) {
+                                     bool fp16, uint32_t* status) {
   pdl_launch_dependents();
   pdl_wait();
+  uint32_t sat = 0;
   const int64_t total = static_cast<int64_t>(M) * F;
   for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < total;
        i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
@@ -778,8 +799,9 @@ __global__ void reduce_swiglu_kernel(Src src, int M, int F, bf16* out_hi, bf16* 
     split_index<Src>(i, M, F, m, f);
     const float g = src(m, static_cast<int>(f));
     const float u = src(m, static_cast<int>(f) + F);
-    store_split1(out_hi, out_lo, static_cast<size_t>(m) * ldo + f, silu_f(g) * u, fp16);
+    store_split1(out_hi, out_lo, static_cast<size_t>(m) * ldo + f, silu_f(g) * u, fp16, sat);
   }
+  report_saturation(status, sat);
 }
 
 // One thread per (row, q|k|v section, head, i < hd/2): sums the pair (i, i + hd/2).
@@ -956,9 +978,10 @@ __global__ void stream_reduce_f32_kernel(StreamSrc src, int M, int N, float* out
 
 // items (ceil(F / 256), ceil(M / kMR)), 256 threads: gate column f, up column f + F
 __global__ void stream_reduce_swiglu_kernel(StreamSrc src, int M, int F, bf16* out_hi,
-                                            bf16* out_lo, int ldo, bool fp16) {
+                                            bf16* out_lo, int ldo, bool fp16, uint32_t* status) {
   pdl_launch_dependents();
   pdl_wait();
+  uint32_t sat = 0;
   const int nx = (F + 255) / 256, ny = (M + kMR - 1) / kMR;
   int item = blockIdx.x, bx, by;
   while (next_item(item, nx, ny, bx, by)) {
@@ -970,9 +993,10 @@ __global__ void stream_reduce_swiglu_kernel(StreamSrc src, int M, int F, bf16* o
 #pragma unroll
     for (int j = 0; j < kMR; ++j) {
       if (m0 + j >= M) break;
-      store_split1(out_hi, out_lo, static_cast<size_t>(m0 + j) * ldo + f, silu_f(g[j]) * u[j], fp16);
+      store_split1(out_hi, out_lo, static_cast<size_t>(m0 + j) * ldo + f, silu_f(g[j]) * u[j], fp16, sat);
     }
   }
+  report_saturation(status, sat);
 }
 
 // items (3d / 256, ceil(M / kMR)), 128 threads; 256 % hd == 0 and d % 256 == 0, so both
@@ -1028,12 +1052,13 @@ __global__ void stream_reduce_qkv_kernel(StreamSrc src, int M, EpiArgs e) {
 __global__ void __maxnreg__(48) stream_reduce_resid_norm_kernel(StreamSrc src, int N, float* h,
                                                                          int ldh, const bf16* w, float eps,
                                                                          bf16* y_hi, bf16* y_lo, int ldy,
-                                                                         bool fp16) {
+                                                                         bool fp16, uint32_t* status) {
   pdl_launch_dependents();
   pdl_wait();
   __shared__ float red[32];
   const int m = blockIdx.x;
   float* hrow = h + static_cast<size_t>(m) * ldh;
+  uint32_t sat = 0;
   float ss = 0.f;
   for (int n = threadIdx.x * 4; n < N; n += blockDim.x * 4) {
     const float4 acc = TileSum(src, n).sum4(m);
@@ -1056,11 +1081,12 @@ __global__ void __maxnreg__(48) stream_reduce_resid_norm_kernel(StreamSrc src, i
     const uint2 ww = *reinterpret_cast<const uint2*>(w + n);
     const float2 w0 = unpack_bf16x2(ww.x), w1 = unpack_bf16x2(ww.y);
     uint2 hi, lo;
-    split_pack2(v.x * r * w0.x, v.y * r * w0.y, hi.x, lo.x, fp16);
-    split_pack2(v.z * r * w1.x, v.w * r * w1.y, hi.y, lo.y, fp16);
+    split_pack2(v.x * r * w0.x, v.y * r * w0.y, hi.x, lo.x, fp16, sat);
+    split_pack2(v.z * r * w1.x, v.w * r * w1.y, hi.y, lo.y, fp16, sat);
     *reinterpret_cast<uint2*>(y_hi + static_cast<size_t>(m) * ldy + n) = hi;
     *reinterpret_cast<uint2*>(y_lo + static_cast<size_t>(m) * ldy + n) = lo;
   }
+  report_saturation(status, sat);
 }
 
 // ----------------------------------------------------------------------------- decode GEMM
@@ -1080,6 +1106,7 @@ struct GemvParams {
   float* ws;
   uint32_t* status;
   bool fp16;            // operand format (weights and activation pair): fp16, else bf16
+  uint64_t wait_limit;  // ns per bounded mbarrier wait
 };
 
 // TR = 256 weight rows per tile, as two M=128 MMAs sharing each activation tile, so the
@@ -1144,6 +1171,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int g_end = min(g_begin + p.per_cta, total);
   const int t_first = g_begin / p.kbt;
   uint32_t* status = p.status;
+  const uint64_t limit = p.wait_limit;
 
   if (warp == 0) {
     if (lane == 0) {
@@ -1174,7 +1202,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       uint32_t phase = (pre == STAGES) ? 1u : 0u;
       for (int i = pre; i < n; ++i) {
         const int g = g_begin + i, t = g / p.kbt, kb = g - t * p.kbt;
-        if (!wait_bounded(empty0 + 8 * stage, phase ^ 1u, abort_flag, status)) break;
+        if (!wait_bounded(empty0 + 8 * stage, phase ^ 1u, abort_flag, status, limit)) break;
         const uint32_t fb = full0 + 8 * stage;
         const uint32_t sw = smem_u32(smem + stage * STAGE_BYTES);
         const uint32_t sx = sw + W_BYTES;
@@ -1190,7 +1218,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
       for (int s = 0; s < STAGES; ++s)
-        if (issued & (1u << s)) wait_drain(full0 + 8 * s, (issued_phase >> s) & 1u);
+        if (issued & (1u << s)) wait_drain(full0 + 8 * s, (issued_phase >> s) & 1u, limit);
     }
   } else if (warp == 1) {
     if (lane == 0) {
@@ -1206,10 +1234,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         g += kb1 - kb0;
         const int acc = it & 1;
         const uint32_t acc_phase = (it >> 1) & 1;
-        if (!wait_bounded(tempty0 + 8 * acc, acc_phase ^ 1u, abort_flag, status)) break;
+        if (!wait_bounded(tempty0 + 8 * acc, acc_phase ^ 1u, abort_flag, status, limit)) break;
         tc_fence_after();
         for (int kb = kb0; kb < kb1; ++kb) {
-          if (!wait_bounded(full0 + 8 * stage, phase, abort_flag, status)) {
+          if (!wait_bounded(full0 + 8 * stage, phase, abort_flag, status, limit)) {
             ok = false;
             break;
           }
@@ -1237,7 +1265,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (ok) tc_commit(tfull0 + 8 * acc);
       }
       tc_commit(drain_bar);
-      wait_drain(drain_bar, 0);
+      wait_drain(drain_bar, 0, limit);
     }
   } else {
     // -------------------------------------------------------------- epilogue warps 2..5
@@ -1251,7 +1279,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int acc = it & 1;
       const uint32_t acc_phase = (it >> 1) & 1;
       int ok = 1;
-      if (lane == 0) ok = wait_bounded(tfull0 + 8 * acc, acc_phase, abort_flag, status) ? 1 : 0;
+      if (lane == 0) ok = wait_bounded(tfull0 + 8 * acc, acc_phase, abort_flag, status, limit) ? 1 : 0;
       ok = __shfl_sync(0xffffffffu, ok, 0);
       if (!ok) break;
       tc_fence_after();
@@ -1337,12 +1365,9 @@ int launch_kernel(const Maps& m, const Params& p, int grid, cudaStream_t stream)
   constexpr int STAGE = (SPLIT ? 2 : 1) * BM * BK * 2 + BN * BK * 2;
   constexpr int STAGES = (196608 / STAGE) < 8 ? (196608 / STAGE) : 8;
   constexpr int smem = STAGES * STAGE + 1024 + 256;
-  static bool attr_set = false;
+  static std::atomic<uint64_t> attr_done{0};
   auto kern = gemm_tc_kernel<BN, STAGES, EPI, SPLIT>;
-  if (!attr_set) {
-    VLA_CUDA_TRY(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem));
-    attr_set = true;
-  }
+  VLA_CUDA_TRY(set_smem_limit(kern, smem, attr_done));
   VLA_CUDA_TRY(launch_pdl(kern, dim3(grid), dim3(kThreads), smem, stream, m.a, m.a2, m.b, m.b2, p));
   note_launch();
   VLA_CUDA_TRY(cudaGetLastError());
@@ -1354,12 +1379,9 @@ int launch_pair_kernel(const Maps& m, const Params& p, int grid, cudaStream_t st
   constexpr int STAGE = (SPLIT ? 2 : 1) * BM * BK * 2 + 128 * BK * 2;
   constexpr int STAGES = (196608 / STAGE) < 8 ? (196608 / STAGE) : 8;
   constexpr int smem = STAGES * STAGE + 1024 + 256;
-  static bool attr_set = false;
+  static std::atomic<uint64_t> attr_done{0};
   auto kern = gemm_tc2_kernel<STAGES, EPI, SPLIT>;
-  if (!attr_set) {
-    VLA_CUDA_TRY(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem));
-    attr_set = true;
-  }
+  VLA_CUDA_TRY(set_smem_limit(kern, smem, attr_done));
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(grid);
   cfg.blockDim = dim3(kThreads);
@@ -1374,6 +1396,7 @@ int launch_pair_kernel(const Maps& m, const Params& p, int grid, cudaStream_t st
   attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 2;
+  VLA_CUDA_TRY(injected_launch_error());
   VLA_CUDA_TRY(cudaLaunchKernelEx(&cfg, kern, m.a, m.a2, m.b, m.b2, p));
   note_launch();
   VLA_CUDA_TRY(cudaGetLastError());
@@ -1426,7 +1449,7 @@ int launch_reduce(const Src& src, const GemmArgs& a, cudaStream_t stream) {
     case EPI_SWIGLU:
       VLA_CUDA_TRY(launch_pdl(reduce_swiglu_kernel<Src>, dim3(blocks_for(static_cast<int64_t>(a.M) * a.N / 2)),
                               dim3(256), 0, stream, src, a.M, a.N / 2, a.epi.out_hi, a.epi.out_lo, a.epi.ldo,
-                              a.epi.fp16));
+                              a.epi.fp16, a.epi.status));
       break;
     case EPI_QKV:
       VLA_CUDA_TRY(launch_pdl(reduce_qkv_kernel<Src>, dim3(blocks_for(static_cast<int64_t>(a.M) * a.N / 2)),
@@ -1482,12 +1505,9 @@ int launch_gemv(const CUtensorMap& w, const CUtensorMap& x, const CUtensorMap& x
   constexpr int STAGE = 256 * BK * 2 + 2 * BNX * BK * 2;
   constexpr int STAGES = (196608 / STAGE) < 8 ? (196608 / STAGE) : 8;
   constexpr int smem = STAGES * STAGE + 1024 + 256;
-  static bool attr_set = false;
+  static std::atomic<uint64_t> attr_done{0};
   auto kern = gemv_tc_kernel<BNX, STAGES>;
-  if (!attr_set) {
-    VLA_CUDA_TRY(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem));
-    attr_set = true;
-  }
+  VLA_CUDA_TRY(set_smem_limit(kern, smem, attr_done));
   VLA_CUDA_TRY(launch_pdl(kern, dim3(grid), dim3(kThreads), smem, stream, w, x, x2, p));
   note_launch();
   VLA_CUDA_TRY(cudaGetLastError());
@@ -1495,6 +1515,10 @@ int launch_gemv(const CUtensorMap& w, const CUtensorMap& x, const CUtensorMap& x
 }
 
 }  // namespace
+
+std::atomic<int> g_test_stall{0};
+
+void gemm_stall_next_launch() { g_test_stall.store(1); }
 
 int gemm_effective_splits(int K, int splits) {
   const int kbt = (K + BK - 1) / BK;
@@ -1542,6 +1566,7 @@ int gemm_launch(const GemmArgs& a, cudaStream_t stream, int num_sms, GemmCost* c
   p.kb_total = kbt;
   p.kb_per_split = (kbt + splits - 1) / splits;
   p.epi = a.epi;
+  p.wait_limit = g_wait_limit_ns.load(std::memory_order_relaxed);
 
   Maps maps;
   CUtensorMap &ma = maps.a, &mb = maps.b, &mb2 = maps.b2;
@@ -1585,6 +1610,7 @@ int gemm_launch(const GemmArgs& a, cudaStream_t stream, int num_sms, GemmCost* c
     return VLA_OK;
   }
   const int grid = static_cast<int>(units < num_sms ? units : num_sms);
+  p.stall = g_test_stall.exchange(0);  // failure injection: consumed by one tile-GEMM launch
   if (split)
     rc = (BN == 256) ? dispatch_epi<256, true>(run_epi, maps, p, grid, stream)
                      : dispatch_epi<128, true>(run_epi, maps, p, grid, stream);
@@ -1640,6 +1666,7 @@ int gemv_launch(const GemmArgs& a, cudaStream_t stream, int num_sms, GemmCost* c
   p.ws = a.workspace;
   p.status = a.epi.status;
   p.fp16 = fp16;
+  p.wait_limit = g_wait_limit_ns.load(std::memory_order_relaxed);
   int rc;
   switch (pl.bnx) {
     case 16: rc = launch_gemv<16>(mw, mx, mx2, p, pl.grid, stream); break;
@@ -1658,7 +1685,7 @@ int gemv_launch(const GemmArgs& a, cudaStream_t stream, int num_sms, GemmCost* c
       if (resid && a.epi.norm_w) {
         VLA_CUDA_TRY(launch_pdl(stream_reduce_resid_norm_kernel, dim3(a.M), dim3(1024), 0, stream, src, a.N,
                                 a.epi.resid, a.epi.ldr, a.epi.norm_w, a.epi.norm_eps, a.epi.norm_hi,
-                                a.epi.norm_lo, a.epi.ldn, fp16));
+                                a.epi.norm_lo, a.epi.ldn, fp16, a.epi.status));
         break;
       }
       VLA_CUDA_TRY(launch_pdl(stream_reduce_f32_kernel, grid_for((a.N + 255) / 256), dim3(256), 0, stream, src,
@@ -1668,7 +1695,8 @@ int gemv_launch(const GemmArgs& a, cudaStream_t stream, int num_sms, GemmCost* c
     }
     case EPI_SWIGLU:
       VLA_CUDA_TRY(launch_pdl(stream_reduce_swiglu_kernel, grid_for((a.N / 2 + 255) / 256), dim3(256), 0,
-                              stream, src, a.M, a.N / 2, a.epi.out_hi, a.epi.out_lo, a.epi.ldo, fp16));
+                              stream, src, a.M, a.N / 2, a.epi.out_hi, a.epi.out_lo, a.epi.ldo, fp16,
+                              a.epi.status));
       break;
     case EPI_QKV:
       if (256 % a.epi.hd == 0 && a.epi.d % 256 == 0) {
@@ -1761,8 +1789,9 @@ extern "C" int vla_op_gemm_bf16_noalloc(const void* A, const void* A_lo, int lda
     if (rc != VLA_OK) return rc;
     g.workspace_bytes = kNoAllocScratchFloats * sizeof(float);
   }
+  if (const int rs = op_status_word(&g.epi.status)) return rs;
   int dev = 0;
-  cudaGetDevice(&dev);
+  VLA_CUDA_TRY(cudaGetDevice(&dev));
   int n_sms = 0;
   if (cudaDeviceGetAttribute(&n_sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n_sms <= 0)
     n_sms = 148;

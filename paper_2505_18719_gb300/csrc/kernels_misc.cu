@@ -8,6 +8,9 @@
 namespace vla {
 
 int64_t g_launch_count = 0;
+std::atomic<int64_t> g_inject_countdown{0};
+std::atomic<int> g_inject_error{0};
+std::atomic<uint64_t> g_wait_limit_ns{kDefaultWaitLimitNs};
 
 namespace {
 
@@ -42,14 +45,15 @@ __global__ void __launch_bounds__(256) assemble_kernel(const RowInfo* __restrict
   }
 }
 
-__global__ void __launch_bounds__(256) rmsnorm_kernel(const float* __restrict__ h,
+__global__ void __launch_bounds__(256) rmsnorm_kernel(const float* __restrict__ h, int ldh,
                                                       const bf16* __restrict__ w, int d,
                                                       float eps, bf16* __restrict__ y_hi,
-                                                      bf16* __restrict__ y_lo, bool fp16) {
+                                                      bf16* __restrict__ y_lo, bool fp16,
+                                                      uint32_t* status) {
   pdl_launch_dependents();
   pdl_wait();
   __shared__ float red[8];
-  const float* row = h + static_cast<size_t>(blockIdx.x) * d;
+  const float* row = h + static_cast<size_t>(blockIdx.x) * ldh;
   float ss = 0.f;
   for (int c = threadIdx.x * 4; c < d; c += blockDim.x * 4) {
     const float4 v = *reinterpret_cast<const float4*>(row + c);
@@ -62,16 +66,18 @@ __global__ void __launch_bounds__(256) rmsnorm_kernel(const float* __restrict__ 
   for (int i = 0; i < (blockDim.x >> 5); ++i) tot += red[i];
   const float r = rsqrtf(tot / static_cast<float>(d) + eps);
   const size_t off = static_cast<size_t>(blockIdx.x) * d;
+  uint32_t sat = 0;
   for (int c = threadIdx.x * 4; c < d; c += blockDim.x * 4) {
     const float4 v = *reinterpret_cast<const float4*>(row + c);
     const uint2 ww = *reinterpret_cast<const uint2*>(w + c);
     const float2 w0 = unpack_bf16x2(ww.x), w1 = unpack_bf16x2(ww.y);
     uint2 hi, lo;
-    split_pack2(v.x * r * w0.x, v.y * r * w0.y, hi.x, lo.x, fp16);
-    split_pack2(v.z * r * w1.x, v.w * r * w1.y, hi.y, lo.y, fp16);
+    split_pack2(v.x * r * w0.x, v.y * r * w0.y, hi.x, lo.x, fp16, sat);
+    split_pack2(v.z * r * w1.x, v.w * r * w1.y, hi.y, lo.y, fp16, sat);
     *reinterpret_cast<uint2*>(y_hi + off + c) = hi;
     *reinterpret_cast<uint2*>(y_lo + off + c) = lo;
   }
+  report_saturation(status, sat);
 }
 
 __global__ void gather_rows_kernel(const float* __restrict__ src, const int* __restrict__ idx,
@@ -107,10 +113,11 @@ int assemble_launch(const RowInfo* rows, int n_rows, const bf16* visual, const i
   return VLA_OK;
 }
 
-int rmsnorm_launch(const float* h, const bf16* w, int M, int d, float eps, bf16* y_hi,
-                   bf16* y_lo, cudaStream_t s, bool fp16) {
+int rmsnorm_launch(const float* h, int ldh, const bf16* w, int M, int d, float eps, bf16* y_hi,
+                   bf16* y_lo, cudaStream_t s, bool fp16, uint32_t* status) {
   if (M <= 0) return VLA_OK;
-  VLA_CUDA_TRY(launch_pdl(rmsnorm_kernel, dim3(M), dim3(256), 0, s, h, w, d, eps, y_hi, y_lo, fp16));
+  VLA_CUDA_TRY(launch_pdl(rmsnorm_kernel, dim3(M), dim3(256), 0, s, h, ldh, w, d, eps, y_hi, y_lo, fp16,
+                          status));
   note_launch();
   VLA_CUDA_TRY(cudaGetLastError());
   return VLA_OK;
@@ -169,6 +176,7 @@ int bf16_to_f16_launch(const bf16* src, f16* dst, size_t n, int* out_of_range, i
   const size_t n8 = n / 8;
   const size_t want = (n8 + 255) / 256;
   const int grid = static_cast<int>(want < static_cast<size_t>(num_sms) * 8 ? want : static_cast<size_t>(num_sms) * 8);
+  VLA_CUDA_TRY(injected_launch_error());
   bf16_to_f16_kernel<<<grid, 256, 0, s>>>(src, dst, n8, out_of_range);
   note_launch();
   VLA_CUDA_TRY(cudaGetLastError());

@@ -10,10 +10,11 @@ int assemble_launch(const RowInfo* rows, int n_rows, const bf16* visual, const i
                     const int* tokens, const bf16* embed, int d, int vocab, float* h,
                     uint32_t* status, cudaStream_t s);
 
-// y[m] = h[m] / sqrt(mean(h[m]^2) + eps) * w, h f32 [M, d], written as the operand pair
-// (y_hi, y_lo) [M, d] with y_hi + y_lo ~ y, fp16 if `fp16` else bf16.
-int rmsnorm_launch(const float* h, const bf16* w, int M, int d, float eps, bf16* y_hi,
-                   bf16* y_lo, cudaStream_t s, bool fp16);
+// y[m] = h[m] / sqrt(mean(h[m]^2) + eps) * w, h f32 [M, d] (row stride ldh), written as the
+// operand pair (y_hi, y_lo) [M, d] with y_hi + y_lo ~ y, fp16 if `fp16` else bf16; a finite
+// value beyond the fp16 range is stored as +-65504 and sets VLA_STATUS_SATURATED in *status.
+int rmsnorm_launch(const float* h, int ldh, const bf16* w, int M, int d, float eps, bf16* y_hi,
+                   bf16* y_lo, cudaStream_t s, bool fp16, uint32_t* status);
 
 // dst[i] = fp16(src[i]) for n bf16 values (n % 8 == 0, both 16-byte aligned).  A value outside
 // the finite fp16 range (|x| > 65504, or not finite) is clamped to +-65504 and sets

@@ -5,8 +5,6 @@
 
 namespace vla {
 
-constexpr uint64_t kWaitLimitNs = 1000000000ull;  // 1 s per mbarrier wait
-
 // ----------------------------------------------------------------------------- PTX helpers
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
@@ -160,9 +158,10 @@ __device__ __forceinline__ void bulk_load(uint32_t dst, const void* src, uint32_
       : "memory");
 }
 
-// Bounded wait.  Returns false when this CTA is aborting (timeout here or elsewhere).
+// Bounded wait (limit_ns per wait: the launch's copy of g_wait_limit_ns, 1 s by default).
+// Returns false when this CTA is aborting (timeout here or elsewhere in the CTA).
 __device__ __forceinline__ bool wait_bounded(uint32_t bar, uint32_t parity, volatile int* abort_flag,
-                                             uint32_t* status) {
+                                             uint32_t* status, uint64_t limit_ns) {
   if (mbar_try_wait(bar, parity)) return true;
   const uint64_t t0 = globaltimer();
   uint32_t n = 0;
@@ -170,7 +169,7 @@ __device__ __forceinline__ bool wait_bounded(uint32_t bar, uint32_t parity, vola
     if (mbar_try_wait(bar, parity)) return true;
     if (((++n) & 63u) == 0) {
       if (*abort_flag) return false;
-      if (globaltimer() - t0 > kWaitLimitNs) {
+      if (globaltimer() - t0 > limit_ns) {
         *abort_flag = 1;
         if (status) atomicOr(status, VLA_STATUS_TIMEOUT);
         return false;
@@ -179,10 +178,10 @@ __device__ __forceinline__ bool wait_bounded(uint32_t bar, uint32_t parity, vola
   }
 }
 // Wait used while draining: ignores the abort flag, bounded by time only.
-__device__ __forceinline__ void wait_drain(uint32_t bar, uint32_t parity) {
+__device__ __forceinline__ void wait_drain(uint32_t bar, uint32_t parity, uint64_t limit_ns) {
   const uint64_t t0 = globaltimer();
   while (!mbar_try_wait(bar, parity)) {
-    if (globaltimer() - t0 > kWaitLimitNs) return;
+    if (globaltimer() - t0 > limit_ns) return;
   }
 }
 

@@ -29,6 +29,7 @@ VLA_STATUS_BAD_TOKEN = 0x1
 VLA_STATUS_NONFINITE = 0x2
 VLA_STATUS_TIMEOUT = 0x4
 VLA_STATUS_BAD_FORCED = 0x8
+VLA_STATUS_SATURATED = 0x10
 
 KCLASS = ("gemm_prefill", "gemm_decode", "attn_prefill", "attn_decode", "head", "other")
 
@@ -101,6 +102,11 @@ def load(path: str = LIB_PATH):
         "vla_op_attn_decode": (i32, [vp, vp, i32, i32, i32, i32, vp, vp, i32, i32, i32, vp, vp, vp, ctypes.c_size_t, vp]),
         "vla_op_attn_decode_workspace_bytes": (ctypes.c_size_t, [i32, i32, i32, i32, i32]),
         "vla_op_attn_chunk": (i32, [vp, vp, i32, i32, i32, i32, vp, i32, i32, vp, vp, vp, vp]),
+        "vla_op_rmsnorm": (i32, [vp, i32, i32, i32, vp, f32, vp, vp, i32, vp]),
+        "vla_op_read_status": (i32, [vp, ctypes.POINTER(u32)]),
+        "vla_test_inject_launch_error": (i32, [i64, i32]),
+        "vla_test_set_wait_limit_ns": (i32, [ctypes.c_uint64]),
+        "vla_test_stall_next_gemm": (i32, []),
     }
     for name, (res, args) in sig.items():
         f = getattr(lib, name)
@@ -284,6 +290,30 @@ def vla_op_attn_decode(q_ptr, kv_ptr, max_env, H, hd, cap, env_ptr, pos_ptr, B, 
 
 def vla_op_attn_decode_workspace_bytes(B, H, hd, max_ctx, max_keys_per_cta=0) -> int:
     return load().vla_op_attn_decode_workspace_bytes(B, H, hd, max_ctx, max_keys_per_cta)
+
+
+def vla_op_rmsnorm(h_ptr, ldh, M, d, w_ptr, eps, y_hi_ptr, y_lo_ptr, fp16=True, stream=0) -> int:
+    return load().vla_op_rmsnorm(h_ptr or None, ldh, M, d, w_ptr or None, float(eps), y_hi_ptr or None,
+                                 y_lo_ptr or None, 1 if fp16 else 0, stream or None)
+
+
+def vla_op_read_status(stream=0):
+    """(rc, status bits) of the op entry points on the current device; clears the word."""
+    st = ctypes.c_uint32(0)
+    rc = load().vla_op_read_status(stream or None, ctypes.byref(st))
+    return rc, st.value
+
+
+def vla_test_inject_launch_error(nth_launch: int, cuda_error: int) -> int:
+    return load().vla_test_inject_launch_error(int(nth_launch), int(cuda_error))
+
+
+def vla_test_set_wait_limit_ns(limit_ns: int) -> int:
+    return load().vla_test_set_wait_limit_ns(int(limit_ns))
+
+
+def vla_test_stall_next_gemm() -> int:
+    return load().vla_test_stall_next_gemm()
 
 
 # ---------------------------------------------------------------------------- convenience

@@ -18,6 +18,7 @@ import torch
 
 import oracle.vla_oracle as O
 from paper_2505_18719_gb300 import inputs as I
+from tests import attribution as A
 from paper_2505_18719_gb300 import vla as V
 
 TOL = 2e-2
@@ -75,8 +76,8 @@ def run_parity(wl: I.Workload, weights_cpu=None, weights_dev=None, n_check: Opti
     max_tokens = wl.batch * (wl.n_visual + (wl.text_len or wl.text_len_range[1]) + 8)
     pol = V.Policy(sh, weights_dev, wl.batch, wl.kv_capacity, max_tokens)
     orc = O.Oracle(O.shape_from(sh), weights_cpu, wl.batch, cache_f64=cache_f64)
-    emu = O.Oracle(O.shape_from(sh), weights_cpu, wl.batch, cache_f64=cache_f64,
-                   rounding=O.GPU_PATH) if attribution else None
+    emu = A.AttributionOracle(O.shape_from(sh), weights_cpu, wl.batch, cache_f64=cache_f64,
+                              rounding=A.GPU_PATH) if attribution else None
     base = sh.vocab - sh.n_bins
     reports = []
     envs = None

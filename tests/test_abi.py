@@ -63,3 +63,11 @@ def test_host_argument_errors_without_gpu(lib):
     assert "vla_op_gemm_decode_f16" in V.vla_last_error(None)
     assert lib.vla_op_action_head(None, 0, 0, 0, None, None, 1e-6, None, 1.0, None, None, None, None,
                                   None, None, None) == V.VLA_ERR_ARG
+    assert lib.vla_op_rmsnorm(None, 0, 0, 0, None, 1e-6, None, None, 1, None) == V.VLA_ERR_ARG
+    assert "vla_op_rmsnorm" in V.vla_last_error(None)
+    assert lib.vla_op_read_status(None, None) == V.VLA_ERR_ARG
+    # failure-injection hooks: argument checks, and arming / disarming touch no device
+    assert lib.vla_test_inject_launch_error(-1, 701) == V.VLA_ERR_ARG
+    assert lib.vla_test_inject_launch_error(3, 0) == V.VLA_ERR_ARG
+    assert lib.vla_test_inject_launch_error(0, 0) == V.VLA_OK
+    assert lib.vla_test_set_wait_limit_ns(0) == V.VLA_OK

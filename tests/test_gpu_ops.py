@@ -288,3 +288,26 @@ def test_decode_gemm_f16_matches_fp64(M, N, K):
     torch.cuda.synchronize()
     err = (C.cpu().double() - (A.double() + A_lo.double()) @ W.double().T).abs().max().item()
     assert err < 2e-5 * math.sqrt(K) * 8, err
+
+
+# ------------------------------------------------------------------ RMSNorm (operand-pair output)
+@pytest.mark.parametrize("fp16", [True, False])
+def test_rmsnorm_matches_fp64(fp16):
+    M, d, ldh = 37, 4096, 4100
+    h = I.normal_bf16((M, ldh), 95, 1, 3.0).float()
+    w = I.normal_bf16((d,), 95, 2, 1.0, mean=1.0)
+    hd_, wd = h.cuda(), w.cuda()
+    dt = torch.float16 if fp16 else torch.bfloat16
+    yh = torch.empty(M, d, dtype=dt, device="cuda")
+    yl = torch.empty_like(yh)
+    assert V.vla_op_rmsnorm(hd_.data_ptr(), ldh, M, d, wd.data_ptr(), 1e-6, yh.data_ptr(), yl.data_ptr(),
+                            fp16) == 0, V.vla_last_error()
+    assert V.vla_op_read_status() == (0, 0)
+    x = h[:, :d].double()
+    ref = O.rms_norm(x, w.double(), 1e-6)
+    got = yh.cpu().double() + yl.cpu().double()
+    # the pair keeps ~21 (fp16) / ~16 (bf16) significant bits; fp32 math before the split
+    rel = (got - ref).abs().max().item() / ref.abs().max().item()
+    assert rel < (2e-6 if fp16 else 2e-5), rel
+    # hi alone is the round-to-nearest of the value in that format
+    assert (yh.cpu().double() - ref).abs().max().item() <= ref.abs().max().item() * (2.0 ** -11 if fp16 else 2.0 ** -8)
