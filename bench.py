@@ -223,6 +223,7 @@ CASES = {
     "gemm_decode_o": (64, 4096, 4096, 128, 5, True),
     # weight-streaming decode GEMM (swap-AB, stream-K): block_n / splits unused
     "gemv_decode_qkv": (64, 12288, 4096, 0, 0, True),
+    "gemv_decode_o": (64, 4096, 4096, 0, 0, True),
     "gemv_decode_gate_up": (64, 22016, 4096, 0, 0, True),
     "gemv_decode_down": (64, 4096, 11008, 0, 0, True),
     "attn_decode": None,                                       # see run_attn_case

@@ -23,7 +23,10 @@
  *    Its input activation is carried as an fp16 pair hi + lo (~21 significant bits); the
  *    weight-streaming GEMMs (calls of at most 128 rows: decode steps of up to 128 envs)
  *    multiply both halves, the tile GEMMs (prefill, score, larger decode batches) both halves
- *    for q|k|v, o and down and hi alone for gate|up.  K/V are cached in fp16.  A finite
+ *    for q|k|v and hi alone for o, gate|up and down.  K/V are cached in fp16 plus a 4-bit
+ *    residual per element (value = hi + (2c - 15) ulp(hi) / 32, within ulp(hi) / 32 of the
+ *    computed key / value); the chunk attention of prefill and score reads both, the decode
+ *    attention the fp16 part.  A finite
  *    activation beyond the fp16 range (|x| > 65504) is stored as +-65504 and raises
  *    VLA_STATUS_SATURATED in the status word (reported by the next vla_sync).
  *  - Calls are asynchronous on the handle's stream.  Host-checkable errors return at once,
@@ -95,7 +98,8 @@ typedef struct {
 
 /* Create a handle on the current CUDA device.  `cuda_stream` is a cudaStream_t (NULL =
  * the legacy default stream).  Allocates the KV cache
- * (n_layers * max_batch * 2 * d_model * kv_capacity fp16), the fp16 copy of the projection
+ * (n_layers * max_batch * 2 * d_model * kv_capacity fp16, and half a byte per element for its
+ * residual codes), the fp16 copy of the projection
  * matrices (n_layers * (4 d^2 + 3 d_ffn d) fp16) and workspaces, then fills the copy from the
  * bf16 weights and waits for it.  A bf16 weight with 2^-14 <= |w| <= 65504 is exact in
  * fp16; a smaller one rounds to a multiple of 2^-24.

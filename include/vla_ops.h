@@ -141,6 +141,22 @@ int vla_op_attn_chunk(const float* q, const void* kv, int max_env, int H, int hd
                       const int32_t* tiles_host, int n_tiles, int rows, int32_t* tiles_dev,
                       void* out_hi, void* out_lo, void* cuda_stream);
 
+/* The engine's chunk attention (§3.1 self-attention over the env's whole multi-turn context,
+ * §3.3; the prefill chunks and the PPO ratio pass of Eq. 2) on the tcgen05 tensor cores, with
+ * the cache read at its full stored precision:
+ *   q, tiles_host, tiles_dev, rows, out_hi / out_lo as vla_op_attn_chunk, but tiles of up to 128
+ *   rows (1 <= nrows <= 128);
+ *   kv       fp16 cache [env][K,V][H][cap][hd] (one layer, max_env envs), 16-byte aligned;
+ *   kv_res   its 4-bit residual codes, one byte per element pair of the same layout (element 2i
+ *            in the low nibble of byte i), 16-byte aligned: code c of value x with fp16 part
+ *            hi = fp16(x) is c = 8 + clamp(floor((x - hi) / ulp(hi) * 16), -8, 7), and the value
+ *            read is hi + (2c - 15) ulp(hi) / 32, ulp(hi) = 2^(e-25) for hi's biased exponent
+ *            e >= 1, 2^-24 for e = 0.
+ * A pipeline wait that runs out sets VLA_STATUS_TIMEOUT in the op status word.  hd in {64, 128}. */
+int vla_op_attn_chunk_res(const float* q, const void* kv, const void* kv_res, int max_env, int H, int hd,
+                          int cap, const int32_t* tiles_host, int n_tiles, int rows, int32_t* tiles_dev,
+                          void* out_hi, void* out_lo, void* cuda_stream);
+
 /* Number of SMs the kernels size their persistent grids for (device property). */
 int vla_op_num_sms(void);
 

@@ -29,15 +29,46 @@ struct RowInfo {
   int env, pos, kind, idx;
 };
 
-// KV cache geometry: [layer][env][2 (K,V)][H][cap][hd] fp16.
+// KV cache geometry: [layer][env][2 (K,V)][H][cap][hd] fp16, plus a residual plane of the same
+// geometry with one 4-bit code per element (two per byte: element 2i in the low nibble of byte
+// i, 2i+1 in the high nibble), so element offset o has its code in byte o / 2 of `res`.
 struct KVLayout {
   f16* base;          // whole cache
+  uint8_t* res;       // residual codes (null: not written)
   int64_t layer_stride;
   int64_t env_stride;  // 2 * H * cap * hd
   int64_t kv_stride;   // H * cap * hd (V follows K)
   int64_t head_stride; // cap * hd
   int cap;
 };
+
+// 4-bit residual of a cached key / value x around hi = fp16(x): the code c in [0, 15] names the
+// cell [(c - 8) / 16, (c - 7) / 16) of (x - hi) / ulp(hi) (clamped at both ends), and the value
+// read back is hi + (2c - 15) ulp(hi) / 32, the cell's midpoint, within ulp(hi) / 32 of x: four
+// bits past fp16's eleven.  ulp(hi) = 2^(e - 25) for the biased exponent e >= 1, 2^-24 for e = 0.
+// x - hi is exact in fp32 and the scaling is by a power of two, so the code is exact.
+__device__ __forceinline__ uint32_t kv_res_code(float x, f16 hi) {
+  const uint32_t e = (__half_as_ushort(hi) >> 10) & 31u;
+  const uint32_t ee = e ? e : 1u;
+  const float scale = __uint_as_float((156u - ee) << 23);  // 16 / ulp(hi) = 2^(29 - ee)
+  float j = floorf((x - __half2float(hi)) * scale);
+  j = fminf(fmaxf(j, -8.f), 7.f);  // a NaN lands on -8: its value is NaN through hi anyway
+  return static_cast<uint32_t>(static_cast<int>(j) + 8);
+}
+__device__ __forceinline__ float kv_res_value(f16 hi, uint32_t c) {
+  const uint32_t e = (__half_as_ushort(hi) >> 10) & 31u;
+  const uint32_t ee = e ? e : 1u;
+  return __half2float(hi) + static_cast<float>(2 * static_cast<int>(c) - 15) * __uint_as_float((ee + 97u) << 23);
+}
+// Residual value alone, (2c - 15) ulp(hi) / 32, rounded to fp16 (the MMA operand of the low part).
+__device__ __forceinline__ f16 kv_res_lo(f16 hi, uint32_t c) {
+  const uint32_t e = (__half_as_ushort(hi) >> 10) & 31u;
+  const uint32_t ee = e ? e : 1u;
+  return __float2half_rn(static_cast<float>(2 * static_cast<int>(c) - 15) * __uint_as_float((ee + 97u) << 23));
+}
+// Stores x as fp16 at dst[i] and its code into the residual plane (for an even/odd pair, the
+// caller combines two codes into one byte).
+__device__ __forceinline__ f16 kv_hi(float x) { return __float2half_rn(x); }
 
 // ----------------------------------------------------------------------------- bf16 helpers
 __device__ __forceinline__ float bf2f(bf16 x) { return __bfloat162float(x); }

@@ -135,6 +135,7 @@ struct vla_handle {
   const bf16* head_rows = nullptr;
   // owned device memory
   f16* kv = nullptr;      // KV cache [L][B][2][H][cap][hd] fp16
+  uint8_t* kv_res = nullptr;  // its 4-bit residual codes, two per byte (KVLayout)
   KVLayout kvl{};
   float* h = nullptr;    // residual stream f32 [T, d]
   bf16* y = nullptr;     // RMSNorm output, operand pair: hi [T, d] then lo [T, d]
@@ -243,13 +244,14 @@ void prof_harvest(vla_handle* h) {
 }
 
 // Projections whose tile GEMMs (M > 128 rows: prefill, score, decode of more than 128 envs)
-// also multiply the low half of the activation pair.  An fp16 activation alone is within 2^-11
-// relative of its value.  gate|up, 45 % of the projection work, takes hi alone: its rounding
-// adds ~0.01 to the 7B action-bin logits, next to the ~0.012 the fp16 KV cache already costs.
+// also multiply the low half of the activation pair: q|k|v alone.  An fp16 activation alone is
+// within 2^-11 relative of its value; with the KV cache carrying a 4-bit residual (read in full
+// by the chunk attention), o, gate|up and down on hi alone keep the 7B action-bin logits closer
+// to the exact model than all-but-gate|up pairs over a plain fp16 cache did.
 // The weight-streaming GEMMs (M <= 128) always take both halves: they are bound by reading the
 // weights, so the second MMA costs nothing there.
 enum : unsigned { kProjQkv = 1, kProjO = 2, kProjGateUp = 4, kProjDown = 8 };
-constexpr unsigned kTileLoMask = kProjQkv | kProjO | kProjDown;
+constexpr unsigned kTileLoMask = kProjQkv;
 
 // A is the operand pair: hi at A, lo at A + a_plane (fp16 when h->fp16, else bf16).
 // The GEMM that will consume h->y after a residual GEMM's RMSNorm (its N, K and epilogue).
@@ -404,7 +406,8 @@ int forward_layers(vla_handle* h, int M, const RowInfo* rows_dev, bool decode, i
       prof_end(h, ev, VLA_KCLASS_ATTN_DECODE, 0, 0);
     } else {
       ev = prof_begin(h, VLA_KCLASS_ATTN_PREFILL);
-      rc = attn_chunk_launch(h->q, h->ao, h->ao + pd, h->tiles, n_tiles, h->kvl, l, H, hd, h->stream, h->fp16);
+      rc = attn_chunk_tc_launch(h->q, h->ao, h->ao + pd, h->tiles, n_tiles, h->kvl, l, H, hd, h->status, h->stream,
+                                h->fp16);
       prof_end(h, ev, VLA_KCLASS_ATTN_PREFILL, 0, 0);
     }
     if (rc) return fail(h, rc, t_err);
@@ -574,6 +577,7 @@ int vla_create(const vla_config* cfg, const vla_weights* w, void* cuda_stream, v
     return cudaMalloc(p, bytes) == cudaSuccess;
   };
   bool ok = alloc(reinterpret_cast<void**>(&h->kv), static_cast<size_t>(L) * h->kvl.layer_stride * sizeof(f16)) &&
+            alloc(reinterpret_cast<void**>(&h->kv_res), static_cast<size_t>(L) * h->kvl.layer_stride / 2) &&
             alloc(reinterpret_cast<void**>(&h->h), T * d * sizeof(float)) &&
             alloc(reinterpret_cast<void**>(&h->y), 2 * T * d * sizeof(bf16)) &&
             alloc(reinterpret_cast<void**>(&h->q), T * d * sizeof(float)) &&
@@ -607,6 +611,7 @@ int vla_create(const vla_config* cfg, const vla_weights* w, void* cuda_stream, v
     return set_err(nullptr, VLA_ERR_OOM, "vla_create: device allocation failed");
   }
   h->kvl.base = h->kv;
+  h->kvl.res = h->kv_res;
   {
     const size_t dd = static_cast<size_t>(d) * d, fd = static_cast<size_t>(F) * d;
     f16* p = h->w16;
@@ -698,8 +703,8 @@ int vla_prefill(vla_handle* h, int batch, const void* visual, int n_visual, cons
     if (h->has_pending[b]) rows[r++] = RowInfo{b, pos++, ROW_TOKEN, b};
     for (int j = 0; j < n_visual; ++j) rows[r++] = RowInfo{b, pos++, ROW_VISUAL, b * n_visual + j};
     for (int j = 0; j < lengths[b]; ++j) rows[r++] = RowInfo{b, pos++, ROW_TEXT, b * max_len + j};
-    for (int t0 = 0; t0 < chunk[b]; t0 += 64)
-      tiles[n_tiles++] = AttnTile{b, r0 + t0, std::min(64, chunk[b] - t0), h->len[b] + t0};
+    for (int t0 = 0; t0 < chunk[b]; t0 += 128)
+      tiles[n_tiles++] = AttnTile{b, r0 + t0, std::min(128, chunk[b] - t0), h->len[b] + t0};
     last[b] = r - 1;
   }
   int* sidx = reinterpret_cast<int*>(tiles + n_tiles);
@@ -1012,7 +1017,7 @@ void vla_destroy(vla_handle* h) {
   if (!h) return;
   DeviceGuard dev_guard(h->dev);  // best effort: the handle is freed whatever happens
   cudaStreamSynchronize(h->stream);
-  void* bufs[] = {h->kv, h->h, h->y, h->q, h->ao, h->u, h->ws, h->h_last, h->head_in, h->head_z, h->head_entropy, h->q_last, h->ss_part, h->last_rows, h->rope,
+  void* bufs[] = {h->kv, h->kv_res, h->h, h->y, h->q, h->ao, h->u, h->ws, h->h_last, h->head_in, h->head_z, h->head_entropy, h->q_last, h->ss_part, h->last_rows, h->rope,
                   h->rows, h->tiles, h->sidx, h->didx, h->fed, h->pending, h->status, h->part_o,
                   h->part_ml, h->attn_tickets, h->w16, h->w16_range};
   for (void* p : bufs)
@@ -1298,6 +1303,40 @@ int vla_op_attn_chunk(const float* q, const void* kv, int max_env, int H, int hd
   const int rc = attn_chunk_launch(q, static_cast<bf16*>(out_hi), static_cast<bf16*>(out_lo),
                                    reinterpret_cast<const AttnTile*>(tiles_dev), n_tiles, L, 0, H, hd, st, false);
   if (rc != VLA_OK && rc != VLA_ERR_CUDA) return set_err(nullptr, rc, "vla_op_attn_chunk: unsupported arguments");
+  return rc;
+}
+
+int vla_op_attn_chunk_res(const float* q, const void* kv, const void* kv_res, int max_env, int H, int hd, int cap,
+                          const int32_t* tiles_host, int n_tiles, int rows, int32_t* tiles_dev, void* out_hi,
+                          void* out_lo, void* cuda_stream) {
+  if (!q || !kv || !kv_res || !tiles_host || !tiles_dev || !out_hi || !out_lo || max_env < 1 || H < 1 || cap < 1 ||
+      n_tiles < 1 || rows < 1 || (hd != 64 && hd != 128))
+    return set_err(nullptr, VLA_ERR_ARG, "vla_op_attn_chunk_res: bad argument");
+  for (int i = 0; i < n_tiles; ++i) {
+    const int32_t* t = tiles_host + 4 * i;
+    if (t[0] < 0 || t[0] >= max_env || t[2] < 1 || t[2] > 128 || t[3] < 0 || t[3] + t[2] > cap || t[1] < 0 ||
+        t[1] + t[2] > rows)
+      return set_err(nullptr, VLA_ERR_ARG, "vla_op_attn_chunk_res: tile outside the buffers");
+  }
+  uint32_t* status = nullptr;
+  if (const int rs = op_status_word(&status)) return rs;
+  cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
+  if (cudaMemcpyAsync(tiles_dev, tiles_host, static_cast<size_t>(n_tiles) * 4 * sizeof(int32_t),
+                      cudaMemcpyHostToDevice, st) != cudaSuccess)
+    return cuda_fail(cudaGetLastError(), "vla_op_attn_chunk_res: tile copy");
+  KVLayout L{};
+  L.base = static_cast<f16*>(const_cast<void*>(kv));
+  L.res = static_cast<uint8_t*>(const_cast<void*>(kv_res));
+  L.cap = cap;
+  L.head_stride = static_cast<int64_t>(cap) * hd;
+  L.kv_stride = static_cast<int64_t>(H) * L.head_stride;
+  L.env_stride = 2 * L.kv_stride;
+  L.layer_stride = static_cast<int64_t>(max_env) * L.env_stride;
+  const int rc = attn_chunk_tc_launch(q, static_cast<bf16*>(out_hi), static_cast<bf16*>(out_lo),
+                                      reinterpret_cast<const AttnTile*>(tiles_dev), n_tiles, L, 0, H, hd, status, st,
+                                      false);
+  if (rc != VLA_OK && rc != VLA_ERR_CUDA)
+    return set_err(nullptr, rc, "vla_op_attn_chunk_res: unsupported arguments or misaligned buffers");
   return rc;
 }
 

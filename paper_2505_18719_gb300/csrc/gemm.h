@@ -88,6 +88,11 @@ int gemm_launch(const GemmArgs& a, cudaStream_t stream, int num_sms, GemmCost* c
 // (EPI_RESID with norm_w set: fused with the following RMSNorm).
 size_t gemv_workspace_bytes(int M, int N, int K, int num_sms);
 
+// 2-D tensor map of 2-byte elements (bf16, or fp16 when fp16) over [rows, cols] (row stride ld
+// elements), box {64, box_rows}, 128-byte swizzle.
+bool make_tensor_map_2d(CUtensorMap* m, const void* ptr, int64_t rows, int64_t cols, int64_t ld, int box_rows,
+                        bool fp16);
+
 // Failure injection (test hook): in the next single-CTA tile GEMM launch, CTA 0 leaves its first
 // pipeline stage unfilled; its bounded wait on that stage runs out (VLA_STATUS_TIMEOUT).
 void gemm_stall_next_launch();

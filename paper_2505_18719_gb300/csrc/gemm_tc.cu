@@ -113,6 +113,25 @@ __device__ __forceinline__ void store_f16x16(f16* dst, const float (&v)[16]) {
   reinterpret_cast<uint4*>(dst)[0] = a;
   reinterpret_cast<uint4*>(dst)[1] = b;
 }
+// 16 values as fp16 at dst and their 4-bit residual codes (8 bytes) at res, when res is set.
+__device__ __forceinline__ void store_kv16(f16* dst, uint8_t* res, const float (&v)[16]) {
+  store_f16x16(dst, v);
+  if (!res) return;
+  uint32_t w[2] = {0u, 0u};
+#pragma unroll
+  for (int i = 0; i < 16; ++i) w[i >> 3] |= kv_res_code(v[i], __float2half_rn(v[i])) << (4 * (i & 7));
+  *reinterpret_cast<uint2*>(res) = make_uint2(w[0], w[1]);
+}
+// Stores the fp16 value of x at dst[i] and, when res is set, the residual byte of the element
+// pair (i, i + 1) at res[i / 2]: lane l holds element i and lane l + 1 element i + 1 (i even on
+// even lanes); every lane of the warp must call this together.
+__device__ __forceinline__ void store_kv_pairlanes(f16* dst, uint8_t* res, int i, float x) {
+  const f16 h = __float2half_rn(x);
+  dst[i] = h;
+  const uint32_t c = res ? kv_res_code(x, h) : 0u;
+  const uint32_t c_next = __shfl_down_sync(0xffffffffu, c, 1);
+  if (res && (i & 1) == 0) res[i >> 1] = static_cast<uint8_t>(c | (c_next << 4));
+}
 __device__ __forceinline__ void store_f32x16(float* dst, const float (&v)[16]) {
 #pragma unroll
   for (int i = 0; i < 4; ++i)
@@ -277,13 +296,14 @@ __device__ __forceinline__ void epilogue_qkv(const Params& p, uint32_t trow, int
     const uint32_t tcol = trow + hh * hd;
     if (sec == 2) {
       f16* dst = row_ok ? kv_row + static_cast<int64_t>(head) * kv.head_stride : nullptr;
+      uint8_t* rdst = (row_ok && kv.res) ? kv.res + (dst - kv.base) / 2 : nullptr;
 #pragma unroll 1
       for (int j = 0; j < hd; j += 16) {
         float v[16];
         ld16f(tcol + j, v);
 #pragma unroll
         for (int i = 0; i < 16; ++i) v[i] *= rs;
-        if (row_ok) store_f16x16(dst + j, v);
+        if (row_ok) store_kv16(dst + j, rdst ? rdst + j / 2 : nullptr, v);
       }
     } else {
 #pragma unroll 1
@@ -307,8 +327,9 @@ __device__ __forceinline__ void epilogue_qkv(const Params& p, uint32_t trow, int
           store_f32x16(dst + half + j, rb);
         } else {
           f16* dst = kv_row + static_cast<int64_t>(head) * kv.head_stride;
-          store_f16x16(dst + j, ra);
-          store_f16x16(dst + half + j, rb);
+          uint8_t* rdst = kv.res ? kv.res + (dst - kv.base) / 2 : nullptr;
+          store_kv16(dst + j, rdst ? rdst + j / 2 : nullptr, ra);
+          store_kv16(dst + half + j, rdst ? rdst + (half + j) / 2 : nullptr, rb);
         }
       }
     }
@@ -804,7 +825,9 @@ __global__ void reduce_swiglu_kernel(Src src, int M, int F, bf16* out_hi, bf16* 
   report_saturation(status, sat);
 }
 
-// One thread per (row, q|k|v section, head, i < hd/2): sums the pair (i, i + hd/2).
+// One thread per (row, q|k|v section, head, i < hd/2): sums the pair (i, i + hd/2).  Rotary
+// index i runs along the lanes (hd/2 is a multiple of 32), so the residual byte of elements
+// (i, i + 1) is assembled from two neighbouring lanes.
 template <class Src>
 __global__ void reduce_qkv_kernel(Src src, int M, EpiArgs e) {
   pdl_launch_dependents();
@@ -839,8 +862,9 @@ __global__ void reduce_qkv_kernel(Src src, int M, EpiArgs e) {
       f16* dst = e.kv.base + static_cast<int64_t>(e.layer) * e.kv.layer_stride +
                  static_cast<int64_t>(ri.env) * e.kv.env_stride + (sec == 2 ? e.kv.kv_stride : 0) +
                  static_cast<int64_t>(head) * e.kv.head_stride + static_cast<int64_t>(ri.pos) * hd;
-      dst[i] = __float2half_rn(a);
-      dst[i + half] = __float2half_rn(b);
+      uint8_t* res = e.kv.res ? e.kv.res + (dst - e.kv.base) / 2 : nullptr;
+      store_kv_pairlanes(dst, res, i, a);
+      store_kv_pairlanes(dst, res, i + half, b);
     }
   }
 }
@@ -1038,8 +1062,9 @@ __global__ void stream_reduce_qkv_kernel(StreamSrc src, int M, EpiArgs e) {
         f16* dst = e.kv.base + static_cast<int64_t>(e.layer) * e.kv.layer_stride +
                    static_cast<int64_t>(ri.env) * e.kv.env_stride + (sec == 2 ? e.kv.kv_stride : 0) +
                    static_cast<int64_t>(head) * e.kv.head_stride + static_cast<int64_t>(ri.pos) * hd;
-        dst[i] = __float2half_rn(x);
-        dst[i + half] = __float2half_rn(y);
+        uint8_t* res = e.kv.res ? e.kv.res + (dst - e.kv.base) / 2 : nullptr;
+        store_kv_pairlanes(dst, res, i, x);
+        store_kv_pairlanes(dst, res, i + half, y);
       }
     }
   }
@@ -1515,6 +1540,12 @@ int launch_gemv(const CUtensorMap& w, const CUtensorMap& x, const CUtensorMap& x
 }
 
 }  // namespace
+
+// Exported for the attention kernels (tiles of the KV cache).
+bool make_tensor_map_2d(CUtensorMap* m, const void* ptr, int64_t rows, int64_t cols, int64_t ld, int box_rows,
+                        bool fp16) {
+  return make_map(m, ptr, rows, cols, ld, box_rows, fp16);
+}
 
 std::atomic<int> g_test_stall{0};
 

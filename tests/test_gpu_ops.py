@@ -311,3 +311,72 @@ def test_rmsnorm_matches_fp64(fp16):
     assert rel < (2e-6 if fp16 else 2e-5), rel
     # hi alone is the round-to-nearest of the value in that format
     assert (yh.cpu().double() - ref).abs().max().item() <= ref.abs().max().item() * (2.0 ** -11 if fp16 else 2.0 ** -8)
+
+
+# ------------------------------------------------------------------ tcgen05 chunk attention (fp16 + 4-bit residual cache)
+def _encode_res4(x32: np.ndarray):
+    """Host encoding of the cache's 4-bit residual, written from its definition: hi = fp16(x),
+    code c = 8 + clamp(floor((x - hi) / ulp(hi) * 16), -8, 7), value hi + (2c - 15) ulp(hi) / 32
+    with ulp(hi) = 2^(e-25) (biased exponent e >= 1) or 2^-24.  Returns (hi, packed codes, value)."""
+    hi = x32.astype(np.float16)
+    e = ((hi.view(np.uint16) >> 10) & 31).astype(np.int64)
+    ee = np.maximum(e, 1)
+    j = np.floor((x32.astype(np.float64) - hi.astype(np.float64)) * np.ldexp(1.0, 29 - ee))
+    c = (np.clip(j, -8, 7) + 8).astype(np.uint8)
+    value = hi.astype(np.float64) + (2.0 * c - 15.0) * np.ldexp(1.0, ee - 30)
+    packed = (c[..., 0::2] | (c[..., 1::2] << 4)).astype(np.uint8)
+    return hi, packed, value
+
+
+@pytest.mark.parametrize("hd", [128, 64])
+def test_chunk_attention_tc_matches_fp64(hd):
+    """The tcgen05 chunk attention vs brute-force causal softmax attention in fp64 over the values
+    the cache stores (fp16 + residual): chunks of 1..200 rows after 0..300 cached positions, tiles
+    of <= 128 rows, a context reaching the last cache position (cap not a multiple of 64)."""
+    H, cap, max_env = 3, 400, 6
+    chunks = [(0, 0, 1), (1, 0, 127), (2, 0, 128), (3, 7, 200), (4, 300, 100), (5, 100, 64)]  # (env, past, n)
+    rows = sum(n for _, _, n in chunks)
+    x = (I.normal_bf16((max_env, 2, H, cap, hd), 93, hd, 1.0).float()
+         + I.normal_bf16((max_env, 2, H, cap, hd), 93, 7 + hd, 2.0 ** -9).float()).numpy()
+    hi, packed, value = _encode_res4(x)
+    q = I.normal_bf16((rows, H * hd), 93, 1000 + hd, 1.0).float()
+    tiles, qpos, qenv = [], [], []
+    r = 0
+    for env, past, n in chunks:
+        for t0 in range(0, n, 128):
+            tiles.append((env, r + t0, min(128, n - t0), past + t0))
+        qpos += [past + i for i in range(n)]
+        qenv += [env] * n
+        r += n
+    tiles_dev = torch.zeros(len(tiles) * 4, dtype=torch.int32, device="cuda")
+    oh = torch.full((rows, H * hd), float("nan"), dtype=torch.bfloat16, device="cuda")
+    ol = torch.full_like(oh, float("nan"))
+    qd = q.cuda()
+    kvd = torch.from_numpy(hi).cuda()
+    rsd = torch.from_numpy(packed).cuda()
+    assert V.vla_op_read_status()[0] == 0
+    rc = V.vla_op_attn_chunk_res(qd.data_ptr(), kvd.data_ptr(), rsd.data_ptr(), max_env, H, hd, cap, tiles, rows,
+                                 tiles_dev.data_ptr(), oh.data_ptr(), ol.data_ptr())
+    assert rc == 0, V.vla_last_error(None)
+    assert V.vla_op_read_status() == (0, 0)
+    out = oh.cpu().double() + ol.cpu().double()
+    kv64 = torch.from_numpy(value)
+    kvhi = torch.from_numpy(hi.astype(np.float64))
+    err = err_hi = 0.0
+    for i in range(rows):
+        env, p = qenv[i], qpos[i]
+        for hh in range(H):
+            qi = q[i, hh * hd:(hh + 1) * hd].double()
+            o = out[i, hh * hd:(hh + 1) * hd]
+            K, Vv = kv64[env, 0, hh, :p + 1], kv64[env, 1, hh, :p + 1]
+            w = torch.softmax(K @ qi / math.sqrt(hd), dim=0)
+            err = max(err, float((o - w @ Vv).abs().max()))
+            Kh, Vh = kvhi[env, 0, hh, :p + 1], kvhi[env, 1, hh, :p + 1]
+            wh = torch.softmax(Kh @ qi / math.sqrt(hd), dim=0)
+            err_hi = max(err_hi, float((o - wh @ Vh).abs().max()))
+    # hi / lo products in fp32, the bf16 output pair (~16 bits): far below the fp16 cache's own error
+    assert err < 1e-4, err
+    assert err_hi > 4 * err, (err, err_hi)   # the residual is read, not just the fp16 part
+    bad = [(0, 0, 129, 0)]
+    assert V.vla_op_attn_chunk_res(qd.data_ptr(), kvd.data_ptr(), rsd.data_ptr(), max_env, H, hd, cap, bad, rows,
+                                   tiles_dev.data_ptr(), oh.data_ptr(), ol.data_ptr()) == V.VLA_ERR_ARG
