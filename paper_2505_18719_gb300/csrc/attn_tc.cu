@@ -8,19 +8,21 @@
 // each product takes three MMAs into one fp32 accumulator:
 //   S = Q_hi K_hi^T + Q_lo K_hi^T + Q_hi K_lo^T,    O += P_hi V_hi + P_lo V_hi + P_hi V_lo.
 //
-// Roles (320 threads):
-//   warp 0     TMA producer: per 64-key block, K_hi and V_hi (tensor map over the whole cache,
-//              128-byte swizzle) and the two residual byte ranges (bulk copies), two stages;
-//   warp 1     TMEM owner (512 columns) and MMA issuer: S = Q K^T with Q read from TMEM (A
-//              operand) and K from shared memory; O += P V with P from TMEM and V^T from shared
-//              memory; S is double-buffered so block b+1's scores run during block b's softmax;
-//   warps 2-5  softmax, one query row per thread (= its TMEM lane): write Q into TMEM, read each
-//              S block, online softmax in the exp2 domain with a lazily moved reference max (O
-//              and the row sum are rescaled only when the block max exceeds it by more than 8,
-//              so P <= 2^8), write P into TMEM, and finally O / l as the output pair;
-//   warps 6-9  converters: K_lo from K_hi and its residual codes (same swizzled layout), and
-//              V^T_hi / V^T_lo (keys along the rows' 128 bytes, the K-major B operand of P V),
-//              with keys past the last visible one zeroed.
+// Roles (448 threads):
+//   warp 0      TMA producer: per 64-key block, K_hi and V_hi (tensor map over the whole cache,
+//               128-byte swizzle) and the two residual byte ranges (bulk copies), three stages;
+//   warp 1      TMEM owner (512 columns) and MMA issuer: S = Q K^T with Q read from TMEM (A
+//               operand) and K from shared memory (K-major B); O += P V with P from TMEM and V
+//               straight from the cache rows (keys x dims, the MN-major B operand); S is
+//               double-buffered, and the issuer takes whichever of "S of the next block" and
+//               "P V of the oldest pending block" is ready first;
+//   warps 2-5   softmax, one query row per thread (= its TMEM lane): write Q into TMEM, read each
+//               S block, online softmax in the exp2 domain with a lazily moved reference max (O
+//               and the row sum are rescaled only when the block max exceeds it by more than 8,
+//               so P <= 2^8), write P into TMEM, and finally O / l as the output pair;
+//   warps 6-13  converters: K_lo and V_lo from the hi parts and their residual codes, in the hi
+//               parts' own swizzled layout; values of keys past the last visible one are zeroed
+//               (their P is 0, and a stale NaN would still poison the product).
 // TMEM columns: S0 [0,64) S1 [64,128) O [128,128+HD) Q_hi [256,256+HD/2) Q_lo [256+HD/2,256+HD)
 // P_hi [384,416) P_lo [416,448).  Every wait is bounded; on a timeout the CTA records
 // VLA_STATUS_TIMEOUT, drains its copies and MMAs, frees TMEM and writes nothing.
@@ -34,23 +36,31 @@ namespace vla {
 
 namespace {
 
-constexpr int kAtThreads = 320;
+constexpr int kAtWarps = 14;
+constexpr int kAtThreads = 32 * kAtWarps;
+constexpr int kConvWarps = kAtWarps - 6;
+constexpr int kStages = 3;
 constexpr int kKeys = 64;  // keys per block
 constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kColS = 0, kColO = 128, kColQ = 256, kColP = 384;
 
-__device__ __forceinline__ uint64_t sdesc_sw128(uint32_t saddr) {
+// Shared-memory matrix descriptor, 128-byte swizzle: atoms of 8 rows x 128 bytes, 1024 bytes
+// apart along the rows (SBO); for an MN-major operand the 64-element column blocks lie `lbo`
+// bytes apart (LBO; unused for K-major).
+__device__ __forceinline__ uint64_t sdesc_sw128(uint32_t saddr, uint32_t lbo = 16) {
   uint64_t d = 0;
   d |= static_cast<uint64_t>((saddr & 0x3FFFFu) >> 4);
-  d |= static_cast<uint64_t>(1) << 16;          // LBO (unused for swizzled K-major)
-  d |= static_cast<uint64_t>(1024 >> 4) << 32;  // SBO: 8-row groups 1024 bytes apart
+  d |= static_cast<uint64_t>(lbo >> 4) << 16;
+  d |= static_cast<uint64_t>(1024 >> 4) << 32;
   d |= static_cast<uint64_t>(1) << 46;          // descriptor version
   d |= static_cast<uint64_t>(2) << 61;          // 128-byte swizzle
   return d;
 }
-// kind::f16, fp16 A and B (format fields 0), fp32 D, both K-major, M = 128, N.
-__device__ __forceinline__ constexpr uint32_t idesc_f16(int N) {
-  return (1u << 4) | (static_cast<uint32_t>(N >> 3) << 17) | (static_cast<uint32_t>(128 >> 4) << 24);
+// kind::f16, fp16 A and B (format fields 0), fp32 D, M = 128, N; A K-major, B K-major or
+// MN-major (bit 16).
+__device__ __forceinline__ constexpr uint32_t idesc_f16(int N, bool b_mn_major = false) {
+  return (1u << 4) | (b_mn_major ? (1u << 16) : 0u) | (static_cast<uint32_t>(N >> 3) << 17) |
+         (static_cast<uint32_t>(128 >> 4) << 24);
 }
 // D (TMEM) (+)= A (TMEM) * B (shared memory)
 __device__ __forceinline__ void mma_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t bdesc, uint32_t idesc,
@@ -73,22 +83,31 @@ __device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t (&r)[16
 __device__ __forceinline__ void tmem_wait_st() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
 __device__ __forceinline__ void fence_async_smem() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
 
-__device__ __forceinline__ uint32_t pack_h2(f16 a, f16 b) {
-  __half2 v = __halves2half2(a, b);
-  return *reinterpret_cast<uint32_t*>(&v);
+__device__ __forceinline__ __half2 u32_h2(uint32_t v) { return *reinterpret_cast<__half2*>(&v); }
+__device__ __forceinline__ uint32_t h2_u32(__half2 v) { return *reinterpret_cast<uint32_t*>(&v); }
+// (a, b) -> fp16 pairs hi = fp16(x), lo = fp16(x - hi), with packed conversions.
+__device__ __forceinline__ void split_h2(float a, float b, uint32_t& hi, uint32_t& lo) {
+  const __half2 h = __floats2half2_rn(a, b);
+  const float2 f = __half22float2(h);
+  hi = h2_u32(h);
+  lo = h2_u32(__floats2half2_rn(a - f.x, b - f.y));
 }
-// Low part of 8 cached fp16 values (one 16-byte chunk) from their 4-bit codes (4 bytes).
+// Low parts of 8 cached fp16 values (one 16-byte chunk) from their 4-bit codes (4 bytes, element
+// 2i in the low nibble of byte i): per element (2c - 15) * 2^(e - 30), e the value's fp16 exponent
+// field, in fp16 arithmetic with no conversion instruction.  2c goes into the mantissa of 1024
+// (fp16 bits 0x6400 | 2c), so 1024 + 2c - 1039 = 2c - 15 exactly; 2^(e - 30) is the value with
+// mantissa and sign cleared (2^(e-15)) times 2^-15.  Exact for e >= 6; below that the term is
+// under 2^-21 in magnitude and comes out as zero or a rounded subnormal.
 __device__ __forceinline__ uint4 res_lo8(uint4 hi, uint32_t codes) {
-  const uint32_t w[4] = {hi.x, hi.y, hi.z, hi.w};
-  uint32_t o[4];
-#pragma unroll
-  for (int k = 0; k < 4; ++k) {
-    const f16 a = __ushort_as_half(static_cast<unsigned short>(w[k] & 0xFFFFu));
-    const f16 b = __ushort_as_half(static_cast<unsigned short>(w[k] >> 16));
-    const uint32_t byte = (codes >> (8 * k)) & 0xFFu;
-    o[k] = pack_h2(kv_res_lo(a, byte & 15u), kv_res_lo(b, byte >> 4));
-  }
-  return make_uint4(o[0], o[1], o[2], o[3]);
+  const uint32_t twice_lo = (codes << 1) & 0x1E1E1E1Eu;  // 2c of each byte's low nibble
+  const uint32_t twice_hi = (codes >> 3) & 0x1E1E1E1Eu;  // 2c of each byte's high nibble
+  auto pair = [&](uint32_t h2, uint32_t sel) {
+    const uint32_t w = (__byte_perm(twice_lo, twice_hi, sel) & 0x00FF00FFu) | 0x64006400u;
+    const __half2 k = __hsub2(u32_h2(w), u32_h2(0x640F640Fu));                      // 2c - 15
+    const __half2 s = __hmul2(u32_h2(h2 & 0x7C007C00u), u32_h2(0x02000200u));       // 2^(e - 30)
+    return h2_u32(__hmul2(k, s));
+  };
+  return make_uint4(pair(hi.x, 0x0400u), pair(hi.y, 0x0501u), pair(hi.z, 0x0602u), pair(hi.w, 0x0703u));
 }
 
 struct AtParams {
@@ -110,25 +129,28 @@ template <int HD>
 struct AtSmem {
   static constexpr int K_BYTES = kKeys * HD * 2;        // one 64-key tile of K (or V), fp16
   static constexpr int R_BYTES = kKeys * HD / 2;        // its residual codes
-  // stage: K_hi | K_lo | V_hi (TMA) | V^T_hi | V^T_lo | K codes | V codes
-  static constexpr int STAGE = 5 * K_BYTES + 2 * R_BYTES;
-  static constexpr int SMEM = 1024 + 2 * STAGE + 256;
+  // a stage: K_hi | V_hi | K_lo | V_lo | K codes | V codes (each tile 1024-byte aligned)
+  static constexpr int STAGE = 4 * K_BYTES + 2 * R_BYTES;
+  static constexpr int SMEM = 1024 + kStages * STAGE + 256;
+  static_assert(STAGE % 1024 == 0, "stage alignment");
 };
 
 template <int HD>
 __global__ void __launch_bounds__(kAtThreads, 1)
     attn_chunk_tc_kernel(const __grid_constant__ CUtensorMap tmKV, const AtParams p) {
   using Sm = AtSmem<HD>;
-  constexpr int KB = HD / 64;  // 64-element k-blocks of one K row
+  constexpr int KB = HD / 64;  // 64-element column blocks of one K / V row
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + 2 * Sm::STAGE);
-  // full[2] conv[2] sfull[2] sfree[2] stfree[2] pfull pdone qready drain
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + kStages * Sm::STAGE);
+  // full[3] (loaded) conv[3] (low parts written) stfree[3] (the MMAs are done with the stage)
+  // sfull[2] sfree[2] pfull pdone qready drain
   const uint32_t b0 = smem_u32(bars);
   auto BAR = [&](int i) { return b0 + 8u * static_cast<uint32_t>(i); };
-  const uint32_t FULL = 0, CONV = 2, SFULL = 4, SFREE = 6, STFREE = 8, PFULL = 10, PDONE = 11, QREADY = 12, DRAIN = 13;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 16);
+  const uint32_t FULL = 0, CONV = 3, STFREE = 6, SFULL = 9, SFREE = 11, PFULL = 13, PDONE = 14, QREADY = 15,
+                 DRAIN = 16;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 17);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   pdl_launch_dependents();
@@ -143,16 +165,15 @@ __global__ void __launch_bounds__(kAtThreads, 1)
   const uint64_t limit = p.wait_limit;
 
   if (threadIdx.x == 0) {
-    mbar_init(BAR(FULL), 1);
-    mbar_init(BAR(FULL + 1), 1);
-    mbar_init(BAR(CONV), 4);
-    mbar_init(BAR(CONV + 1), 4);
-    mbar_init(BAR(SFULL), 1);
-    mbar_init(BAR(SFULL + 1), 1);
-    mbar_init(BAR(SFREE), 4);
-    mbar_init(BAR(SFREE + 1), 4);
-    mbar_init(BAR(STFREE), 1);
-    mbar_init(BAR(STFREE + 1), 1);
+    for (int s = 0; s < kStages; ++s) {
+      mbar_init(BAR(FULL + s), 1);
+      mbar_init(BAR(CONV + s), kConvWarps);
+      mbar_init(BAR(STFREE + s), 1);
+    }
+    for (int s = 0; s < 2; ++s) {
+      mbar_init(BAR(SFULL + s), 1);
+      mbar_init(BAR(SFREE + s), 4);
+    }
     mbar_init(BAR(PFULL), 4);
     mbar_init(BAR(PDONE), 1);
     mbar_init(BAR(QREADY), 4);
@@ -180,11 +201,10 @@ __global__ void __launch_bounds__(kAtThreads, 1)
       pdl_wait();  // the chunk's own keys / values were written by the q|k|v projection
       uint32_t issued = 0, issued_phase = 0;
       for (int b = 0; b < nb; ++b) {
-        const int st = b & 1;
-        if (b >= 2 && !wait_bounded(BAR(STFREE + st), ((b >> 1) - 1) & 1, abort_flag, status, limit)) break;
-        uint8_t* sp = stage_ptr(st);
-        const uint32_t s_khi = smem_u32(sp), s_vhi = s_khi + 2 * Sm::K_BYTES;
-        const uint32_t s_kr = s_khi + 5 * Sm::K_BYTES, s_vr = s_kr + Sm::R_BYTES;
+        const int st = b % kStages, round = b / kStages;
+        if (round >= 1 && !wait_bounded(BAR(STFREE + st), (round - 1) & 1, abort_flag, status, limit)) break;
+        const uint32_t s_khi = smem_u32(stage_ptr(st)), s_vhi = s_khi + Sm::K_BYTES;
+        const uint32_t s_kr = s_khi + 4 * Sm::K_BYTES, s_vr = s_kr + Sm::R_BYTES;
         const int key0 = b * kKeys;
         const int rows = min(kKeys, p.cap - key0);  // residual rows inside this (env, head)
         const uint32_t rbytes = static_cast<uint32_t>(rows) * (HD / 2);
@@ -197,60 +217,67 @@ __global__ void __launch_bounds__(kAtThreads, 1)
         bulk_load(s_kr, p.res + (krow0 + key0) * (HD / 2), rbytes, BAR(FULL + st));
         bulk_load(s_vr, p.res + (vrow0 + key0) * (HD / 2), rbytes, BAR(FULL + st));
         issued |= 1u << st;
-        issued_phase = (issued_phase & ~(1u << st)) | (static_cast<uint32_t>((b >> 1) & 1) << st);
+        issued_phase = (issued_phase & ~(1u << st)) | (static_cast<uint32_t>(round & 1) << st);
       }
-      for (int st = 0; st < 2; ++st)
+      for (int st = 0; st < kStages; ++st)
         if (issued & (1u << st)) wait_drain(BAR(FULL + st), (issued_phase >> st) & 1u, limit);
     }
   } else if (warp == 1) {
     if (lane == 0) {
       // ------------------------------------------------------------------ MMA issuer
-      const uint32_t IS = idesc_f16(kKeys), IO = idesc_f16(HD);
+      const uint32_t IS = idesc_f16(kKeys), IO = idesc_f16(HD, true);
       const uint32_t tS0 = tmem + kColS, tO = tmem + kColO;
       const uint32_t tQh = tmem + kColQ, tQl = tmem + kColQ + HD / 2;
       const uint32_t tPh = tmem + kColP, tPl = tmem + kColP + kKeys / 2;
       bool ok = wait_bounded(BAR(QREADY), 0, abort_flag, status, limit);
-      auto issue_o = [&](int bb) -> bool {
-        if (!wait_bounded(BAR(PFULL), bb & 1, abort_flag, status, limit)) return false;
-        tc_fence_after();
-        const uint32_t s_vth = smem_u32(stage_ptr(bb & 1)) + 3 * Sm::K_BYTES;
-        const uint32_t s_vtl = s_vth + Sm::K_BYTES;
+      int bs = 0, bo = 0;  // next block whose S, whose P V is to be issued
+      uint64_t t_last = globaltimer();
+      uint32_t spins = 0;
+      while (ok && bo < nb) {
+        if (bo < bs && mbar_test_wait(BAR(PFULL), bo & 1)) {
+          // O += P V of block bo; the commit frees its stage and hands O / P back to the softmax
+          tc_fence_after();
+          const uint32_t s_vhi = smem_u32(stage_ptr(bo % kStages)) + Sm::K_BYTES;
+          const uint32_t s_vlo = s_vhi + 2 * Sm::K_BYTES;
 #pragma unroll
-        for (int k = 0; k < kKeys / 16; ++k) {
-          const uint64_t dh = sdesc_sw128(s_vth + k * 32), dl = sdesc_sw128(s_vtl + k * 32);
-          mma_ts(tO, tPh + k * 8, dh, IO, (bb > 0 || k > 0) ? 1u : 0u);
-          mma_ts(tO, tPl + k * 8, dh, IO, 1u);
-          mma_ts(tO, tPh + k * 8, dl, IO, 1u);
-        }
-        tc_commit(BAR(PDONE));
-        tc_commit(BAR(STFREE + (bb & 1)));
-        return true;
-      };
-      for (int b = 0; b < nb && ok; ++b) {
-        const int st = b & 1;
-        if (!wait_bounded(BAR(CONV + st), (b >> 1) & 1, abort_flag, status, limit)) {
-          ok = false;
-          break;
-        }
-        if (b >= 2 && !wait_bounded(BAR(SFREE + st), ((b >> 1) - 1) & 1, abort_flag, status, limit)) {
-          ok = false;
-          break;
-        }
-        tc_fence_after();
-        const uint32_t s_khi = smem_u32(stage_ptr(st)), s_klo = s_khi + Sm::K_BYTES;
-        const uint32_t tS = tS0 + st * kKeys;
+          for (int k = 0; k < kKeys / 16; ++k) {
+            const uint64_t dh = sdesc_sw128(s_vhi + k * 2048, kKeys * 128);
+            const uint64_t dl = sdesc_sw128(s_vlo + k * 2048, kKeys * 128);
+            mma_ts(tO, tPh + k * 8, dh, IO, (bo > 0 || k > 0) ? 1u : 0u);
+            mma_ts(tO, tPl + k * 8, dh, IO, 1u);
+            mma_ts(tO, tPh + k * 8, dl, IO, 1u);
+          }
+          tc_commit(BAR(PDONE));
+          tc_commit(BAR(STFREE + bo % kStages));
+          ++bo;
+          t_last = globaltimer();
+        } else if (bs < nb && mbar_test_wait(BAR(CONV + bs % kStages), (bs / kStages) & 1) &&
+                   (bs < 2 || mbar_test_wait(BAR(SFREE + (bs & 1)), ((bs >> 1) - 1) & 1))) {
+          // S of block bs into buffer bs & 1
+          tc_fence_after();
+          const uint32_t s_khi = smem_u32(stage_ptr(bs % kStages)), s_klo = s_khi + 2 * Sm::K_BYTES;
+          const uint32_t tS = tS0 + (bs & 1) * kKeys;
 #pragma unroll
-        for (int k = 0; k < HD / 16; ++k) {
-          const uint32_t off = (k >> 2) * (kKeys * 128) + (k & 3) * 32;
-          const uint64_t dh = sdesc_sw128(s_khi + off), dl = sdesc_sw128(s_klo + off);
-          mma_ts(tS, tQh + k * 8, dh, IS, k > 0 ? 1u : 0u);
-          mma_ts(tS, tQl + k * 8, dh, IS, 1u);
-          mma_ts(tS, tQh + k * 8, dl, IS, 1u);
+          for (int k = 0; k < HD / 16; ++k) {
+            const uint32_t off = (k >> 2) * (kKeys * 128) + (k & 3) * 32;
+            const uint64_t dh = sdesc_sw128(s_khi + off), dl = sdesc_sw128(s_klo + off);
+            mma_ts(tS, tQh + k * 8, dh, IS, k > 0 ? 1u : 0u);
+            mma_ts(tS, tQl + k * 8, dh, IS, 1u);
+            mma_ts(tS, tQh + k * 8, dl, IS, 1u);
+          }
+          tc_commit(BAR(SFULL + (bs & 1)));
+          ++bs;
+          t_last = globaltimer();
+        } else if (((++spins) & 63u) == 0) {
+          if (*abort_flag) {
+            ok = false;
+          } else if (globaltimer() - t_last > limit) {
+            *abort_flag = 1;
+            if (status) atomicOr(status, VLA_STATUS_TIMEOUT);
+            ok = false;
+          }
         }
-        tc_commit(BAR(SFULL + st));
-        if (b >= 1 && !issue_o(b - 1)) ok = false;
       }
-      if (ok && nb > 0) issue_o(nb - 1);
       tc_commit(BAR(DRAIN));
       wait_drain(BAR(DRAIN), 0, limit);
     }
@@ -267,17 +294,23 @@ __global__ void __launch_bounds__(kAtThreads, 1)
     {
       const float* qrow = p.q + static_cast<size_t>(tile.row0 + (valid ? r : 0)) * dcols + head * HD;
 #pragma unroll 1
-      for (int c = 0; c < HD; c += 32) {
-        uint32_t hi[16], lo[16];
+      for (int c = 0; c < HD; c += 64) {
+        float4 x[16];  // 64 values in flight
 #pragma unroll
-        for (int i = 0; i < 16; ++i) {
-          const float2 x = valid ? *reinterpret_cast<const float2*>(qrow + c + 2 * i) : make_float2(0.f, 0.f);
-          const f16 h0 = __float2half_rn(x.x), h1 = __float2half_rn(x.y);
-          hi[i] = pack_h2(h0, h1);
-          lo[i] = pack_h2(__float2half_rn(x.x - __half2float(h0)), __float2half_rn(x.y - __half2float(h1)));
+        for (int i = 0; i < 16; ++i)
+          x[i] = valid ? __ldg(reinterpret_cast<const float4*>(qrow + c) + i) : make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+        for (int half = 0; half < 2; ++half) {
+          uint32_t hi[16], lo[16];
+#pragma unroll
+          for (int i = 0; i < 8; ++i) {
+            const float4 v = x[half * 8 + i];
+            split_h2(v.x, v.y, hi[2 * i], lo[2 * i]);
+            split_h2(v.z, v.w, hi[2 * i + 1], lo[2 * i + 1]);
+          }
+          tmem_st16(tmem + lane_off + kColQ + (c + 32 * half) / 2, hi);
+          tmem_st16(tmem + lane_off + kColQ + HD / 2 + (c + 32 * half) / 2, lo);
         }
-        tmem_st16(tmem + lane_off + kColQ + c / 2, hi);
-        tmem_st16(tmem + lane_off + kColQ + HD / 2 + c / 2, lo);
       }
       tmem_wait_st();
       tc_fence_before();
@@ -349,9 +382,7 @@ __global__ void __launch_bounds__(kAtThreads, 1)
         for (int i = 0; i < 16; ++i) {
           const float p0 = exp2f(s[c + 2 * i] - m_ref), p1 = exp2f(s[c + 2 * i + 1] - m_ref);
           ps += p0 + p1;
-          const f16 h0 = __float2half_rn(p0), h1 = __float2half_rn(p1);
-          hi[i] = pack_h2(h0, h1);
-          lo[i] = pack_h2(__float2half_rn(p0 - __half2float(h0)), __float2half_rn(p1 - __half2float(h1)));
+          split_h2(p0, p1, hi[i], lo[i]);
         }
         tmem_st16(tmem + lane_off + kColP + c / 2, hi);
         tmem_st16(tmem + lane_off + kColP + kKeys / 2 + c / 2, lo);
@@ -392,54 +423,32 @@ __global__ void __launch_bounds__(kAtThreads, 1)
       }
     }
   } else {
-    // ------------------------------------------------------------------ converters (warps 6-9)
-    const int t = threadIdx.x - 6 * 32;  // 0..127
+    // ------------------------------------------------------------------ converters (warps 6-13)
+    const int t = threadIdx.x - 6 * 32;
+    constexpr int CH = HD / 8;  // 16-byte chunks of one row
     for (int b = 0; b < nb; ++b) {
-      const int st = b & 1;
+      const int st = b % kStages;
       int w_ok = 1;
-      if (lane == 0) w_ok = wait_bounded(BAR(FULL + st), (b >> 1) & 1, abort_flag, status, limit) ? 1 : 0;
+      if (lane == 0) w_ok = wait_bounded(BAR(FULL + st), (b / kStages) & 1, abort_flag, status, limit) ? 1 : 0;
       if (!__shfl_sync(0xffffffffu, w_ok, 0)) break;
       uint8_t* sp = stage_ptr(st);
-      const uint8_t* khi = sp;
-      uint8_t* klo = sp + Sm::K_BYTES;
-      const uint8_t* vhi = sp + 2 * Sm::K_BYTES;
-      uint8_t* vth = sp + 3 * Sm::K_BYTES;
-      uint8_t* vtl = sp + 4 * Sm::K_BYTES;
-      const uint8_t* kr = sp + 5 * Sm::K_BYTES;
-      const uint8_t* vr = kr + Sm::R_BYTES;
-      const int key0 = b * kKeys;
-      // K_lo: chunk index fastest over lanes (conflict-free code reads and swizzled accesses)
-      for (int ch = t; ch < kKeys * (HD / 8); ch += 128) {
-        const int c = ch % (HD / 8), key = ch / (HD / 8);
+      const int live = n_keys - b * kKeys;  // keys of this block visible to some row
+      // chunk index fastest over lanes: 8 lanes read one swizzled 128-byte row, a warp reads 128
+      // consecutive code bytes
+#pragma unroll 2
+      for (int ch = t; ch < 2 * kKeys * CH; ch += 32 * kConvWarps) {
+        const int w = ch / (kKeys * CH);  // 0: K, 1: V
+        const int c = ch % CH, key = (ch / CH) % kKeys;
         const int off = (c >> 3) * (kKeys * 128) + key * 128 + (((c & 7) ^ (key & 7)) << 4);
-        const uint4 hv = *reinterpret_cast<const uint4*>(khi + off);
-        const uint32_t codes = *reinterpret_cast<const uint32_t*>(kr + key * (HD / 2) + c * 4);
-        *reinterpret_cast<uint4*>(klo + off) = res_lo8(hv, codes);
-      }
-      // V^T_hi, V^T_lo: key fastest over lanes (conflict-free transposed stores); a thread takes
-      // 32 dims of one key (16 bytes of codes), keys past the last visible one are zero
-      for (int it = t; it < kKeys * (HD / 32); it += 128) {
-        const int key = it % kKeys, g = it / kKeys;
-        const bool live = key0 + key < n_keys;
-        const uint4 cw = *reinterpret_cast<const uint4*>(vr + key * (HD / 2) + g * 16);
-        const uint32_t cws[4] = {cw.x, cw.y, cw.z, cw.w};
-#pragma unroll
-        for (int j = 0; j < 4; ++j) {
-          const int c = g * 4 + j;  // 8-dim chunk
-          const int off = (c >> 3) * (kKeys * 128) + key * 128 + (((c & 7) ^ (key & 7)) << 4);
-          uint4 hv = *reinterpret_cast<const uint4*>(vhi + off);
-          uint4 lv = res_lo8(hv, cws[j]);
-          if (!live) hv = lv = make_uint4(0u, 0u, 0u, 0u);
-          const uint32_t hw[4] = {hv.x, hv.y, hv.z, hv.w}, lw[4] = {lv.x, lv.y, lv.z, lv.w};
-#pragma unroll
-          for (int e = 0; e < 8; ++e) {
-            const int d = c * 8 + e;
-            const int toff = d * 128 + ((((key >> 3) ^ (d & 7))) << 4) + (key & 7) * 2;
-            const uint16_t hb = static_cast<uint16_t>(hw[e >> 1] >> (16 * (e & 1)));
-            const uint16_t lb = static_cast<uint16_t>(lw[e >> 1] >> (16 * (e & 1)));
-            *reinterpret_cast<uint16_t*>(vth + toff) = hb;
-            *reinterpret_cast<uint16_t*>(vtl + toff) = lb;
-          }
+        uint4* hi = reinterpret_cast<uint4*>(sp + w * Sm::K_BYTES + off);
+        uint4* lo = reinterpret_cast<uint4*>(sp + (2 + w) * Sm::K_BYTES + off);
+        if (w == 1 && key >= live) {
+          *hi = make_uint4(0u, 0u, 0u, 0u);
+          *lo = make_uint4(0u, 0u, 0u, 0u);
+        } else {
+          const uint32_t codes =
+              *reinterpret_cast<const uint32_t*>(sp + 4 * Sm::K_BYTES + w * Sm::R_BYTES + key * (HD / 2) + c * 4);
+          *lo = res_lo8(*hi, codes);
         }
       }
       fence_async_smem();  // the MMAs (async proxy) read what these generic stores wrote
