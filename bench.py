@@ -230,6 +230,8 @@ CASES = {
     "learning": None,                                          # see run_learning_case
     "attn_chunk": None,                                        # see run_attn_chunk_case
     "attn_score": None,                                        # 6 rows per env after the prefix
+    "attn_chunk_res": None,                                    # the same over fp16 + 4-bit residual
+    "attn_score_res": None,
     # the same prefill shapes on CTA pairs (2-SM MMAs, 256 x 256 tiles)
     "pair_prefill_qkv": (4608, 12288, 4096, 256, 1, True),
     "pair_prefill_down": (4608, 4096, 11008, 256, 1, True),
@@ -310,7 +312,9 @@ def run_attn_case(args):
 
 def run_attn_chunk_case(args):
     """Prefill chunk attention of one layer of the bench step: 64 envs, 256 visual + U{16..48}
-    text rows each, 32 heads x 128, in tiles of <= 64 query rows."""
+    text rows each, 32 heads x 128.  attn_chunk / attn_score: the fp16-cache kernel, tiles of
+    <= 64 query rows; attn_chunk_res / attn_score_res: the tcgen05 kernel over the fp16 +
+    4-bit residual cache (the engine's form), tiles of <= 128 rows."""
     import torch
     import __graft_entry__
     __graft_entry__.build()
@@ -318,24 +322,31 @@ def run_attn_chunk_case(args):
     from paper_2505_18719_gb300 import vla as V
     B, H, hd, cap = 64, 32, 128, 320
     prefix = (256 + I.randint_i32((B,), 5, 7, 16, 48)).tolist()
-    score = args.case == "attn_score"       # the score pass: 6 rows per env after its prefix
+    score = args.case.startswith("attn_score")   # the score pass: 6 rows per env after its prefix
+    res = args.case.endswith("_res")
+    tile_rows = 128 if res else 64
     lens = [6] * B if score else prefix
     past = prefix if score else [0] * B
     rows = sum(lens)
     kv = I.normal_bf16((B, 2, H, cap, hd), 5, 1, 1.0).cuda().half()
+    codes = I.randint_i32((B * 2 * H * cap * hd // 2,), 5, 3, 0, 256).to(torch.uint8).cuda() if res else None
     q = I.normal_bf16((rows, H * hd), 5, 2, 1.0).cuda().float()
     tiles, r = [], 0
     for b, n in enumerate(lens):
-        for t0 in range(0, n, 64):
-            tiles.append((b, r + t0, min(64, n - t0), past[b] + t0))
+        for t0 in range(0, n, tile_rows):
+            tiles.append((b, r + t0, min(tile_rows, n - t0), past[b] + t0))
         r += n
     tiles_dev = torch.zeros(len(tiles) * 4, dtype=torch.int32, device="cuda")
     oh = torch.empty(rows, H * hd, dtype=torch.bfloat16, device="cuda")
     ol = torch.empty_like(oh)
 
     def launch():
-        rc = V.vla_op_attn_chunk(q.data_ptr(), kv.data_ptr(), B, H, hd, cap, tiles, rows, tiles_dev.data_ptr(),
-                                 oh.data_ptr(), ol.data_ptr())
+        if res:
+            rc = V.vla_op_attn_chunk_res(q.data_ptr(), kv.data_ptr(), codes.data_ptr(), B, H, hd, cap, tiles, rows,
+                                         tiles_dev.data_ptr(), oh.data_ptr(), ol.data_ptr())
+        else:
+            rc = V.vla_op_attn_chunk(q.data_ptr(), kv.data_ptr(), B, H, hd, cap, tiles, rows, tiles_dev.data_ptr(),
+                                     oh.data_ptr(), ol.data_ptr())
         assert rc == 0, V.vla_last_error(None)
 
     for _ in range(args.warmup):
@@ -349,11 +360,11 @@ def run_attn_chunk_case(args):
     torch.cuda.synchronize()
     ms = e0.elapsed_time(e1) / args.steps
     flops = sum(2.0 * H * hd * n * (n + 1 + 2 * p) for n, p in zip(lens, past))   # causal QK^T + PV
-    kv_bytes = sum((p + n) * 2.0 * H * hd * 2 for n, p in zip(lens, past))
+    kv_bytes = sum((p + n) * 2.0 * H * hd * (2.5 if res else 2) for n, p in zip(lens, past))
     _, tf_burst, _, kind = peaks()
     print(json.dumps({"case": args.case, "B": B, "H": H, "hd": hd, "rows": rows, "tiles": len(tiles), "ms": ms,
                       "tflops": flops / ms / 1e9, "tc_frac_of_burst": flops / ms / 1e9 / tf_burst,
-                      "issued_mma_tflops": 2 * flops / ms / 1e9, "kv_gbs": kv_bytes / ms / 1e6, "peaks": kind}))
+                      "issued_mma_tflops": (3 if res else 2) * flops / ms / 1e9, "kv_gbs": kv_bytes / ms / 1e6, "peaks": kind}))
     return 0
 
 
@@ -407,7 +418,7 @@ def run_case(args):
         return run_attn_case(args)
     if args.case == "learning":
         return run_learning_case(args)
-    if args.case in ("attn_chunk", "attn_score"):
+    if args.case.startswith(("attn_chunk", "attn_score")):
         return run_attn_chunk_case(args)
     M, N, K, bn, splits, split_a = CASES[args.case]
     fp16 = args.case.endswith("_f16")

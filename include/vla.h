@@ -25,8 +25,7 @@
  *    multiply both halves, the tile GEMMs (prefill, score, larger decode batches) both halves
  *    for q|k|v and hi alone for o, gate|up and down.  K/V are cached in fp16 plus a 4-bit
  *    residual per element (value = hi + (2c - 15) ulp(hi) / 32, within ulp(hi) / 32 of the
- *    computed key / value); the chunk attention of prefill and score reads both, the decode
- *    attention the fp16 part.  A finite
+ *    computed key / value), and every attention reads both.  A finite
  *    activation beyond the fp16 range (|x| > 65504) is stored as +-65504 and raises
  *    VLA_STATUS_SATURATED in the status word (reported by the next vla_sync).
  *  - Calls are asynchronous on the handle's stream.  Host-checkable errors return at once,

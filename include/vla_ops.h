@@ -152,7 +152,9 @@ int vla_op_attn_chunk(const float* q, const void* kv, int max_env, int H, int hd
  *            hi = fp16(x) is c = 8 + clamp(floor((x - hi) / ulp(hi) * 16), -8, 7), and the value
  *            read is hi + (2c - 15) ulp(hi) / 32, ulp(hi) = 2^(e-25) for hi's biased exponent
  *            e >= 1, 2^-24 for e = 0.
- * A pipeline wait that runs out sets VLA_STATUS_TIMEOUT in the op status word.  hd in {64, 128}. */
+ * Cache positions past a tile's last visible key may hold anything (NaN included): they do not
+ * reach the output.  A pipeline wait that runs out sets VLA_STATUS_TIMEOUT in the op status
+ * word.  hd in {64, 128}. */
 int vla_op_attn_chunk_res(const float* q, const void* kv, const void* kv_res, int max_env, int H, int hd,
                           int cap, const int32_t* tiles_host, int n_tiles, int rows, int32_t* tiles_dev,
                           void* out_hi, void* out_lo, void* cuda_stream);

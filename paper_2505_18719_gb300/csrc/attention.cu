@@ -269,7 +269,8 @@ __global__ void __launch_bounds__(128) attn_chunk_mma_kernel(const float* __rest
 }
 
 // ---------------------------------------------------------------------------------- decode
-// One query per (env, head, key range): 16 lanes x 16 bytes read one 128-element fp16 key row,
+// One query per (env, head, key range): 16 lanes x 16 bytes read one 128-element fp16 key row
+// (with RES, also its 4-bit residual codes, 4 bytes per lane, and use hi + lo as the cached value),
 // each lane group loads 4 key rows (K and V) before using any (memory-level parallelism), the
 // dot products reduce with xor shuffles inside the group, online softmax per lane group; the
 // groups of the CTA merge through shared memory into one partial (max, sum, unnormalised
@@ -281,8 +282,8 @@ __global__ void __launch_bounds__(128) attn_chunk_mma_kernel(const float* __rest
 // at once (one wave, no tail).  No minimum-blocks bound is given: capping at 64 forces a small
 // spill in the 64-dim variant.
 constexpr int kDecodeWarps = 2;
-template <int HD, int NW = kDecodeWarps>
-__global__ void __launch_bounds__(NW * 32) attn_decode_kernel(const float* __restrict__ q,
+template <int HD, bool RES, int NW = kDecodeWarps>
+__global__ void __launch_bounds__(NW * 32, RES ? 14 : 1) attn_decode_kernel(const float* __restrict__ q,
                                                           const RowInfo* __restrict__ rows,
                                                           KVLayout kv, int layer, int H,
                                                           int chunk, int S, float scale_log2,
@@ -325,6 +326,9 @@ __global__ void __launch_bounds__(NW * 32) attn_decode_kernel(const float* __res
                      static_cast<int64_t>(ri.env) * kv.env_stride +
                      static_cast<int64_t>(head) * kv.head_stride;
   const f16* vbase = kbase + kv.kv_stride;
+  // RES: the residual codes of the same elements (half a byte each), read with the fp16 parts
+  const uint8_t* kres = RES ? kv.res + (kbase - kv.base) / 2 : nullptr;
+  const uint8_t* vres = RES ? kres + kv.kv_stride / 2 : nullptr;
 
   float m = -INFINITY, l = 0.f, o[8];
 #pragma unroll
@@ -332,14 +336,20 @@ __global__ void __launch_bounds__(NW * 32) attn_decode_kernel(const float* __res
 
   for (int key0 = k_begin + warp * KPI * U; key0 < k_end; key0 += NW * KPI * U) {
     uint4 kk[U], vv[U];
+    uint32_t kc[U], vc[U];
 #pragma unroll
     for (int u = 0; u < U; ++u) {
       const int key = key0 + u * KPI + sub;
       kk[u] = make_uint4(0, 0, 0, 0);
       vv[u] = make_uint4(0, 0, 0, 0);
+      kc[u] = vc[u] = 0u;  // fp16 parts of 0: low parts 0 whatever the codes
       if (key < k_end) {
         kk[u] = *reinterpret_cast<const uint4*>(kbase + static_cast<int64_t>(key) * HD + part * 8);
         vv[u] = *reinterpret_cast<const uint4*>(vbase + static_cast<int64_t>(key) * HD + part * 8);
+        if (RES) {
+          kc[u] = *reinterpret_cast<const uint32_t*>(kres + static_cast<int64_t>(key) * (HD / 2) + part * 4);
+          vc[u] = *reinterpret_cast<const uint32_t*>(vres + static_cast<int64_t>(key) * (HD / 2) + part * 4);
+        }
       }
     }
 #pragma unroll
@@ -353,6 +363,16 @@ __global__ void __launch_bounds__(NW * 32) attn_decode_kernel(const float* __res
         acc = fmaf(qv[2 * e], f.x, acc);
         acc = fmaf(qv[2 * e + 1], f.y, acc);
       }
+      if (RES) {
+        const uint4 kl = kv_res_lo8(kk[u], kc[u]);
+        const uint32_t wl[4] = {kl.x, kl.y, kl.z, kl.w};
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const float2 f = unpack_f16x2(wl[e]);
+          acc = fmaf(qv[2 * e], f.x, acc);
+          acc = fmaf(qv[2 * e + 1], f.y, acc);
+        }
+      }
       // reduce across the LPK lanes of this key row (a row's lanes share `valid`; the xor
       // offsets stay inside the group)
 #pragma unroll
@@ -363,11 +383,20 @@ __global__ void __launch_bounds__(NW * 32) attn_decode_kernel(const float* __res
         const float p = exp2f(acc - m_new);
         l = l * alpha + p;
         const uint32_t v4[4] = {vv[u].x, vv[u].y, vv[u].z, vv[u].w};
+        uint32_t vl4[4] = {0u, 0u, 0u, 0u};
+        if (RES) {
+          const uint4 vl = kv_res_lo8(vv[u], vc[u]);
+          vl4[0] = vl.x;
+          vl4[1] = vl.y;
+          vl4[2] = vl.z;
+          vl4[3] = vl.w;
+        }
 #pragma unroll
         for (int e = 0; e < 4; ++e) {
           const float2 f = unpack_f16x2(v4[e]);
-          o[2 * e] = fmaf(p, f.x, o[2 * e] * alpha);
-          o[2 * e + 1] = fmaf(p, f.y, o[2 * e + 1] * alpha);
+          const float2 fl = unpack_f16x2(vl4[e]);
+          o[2 * e] = fmaf(p, f.x + fl.x, o[2 * e] * alpha);
+          o[2 * e + 1] = fmaf(p, f.y + fl.y, o[2 * e + 1] * alpha);
         }
         m = m_new;
       }
@@ -483,12 +512,15 @@ int attn_decode_launch(const float* q, bf16* out_hi, bf16* out_lo, const RowInfo
   const int c = ((max_ctx + S - 1) / S + 15) / 16 * 16;
   const float scale_log2 = 1.4426950408889634f / sqrtf(static_cast<float>(hd));
   dim3 grid(S, H, B);
+  auto go = [&](auto kern) {
+    return launch_pdl(kern, grid, dim3(kDecodeWarps * 32), 0, stream, q, rows, kv, layer, H, c, S, scale_log2, part_o,
+                      part_ml, counters, out_hi, out_lo, fp16);
+  };
+  const bool res = kv.res != nullptr;
   if (hd == 128) {
-    VLA_CUDA_TRY(launch_pdl(attn_decode_kernel<128>, grid, dim3(kDecodeWarps * 32), 0, stream, q, rows, kv, layer, H,
-                            c, S, scale_log2, part_o, part_ml, counters, out_hi, out_lo, fp16));
+    VLA_CUDA_TRY(res ? go(attn_decode_kernel<128, true>) : go(attn_decode_kernel<128, false>));
   } else if (hd == 64) {
-    VLA_CUDA_TRY(launch_pdl(attn_decode_kernel<64>, grid, dim3(kDecodeWarps * 32), 0, stream, q, rows, kv, layer, H,
-                            c, S, scale_log2, part_o, part_ml, counters, out_hi, out_lo, fp16));
+    VLA_CUDA_TRY(res ? go(attn_decode_kernel<64, true>) : go(attn_decode_kernel<64, false>));
   } else {
     return VLA_ERR_UNSUPPORTED;
   }

@@ -1,7 +1,9 @@
 // Chunk causal attention on the tcgen05 tensor cores (paper §3.1: the policy's Llama-2
 // self-attention; §3.3: every chunk of a multi-turn trajectory attends to the whole context):
 // query tiles of up to 128 rows of one env (a prefill chunk, or the teacher-forced action rows
-// of the PPO ratio pass, Eq. 2) against keys 0..pos of that env, one CTA per (tile, head).
+// of the PPO ratio pass, Eq. 2) against keys 0..pos of that env.  Persistent: one CTA per SM
+// takes the (tile, head) items blockIdx.x, blockIdx.x + gridDim.x, ..., and every pipeline
+// (copies, conversions, MMAs, softmax, output) runs on across item boundaries.
 //
 // Precision: the cached keys / values are fp16 plus a 4-bit residual (KVLayout), read here as
 // the pair hi + lo; the queries (fp32) and the softmax weights are split into fp16 pairs too, and
@@ -9,23 +11,28 @@
 //   S = Q_hi K_hi^T + Q_lo K_hi^T + Q_hi K_lo^T,    O += P_hi V_hi + P_lo V_hi + P_hi V_lo.
 //
 // Roles (448 threads):
-//   warp 0      TMA producer: per 64-key block, K_hi and V_hi (tensor map over the whole cache,
-//               128-byte swizzle) and the two residual byte ranges (bulk copies), three stages;
-//   warp 1      TMEM owner (512 columns) and MMA issuer: S = Q K^T with Q read from TMEM (A
-//               operand) and K from shared memory (K-major B); O += P V with P from TMEM and V
-//               straight from the cache rows (keys x dims, the MN-major B operand); S is
-//               double-buffered, and the issuer takes whichever of "S of the next block" and
-//               "P V of the oldest pending block" is ready first;
-//   warps 2-5   softmax, one query row per thread (= its TMEM lane): write Q into TMEM, read each
-//               S block, online softmax in the exp2 domain with a lazily moved reference max (O
-//               and the row sum are rescaled only when the block max exceeds it by more than 8,
-//               so P <= 2^8), write P into TMEM, and finally O / l as the output pair;
-//   warps 6-13  converters: K_lo and V_lo from the hi parts and their residual codes, in the hi
-//               parts' own swizzled layout; values of keys past the last visible one are zeroed
-//               (their P is 0, and a stale NaN would still poison the product).
-// TMEM columns: S0 [0,64) S1 [64,128) O [128,128+HD) Q_hi [256,256+HD/2) Q_lo [256+HD/2,256+HD)
-// P_hi [384,416) P_lo [416,448).  Every wait is bounded; on a timeout the CTA records
-// VLA_STATUS_TIMEOUT, drains its copies and MMAs, frees TMEM and writes nothing.
+//   warp 0       TMA producer: per 64-key block, K_hi and V_hi (tensor map over the whole cache,
+//                128-byte swizzle) and the two residual byte ranges (bulk copies), three stages;
+//   warp 1       TMEM owner (512 columns) and MMA issuer: S = Q K^T with Q read from TMEM (A
+//                operand) and K from shared memory (K-major B); O += P V with P from TMEM and V
+//                straight from the cache rows (keys x dims, the MN-major B operand); it takes
+//                whichever of "S of the next block" and "P V of the oldest pending block" is
+//                ready first;
+//   warps 2-9    softmax, two warps per TMEM lane quarter (one query row per thread, each warp
+//                of the pair half of the block's 64 keys and half of O's columns; the pair
+//                exchanges row maxima and sums through shared memory): online softmax in the
+//                exp2 domain with a lazily moved reference max (O and the row sum are rescaled
+//                only when the block max exceeds it by more than 8, so P <= 2^8), P written over
+//                the S columns it came from; after an item's first block they write the previous
+//                item's O / l as the output operand pair;
+//   warps 10-13  workers: K_lo and V_lo from the hi parts and their residual codes, in the hi
+//                parts' own swizzled layout, values of keys past the last visible one zeroed
+//                (their P is 0, and a stale NaN would still poison the product); and each item's
+//                Q rows (times log2(e) / sqrt(hd)) as an fp16 pair into TMEM once the previous
+//                item's last S is done.
+// TMEM columns: S/P [0,64) [64,128); O [128,128+HD) [128+HD,128+2HD) (items alternate);
+// Q_hi [128+2HD,128+2.5HD) Q_lo [128+2.5HD,128+3HD).  Every wait is bounded; on a timeout the CTA
+// records VLA_STATUS_TIMEOUT, drains its copies and MMAs, frees TMEM and stops.
 #include <atomic>
 
 #include "attention.h"
@@ -38,11 +45,13 @@ namespace {
 
 constexpr int kAtWarps = 14;
 constexpr int kAtThreads = 32 * kAtWarps;
-constexpr int kConvWarps = kAtWarps - 6;
+constexpr int kSoftWarps = 8;   // warps 2..9
+constexpr int kWorkWarp0 = 10;  // warps 10..13
+constexpr int kWorkWarps = 4;
 constexpr int kStages = 3;
 constexpr int kKeys = 64;  // keys per block
 constexpr uint32_t kTmemCols = 512;
-constexpr uint32_t kColS = 0, kColO = 128, kColQ = 256, kColP = 384;
+constexpr uint32_t kColS = 0, kColO = 128;
 
 // Shared-memory matrix descriptor, 128-byte swizzle: atoms of 8 rows x 128 bytes, 1024 bytes
 // apart along the rows (SBO); for an MN-major operand the 64-element column blocks lie `lbo`
@@ -83,7 +92,6 @@ __device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t (&r)[16
 __device__ __forceinline__ void tmem_wait_st() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
 __device__ __forceinline__ void fence_async_smem() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
 
-__device__ __forceinline__ __half2 u32_h2(uint32_t v) { return *reinterpret_cast<__half2*>(&v); }
 __device__ __forceinline__ uint32_t h2_u32(__half2 v) { return *reinterpret_cast<uint32_t*>(&v); }
 // (a, b) -> fp16 pairs hi = fp16(x), lo = fp16(x - hi), with packed conversions.
 __device__ __forceinline__ void split_h2(float a, float b, uint32_t& hi, uint32_t& lo) {
@@ -92,22 +100,11 @@ __device__ __forceinline__ void split_h2(float a, float b, uint32_t& hi, uint32_
   hi = h2_u32(h);
   lo = h2_u32(__floats2half2_rn(a - f.x, b - f.y));
 }
-// Low parts of 8 cached fp16 values (one 16-byte chunk) from their 4-bit codes (4 bytes, element
-// 2i in the low nibble of byte i): per element (2c - 15) * 2^(e - 30), e the value's fp16 exponent
-// field, in fp16 arithmetic with no conversion instruction.  2c goes into the mantissa of 1024
-// (fp16 bits 0x6400 | 2c), so 1024 + 2c - 1039 = 2c - 15 exactly; 2^(e - 30) is the value with
-// mantissa and sign cleared (2^(e-15)) times 2^-15.  Exact for e >= 6; below that the term is
-// under 2^-21 in magnitude and comes out as zero or a rounded subnormal.
-__device__ __forceinline__ uint4 res_lo8(uint4 hi, uint32_t codes) {
-  const uint32_t twice_lo = (codes << 1) & 0x1E1E1E1Eu;  // 2c of each byte's low nibble
-  const uint32_t twice_hi = (codes >> 3) & 0x1E1E1E1Eu;  // 2c of each byte's high nibble
-  auto pair = [&](uint32_t h2, uint32_t sel) {
-    const uint32_t w = (__byte_perm(twice_lo, twice_hi, sel) & 0x00FF00FFu) | 0x64006400u;
-    const __half2 k = __hsub2(u32_h2(w), u32_h2(0x640F640Fu));                      // 2c - 15
-    const __half2 s = __hmul2(u32_h2(h2 & 0x7C007C00u), u32_h2(0x02000200u));       // 2^(e - 30)
-    return h2_u32(__hmul2(k, s));
-  };
-  return make_uint4(pair(hi.x, 0x0400u), pair(hi.y, 0x0501u), pair(hi.z, 0x0602u), pair(hi.w, 0x0703u));
+// 2^x (MUFU approximation, flush-to-zero; 2^-inf = 0)
+__device__ __forceinline__ float ex2(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
 }
 
 struct AtParams {
@@ -119,7 +116,8 @@ struct AtParams {
   int64_t layer_row0;      // first cache row (of HD elements) of this layer
   int64_t env_rows, kv_rows, head_rows;  // row strides: env, K->V, head (= cap)
   int cap, H;
-  float scale_log2;
+  int n_items;             // tiles x heads
+  float scale_log2;        // log2(e) / sqrt(HD), folded into the queries
   bool fp16;
   uint32_t* status;
   uint64_t wait_limit;
@@ -131,53 +129,85 @@ struct AtSmem {
   static constexpr int R_BYTES = kKeys * HD / 2;        // its residual codes
   // a stage: K_hi | V_hi | K_lo | V_lo | K codes | V codes (each tile 1024-byte aligned)
   static constexpr int STAGE = 4 * K_BYTES + 2 * R_BYTES;
-  static constexpr int SMEM = 1024 + kStages * STAGE + 256;
+  static constexpr int BARS = 256;                      // mbarriers, TMEM address, abort flag
+  // + the softmax pairs' exchange: row maxima [2 blocks][2 halves][128] and partial row sums
+  // [2 items][2 halves][128]
+  static constexpr int SMEM = 1024 + kStages * STAGE + BARS + 2 * (2 * 2 * 128 * 4);
   static_assert(STAGE % 1024 == 0, "stage alignment");
 };
+
+// The j-th item of this CTA: (tile, head) number blockIdx.x + j * gridDim.x, tile-major.
+struct Item {
+  AttnTile tile;
+  int head, n_keys, nb;
+  int64_t krow0;  // first K row of (env, head) in the cache
+};
+__device__ __forceinline__ Item get_item(const AtParams& p, int j) {
+  const int w = static_cast<int>(blockIdx.x) + j * static_cast<int>(gridDim.x);
+  Item it;
+  it.tile = p.tiles[w / p.H];
+  it.head = w % p.H;
+  it.n_keys = it.tile.pos0 + it.tile.nrows;
+  it.nb = (it.n_keys + kKeys - 1) / kKeys;
+  it.krow0 = p.layer_row0 + it.tile.env * p.env_rows + it.head * p.head_rows;
+  return it;
+}
+
+// Bounded wait by lane 0, the verdict shared by the warp.
+__device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, volatile int* abort_flag, uint32_t* status,
+                                          uint64_t limit) {
+  int ok = 1;
+  if ((threadIdx.x & 31) == 0) ok = wait_bounded(bar, parity, abort_flag, status, limit) ? 1 : 0;
+  return __shfl_sync(0xffffffffu, ok, 0) != 0;
+}
 
 template <int HD>
 __global__ void __launch_bounds__(kAtThreads, 1)
     attn_chunk_tc_kernel(const __grid_constant__ CUtensorMap tmKV, const AtParams p) {
   using Sm = AtSmem<HD>;
   constexpr int KB = HD / 64;  // 64-element column blocks of one K / V row
+  constexpr uint32_t kColQ = kColO + 2 * HD;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + kStages * Sm::STAGE);
-  // full[3] (loaded) conv[3] (low parts written) stfree[3] (the MMAs are done with the stage)
-  // sfull[2] sfree[2] pfull pdone qready drain
+  float* xbuf = reinterpret_cast<float*>(smem + kStages * Sm::STAGE + Sm::BARS);  // [2][2][128] row maxima
+  float* lbuf = xbuf + 2 * 2 * 128;                                                // [2][2][128] row sums
   const uint32_t b0 = smem_u32(bars);
   auto BAR = [&](int i) { return b0 + 8u * static_cast<uint32_t>(i); };
-  const uint32_t FULL = 0, CONV = 3, STFREE = 6, SFULL = 9, SFREE = 11, PFULL = 13, PDONE = 14, QREADY = 15,
-                 DRAIN = 16;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 17);
+  // per stage: full (loaded), conv (low parts written), stfree (MMAs done with it); per S/P
+  // buffer: sfull (S written), sfree (P V done with it), pfull (P written); pdone (the latest
+  // P V done); qready / qfree (Q written / the item's last S done); per item parity: odone (O
+  // final); drain; per lane quarter and block parity: xch (the softmax pair's exchange written)
+  const int FULL = 0, CONV = 3, STFREE = 6, SFULL = 9, SFREE = 11, PFULL = 13, PDONE = 15, QREADY = 16,
+            QFREE = 17, ODONE = 18, DRAIN = 20, XCH = 21;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 29);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   pdl_launch_dependents();
-  const AttnTile tile = p.tiles[blockIdx.x];
-  const int head = blockIdx.y;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int n_keys = tile.pos0 + tile.nrows;
-  const int nb = (n_keys + kKeys - 1) / kKeys;
-  const int64_t krow0 = p.layer_row0 + tile.env * p.env_rows + head * p.head_rows;  // K rows of (env, head)
-  const int64_t vrow0 = krow0 + p.kv_rows;
+  const int n_my = (p.n_items - static_cast<int>(blockIdx.x) + static_cast<int>(gridDim.x) - 1) /
+                   static_cast<int>(gridDim.x);
   uint32_t* status = p.status;
   const uint64_t limit = p.wait_limit;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
       mbar_init(BAR(FULL + s), 1);
-      mbar_init(BAR(CONV + s), kConvWarps);
+      mbar_init(BAR(CONV + s), kWorkWarps);
       mbar_init(BAR(STFREE + s), 1);
     }
     for (int s = 0; s < 2; ++s) {
       mbar_init(BAR(SFULL + s), 1);
-      mbar_init(BAR(SFREE + s), 4);
+      mbar_init(BAR(SFREE + s), 1);
+      mbar_init(BAR(PFULL + s), kSoftWarps);
+      mbar_init(BAR(ODONE + s), 1);
     }
-    mbar_init(BAR(PFULL), 4);
     mbar_init(BAR(PDONE), 1);
-    mbar_init(BAR(QREADY), 4);
+    mbar_init(BAR(QREADY), kWorkWarps);
+    mbar_init(BAR(QFREE), 1);
     mbar_init(BAR(DRAIN), 1);
+    for (int s = 0; s < 8; ++s) mbar_init(BAR(XCH + s), 2);
     *abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmKV)) : "memory");
@@ -198,26 +228,36 @@ __global__ void __launch_bounds__(kAtThreads, 1)
   if (warp == 0) {
     if (lane == 0) {
       // ------------------------------------------------------------------ producer
-      pdl_wait();  // the chunk's own keys / values were written by the q|k|v projection
+      pdl_wait();  // the chunks' own keys / values were written by the q|k|v projection
       uint32_t issued = 0, issued_phase = 0;
-      for (int b = 0; b < nb; ++b) {
-        const int st = b % kStages, round = b / kStages;
-        if (round >= 1 && !wait_bounded(BAR(STFREE + st), (round - 1) & 1, abort_flag, status, limit)) break;
-        const uint32_t s_khi = smem_u32(stage_ptr(st)), s_vhi = s_khi + Sm::K_BYTES;
-        const uint32_t s_kr = s_khi + 4 * Sm::K_BYTES, s_vr = s_kr + Sm::R_BYTES;
-        const int key0 = b * kKeys;
-        const int rows = min(kKeys, p.cap - key0);  // residual rows inside this (env, head)
-        const uint32_t rbytes = static_cast<uint32_t>(rows) * (HD / 2);
-        mbar_arrive_expect_tx(BAR(FULL + st), 2u * Sm::K_BYTES + 2u * rbytes);
+      bool ok = true;
+      int g = 0;  // block number over all of this CTA's items
+      for (int j = 0; j < n_my && ok; ++j) {
+        const Item it = get_item(p, j);
+        const int64_t vrow0 = it.krow0 + p.kv_rows;
+        for (int b = 0; b < it.nb; ++b, ++g) {
+          const int st = g % kStages, round = g / kStages;
+          if (round >= 1 && !wait_bounded(BAR(STFREE + st), (round - 1) & 1, abort_flag, status, limit)) {
+            ok = false;
+            break;
+          }
+          const uint32_t s_khi = smem_u32(stage_ptr(st)), s_vhi = s_khi + Sm::K_BYTES;
+          const uint32_t s_kr = s_khi + 4 * Sm::K_BYTES, s_vr = s_kr + Sm::R_BYTES;
+          const int key0 = b * kKeys;
+          const int rows = min(kKeys, p.cap - key0);  // residual rows inside this (env, head)
+          const uint32_t rbytes = static_cast<uint32_t>(rows) * (HD / 2);
+          mbar_arrive_expect_tx(BAR(FULL + st), 2u * Sm::K_BYTES + 2u * rbytes);
 #pragma unroll
-        for (int kb = 0; kb < KB; ++kb) {
-          tma_load_2d(s_khi + kb * (kKeys * 128), &tmKV, BAR(FULL + st), kb * 64, static_cast<int>(krow0 + key0));
-          tma_load_2d(s_vhi + kb * (kKeys * 128), &tmKV, BAR(FULL + st), kb * 64, static_cast<int>(vrow0 + key0));
+          for (int kb = 0; kb < KB; ++kb) {
+            tma_load_2d(s_khi + kb * (kKeys * 128), &tmKV, BAR(FULL + st), kb * 64,
+                        static_cast<int>(it.krow0 + key0));
+            tma_load_2d(s_vhi + kb * (kKeys * 128), &tmKV, BAR(FULL + st), kb * 64, static_cast<int>(vrow0 + key0));
+          }
+          bulk_load(s_kr, p.res + (it.krow0 + key0) * (HD / 2), rbytes, BAR(FULL + st));
+          bulk_load(s_vr, p.res + (vrow0 + key0) * (HD / 2), rbytes, BAR(FULL + st));
+          issued |= 1u << st;
+          issued_phase = (issued_phase & ~(1u << st)) | (static_cast<uint32_t>(round & 1) << st);
         }
-        bulk_load(s_kr, p.res + (krow0 + key0) * (HD / 2), rbytes, BAR(FULL + st));
-        bulk_load(s_vr, p.res + (vrow0 + key0) * (HD / 2), rbytes, BAR(FULL + st));
-        issued |= 1u << st;
-        issued_phase = (issued_phase & ~(1u << st)) | (static_cast<uint32_t>(round & 1) << st);
       }
       for (int st = 0; st < kStages; ++st)
         if (issued & (1u << st)) wait_drain(BAR(FULL + st), (issued_phase >> st) & 1u, limit);
@@ -226,47 +266,66 @@ __global__ void __launch_bounds__(kAtThreads, 1)
     if (lane == 0) {
       // ------------------------------------------------------------------ MMA issuer
       const uint32_t IS = idesc_f16(kKeys), IO = idesc_f16(HD, true);
-      const uint32_t tS0 = tmem + kColS, tO = tmem + kColO;
       const uint32_t tQh = tmem + kColQ, tQl = tmem + kColQ + HD / 2;
-      const uint32_t tPh = tmem + kColP, tPl = tmem + kColP + kKeys / 2;
-      bool ok = wait_bounded(BAR(QREADY), 0, abort_flag, status, limit);
-      int bs = 0, bo = 0;  // next block whose S, whose P V is to be issued
+      // descriptors of stage 0's tiles; another stage (or k step) adds its byte offset / 16
+      const uint64_t dK0 = sdesc_sw128(smem_u32(stage_ptr(0)));
+      const uint64_t dV0 = sdesc_sw128(smem_u32(stage_ptr(0)) + Sm::K_BYTES, kKeys * 128);
+      constexpr uint64_t kStageStep = Sm::STAGE >> 4, kLoStep = (2 * Sm::K_BYTES) >> 4;
+      bool ok = true;
+      // S cursor (item js, block bs, global block gs) and P V cursor (jo, bo, go)
+      int js = 0, bs = 0, gs = 0, nbs = get_item(p, 0).nb;
+      int jo = 0, bo = 0, go = 0, nbo = nbs;
       uint64_t t_last = globaltimer();
       uint32_t spins = 0;
-      while (ok && bo < nb) {
-        if (bo < bs && mbar_test_wait(BAR(PFULL), bo & 1)) {
-          // O += P V of block bo; the commit frees its stage and hands O / P back to the softmax
+      while (ok && jo < n_my) {
+        bool did = false;
+        if (go < gs && mbar_test_wait(BAR(PFULL + (go & 1)), (go >> 1) & 1)) {
+          // O(jo) (+)= P V of block go
           tc_fence_after();
-          const uint32_t s_vhi = smem_u32(stage_ptr(bo % kStages)) + Sm::K_BYTES;
-          const uint32_t s_vlo = s_vhi + 2 * Sm::K_BYTES;
+          const uint64_t dvh = dV0 + (go % kStages) * kStageStep;
+          const uint32_t tO = tmem + kColO + (jo & 1) * HD;
+          const uint32_t tPh = tmem + kColS + (go & 1) * kKeys, tPl = tPh + kKeys / 2;
 #pragma unroll
           for (int k = 0; k < kKeys / 16; ++k) {
-            const uint64_t dh = sdesc_sw128(s_vhi + k * 2048, kKeys * 128);
-            const uint64_t dl = sdesc_sw128(s_vlo + k * 2048, kKeys * 128);
+            const uint64_t dh = dvh + k * (2048 >> 4), dl = dh + kLoStep;
             mma_ts(tO, tPh + k * 8, dh, IO, (bo > 0 || k > 0) ? 1u : 0u);
             mma_ts(tO, tPl + k * 8, dh, IO, 1u);
             mma_ts(tO, tPh + k * 8, dl, IO, 1u);
           }
           tc_commit(BAR(PDONE));
-          tc_commit(BAR(STFREE + bo % kStages));
-          ++bo;
-          t_last = globaltimer();
-        } else if (bs < nb && mbar_test_wait(BAR(CONV + bs % kStages), (bs / kStages) & 1) &&
-                   (bs < 2 || mbar_test_wait(BAR(SFREE + (bs & 1)), ((bs >> 1) - 1) & 1))) {
-          // S of block bs into buffer bs & 1
+          tc_commit(BAR(SFREE + (go & 1)));
+          tc_commit(BAR(STFREE + go % kStages));
+          if (bo == nbo - 1) tc_commit(BAR(ODONE + (jo & 1)));
+          ++go;
+          if (++bo == nbo) {
+            bo = 0;
+            if (++jo < n_my) nbo = get_item(p, jo).nb;
+          }
+          did = true;
+        } else if (js < n_my && mbar_test_wait(BAR(CONV + gs % kStages), (gs / kStages) & 1) &&
+                   (gs < 2 || mbar_test_wait(BAR(SFREE + (gs & 1)), ((gs >> 1) - 1) & 1)) &&
+                   (bs > 0 || mbar_test_wait(BAR(QREADY), js & 1))) {
+          // S of block gs into buffer gs & 1
           tc_fence_after();
-          const uint32_t s_khi = smem_u32(stage_ptr(bs % kStages)), s_klo = s_khi + 2 * Sm::K_BYTES;
-          const uint32_t tS = tS0 + (bs & 1) * kKeys;
+          const uint64_t dkh = dK0 + (gs % kStages) * kStageStep;
+          const uint32_t tS = tmem + kColS + (gs & 1) * kKeys;
 #pragma unroll
           for (int k = 0; k < HD / 16; ++k) {
-            const uint32_t off = (k >> 2) * (kKeys * 128) + (k & 3) * 32;
-            const uint64_t dh = sdesc_sw128(s_khi + off), dl = sdesc_sw128(s_klo + off);
+            const uint64_t dh = dkh + (((k >> 2) * (kKeys * 128) + (k & 3) * 32) >> 4), dl = dh + kLoStep;
             mma_ts(tS, tQh + k * 8, dh, IS, k > 0 ? 1u : 0u);
             mma_ts(tS, tQl + k * 8, dh, IS, 1u);
             mma_ts(tS, tQh + k * 8, dl, IS, 1u);
           }
-          tc_commit(BAR(SFULL + (bs & 1)));
-          ++bs;
+          tc_commit(BAR(SFULL + (gs & 1)));
+          if (bs == nbs - 1) tc_commit(BAR(QFREE));
+          ++gs;
+          if (++bs == nbs) {
+            bs = 0;
+            if (++js < n_my) nbs = get_item(p, js).nb;
+          }
+          did = true;
+        }
+        if (did) {
           t_last = globaltimer();
         } else if (((++spins) & 63u) == 0) {
           if (*abort_flag) {
@@ -281,18 +340,174 @@ __global__ void __launch_bounds__(kAtThreads, 1)
       tc_commit(BAR(DRAIN));
       wait_drain(BAR(DRAIN), 0, limit);
     }
-  } else if (warp < 6) {
-    // ------------------------------------------------------------------ softmax (row per thread)
+  } else if (warp < kWorkWarp0) {
+    // ------------------------------------------------------------------ softmax (warps 2-9)
     const int q4 = warp & 3;                 // TMEM lane quarter of this warp
+    const int hf = (warp - 2) >> 2;          // which 32 keys of a block, and which half of O's columns
     const int r = q4 * 32 + lane;            // query row in the tile
-    const bool valid = r < tile.nrows;
-    const int qpos = tile.pos0 + min(r, tile.nrows - 1);
     const uint32_t lane_off = static_cast<uint32_t>(q4 * 32) << 16;
     const int dcols = p.H * HD;
-    pdl_wait();
-    // Q row -> fp16 pair in TMEM (A operand of S)
-    {
-      const float* qrow = p.q + static_cast<size_t>(tile.row0 + (valid ? r : 0)) * dcols + head * HD;
+    uint32_t sat = 0;  // convex combinations of the cached values: the fp16 split never saturates
+    pdl_wait();        // the output may still be read by the previous kernel's predecessors
+    // item jp's output, O / l as the operand pair: this warp's rows, its half of the columns
+    auto epilogue = [&](int jp, float l_tot) -> bool {
+      if (!warp_wait(BAR(ODONE + (jp & 1)), (jp >> 1) & 1, abort_flag, status, limit)) return false;
+      tc_fence_after();
+      const Item it = get_item(p, jp);
+      const bool valid = r < it.tile.nrows;
+      const float inv = 1.f / l_tot;
+      const size_t off = static_cast<size_t>(it.tile.row0 + (valid ? r : 0)) * dcols + it.head * HD + hf * (HD / 2);
+      const uint32_t tO = tmem + lane_off + kColO + (jp & 1) * HD + hf * (HD / 2);
+#pragma unroll 1
+      for (int c = 0; c < HD / 2; c += 16) {
+        uint32_t v[16];
+        tmem_ld16(tO + c, v);
+        tmem_wait_ld();
+        if (valid) {
+          uint32_t h[8], lo[8];
+#pragma unroll
+          for (int i = 0; i < 8; ++i)
+            split_pack2(__uint_as_float(v[2 * i]) * inv, __uint_as_float(v[2 * i + 1]) * inv, h[i], lo[i], p.fp16,
+                        sat);
+          uint4* dh = reinterpret_cast<uint4*>(p.out_hi + off + c);
+          uint4* dl = reinterpret_cast<uint4*>(p.out_lo + off + c);
+          dh[0] = make_uint4(h[0], h[1], h[2], h[3]);
+          dh[1] = make_uint4(h[4], h[5], h[6], h[7]);
+          dl[0] = make_uint4(lo[0], lo[1], lo[2], lo[3]);
+          dl[1] = make_uint4(lo[4], lo[5], lo[6], lo[7]);
+        }
+      }
+      return true;
+    };
+    // the pair's exchange at block g: this warp's value in, the partner's out
+    auto exchange = [&](float* buf, int g, float v, float& other) -> bool {
+      buf[hf * 128 + r] = v;
+      __syncwarp();
+      if (lane == 0) mbar_arrive(BAR(XCH + 2 * q4 + (g & 1)));
+      if (!warp_wait(BAR(XCH + 2 * q4 + (g & 1)), (g >> 1) & 1, abort_flag, status, limit)) return false;
+      other = buf[(hf ^ 1) * 128 + r];
+      return true;
+    };
+    bool ok = true;
+    int g = 0;
+    float l_prev = 0.f;  // the previous item's partial row sum (this warp's keys)
+    for (int j = 0; j < n_my && ok; ++j) {
+      const Item it = get_item(p, j);
+      const int qpos = it.tile.pos0 + min(r, it.tile.nrows - 1);
+      const uint32_t tO = tmem + lane_off + kColO + (j & 1) * HD + hf * (HD / 2);
+      float m_ref = -INFINITY, l = 0.f;
+      for (int b = 0; b < it.nb; ++b, ++g) {
+        if (!warp_wait(BAR(SFULL + (g & 1)), (g >> 1) & 1, abort_flag, status, limit)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t tS = tmem + lane_off + kColS + (g & 1) * kKeys;
+        float s[32];
+        {
+          uint32_t v0[16], v1[16];
+          tmem_ld16(tS + hf * 32, v0);
+          tmem_ld16(tS + hf * 32 + 16, v1);
+          tmem_wait_ld();
+#pragma unroll
+          for (int i = 0; i < 16; ++i) {
+            s[i] = __uint_as_float(v0[i]);
+            s[16 + i] = __uint_as_float(v1[i]);
+          }
+        }
+        const int key0 = b * kKeys + hf * 32;
+        if (__any_sync(0xffffffffu, key0 + 31 > qpos)) {
+#pragma unroll
+          for (int c = 0; c < 32; ++c) s[c] = (key0 + c <= qpos) ? s[c] : -INFINITY;
+        }
+        float mb = s[0];
+#pragma unroll
+        for (int c = 1; c < 32; ++c) mb = fmaxf(mb, s[c]);
+        // the pair's block maximum of row r (past the exchange both warps have read their S
+        // columns, so P may overwrite them); an item's first block also carries the previous
+        // item's partial row sums
+        if (b == 0 && j > 0) lbuf[((j - 1) & 1) * 256 + hf * 128 + r] = l_prev;
+        float mo;
+        if (!exchange(xbuf + (g & 1) * 256, g, mb, mo)) {
+          ok = false;
+          break;
+        }
+        mb = fmaxf(mb, mo);
+        float alpha = 1.f;
+        if (mb > m_ref + 8.f) {
+          // first block (m_ref = -inf) or a max well above the reference: move it
+          alpha = ex2(m_ref - mb);  // 0 on the first block
+          m_ref = mb;
+          l *= alpha;
+        }
+        if (b >= 1 && __any_sync(0xffffffffu, alpha != 1.f)) {
+          // O is the MMAs' until the previous block's P V is done
+          if (!warp_wait(BAR(PDONE), (g - 1) & 1, abort_flag, status, limit)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+#pragma unroll 1
+          for (int c = 0; c < HD / 2; c += 16) {
+            uint32_t v[16];
+            tmem_ld16(tO + c, v);
+            tmem_wait_ld();
+#pragma unroll
+            for (int i = 0; i < 16; ++i) v[i] = __float_as_uint(__uint_as_float(v[i]) * alpha);
+            tmem_st16(tO + c, v);
+          }
+        }
+        // P over the S columns: hi of keys 2c, 2c + 1 in column c, lo 32 columns further
+        {
+          uint32_t hi[16], lo[16];
+          float ps = 0.f;
+#pragma unroll
+          for (int i = 0; i < 16; ++i) {
+            const float p0 = ex2(s[2 * i] - m_ref), p1 = ex2(s[2 * i + 1] - m_ref);
+            ps += p0 + p1;
+            split_h2(p0, p1, hi[i], lo[i]);
+          }
+          l += ps;
+          tmem_st16(tS + hf * 16, hi);
+          tmem_st16(tS + kKeys / 2 + hf * 16, lo);
+        }
+        tmem_wait_st();
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(BAR(PFULL + (g & 1)));
+        if (b == 0 && j > 0) {
+          const float l_tot = l_prev + lbuf[((j - 1) & 1) * 256 + (hf ^ 1) * 128 + r];
+          if (!epilogue(j - 1, l_tot)) {
+            ok = false;
+            break;
+          }
+        }
+      }
+      l_prev = l;
+    }
+    if (ok) {
+      // the last item: its row sums through one more exchange, then its output
+      const int j = n_my - 1;
+      float lo_sum;
+      if (exchange(lbuf + (j & 1) * 256, g, l_prev, lo_sum)) epilogue(j, l_prev + lo_sum);
+    }
+    report_saturation(status, sat);
+  } else {
+    // ------------------------------------------------------------------ workers (warps 10-13)
+    const int q4 = warp & 3;
+    const int r = q4 * 32 + lane;            // Q row written by this thread (its TMEM lane)
+    const uint32_t lane_off = static_cast<uint32_t>(q4 * 32) << 16;
+    const int t = threadIdx.x - kWorkWarp0 * 32;
+    const int dcols = p.H * HD;
+    constexpr int CH = HD / 8;                                 // 16-byte chunks of one row
+    constexpr int ITER = 2 * kKeys * CH / (32 * kWorkWarps);   // chunks per thread and block
+    constexpr int KSTEP = 32 * kWorkWarps / CH;                // rows between a thread's chunks
+    static_assert((32 * kWorkWarps) % CH == 0 && ITER % 2 == 0, "converter tiling");
+    pdl_wait();  // the queries were written by the q|k|v projection
+    // Q rows of an item, times log2(e) / sqrt(HD), -> fp16 pair in TMEM (A operand of S)
+    auto write_q = [&](const Item& it) {
+      const bool valid = r < it.tile.nrows;
+      const float* qrow = p.q + static_cast<size_t>(it.tile.row0 + (valid ? r : 0)) * dcols + it.head * HD;
 #pragma unroll 1
       for (int c = 0; c < HD; c += 64) {
         float4 x[16];  // 64 values in flight
@@ -305,8 +520,8 @@ __global__ void __launch_bounds__(kAtThreads, 1)
 #pragma unroll
           for (int i = 0; i < 8; ++i) {
             const float4 v = x[half * 8 + i];
-            split_h2(v.x, v.y, hi[2 * i], lo[2 * i]);
-            split_h2(v.z, v.w, hi[2 * i + 1], lo[2 * i + 1]);
+            split_h2(v.x * p.scale_log2, v.y * p.scale_log2, hi[2 * i], lo[2 * i]);
+            split_h2(v.z * p.scale_log2, v.w * p.scale_log2, hi[2 * i + 1], lo[2 * i + 1]);
           }
           tmem_st16(tmem + lane_off + kColQ + (c + 32 * half) / 2, hi);
           tmem_st16(tmem + lane_off + kColQ + HD / 2 + (c + 32 * half) / 2, lo);
@@ -316,144 +531,66 @@ __global__ void __launch_bounds__(kAtThreads, 1)
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(BAR(QREADY));
-    }
-    float m_ref = -INFINITY, l = 0.f;
+    };
+    auto prefetch_q = [&](const Item& it) {
+      if (r < it.tile.nrows) {
+        const float* qrow = p.q + static_cast<size_t>(it.tile.row0 + r) * dcols + it.head * HD;
+#pragma unroll
+        for (int c = 0; c < HD; c += 32) asm volatile("prefetch.global.L2 [%0];" ::"l"(qrow + c));
+      }
+    };
     bool ok = true;
-    for (int b = 0; b < nb && ok; ++b) {
-      const int st = b & 1;
-      int w_ok = 1;
-      if (lane == 0) w_ok = wait_bounded(BAR(SFULL + st), (b >> 1) & 1, abort_flag, status, limit) ? 1 : 0;
-      if (!__shfl_sync(0xffffffffu, w_ok, 0)) {
-        ok = false;
-        break;
-      }
-      tc_fence_after();
-      float s[kKeys];
-#pragma unroll
-      for (int c = 0; c < kKeys; c += 16) {
-        uint32_t v[16];
-        tmem_ld16(tmem + lane_off + kColS + st * kKeys + c, v);
-        tmem_wait_ld();
-#pragma unroll
-        for (int i = 0; i < 16; ++i) s[c + i] = __uint_as_float(v[i]);
-      }
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(BAR(SFREE + st));
-      const int key0 = b * kKeys;
-      float mb = -INFINITY;
-#pragma unroll
-      for (int c = 0; c < kKeys; ++c) {
-        s[c] = (key0 + c <= qpos) ? s[c] * p.scale_log2 : -INFINITY;
-        mb = fmaxf(mb, s[c]);
-      }
-      // O and P are the MMA's until block b-1's products are done
-      if (b >= 1) {
-        if (lane == 0) w_ok = wait_bounded(BAR(PDONE), (b - 1) & 1, abort_flag, status, limit) ? 1 : 0;
-        if (!__shfl_sync(0xffffffffu, w_ok, 0)) {
+    int g = 0;
+    for (int j = 0; j < n_my && ok; ++j) {
+      const Item it = get_item(p, j);
+      for (int b = 0; b < it.nb; ++b, ++g) {
+        const int st = g % kStages;
+        if (!warp_wait(BAR(FULL + st), (g / kStages) & 1, abort_flag, status, limit)) {
           ok = false;
           break;
         }
-        tc_fence_after();
-      }
-      float alpha = 1.f;
-      if (mb > m_ref + 8.f) {
-        // first block (m_ref = -inf) or a max well above the reference: move it
-        alpha = exp2f(m_ref - mb);  // 0 on the first block
-        m_ref = mb;
-        l *= alpha;
-      }
-      if (b >= 1 && __any_sync(0xffffffffu, alpha != 1.f)) {
-#pragma unroll 1
-        for (int c = 0; c < HD; c += 16) {
-          uint32_t v[16];
-          tmem_ld16(tmem + lane_off + kColO + c, v);
-          tmem_wait_ld();
+        // K_lo, V_lo: a thread's chunks all sit in one column c (the stride over chunks is a
+        // multiple of CH), rows key0t, key0t + KSTEP, ...: loads first, then decode and stores
+        uint8_t* sp = stage_ptr(st);
+        const int live = it.n_keys - b * kKeys;  // keys of this block visible to some row
+        const int c = t % CH, key0t = t / CH;
+        const int coff = (c >> 3) * (kKeys * 128) + key0t * 128 + (((c & 7) ^ (key0t & 7)) << 4);
+        uint4 hv[ITER];
+        uint32_t cv[ITER];
 #pragma unroll
-          for (int i = 0; i < 16; ++i) v[i] = __float_as_uint(__uint_as_float(v[i]) * alpha);
-          tmem_st16(tmem + lane_off + kColO + c, v);
+        for (int i = 0; i < ITER; ++i) {
+          const int w = i / (ITER / 2), key = key0t + (i % (ITER / 2)) * KSTEP;
+          hv[i] = *reinterpret_cast<const uint4*>(sp + w * Sm::K_BYTES + coff + (i % (ITER / 2)) * KSTEP * 128);
+          cv[i] = *reinterpret_cast<const uint32_t*>(sp + 4 * Sm::K_BYTES + w * Sm::R_BYTES + key * (HD / 2) + c * 4);
         }
-      }
-      float ps = 0.f;
 #pragma unroll
-      for (int c = 0; c < kKeys; c += 32) {
-        uint32_t hi[16], lo[16];
-#pragma unroll
-        for (int i = 0; i < 16; ++i) {
-          const float p0 = exp2f(s[c + 2 * i] - m_ref), p1 = exp2f(s[c + 2 * i + 1] - m_ref);
-          ps += p0 + p1;
-          split_h2(p0, p1, hi[i], lo[i]);
-        }
-        tmem_st16(tmem + lane_off + kColP + c / 2, hi);
-        tmem_st16(tmem + lane_off + kColP + kKeys / 2 + c / 2, lo);
-      }
-      l += ps;
-      tmem_wait_st();
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(BAR(PFULL));
-    }
-    if (ok && nb > 0) {
-      int w_ok = 1;
-      if (lane == 0) w_ok = wait_bounded(BAR(PDONE), (nb - 1) & 1, abort_flag, status, limit) ? 1 : 0;
-      if (__shfl_sync(0xffffffffu, w_ok, 0)) {
-        tc_fence_after();
-        const float inv = 1.f / l;
-        const size_t off = static_cast<size_t>(tile.row0 + (valid ? r : 0)) * dcols + head * HD;
-        uint32_t sat = 0;  // convex combinations of the cached values: the fp16 split never saturates
-#pragma unroll 1
-        for (int c = 0; c < HD; c += 16) {
-          uint32_t v[16];
-          tmem_ld16(tmem + lane_off + kColO + c, v);
-          tmem_wait_ld();
-          if (valid) {
-            uint32_t h[8], lo[8];
-#pragma unroll
-            for (int i = 0; i < 8; ++i)
-              split_pack2(__uint_as_float(v[2 * i]) * inv, __uint_as_float(v[2 * i + 1]) * inv, h[i], lo[i], p.fp16,
-                          sat);
-            uint4* dh = reinterpret_cast<uint4*>(p.out_hi + off + c);
-            uint4* dl = reinterpret_cast<uint4*>(p.out_lo + off + c);
-            dh[0] = make_uint4(h[0], h[1], h[2], h[3]);
-            dh[1] = make_uint4(h[4], h[5], h[6], h[7]);
-            dl[0] = make_uint4(lo[0], lo[1], lo[2], lo[3]);
-            dl[1] = make_uint4(lo[4], lo[5], lo[6], lo[7]);
+        for (int i = 0; i < ITER; ++i) {
+          const int w = i / (ITER / 2), key = key0t + (i % (ITER / 2)) * KSTEP;
+          const int off = coff + (i % (ITER / 2)) * KSTEP * 128;
+          uint4* lo = reinterpret_cast<uint4*>(sp + (2 + w) * Sm::K_BYTES + off);
+          if (w == 1 && key >= live) {
+            *reinterpret_cast<uint4*>(sp + Sm::K_BYTES + off) = make_uint4(0u, 0u, 0u, 0u);
+            *lo = make_uint4(0u, 0u, 0u, 0u);
+          } else {
+            *lo = kv_res_lo8(hv[i], cv[i]);
           }
         }
-      }
-    }
-  } else {
-    // ------------------------------------------------------------------ converters (warps 6-13)
-    const int t = threadIdx.x - 6 * 32;
-    constexpr int CH = HD / 8;  // 16-byte chunks of one row
-    for (int b = 0; b < nb; ++b) {
-      const int st = b % kStages;
-      int w_ok = 1;
-      if (lane == 0) w_ok = wait_bounded(BAR(FULL + st), (b / kStages) & 1, abort_flag, status, limit) ? 1 : 0;
-      if (!__shfl_sync(0xffffffffu, w_ok, 0)) break;
-      uint8_t* sp = stage_ptr(st);
-      const int live = n_keys - b * kKeys;  // keys of this block visible to some row
-      // chunk index fastest over lanes: 8 lanes read one swizzled 128-byte row, a warp reads 128
-      // consecutive code bytes
-#pragma unroll 2
-      for (int ch = t; ch < 2 * kKeys * CH; ch += 32 * kConvWarps) {
-        const int w = ch / (kKeys * CH);  // 0: K, 1: V
-        const int c = ch % CH, key = (ch / CH) % kKeys;
-        const int off = (c >> 3) * (kKeys * 128) + key * 128 + (((c & 7) ^ (key & 7)) << 4);
-        uint4* hi = reinterpret_cast<uint4*>(sp + w * Sm::K_BYTES + off);
-        uint4* lo = reinterpret_cast<uint4*>(sp + (2 + w) * Sm::K_BYTES + off);
-        if (w == 1 && key >= live) {
-          *hi = make_uint4(0u, 0u, 0u, 0u);
-          *lo = make_uint4(0u, 0u, 0u, 0u);
-        } else {
-          const uint32_t codes =
-              *reinterpret_cast<const uint32_t*>(sp + 4 * Sm::K_BYTES + w * Sm::R_BYTES + key * (HD / 2) + c * 4);
-          *lo = res_lo8(*hi, codes);
+        fence_async_smem();  // the MMAs (async proxy) read what these generic stores wrote
+        __syncwarp();
+        if (lane == 0) mbar_arrive(BAR(CONV + st));
+        if (b == 0) {
+          // this item's queries, once the previous item's last S is done
+          if (j > 0) {
+            if (!warp_wait(BAR(QFREE), (j - 1) & 1, abort_flag, status, limit)) {
+              ok = false;
+              break;
+            }
+            tc_fence_after();
+          }
+          write_q(it);
+          if (j + 1 < n_my) prefetch_q(get_item(p, j + 1));
         }
       }
-      fence_async_smem();  // the MMAs (async proxy) read what these generic stores wrote
-      __syncwarp();
-      if (lane == 0) mbar_arrive(BAR(CONV + st));
     }
   }
 
@@ -469,9 +606,10 @@ __global__ void __launch_bounds__(kAtThreads, 1)
 }  // namespace
 
 int attn_chunk_tc_launch(const float* q, bf16* out_hi, bf16* out_lo, const AttnTile* tiles, int n_tiles,
-                         KVLayout kv, int layer, int H, int hd, uint32_t* status, cudaStream_t stream, bool fp16) {
+                         KVLayout kv, int layer, int H, int hd, uint32_t* status, cudaStream_t stream, bool fp16,
+                         int num_sms) {
   if (n_tiles <= 0) return VLA_OK;
-  if (!kv.res || (hd != 64 && hd != 128)) return VLA_ERR_UNSUPPORTED;
+  if (!kv.res || (hd != 64 && hd != 128) || num_sms <= 0) return VLA_ERR_UNSUPPORTED;
   if ((reinterpret_cast<uintptr_t>(kv.base) & 15) || (reinterpret_cast<uintptr_t>(kv.res) & 15))
     return VLA_ERR_ARG;
   AtParams p{};
@@ -487,6 +625,7 @@ int attn_chunk_tc_launch(const float* q, bf16* out_hi, bf16* out_lo, const AttnT
   p.layer_row0 = static_cast<int64_t>(layer) * (kv.layer_stride / hd);
   p.cap = kv.cap;
   p.H = H;
+  p.n_items = n_tiles * H;
   p.scale_log2 = 1.4426950408889634f / sqrtf(static_cast<float>(hd));
   p.fp16 = fp16;
   p.status = status;
@@ -498,7 +637,8 @@ int attn_chunk_tc_launch(const float* q, bf16* out_hi, bf16* out_lo, const AttnT
   CUtensorMap map;
   if (!make_tensor_map_2d(&map, kv.base, total_rows, hd, hd, kKeys, true))
     return cuda_fail(cudaErrorInvalidValue, "tensor map (KV cache)");
-  dim3 grid(n_tiles, H);
+  // persistent: one CTA per SM (each holds ~220 KB of shared memory and all 512 TMEM columns)
+  const dim3 grid(std::min(p.n_items, num_sms));
   if (hd == 128) {
     static std::atomic<uint64_t> attr_done{0};
     VLA_CUDA_TRY(set_smem_limit(attn_chunk_tc_kernel<128>, AtSmem<128>::SMEM, attr_done));

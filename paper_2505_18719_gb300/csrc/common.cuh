@@ -55,20 +55,27 @@ __device__ __forceinline__ uint32_t kv_res_code(float x, f16 hi) {
   j = fminf(fmaxf(j, -8.f), 7.f);  // a NaN lands on -8: its value is NaN through hi anyway
   return static_cast<uint32_t>(static_cast<int>(j) + 8);
 }
-__device__ __forceinline__ float kv_res_value(f16 hi, uint32_t c) {
-  const uint32_t e = (__half_as_ushort(hi) >> 10) & 31u;
-  const uint32_t ee = e ? e : 1u;
-  return __half2float(hi) + static_cast<float>(2 * static_cast<int>(c) - 15) * __uint_as_float((ee + 97u) << 23);
+// Low parts of 8 cached fp16 values (one 16-byte chunk) from their 4-bit codes (4 bytes, element
+// 2i in the low nibble of byte i): per element (2c - 15) * 2^(e - 30) = (2c - 15) ulp(hi) / 32, e
+// the value's fp16 exponent field, in fp16 arithmetic with no conversion instruction.  2c goes
+// into the mantissa of 1024 (fp16 bits 0x6400 | 2c), so 1024 + 2c - 1039 = 2c - 15 exactly;
+// 2^(e - 30) is the value with mantissa and sign cleared (2^(e-15)) times 2^-15.  Exact for
+// e >= 6; below that the term is under 2^-21 in magnitude and comes out as zero or a rounded
+// subnormal.
+__device__ __forceinline__ uint4 kv_res_lo8(uint4 hi, uint32_t codes) {
+  const uint32_t twice_lo = (codes << 1) & 0x1E1E1E1Eu;  // 2c of each byte's low nibble
+  const uint32_t twice_hi = (codes >> 3) & 0x1E1E1E1Eu;  // 2c of each byte's high nibble
+  auto pair = [&](uint32_t h2, uint32_t sel) {
+    uint32_t w = (__byte_perm(twice_lo, twice_hi, sel) & 0x00FF00FFu) | 0x64006400u;
+    uint32_t e = h2 & 0x7C007C00u;
+    const uint32_t c1039 = 0x640F640Fu, c2m15 = 0x02000200u;
+    const __half2 k = __hsub2(*reinterpret_cast<const __half2*>(&w), *reinterpret_cast<const __half2*>(&c1039));
+    const __half2 sc = __hmul2(*reinterpret_cast<const __half2*>(&e), *reinterpret_cast<const __half2*>(&c2m15));
+    const __half2 r = __hmul2(k, sc);
+    return *reinterpret_cast<const uint32_t*>(&r);
+  };
+  return make_uint4(pair(hi.x, 0x0400u), pair(hi.y, 0x0501u), pair(hi.z, 0x0602u), pair(hi.w, 0x0703u));
 }
-// Residual value alone, (2c - 15) ulp(hi) / 32, rounded to fp16 (the MMA operand of the low part).
-__device__ __forceinline__ f16 kv_res_lo(f16 hi, uint32_t c) {
-  const uint32_t e = (__half_as_ushort(hi) >> 10) & 31u;
-  const uint32_t ee = e ? e : 1u;
-  return __float2half_rn(static_cast<float>(2 * static_cast<int>(c) - 15) * __uint_as_float((ee + 97u) << 23));
-}
-// Stores x as fp16 at dst[i] and its code into the residual plane (for an even/odd pair, the
-// caller combines two codes into one byte).
-__device__ __forceinline__ f16 kv_hi(float x) { return __float2half_rn(x); }
 
 // ----------------------------------------------------------------------------- bf16 helpers
 __device__ __forceinline__ float bf2f(bf16 x) { return __bfloat162float(x); }

@@ -407,7 +407,7 @@ int forward_layers(vla_handle* h, int M, const RowInfo* rows_dev, bool decode, i
     } else {
       ev = prof_begin(h, VLA_KCLASS_ATTN_PREFILL);
       rc = attn_chunk_tc_launch(h->q, h->ao, h->ao + pd, h->tiles, n_tiles, h->kvl, l, H, hd, h->status, h->stream,
-                                h->fp16);
+                                h->fp16, h->num_sms);
       prof_end(h, ev, VLA_KCLASS_ATTN_PREFILL, 0, 0);
     }
     if (rc) return fail(h, rc, t_err);
@@ -1334,7 +1334,7 @@ int vla_op_attn_chunk_res(const float* q, const void* kv, const void* kv_res, in
   L.layer_stride = static_cast<int64_t>(max_env) * L.env_stride;
   const int rc = attn_chunk_tc_launch(q, static_cast<bf16*>(out_hi), static_cast<bf16*>(out_lo),
                                       reinterpret_cast<const AttnTile*>(tiles_dev), n_tiles, L, 0, H, hd, status, st,
-                                      false);
+                                      false, query_num_sms());
   if (rc != VLA_OK && rc != VLA_ERR_CUDA)
     return set_err(nullptr, rc, "vla_op_attn_chunk_res: unsupported arguments or misaligned buffers");
   return rc;

@@ -70,14 +70,12 @@ class Rounding:
 EXACT = Rounding()
 # The GPU path: fp16 activation pairs (fp16 weights hold the bf16 ones exactly above 2^-14),
 # fp32 queries, K/V cached as fp16 + 4-bit residual; the multi-row projections use the pair for
-# q|k|v only (hi alone for o, gate|up and down); single-row (decode) attention reads the fp16
-# part alone.  Approximate where the GPU's choice follows the whole call's rows rather than one
+# q|k|v only (hi alone for o, gate|up and down); every attention reads the cache at its stored
+# precision.  Approximate where the GPU's choice follows the whole call's rows rather than one
 # env's chunk (the last prefill layer runs o, gate|up and down on each env's final row through
-# the two-half weight-streaming GEMM and reads the cache through the decode attention; decode of
-# more than 128 envs runs the tile GEMMs).
+# the two-half weight-streaming GEMM; decode of more than 128 envs runs the tile GEMMs).
 GPU_PATH = Rounding(act=round_f16_pair, q=lambda x: x.to(torch.float32).to(F64), kv=round_f16_r4,
-                    act_chunk={"o": round_f16, "gate_up": round_f16, "down": round_f16},
-                    kv_read_decode=round_f16)
+                    act_chunk={"o": round_f16, "gate_up": round_f16, "down": round_f16})
 
 
 def layer_forward_rounded(shape: O.Shape, lw: dict, h, pos, k_cache, v_cache, rnd: Rounding):

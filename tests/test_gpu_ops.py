@@ -332,13 +332,16 @@ def _encode_res4(x32: np.ndarray):
 def test_chunk_attention_tc_matches_fp64(hd):
     """The tcgen05 chunk attention vs brute-force causal softmax attention in fp64 over the values
     the cache stores (fp16 + residual): chunks of 1..200 rows after 0..300 cached positions, tiles
-    of <= 128 rows, a context reaching the last cache position (cap not a multiple of 64)."""
+    of <= 128 rows, a context reaching the last cache position (cap not a multiple of 64).  Cache
+    positions past each env's context hold NaN, as stale rows may: they must not reach the output."""
     H, cap, max_env = 3, 400, 6
     chunks = [(0, 0, 1), (1, 0, 127), (2, 0, 128), (3, 7, 200), (4, 300, 100), (5, 100, 64)]  # (env, past, n)
     rows = sum(n for _, _, n in chunks)
     x = (I.normal_bf16((max_env, 2, H, cap, hd), 93, hd, 1.0).float()
          + I.normal_bf16((max_env, 2, H, cap, hd), 93, 7 + hd, 2.0 ** -9).float()).numpy()
     hi, packed, value = _encode_res4(x)
+    for env, past, n in chunks:
+        hi[env, :, :, past + n:] = np.float16("nan")
     q = I.normal_bf16((rows, H * hd), 93, 1000 + hd, 1.0).float()
     tiles, qpos, qenv = [], [], []
     r = 0
@@ -380,3 +383,64 @@ def test_chunk_attention_tc_matches_fp64(hd):
     bad = [(0, 0, 129, 0)]
     assert V.vla_op_attn_chunk_res(qd.data_ptr(), kvd.data_ptr(), rsd.data_ptr(), max_env, H, hd, cap, bad, rows,
                                    tiles_dev.data_ptr(), oh.data_ptr(), ol.data_ptr()) == V.VLA_ERR_ARG
+
+
+def _decode_res4(hi: np.ndarray, packed: np.ndarray) -> np.ndarray:
+    """The cached values from the fp16 parts and their packed 4-bit codes, from the definition:
+    hi + (2c - 15) ulp(hi) / 32 with ulp(hi) = 2^(e-25) (biased exponent e >= 1) or 2^-24."""
+    c = np.empty(hi.shape, dtype=np.int64)
+    c[..., 0::2] = packed & 15
+    c[..., 1::2] = packed >> 4
+    e = ((hi.view(np.uint16) >> 10) & 31).astype(np.int64)
+    return hi.astype(np.float64) + (2.0 * c - 15.0) * np.ldexp(1.0, np.maximum(e, 1) - 30)
+
+
+@pytest.mark.parametrize("score", [False, True])
+def test_chunk_attention_tc_full_size_sampled(score):
+    """The engine's chunk attention at the bench step's size: 64 envs x 32 heads x 128, contexts
+    of 256 + U{16..48} positions in a 320-position cache.  Prefill: each env's whole context as
+    one chunk in tiles of <= 128 rows (192 tiles, 6144 (tile, head) items, ~41 per persistent
+    CTA); score: 6 rows after the context (64 tiles, 2048 items).  Random fp16 parts and residual
+    codes, NaN past each env's last position; sampled (row, head) outputs vs fp64 brute force."""
+    B, H, hd, cap = 64, 32, 128, 320
+    ctx = (256 + I.randint_i32((B,), 97, 3, 16, 49)).tolist()
+    lens = [6] * B if score else [c - 6 for c in ctx]
+    past = [c - 6 for c in ctx] if score else [0] * B
+    hi = I.normal_bf16((B, 2, H, cap, hd), 97, 1, 1.0).float().half().numpy()
+    packed = I.randint_i32((B, 2, H, cap, hd // 2), 97, 2, 0, 256).to(torch.uint8).numpy()
+    for b in range(B):
+        hi[b, :, :, past[b] + lens[b]:] = np.float16("nan")
+    rows = sum(lens)
+    q = I.normal_bf16((rows, H * hd), 97, 4, 1.0).float()
+    tiles, row_env, row_pos, tile_of_row = [], [], [], []
+    r = 0
+    for b, n in enumerate(lens):
+        for t0 in range(0, n, 128):
+            tiles.append((b, r + t0, min(128, n - t0), past[b] + t0))
+        row_env += [b] * n
+        row_pos += [past[b] + i for i in range(n)]
+        r += n
+    tiles_dev = torch.zeros(len(tiles) * 4, dtype=torch.int32, device="cuda")
+    oh = torch.full((rows, H * hd), float("nan"), dtype=torch.bfloat16, device="cuda")
+    ol = torch.full_like(oh, float("nan"))
+    qd, kvd, rsd = q.cuda(), torch.from_numpy(hi).cuda(), torch.from_numpy(packed).cuda()
+    assert V.vla_op_read_status()[0] == 0
+    assert V.vla_op_attn_chunk_res(qd.data_ptr(), kvd.data_ptr(), rsd.data_ptr(), B, H, hd, cap, tiles, rows,
+                                   tiles_dev.data_ptr(), oh.data_ptr(), ol.data_ptr()) == 0
+    assert V.vla_op_read_status() == (0, 0)
+    out = oh.cpu().double() + ol.cpu().double()
+    assert torch.isfinite(out).all()
+    rng = np.random.default_rng(11)
+    picks = [(int(i), int(h)) for i, h in zip(rng.integers(0, rows, 48), rng.integers(0, H, 48))]
+    picks += [(t[1] + t[2] - 1, (k * 7) % H) for k, t in enumerate(tiles[::9])]   # tiles' last rows
+    err = 0.0
+    for i, h in picks:
+        b, p = row_env[i], row_pos[i]
+        K = _decode_res4(hi[b, 0, h, :p + 1], packed[b, 0, h, :p + 1])
+        Vv = _decode_res4(hi[b, 1, h, :p + 1], packed[b, 1, h, :p + 1])
+        qi = q[i, h * hd:(h + 1) * hd].double().numpy()
+        s = K @ qi / math.sqrt(hd)
+        w = np.exp(s - s.max())
+        ref = (w / w.sum()) @ Vv
+        err = max(err, float(np.abs(out[i, h * hd:(h + 1) * hd].numpy() - ref).max()))
+    assert err < 1e-4, err
