@@ -227,6 +227,7 @@ CASES = {
     "gemv_decode_gate_up": (64, 22016, 4096, 0, 0, True),
     "gemv_decode_down": (64, 4096, 11008, 0, 0, True),
     "attn_decode": None,                                       # see run_attn_case
+    "attn_decode_res": None,
     "learning": None,                                          # see run_learning_case
     "attn_chunk": None,                                        # see run_attn_chunk_case
     "attn_score": None,                                        # 6 rows per env after the prefix
@@ -264,7 +265,8 @@ CASES.update({k + "_f16": v for k, v in list(CASES.items()) if v is not None})
 
 
 def run_attn_case(args):
-    """Decode attention for 64 envs x 32 heads at ~290 cached positions (one layer)."""
+    """Decode attention for 64 envs x 32 heads at ~290 cached positions (one layer); attn_decode_res
+    reads the fp16 parts and their 4-bit residual codes (the engine's form)."""
     import torch
     import __graft_entry__
     __graft_entry__.build()
@@ -274,6 +276,8 @@ def run_attn_case(args):
     scale = max(1, args.attn_ctx_scale)
     cap = 320 * scale
     kv = I.normal_bf16((B, 2, H, cap, hd), 5, 1, 1.0).cuda().half()
+    res = args.case.endswith("_res")
+    codes = I.randint_i32((B * 2 * H * cap * hd // 2,), 5, 4, 0, 256).to(torch.uint8).cuda() if res else None
     q = I.normal_bf16((B, H, hd), 5, 2, 1.0).cuda().float()
     ctx = I.randint_i32((B,), 5, 3, 273, 311) * scale
     env = torch.arange(B, dtype=torch.int32, device="cuda")
@@ -287,9 +291,14 @@ def run_attn_case(args):
     stream = torch.cuda.current_stream()
 
     def launch():
-        rc = V.vla_op_attn_decode(q.data_ptr(), kv.data_ptr(), B, H, hd, cap, env.data_ptr(), pos.data_ptr(), B,
-                                  max_ctx, oh.data_ptr(), ol.data_ptr(), ws.data_ptr(), nbytes, stream.cuda_stream,
-                                  keys)
+        if res:
+            rc = V.vla_op_attn_decode_res(q.data_ptr(), kv.data_ptr(), codes.data_ptr(), B, H, hd, cap, env.data_ptr(),
+                                          pos.data_ptr(), B, max_ctx, oh.data_ptr(), ol.data_ptr(), ws.data_ptr(),
+                                          nbytes, stream.cuda_stream, keys)
+        else:
+            rc = V.vla_op_attn_decode(q.data_ptr(), kv.data_ptr(), B, H, hd, cap, env.data_ptr(), pos.data_ptr(), B,
+                                      max_ctx, oh.data_ptr(), ol.data_ptr(), ws.data_ptr(), nbytes,
+                                      stream.cuda_stream, keys)
         assert rc == 0, V.vla_last_error()
 
     for _ in range(args.warmup):
@@ -303,7 +312,7 @@ def run_attn_case(args):
     torch.cuda.synchronize()
     ms = e0.elapsed_time(e1) / args.steps
     hbm, _, _, kind = peaks()
-    bytes_ = float(ctx.sum()) * 2 * H * hd * 2 + B * H * hd * (4 + 4)
+    bytes_ = float(ctx.sum()) * 2 * H * hd * (2.5 if res else 2) + B * H * hd * (4 + 4)
     print(json.dumps({"case": args.case, "B": B, "H": H, "hd": hd, "max_keys_per_cta": keys,
                       "kv_positions": int(ctx.sum()), "ms": ms,
                       "gbs": bytes_ / ms / 1e6, "hbm_frac": bytes_ / ms / 1e6 / hbm, "peaks": kind}))
@@ -414,7 +423,7 @@ def run_case(args):
     __graft_entry__.build()
     from paper_2505_18719_gb300 import inputs as I
     from paper_2505_18719_gb300 import vla as V
-    if args.case == "attn_decode":
+    if args.case in ("attn_decode", "attn_decode_res"):
         return run_attn_case(args)
     if args.case == "learning":
         return run_learning_case(args)

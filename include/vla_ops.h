@@ -125,6 +125,16 @@ int vla_op_attn_decode(const float* q, const void* kv, int max_env, int H, int h
                        size_t workspace_bytes, void* cuda_stream);
 size_t vla_op_attn_decode_workspace_bytes(int B, int H, int hd, int max_ctx, int max_keys_per_cta);
 
+/* The engine's decode attention: vla_op_attn_decode with the cache read at its stored
+ * precision, each value hi + (2c - 15) ulp(hi) / 32 from its fp16 part hi in kv and its 4-bit
+ * code c in kv_res (the layout of vla_op_attn_chunk_res); kv and kv_res 16-byte aligned.  Cache
+ * positions past pos[b] may hold anything (NaN included): they do not reach the output.  Same
+ * workspace as vla_op_attn_decode. */
+int vla_op_attn_decode_res(const float* q, const void* kv, const void* kv_res, int max_env, int H, int hd,
+                           int cap, const int32_t* env, const int32_t* pos, int B, int max_ctx,
+                           int max_keys_per_cta, void* out_hi, void* out_lo, float* workspace,
+                           size_t workspace_bytes, void* cuda_stream);
+
 /* Chunk causal attention (§3.1 self-attention; a prefill or appended chunk of each env attends
  * to its whole cached context, §3.3), the prefill / score kernel on its own:
  *   q          f32 [rows, H*hd] (already rotated), rows packed chunk after chunk;

@@ -69,7 +69,7 @@ __device__ __forceinline__ void split_h2(float a, float b, uint32_t& hi, uint32_
 }
 
 template <int HD>
-__global__ void __launch_bounds__(128) attn_chunk_mma_kernel(const float* __restrict__ q,
+__global__ void __launch_bounds__(128) attn_chunk_mma_kernel(const float* q,
                                                              bf16* __restrict__ out_hi,
                                                              bf16* __restrict__ out_lo,
                                                              const AttnTile* __restrict__ tiles,
@@ -283,8 +283,7 @@ __global__ void __launch_bounds__(128) attn_chunk_mma_kernel(const float* __rest
 // spill in the 64-dim variant.
 constexpr int kDecodeWarps = 2;
 template <int HD, bool RES, int NW = kDecodeWarps>
-__global__ void __launch_bounds__(NW * 32, RES ? 14 : 1) attn_decode_kernel(const float* __restrict__ q,
-                                                          const RowInfo* __restrict__ rows,
+__global__ void __launch_bounds__(NW * 32, RES ? 14 : 1) attn_decode_kernel(const float* q, const RowInfo* rows,
                                                           KVLayout kv, int layer, int H,
                                                           int chunk, int S, float scale_log2,
                                                           float* __restrict__ part_o,
@@ -304,7 +303,11 @@ __global__ void __launch_bounds__(NW * 32, RES ? 14 : 1) attn_decode_kernel(cons
   const int split = blockIdx.x, head = blockIdx.y, b = blockIdx.z;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int sub = lane / LPK, part = lane - sub * LPK;
-  const RowInfo ri = rows[b];
+  // the queries and row table come from the kernels just before (programmatic dependent
+  // launch): read them at L2, never through the non-coherent read-only path
+  RowInfo ri;
+  ri.env = __ldcg(&rows[b].env);
+  ri.pos = __ldcg(&rows[b].pos);
   const int d = H * HD;
   const int k_begin = split * chunk;
   const int k_end = min(k_begin + chunk, ri.pos + 1);
@@ -312,7 +315,7 @@ __global__ void __launch_bounds__(NW * 32, RES ? 14 : 1) attn_decode_kernel(cons
   float qv[8];
   {
     const float4* qp = reinterpret_cast<const float4*>(q + static_cast<size_t>(b) * d + head * HD + part * 8);
-    const float4 q0 = qp[0], q1 = qp[1];
+    const float4 q0 = __ldcg(qp), q1 = __ldcg(qp + 1);
     qv[0] = q0.x * scale_log2;
     qv[1] = q0.y * scale_log2;
     qv[2] = q0.z * scale_log2;

@@ -228,7 +228,7 @@ __global__ void __launch_bounds__(kAtThreads, 1)
   if (warp == 0) {
     if (lane == 0) {
       // ------------------------------------------------------------------ producer
-      pdl_wait();  // the chunks' own keys / values were written by the q|k|v projection
+      pdl_wait_async();  // the chunks' own keys / values were written by the q|k|v projection
       uint32_t issued = 0, issued_phase = 0;
       bool ok = true;
       int g = 0;  // block number over all of this CTA's items
@@ -513,7 +513,7 @@ __global__ void __launch_bounds__(kAtThreads, 1)
         float4 x[16];  // 64 values in flight
 #pragma unroll
         for (int i = 0; i < 16; ++i)
-          x[i] = valid ? __ldg(reinterpret_cast<const float4*>(qrow + c) + i) : make_float4(0.f, 0.f, 0.f, 0.f);
+          x[i] = valid ? __ldcg(reinterpret_cast<const float4*>(qrow + c) + i) : make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll
         for (int half = 0; half < 2; ++half) {
           uint32_t hi[16], lo[16];

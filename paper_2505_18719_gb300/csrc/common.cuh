@@ -189,7 +189,10 @@ __device__ __forceinline__ float silu_f(float x) { return x / (1.0f + expf(-x));
 // Programmatic dependent launch: every kernel of the path is launched with programmatic
 // stream serialization, lets its successor be scheduled early (launch_dependents) and waits
 // for its predecessor's results (wait) before touching any memory the predecessor wrote or
-// reads.  Without the launch attribute both instructions are no-ops.
+// reads.  Data written by earlier kernels of the path is read with coherent loads (plain or
+// ld.global.cg), never through the non-coherent read-only path (__ldg, const __restrict__):
+// a kernel scheduled early can see stale read-only-cache lines there.  Without the launch
+// attribute both instructions are no-ops.
 __device__ __forceinline__ void pdl_launch_dependents() {
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 }

@@ -1239,14 +1239,17 @@ size_t vla_op_attn_decode_workspace_bytes(int B, int H, int hd, int max_ctx, int
          256 + 256;
 }
 
-int vla_op_attn_decode(const float* q, const void* kv, int max_env, int H, int hd, int cap, const int32_t* env,
-                       const int32_t* pos, int B, int max_ctx, int max_keys_per_cta, void* out_hi, void* out_lo,
-                       float* workspace, size_t workspace_bytes, void* cuda_stream) {
+static int op_attn_decode(const char* name, const float* q, const void* kv, const void* kv_res, int max_env, int H,
+                          int hd, int cap, const int32_t* env, const int32_t* pos, int B, int max_ctx,
+                          int max_keys_per_cta, void* out_hi, void* out_lo, float* workspace, size_t workspace_bytes,
+                          void* cuda_stream) {
   const int chunk = max_keys_per_cta > 0 ? max_keys_per_cta : kOpAttnChunk;
+  if ((reinterpret_cast<uintptr_t>(kv) & 15) || (reinterpret_cast<uintptr_t>(kv_res) & 15))
+    return set_err(nullptr, VLA_ERR_ARG, std::string(name) + ": misaligned cache");
   if (!q || !kv || !env || !pos || !out_hi || !out_lo || !workspace || B < 1 || H < 1 || cap < 1 ||
       max_env < 1 || max_ctx < 1 || max_ctx > cap || (hd != 64 && hd != 128) || chunk < 16 ||
       workspace_bytes < vla_op_attn_decode_workspace_bytes(B, H, hd, max_ctx, chunk))
-    return set_err(nullptr, VLA_ERR_ARG, "vla_op_attn_decode: bad argument");
+    return set_err(nullptr, VLA_ERR_ARG, std::string(name) + ": bad argument");
   cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
   // Row table from env / pos (a strided device copy each, no host round trip).
   RowInfo* rows = reinterpret_cast<RowInfo*>(workspace);
@@ -1255,7 +1258,7 @@ int vla_op_attn_decode(const float* q, const void* kv, int max_env, int H, int h
                         cudaMemcpyDeviceToDevice, st) != cudaSuccess ||
       cudaMemcpy2DAsync(&rows[0].pos, sizeof(RowInfo), pos, sizeof(int32_t), sizeof(int32_t), B,
                         cudaMemcpyDeviceToDevice, st) != cudaSuccess)
-    return cuda_fail(cudaGetLastError(), "vla_op_attn_decode: row table");
+    return cuda_fail(cudaGetLastError(), (std::string(name) + ": row table").c_str());
   char* base = reinterpret_cast<char*>(workspace) + ((static_cast<size_t>(B) * sizeof(RowInfo) + 255) / 256) * 256;
   const size_t S = (static_cast<size_t>(max_ctx) + chunk - 1) / chunk;
   float* part_o = reinterpret_cast<float*>(base);
@@ -1263,9 +1266,10 @@ int vla_op_attn_decode(const float* q, const void* kv, int max_env, int H, int h
   float2* part_ml = reinterpret_cast<float2*>(ml_base);
   int* counters = reinterpret_cast<int*>(ml_base + ((static_cast<size_t>(B) * H * S * sizeof(float2) + 255) / 256) * 256);
   if (cudaMemsetAsync(counters, 0, static_cast<size_t>(B) * H * sizeof(int), st) != cudaSuccess)
-    return cuda_fail(cudaGetLastError(), "vla_op_attn_decode: tickets");
+    return cuda_fail(cudaGetLastError(), (std::string(name) + ": tickets").c_str());
   KVLayout L{};
   L.base = static_cast<f16*>(const_cast<void*>(kv));
+  L.res = static_cast<uint8_t*>(const_cast<void*>(kv_res));
   L.cap = cap;
   L.head_stride = static_cast<int64_t>(cap) * hd;
   L.kv_stride = static_cast<int64_t>(H) * L.head_stride;
@@ -1273,8 +1277,23 @@ int vla_op_attn_decode(const float* q, const void* kv, int max_env, int H, int h
   L.layer_stride = static_cast<int64_t>(max_env) * L.env_stride;
   const int rc = attn_decode_launch(q, static_cast<bf16*>(out_hi), static_cast<bf16*>(out_lo), rows, B, max_ctx, L,
                                     0, H, hd, chunk, part_o, part_ml, counters, st, false);
-  if (rc != VLA_OK && rc != VLA_ERR_CUDA) return set_err(nullptr, rc, "vla_op_attn_decode: unsupported arguments");
+  if (rc != VLA_OK && rc != VLA_ERR_CUDA) return set_err(nullptr, rc, std::string(name) + ": unsupported arguments");
   return rc;
+}
+
+int vla_op_attn_decode(const float* q, const void* kv, int max_env, int H, int hd, int cap, const int32_t* env,
+                       const int32_t* pos, int B, int max_ctx, int max_keys_per_cta, void* out_hi, void* out_lo,
+                       float* workspace, size_t workspace_bytes, void* cuda_stream) {
+  return op_attn_decode("vla_op_attn_decode", q, kv, nullptr, max_env, H, hd, cap, env, pos, B, max_ctx,
+                        max_keys_per_cta, out_hi, out_lo, workspace, workspace_bytes, cuda_stream);
+}
+
+int vla_op_attn_decode_res(const float* q, const void* kv, const void* kv_res, int max_env, int H, int hd, int cap,
+                           const int32_t* env, const int32_t* pos, int B, int max_ctx, int max_keys_per_cta,
+                           void* out_hi, void* out_lo, float* workspace, size_t workspace_bytes, void* cuda_stream) {
+  if (!kv_res) return set_err(nullptr, VLA_ERR_ARG, "vla_op_attn_decode_res: bad argument");
+  return op_attn_decode("vla_op_attn_decode_res", q, kv, kv_res, max_env, H, hd, cap, env, pos, B, max_ctx,
+                        max_keys_per_cta, out_hi, out_lo, workspace, workspace_bytes, cuda_stream);
 }
 
 int vla_op_attn_chunk(const float* q, const void* kv, int max_env, int H, int hd, int cap,

@@ -402,7 +402,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp == 0) {
     if (lane == 0) {
       // ------------------------------------------------------------ TMA producer
-      pdl_wait();  // everything this CTA reads or writes is ordered after this wait
+      pdl_wait_async();  // everything this CTA reads or writes is ordered after this wait
       int stage = 0;
       uint32_t phase = 0;
       uint32_t issued = 0, issued_phase = 0;
@@ -624,7 +624,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp == 0) {
     if (lane == 0) {
       // ------------------------------------------------------------ TMA producer (both CTAs)
-      pdl_wait();
+      pdl_wait_async();
       int stage = 0;
       uint32_t phase = 0;
       uint32_t issued = 0, issued_phase = 0;
@@ -1215,7 +1215,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         tma_load_2d_hint(sw, &tmW, full0 + 8 * i, kb * BK, t * TR, pol_w);
         issued |= 1u << i;
       }
-      pdl_wait();
+      pdl_wait_async();
       for (int i = 0; i < pre; ++i) {
         const int g = g_begin + i, t = g / p.kbt, kb = g - t * p.kbt;
         (void)t;

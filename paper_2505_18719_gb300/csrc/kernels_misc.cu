@@ -17,7 +17,7 @@ namespace {
 __global__ void __launch_bounds__(256) assemble_kernel(const RowInfo* __restrict__ rows,
                                                        const bf16* __restrict__ visual,
                                                        const int* __restrict__ ids,
-                                                       const int* __restrict__ tokens,
+                                                       const int* tokens,
                                                        const bf16* __restrict__ embed, int d,
                                                        int vocab, float* __restrict__ h,
                                                        uint32_t* status) {
@@ -45,7 +45,7 @@ __global__ void __launch_bounds__(256) assemble_kernel(const RowInfo* __restrict
   }
 }
 
-__global__ void __launch_bounds__(256) rmsnorm_kernel(const float* __restrict__ h, int ldh,
+__global__ void __launch_bounds__(256) rmsnorm_kernel(const float* h, int ldh,
                                                       const bf16* __restrict__ w, int d,
                                                       float eps, bf16* __restrict__ y_hi,
                                                       bf16* __restrict__ y_lo, bool fp16,
@@ -80,7 +80,7 @@ __global__ void __launch_bounds__(256) rmsnorm_kernel(const float* __restrict__ 
   report_saturation(status, sat);
 }
 
-__global__ void gather_rows_kernel(const float* __restrict__ src, const int* __restrict__ idx,
+__global__ void gather_rows_kernel(const float* src, const int* __restrict__ idx,
                                    int d, float* __restrict__ dst) {
   pdl_launch_dependents();
   pdl_wait();
@@ -90,7 +90,7 @@ __global__ void gather_rows_kernel(const float* __restrict__ src, const int* __r
     *reinterpret_cast<float4*>(o + c) = *reinterpret_cast<const float4*>(s + c);
 }
 
-__global__ void scatter_rows_kernel(const float* __restrict__ src, const int* __restrict__ sidx,
+__global__ void scatter_rows_kernel(const float* src, const int* __restrict__ sidx,
                                     const int* __restrict__ didx, int d, float* __restrict__ dst) {
   pdl_launch_dependents();
   pdl_wait();

@@ -12,7 +12,7 @@ namespace vla {
 namespace {
 
 // One CTA (256 threads) per env: V_b = sum_c h_c r g_c w_c + bias, r = rsqrt(mean h^2 + eps).
-__global__ void __launch_bounds__(256) value_head_kernel(const float* __restrict__ h, int ldh, int d,
+__global__ void __launch_bounds__(256) value_head_kernel(const float* h, int ldh, int d,
                                                          const bf16* __restrict__ gain,
                                                          const bf16* __restrict__ w, float eps,
                                                          float bias, float* __restrict__ out) {
@@ -45,8 +45,8 @@ __global__ void __launch_bounds__(256) value_head_kernel(const float* __restrict
 }
 
 // One thread per env b: A_t = delta_t + gamma lam (1 - done_t) A_{t+1}, walking t = M-1 .. 0.
-__global__ void gae_kernel(const float* __restrict__ r, const float* __restrict__ v,
-                           const float* __restrict__ done, int M, int B, float gamma, float lam,
+__global__ void gae_kernel(const float* r, const float* v,
+                           const float* done, int M, int B, float gamma, float lam,
                            float* __restrict__ adv, float* __restrict__ ret) {
   pdl_launch_dependents();
   pdl_wait();
@@ -65,9 +65,9 @@ __global__ void gae_kernel(const float* __restrict__ r, const float* __restrict_
 }
 
 // One CTA of 1024 threads: thread j sums samples j, j + 1024, ... in order; then a fixed tree.
-__global__ void __launch_bounds__(1024) ppo_clip_kernel(const float* __restrict__ lp_new,
-                                                        const float* __restrict__ lp_old,
-                                                        const float* __restrict__ adv, int N, int A,
+__global__ void __launch_bounds__(1024) ppo_clip_kernel(const float* lp_new,
+                                                        const float* lp_old,
+                                                        const float* adv, int N, int A,
                                                         float eps, float* __restrict__ objective,
                                                         float* __restrict__ ratio,
                                                         float* __restrict__ clip_frac) {

@@ -28,6 +28,12 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
       : "memory");
   return ok != 0;
 }
+// griddepcontrol.wait for a thread that then reads the previous kernels' output through the
+// async proxy (TMA / bulk copies): their generic stores are ordered before those reads.
+__device__ __forceinline__ void pdl_wait_async() {
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  asm volatile("fence.proxy.async.global;" ::: "memory");
+}
 // Non-blocking probe of the same condition (no suspend), for a thread polling several barriers.
 __device__ __forceinline__ bool mbar_test_wait(uint32_t bar, uint32_t parity) {
   uint32_t ok;

@@ -101,6 +101,8 @@ def load(path: str = LIB_PATH):
         "vla_op_num_sms": (i32, []),
         "vla_op_attn_decode": (i32, [vp, vp, i32, i32, i32, i32, vp, vp, i32, i32, i32, vp, vp, vp, ctypes.c_size_t, vp]),
         "vla_op_attn_decode_workspace_bytes": (ctypes.c_size_t, [i32, i32, i32, i32, i32]),
+        "vla_op_attn_decode_res": (i32, [vp, vp, vp, i32, i32, i32, i32, vp, vp, i32, i32, i32, vp, vp, vp,
+                                         ctypes.c_size_t, vp]),
         "vla_op_attn_chunk": (i32, [vp, vp, i32, i32, i32, i32, vp, i32, i32, vp, vp, vp, vp]),
         "vla_op_rmsnorm": (i32, [vp, i32, i32, i32, vp, f32, vp, vp, i32, vp]),
         "vla_op_attn_chunk_res": (i32, [vp, vp, vp, i32, i32, i32, i32, vp, i32, i32, vp, vp, vp, vp]),
@@ -297,6 +299,13 @@ def vla_op_attn_decode(q_ptr, kv_ptr, max_env, H, hd, cap, env_ptr, pos_ptr, B, 
                        ws_ptr, ws_bytes, stream=0, max_keys_per_cta=0) -> int:
     return load().vla_op_attn_decode(q_ptr, kv_ptr, max_env, H, hd, cap, env_ptr, pos_ptr, B, max_ctx,
                                      max_keys_per_cta, out_hi_ptr, out_lo_ptr, ws_ptr, ws_bytes, stream or None)
+
+
+def vla_op_attn_decode_res(q_ptr, kv_ptr, res_ptr, max_env, H, hd, cap, env_ptr, pos_ptr, B, max_ctx, out_hi_ptr,
+                           out_lo_ptr, ws_ptr, ws_bytes, stream=0, max_keys_per_cta=0) -> int:
+    """vla_op_attn_decode over the fp16 cache plus its 4-bit residual codes (res)."""
+    return load().vla_op_attn_decode_res(q_ptr, kv_ptr, res_ptr, max_env, H, hd, cap, env_ptr, pos_ptr, B, max_ctx,
+                                         max_keys_per_cta, out_hi_ptr, out_lo_ptr, ws_ptr, ws_bytes, stream or None)
 
 
 def vla_op_attn_decode_workspace_bytes(B, H, hd, max_ctx, max_keys_per_cta=0) -> int:

@@ -189,6 +189,50 @@ def test_decode_attention_matches_fp64(B, H, hd, cap, ctx):
         assert (got[b] - o).abs().max().item() < 1e-4, b
 
 
+@pytest.mark.parametrize("B,H,hd,cap,ctx", [(3, 2, 64, 64, [1, 7, 64]), (5, 4, 128, 1152, [1, 129, 300, 1116, 161]),
+                                          (64, 32, 128, 320, None)])
+def test_decode_attention_res_matches_fp64(B, H, hd, cap, ctx):
+    """The engine's decode attention, reading fp16 parts and 4-bit residual codes (random), vs
+    brute-force softmax attention in fp64 over the values the cache stores (hi + residual);
+    positions past each context hold NaN."""
+    max_env = B + 1
+    hi = I.normal_bf16((max_env, 2, H, cap, hd), 79, B, 1.0).float().half().numpy()
+    packed = I.randint_i32((max_env, 2, H, cap, hd // 2), 79, 50 + B, 0, 256).to(torch.uint8).numpy()
+    q = I.normal_bf16((B, H, hd), 79, 100 + B, 1.0).float()
+    if ctx is None:
+        ctx = I.randint_i32((B,), 79, 200, 272, 310).tolist()
+    env = torch.tensor([(b * 7 + 1) % max_env for b in range(B)], dtype=torch.int32)
+    pos = torch.tensor([c - 1 for c in ctx], dtype=torch.int32)
+    value = _decode_res4(hi, packed)
+    for b in range(B):
+        hi[int(env[b]), :, :, ctx[b]:] = np.float16("nan")
+    max_ctx = max(ctx)
+    nbytes = V.vla_op_attn_decode_workspace_bytes(B, H, hd, max_ctx, 0)
+    ws = torch.empty(nbytes // 4 + 64, dtype=torch.float32, device="cuda")
+    oh = torch.empty(B, H * hd, dtype=torch.bfloat16, device="cuda")
+    ol = torch.empty(B, H * hd, dtype=torch.bfloat16, device="cuda")
+    kvd, rsd, qd = torch.from_numpy(hi).cuda(), torch.from_numpy(packed).cuda(), q.cuda()
+    envd, posd = env.cuda(), pos.cuda()
+    rc = V.vla_op_attn_decode_res(qd.data_ptr(), kvd.data_ptr(), rsd.data_ptr(), max_env, H, hd, cap, envd.data_ptr(),
+                                  posd.data_ptr(), B, max_ctx, oh.data_ptr(), ol.data_ptr(), ws.data_ptr(), nbytes, 0)
+    assert rc == 0, V.vla_last_error()
+    torch.cuda.synchronize()
+    got = (oh.double() + ol.double()).cpu().reshape(B, H, hd)
+    kv64 = torch.from_numpy(value)
+    err = err_hi = 0.0
+    for b in range(B):
+        e, n = int(env[b]), ctx[b]
+        k, v = kv64[e, 0, :, :n], kv64[e, 1, :, :n]                  # [H, n, hd]
+        sc = torch.einsum("hd,hnd->hn", q[b].double(), k) / math.sqrt(hd)
+        o = torch.einsum("hn,hnd->hd", torch.softmax(sc, -1), v)
+        err = max(err, (got[b] - o).abs().max().item())
+        kh, vh = (torch.from_numpy(hi[e, i, :, :n].astype(np.float64)) for i in (0, 1))
+        sh = torch.einsum("hd,hnd->hn", q[b].double(), kh) / math.sqrt(hd)
+        err_hi = max(err_hi, (got[b] - torch.einsum("hn,hnd->hd", torch.softmax(sh, -1), vh)).abs().max().item())
+    assert err < 1e-4, err
+    assert err_hi > 4 * err, (err, err_hi)   # the residual is read, not just the fp16 part
+
+
 @pytest.mark.parametrize("hd", [64, 128])
 def test_chunk_attention_matches_fp64(hd):
     """Prefill / score chunk attention vs brute-force causal softmax attention in fp64: chunks of
