@@ -38,7 +38,7 @@ WORKLOAD = "7b_b64_ragged_score"
 # that kernel changes): gemm_tc2_kernel, the q|k|v projection of this step's prefill
 # (18385 x 12288 x 4096, fp16 operand pair, case pair_prefill_qkv_18385_f16; fp32 output in
 # the case).
-PROFILED_TRAFFIC = {"bytes": 2.113555e9 + 0.879153e9,
+PROFILED_TRAFFIC = {"bytes": 2.366113e9 + 0.880124e9,
                     "launch": "gemm_tc2_kernel q|k|v (fp16 operands), M=18385 N=12288 K=4096",
                     "algorithmic_bytes": 2.0 * 18385 * 4096 * 2 + 2.0 * 12288 * 4096 + 4.0 * 18385 * 12288,
                     "profile": "profiles/gemm_tc2_prefill_qkv_18385x12288x4096.md"}
@@ -59,8 +59,8 @@ def workload_config(wl, n_gpus):
 
 def phase_work(sh, past, chunk):
     """Algorithmic work of one turn's phases for envs whose chunk of chunk[b] rows lands after
-    past[b] cached positions (7B: 6.476e9 matrix parameters, 16 KB of fp16 K+V per position
-    and layer).  Prefill FLOPs count what the method needs: every row through every layer,
+    past[b] cached positions (7B: 6.476e9 matrix parameters; K+V per position and layer as
+    cached: 16 KB of fp16 parts and 4 KB of 4-bit residual codes).  Prefill FLOPs count what the method needs: every row through every layer,
     except that the last layer only needs q|k|v for all rows (KV cache) and the rest for each
     env's final row; attention FLOPs are the causal ones.  Decode bytes are, per forward, all
     weights + the K/V each env reads (positions 0..pos) and writes + the 256 head rows.
@@ -70,7 +70,7 @@ def phase_work(sh, past, chunk):
     qkv_params = 3 * d * d
     params = L * per_layer
     w_bytes = 2.0 * params
-    kv_tok = 2.0 * 2 * d * L                    # fp16 K and V, all layers
+    kv_tok = 2.5 * 2 * d * L                    # K and V as cached (fp16 + 4-bit residual), all layers
     A = sh.action_dim
     B = len(chunk)
     T = sum(chunk)
@@ -204,7 +204,8 @@ def run_reference(args):
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
         "data": "synthetic (seeded; random-init weights)",
         "config": dict(workload_config(wl, world), sample="1 env per step (prefill + 7 tokens + score)"),
-        "cpu_baseline": {"value": value, "unit": "action tokens/s", "cores": threads, "kind": "oracle",
+        "cpu_baseline": {"value": value, "unit": "action tokens/s", "cores": threads, "host_cpus": os.cpu_count(),
+                         "kind": "oracle",
                          "sample": f"1 of {wl.batch} envs, prefix {prefix} tokens, prefill+decode+score, fp64"},
         "e2e": {"value": value, "unit": "action tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
@@ -736,7 +737,7 @@ def main():
     if rank == 0 and not args.no_cpu_baseline:
         dt, prefix, threads = oracle_sample(wl, w_cpu)
         line["cpu_baseline"] = {"value": A / dt, "unit": "action tokens/s", "cores": threads,
-                                "kind": "oracle",
+                                "host_cpus": os.cpu_count(), "kind": "oracle",
                                 "sample": f"1 of {B} envs (prefix {prefix} tokens): prefill + 7-token decode + score, fp64, {dt:.1f} s"}
     if dist is not None:
         dist.barrier()
