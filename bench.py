@@ -676,12 +676,12 @@ def main():
                 "traffic": PROFILED_TRAFFIC["bytes"] if PROFILED_TRAFFIC else None,
                 "traffic_launch": PROFILED_TRAFFIC,
                 "launches": gp["launches"], "avg_launch_ms": gp["ms"] / max(1, gp["launches"])}
-        # the q|k|v, o and down tile GEMMs multiply both halves of the activation pair, gate|up
-        # hi alone: the MMAs issued are (1 + the paired share of the projection work) x the
-        # algorithmic product
+        # the q|k|v tile GEMMs multiply both halves of the activation pair, o, gate|up and
+        # down hi alone: the MMAs issued are (1 + the paired share of the projection work) x
+        # the algorithmic product
         sh = wl.shape
         d_, f_ = float(sh.d_model), float(sh.d_ffn)
-        paired_share = (4.0 * d_ * d_ + f_ * d_) / (4.0 * d_ * d_ + 3.0 * f_ * d_)
+        paired_share = (3.0 * d_ * d_) / (4.0 * d_ * d_ + 3.0 * f_ * d_)
         roof["issued_mma_frac"] = (1.0 + paired_share) * achieved / tf_sus
     roof_dec = None
     if gd["ms"] > 0:
