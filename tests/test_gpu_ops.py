@@ -488,3 +488,28 @@ def test_chunk_attention_tc_full_size_sampled(score):
         ref = (w / w.sum()) @ Vv
         err = max(err, float(np.abs(out[i, h * hd:(h + 1) * hd].numpy() - ref).max()))
     assert err < 1e-4, err
+
+
+def test_pair_gemm_f16_full_size_sampled():
+    """The prefill q|k|v projection at the bench step's full size, M = 18385 rows (64 envs x
+    (256 + U{16..48})), N = 12288, K = 4096, on CTA pairs with the fp16 activation pair: sampled
+    outputs (random, every tile edge in m and n, the ragged last rows) vs fp64 sums over the same
+    fp16 values, within fp32 accumulation error."""
+    M, N, K = 18385, 12288, 4096
+    A = I.normal_bf16((M, K), 31, 1, 1.0).float().half()
+    A_lo = (I.normal_bf16((M, K), 31, 2, 1.0).float() * 2.0 ** -12).half()
+    W = I.normal_bf16((N, K), 31, 3, 0.02).float().half()
+    C = torch.full((M, N), float("nan"), dtype=torch.float32, device="cuda")
+    Ad, Ald, Wd = A.cuda(), A_lo.cuda(), W.cuda()
+    assert V.vla_op_gemm_pair_f16(Ad.data_ptr(), Ald.data_ptr(), K, Wd.data_ptr(), K, C.data_ptr(), N, M, N, K, 0) == 0
+    torch.cuda.synchronize()
+    rng = np.random.default_rng(3)
+    ms = list(rng.integers(0, M, 40)) + [0, 255, 256, 2047, 2048, M - 256, M - 2, M - 1]
+    ns = list(rng.integers(0, N, 40)) + [0, 255, 256, 4095, 4096, 8191, 8192, N - 1]
+    Cs = C[torch.tensor(ms)][:, torch.tensor(ns)].cpu().double()
+    a = A[ms].double() + A_lo[ms].double()
+    w = W[ns].double()
+    ref = a @ w.T
+    bound = (a.abs() @ w.abs().T) * 3e-5 + 1e-6
+    assert torch.isfinite(Cs).all()
+    assert ((Cs - ref).abs() <= bound).all(), float(((Cs - ref).abs() / bound).max())
