@@ -18,9 +18,10 @@ int attn_chunk_launch(const float* q, bf16* out_hi, bf16* out_lo, const AttnTile
 
 // The same on the tcgen05 tensor cores with the cache read as fp16 + 4-bit residual (kv.res
 // required): tiles of up to 128 rows; status gets VLA_STATUS_TIMEOUT if a pipeline wait runs out.
+// write_lo = false leaves out_lo untouched (for a consumer that reads the hi plane alone).
 int attn_chunk_tc_launch(const float* q, bf16* out_hi, bf16* out_lo, const AttnTile* tiles, int n_tiles,
                          KVLayout kv, int layer, int H, int hd, uint32_t* status, cudaStream_t stream, bool fp16,
-                         int num_sms);
+                         int num_sms, bool write_lo);
 
 // One query per env row b (rows[b] gives env and position); key range split into equal ranges
 // of at most `chunk` keys (a multiple of 16 at least 16); partials in part_o [B*H*S*hd] f32 and part_ml [B*H*S]

@@ -119,6 +119,7 @@ struct AtParams {
   int n_items;             // tiles x heads
   float scale_log2;        // log2(e) / sqrt(HD), folded into the queries
   bool fp16;
+  bool write_lo;           // write out_lo (else hi alone: the consumer reads the hi plane only)
   uint32_t* status;
   uint64_t wait_limit;
 };
@@ -370,11 +371,13 @@ __global__ void __launch_bounds__(kAtThreads, 1)
             split_pack2(__uint_as_float(v[2 * i]) * inv, __uint_as_float(v[2 * i + 1]) * inv, h[i], lo[i], p.fp16,
                         sat);
           uint4* dh = reinterpret_cast<uint4*>(p.out_hi + off + c);
-          uint4* dl = reinterpret_cast<uint4*>(p.out_lo + off + c);
           dh[0] = make_uint4(h[0], h[1], h[2], h[3]);
           dh[1] = make_uint4(h[4], h[5], h[6], h[7]);
-          dl[0] = make_uint4(lo[0], lo[1], lo[2], lo[3]);
-          dl[1] = make_uint4(lo[4], lo[5], lo[6], lo[7]);
+          if (p.write_lo) {
+            uint4* dl = reinterpret_cast<uint4*>(p.out_lo + off + c);
+            dl[0] = make_uint4(lo[0], lo[1], lo[2], lo[3]);
+            dl[1] = make_uint4(lo[4], lo[5], lo[6], lo[7]);
+          }
         }
       }
       return true;
@@ -607,7 +610,7 @@ __global__ void __launch_bounds__(kAtThreads, 1)
 
 int attn_chunk_tc_launch(const float* q, bf16* out_hi, bf16* out_lo, const AttnTile* tiles, int n_tiles,
                          KVLayout kv, int layer, int H, int hd, uint32_t* status, cudaStream_t stream, bool fp16,
-                         int num_sms) {
+                         int num_sms, bool write_lo) {
   if (n_tiles <= 0) return VLA_OK;
   if (!kv.res || (hd != 64 && hd != 128) || num_sms <= 0) return VLA_ERR_UNSUPPORTED;
   if ((reinterpret_cast<uintptr_t>(kv.base) & 15) || (reinterpret_cast<uintptr_t>(kv.res) & 15))
@@ -628,6 +631,7 @@ int attn_chunk_tc_launch(const float* q, bf16* out_hi, bf16* out_lo, const AttnT
   p.n_items = n_tiles * H;
   p.scale_log2 = 1.4426950408889634f / sqrtf(static_cast<float>(hd));
   p.fp16 = fp16;
+  p.write_lo = write_lo;
   p.status = status;
   p.wait_limit = g_wait_limit_ns.load(std::memory_order_relaxed);
   // tensor map over every row of the cache (rows = layers * layer_stride / hd): row coordinates

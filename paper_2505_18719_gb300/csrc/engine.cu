@@ -252,6 +252,9 @@ void prof_harvest(vla_handle* h) {
 // weights, so the second MMA costs nothing there.
 enum : unsigned { kProjQkv = 1, kProjO = 2, kProjGateUp = 4, kProjDown = 8 };
 constexpr unsigned kTileLoMask = kProjQkv;
+// Whether the projection `proj` of an M-row call reads the low half of its activation pair:
+// the weight-streaming GEMM (M <= 128) always does, the tile GEMMs for kTileLoMask only.
+constexpr bool gemm_reads_lo(int M, unsigned proj) { return M <= 128 || (kTileLoMask & proj) != 0; }
 
 // A is the operand pair: hi at A, lo at A + a_plane (fp16 when h->fp16, else bf16).
 // The GEMM that will consume h->y after a residual GEMM's RMSNorm (its N, K and epilogue).
@@ -273,7 +276,7 @@ int run_gemm(vla_handle* h, int cls, const bf16* A, size_t a_plane, int lda, con
                                                  : kProjDown;
   GemmArgs g;
   g.A = A;
-  g.A_lo = (stream_k || (kTileLoMask & proj)) ? A + a_plane : nullptr;
+  g.A_lo = gemm_reads_lo(M, proj) ? A + a_plane : nullptr;
   g.lda = lda;
   g.B = W;
   g.ldb = ldw;
@@ -406,8 +409,9 @@ int forward_layers(vla_handle* h, int M, const RowInfo* rows_dev, bool decode, i
       prof_end(h, ev, VLA_KCLASS_ATTN_DECODE, 0, 0);
     } else {
       ev = prof_begin(h, VLA_KCLASS_ATTN_PREFILL);
+      // the low plane of the output only where the o projection reads it
       rc = attn_chunk_tc_launch(h->q, h->ao, h->ao + pd, h->tiles, n_tiles, h->kvl, l, H, hd, h->status, h->stream,
-                                h->fp16, h->num_sms);
+                                h->fp16, h->num_sms, gemm_reads_lo(M, kProjO));
       prof_end(h, ev, VLA_KCLASS_ATTN_PREFILL, 0, 0);
     }
     if (rc) return fail(h, rc, t_err);
@@ -1353,7 +1357,7 @@ int vla_op_attn_chunk_res(const float* q, const void* kv, const void* kv_res, in
   L.layer_stride = static_cast<int64_t>(max_env) * L.env_stride;
   const int rc = attn_chunk_tc_launch(q, static_cast<bf16*>(out_hi), static_cast<bf16*>(out_lo),
                                       reinterpret_cast<const AttnTile*>(tiles_dev), n_tiles, L, 0, H, hd, status, st,
-                                      false, query_num_sms());
+                                      false, query_num_sms(), true);
   if (rc != VLA_OK && rc != VLA_ERR_CUDA)
     return set_err(nullptr, rc, "vla_op_attn_chunk_res: unsupported arguments or misaligned buffers");
   return rc;
