@@ -165,7 +165,7 @@ __device__ __forceinline__ void store_split1(void* hi, void* lo, size_t i, float
   uint16_t h, l;
   split_bits(x, fp16, h, l, sat);
   static_cast<uint16_t*>(hi)[i] = h;
-  static_cast<uint16_t*>(lo)[i] = l;
+  if (lo) static_cast<uint16_t*>(lo)[i] = l;
 }
 // Raises VLA_STATUS_SATURATED when this thread clamped a value (rare: one atomic per thread that did).
 __device__ __forceinline__ void report_saturation(uint32_t* status, uint32_t sat) {

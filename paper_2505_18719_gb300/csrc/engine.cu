@@ -423,7 +423,8 @@ int forward_layers(vla_handle* h, int M, const RowInfo* rows_dev, bool decode, i
     eo.norm_w = h->ffn_norm[l];
     eo.norm_eps = c.rms_eps;
     eo.norm_hi = h->y;
-    eo.norm_lo = h->y + pd;
+    // the low halves of y and u only where gate|up and down read them
+    eo.norm_lo = gemm_reads_lo(Mr, kProjGateUp) ? h->y + pd : nullptr;
     eo.ldn = d;
     const NextGemm gate_up{2 * F, d, EPI_SWIGLU};
     if ((rc = run_gemm(h, gcls, h->ao, pd, d, h->wo[l], d, Mr, d, d, eo, &gate_up))) return rc;
@@ -431,7 +432,7 @@ int forward_layers(vla_handle* h, int M, const RowInfo* rows_dev, bool decode, i
     EpiArgs eg;
     eg.kind = EPI_SWIGLU;
     eg.out_hi = h->u;
-    eg.out_lo = h->u + pf;
+    eg.out_lo = gemm_reads_lo(Mr, kProjDown) ? h->u + pf : nullptr;
     eg.ldo = F;
     if ((rc = run_gemm(h, gcls, h->y, pd, d, h->wgu[l], d, Mr, 2 * F, d, eg))) return rc;
 

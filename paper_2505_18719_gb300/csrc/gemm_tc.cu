@@ -89,7 +89,8 @@ __device__ __forceinline__ void unit_coords(const Params& p, int u, int& m_blk, 
 }
 
 // ----------------------------------------------------------------------------- epilogues
-// 16 values as operand hi/lo pairs, fp16 if `fp16` else bf16 (two 32-byte stores each).
+// 16 values as operand hi/lo pairs, fp16 if `fp16` else bf16 (two 32-byte stores each); the
+// low half is not stored when lo_dst is null (a consumer that reads only the high half).
 __device__ __forceinline__ void store_split16(bf16* hi_dst, bf16* lo_dst, const float (&v)[16],
                                               bool fp16, uint32_t& sat) {
   uint32_t h[8], l[8];
@@ -97,8 +98,14 @@ __device__ __forceinline__ void store_split16(bf16* hi_dst, bf16* lo_dst, const 
   for (int i = 0; i < 8; ++i) split_pack2(v[2 * i], v[2 * i + 1], h[i], l[i], fp16, sat);
   reinterpret_cast<uint4*>(hi_dst)[0] = make_uint4(h[0], h[1], h[2], h[3]);
   reinterpret_cast<uint4*>(hi_dst)[1] = make_uint4(h[4], h[5], h[6], h[7]);
+  if (!lo_dst) return;
   reinterpret_cast<uint4*>(lo_dst)[0] = make_uint4(l[0], l[1], l[2], l[3]);
   reinterpret_cast<uint4*>(lo_dst)[1] = make_uint4(l[4], l[5], l[6], l[7]);
+}
+// dst + off, or null when dst is null.
+template <class T>
+__device__ __forceinline__ T* opt_at(T* dst, size_t off) {
+  return dst ? dst + off : nullptr;
 }
 __device__ __forceinline__ void store_f16x16(f16* dst, const float (&v)[16]) {
   uint4 a, b;
@@ -227,7 +234,7 @@ __device__ __forceinline__ void epilogue_plain(const Params& p, uint32_t trow, i
       }
       const size_t off = static_cast<size_t>(m) * p.epi.ldn + n;
       if (cnt == 16 && (p.epi.ldn & 7) == 0) {
-        store_split16(p.epi.norm_hi + off, p.epi.norm_lo + off, y, p.epi.fp16, sat);
+        store_split16(p.epi.norm_hi + off, opt_at(p.epi.norm_lo, off), y, p.epi.fp16, sat);
       } else {
 #pragma unroll
         for (int i = 0; i < 16; ++i) {
@@ -259,7 +266,7 @@ __device__ __forceinline__ void epilogue_swiglu(const Params& p, uint32_t trow, 
     for (int i = 0; i < 16; ++i) o[i] = silu_f(g[i] * rs) * (u[i] * rs);
     const size_t off = static_cast<size_t>(m) * p.epi.ldo + f;
     if (f + 16 <= F && ((p.epi.ldo & 7) == 0)) {
-      store_split16(p.epi.out_hi + off, p.epi.out_lo + off, o, p.epi.fp16, sat);
+      store_split16(p.epi.out_hi + off, opt_at(p.epi.out_lo, off), o, p.epi.fp16, sat);
     } else {
 #pragma unroll
       for (int i = 0; i < 16; ++i) {
@@ -1496,7 +1503,7 @@ GemmCost gemm_cost(const GemmArgs& a) {
   double out_bytes;
   switch (a.epi.kind) {
     case EPI_RESID: out_bytes = 8.0 * a.M * a.N; break;
-    case EPI_SWIGLU: out_bytes = 2.0 * a.M * (a.N / 2) * 2; break;
+    case EPI_SWIGLU: out_bytes = 2.0 * a.M * (a.N / 2) * (a.epi.out_lo ? 2 : 1); break;
     case EPI_QKV: out_bytes = 2.0 * a.M * a.N; break;
     default: out_bytes = 4.0 * a.M * a.N;
   }
@@ -1568,8 +1575,9 @@ size_t gemm_workspace_bytes(const GemmArgs& a) {
 int gemm_launch(const GemmArgs& a, cudaStream_t stream, int num_sms, GemmCost* cost) {
   if (a.M < 1 || a.N < 1 || a.K < 1 || !a.A || !a.B) return VLA_ERR_ARG;
   if (a.block_n != 128 && a.block_n != 256) return VLA_ERR_ARG;
-  // a following RMSNorm: only as the deferred form (ss_out), on an unsplit residual GEMM
-  if (a.epi.norm_w && (!a.epi.ss_out || a.epi.kind != EPI_RESID || !a.epi.norm_hi || !a.epi.norm_lo))
+  // a following RMSNorm: only as the deferred form (ss_out), on an unsplit residual GEMM (its
+  // low half is skipped when norm_lo is null)
+  if (a.epi.norm_w && (!a.epi.ss_out || a.epi.kind != EPI_RESID || !a.epi.norm_hi))
     return VLA_ERR_ARG;
   if (a.epi.row_ss && a.epi.kind != EPI_QKV && a.epi.kind != EPI_SWIGLU) return VLA_ERR_ARG;
   if ((a.lda % 8) || (a.ldb % 8) || a.lda < a.K || a.ldb < a.K) return VLA_ERR_ARG;

@@ -75,7 +75,7 @@ __global__ void __launch_bounds__(256) rmsnorm_kernel(const float* h, int ldh,
     split_pack2(v.x * r * w0.x, v.y * r * w0.y, hi.x, lo.x, fp16, sat);
     split_pack2(v.z * r * w1.x, v.w * r * w1.y, hi.y, lo.y, fp16, sat);
     *reinterpret_cast<uint2*>(y_hi + off + c) = hi;
-    *reinterpret_cast<uint2*>(y_lo + off + c) = lo;
+    if (y_lo) *reinterpret_cast<uint2*>(y_lo + off + c) = lo;
   }
   report_saturation(status, sat);
 }
