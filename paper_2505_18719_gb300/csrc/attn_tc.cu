@@ -12,7 +12,9 @@
 //
 // Roles (448 threads):
 //   warp 0       TMA producer: per 64-key block, K_hi and V_hi (tensor map over the whole cache,
-//                128-byte swizzle) and the two residual byte ranges (bulk copies), three stages;
+//                128-byte swizzle) and their residual byte ranges (bulk copies), into two rings of
+//                three slots: a K slot is free again once its block's S is done, a V slot once its
+//                P V is done, so the keys of block g + 3 load while block g's softmax and P V run;
 //   warp 1       TMEM owner (512 columns) and MMA issuer: S = Q K^T with Q read from TMEM (A
 //                operand) and K from shared memory (K-major B); O += P V with P from TMEM and V
 //                straight from the cache rows (keys x dims, the MN-major B operand); it takes
@@ -25,11 +27,11 @@
 //                only when the block max exceeds it by more than 8, so P <= 2^8), P written over
 //                the S columns it came from; after an item's first block they write the previous
 //                item's O / l as the output operand pair;
-//   warps 10-13  workers: K_lo and V_lo from the hi parts and their residual codes, in the hi
-//                parts' own swizzled layout, values of keys past the last visible one zeroed
-//                (their P is 0, and a stale NaN would still poison the product); and each item's
-//                Q rows (times log2(e) / sqrt(hd)) as an fp16 pair into TMEM once the previous
-//                item's last S is done.
+//   warps 10-13  workers, per block: K_lo from K_hi and its residual codes (in K_hi's own swizzled
+//                layout); at an item's first block its Q rows (times log2(e) / sqrt(hd)) as an fp16
+//                pair into TMEM once the previous item's last S is done; then V_lo likewise, values
+//                of keys past the last visible one zeroed (their P is 0, and a stale NaN would
+//                still poison the product).
 // TMEM columns: S/P [0,64) [64,128); O [128,128+HD) [128+HD,128+2HD) (items alternate);
 // Q_hi [128+2HD,128+2.5HD) Q_lo [128+2.5HD,128+3HD).  Every wait is bounded; on a timeout the CTA
 // records VLA_STATUS_TIMEOUT, drains its copies and MMAs, frees TMEM and stops.
@@ -128,13 +130,15 @@ template <int HD>
 struct AtSmem {
   static constexpr int K_BYTES = kKeys * HD * 2;        // one 64-key tile of K (or V), fp16
   static constexpr int R_BYTES = kKeys * HD / 2;        // its residual codes
-  // a stage: K_hi | V_hi | K_lo | V_lo | K codes | V codes (each tile 1024-byte aligned)
-  static constexpr int STAGE = 4 * K_BYTES + 2 * R_BYTES;
-  static constexpr int BARS = 256;                      // mbarriers, TMEM address, abort flag
+  // a slot: hi | lo | codes of one 64-key tile (hi and lo 1024-byte aligned); the K ring's
+  // kStages slots, then the V ring's
+  static constexpr int SLOT = 2 * K_BYTES + R_BYTES;
+  static constexpr int BARS = 512;                      // mbarriers, TMEM address, abort flag
   // + the softmax pairs' exchange: row maxima [2 blocks][2 halves][128] and partial row sums
   // [2 items][2 halves][128]
-  static constexpr int SMEM = 1024 + kStages * STAGE + BARS + 2 * (2 * 2 * 128 * 4);
-  static_assert(STAGE % 1024 == 0, "stage alignment");
+  static constexpr int SMEM = 1024 + 2 * kStages * SLOT + BARS + 2 * (2 * 2 * 128 * 4);
+  static_assert(SLOT % 1024 == 0, "slot alignment");
+  static_assert(SMEM <= 232448, "shared memory per CTA");
 };
 
 // The j-th item of this CTA: (tile, head) number blockIdx.x + j * gridDim.x, tile-major.
@@ -171,18 +175,19 @@ __global__ void __launch_bounds__(kAtThreads, 1)
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + kStages * Sm::STAGE);
-  float* xbuf = reinterpret_cast<float*>(smem + kStages * Sm::STAGE + Sm::BARS);  // [2][2][128] row maxima
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + 2 * kStages * Sm::SLOT);
+  float* xbuf = reinterpret_cast<float*>(smem + 2 * kStages * Sm::SLOT + Sm::BARS);  // [2][2][128] row maxima
   float* lbuf = xbuf + 2 * 2 * 128;                                                // [2][2][128] row sums
   const uint32_t b0 = smem_u32(bars);
   auto BAR = [&](int i) { return b0 + 8u * static_cast<uint32_t>(i); };
-  // per stage: full (loaded), conv (low parts written), stfree (MMAs done with it); per S/P
+  // per K / V slot: full (loaded), conv (low part written), free (its MMAs done); per S/P
   // buffer: sfull (S written), sfree (P V done with it), pfull (P written); pdone (the latest
   // P V done); qready / qfree (Q written / the item's last S done); per item parity: odone (O
   // final); drain; per lane quarter and block parity: xch (the softmax pair's exchange written)
-  const int FULL = 0, CONV = 3, STFREE = 6, SFULL = 9, SFREE = 11, PFULL = 13, PDONE = 15, QREADY = 16,
-            QFREE = 17, ODONE = 18, DRAIN = 20, XCH = 21;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 29);
+  const int FULLK = 0, FULLV = 3, CONVK = 6, CONVV = 9, KFREE = 12, VFREE = 15, SFULL = 18, SFREE = 20,
+            PFULL = 22, PDONE = 24, QREADY = 25, QFREE = 26, ODONE = 27, DRAIN = 29, XCH = 30;
+  static_assert(38 * 8 + 8 <= Sm::BARS, "barrier area");
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 38);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   pdl_launch_dependents();
@@ -194,9 +199,12 @@ __global__ void __launch_bounds__(kAtThreads, 1)
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
-      mbar_init(BAR(FULL + s), 1);
-      mbar_init(BAR(CONV + s), kWorkWarps);
-      mbar_init(BAR(STFREE + s), 1);
+      mbar_init(BAR(FULLK + s), 1);
+      mbar_init(BAR(FULLV + s), 1);
+      mbar_init(BAR(CONVK + s), kWorkWarps);
+      mbar_init(BAR(CONVV + s), kWorkWarps);
+      mbar_init(BAR(KFREE + s), 1);
+      mbar_init(BAR(VFREE + s), 1);
     }
     for (int s = 0; s < 2; ++s) {
       mbar_init(BAR(SFULL + s), 1);
@@ -224,54 +232,58 @@ __global__ void __launch_bounds__(kAtThreads, 1)
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
 
-  auto stage_ptr = [&](int st) { return smem + st * Sm::STAGE; };
+  auto kslot = [&](int st) { return smem + st * Sm::SLOT; };
+  auto vslot = [&](int st) { return smem + (kStages + st) * Sm::SLOT; };
 
   if (warp == 0) {
     if (lane == 0) {
       // ------------------------------------------------------------------ producer
       pdl_wait_async();  // the chunks' own keys / values were written by the q|k|v projection
+      // bit (ring * kStages + slot): a copy was issued there, with the phase it completes
       uint32_t issued = 0, issued_phase = 0;
       bool ok = true;
       int g = 0;  // block number over all of this CTA's items
       for (int j = 0; j < n_my && ok; ++j) {
         const Item it = get_item(p, j);
-        const int64_t vrow0 = it.krow0 + p.kv_rows;
-        for (int b = 0; b < it.nb; ++b, ++g) {
+        for (int b = 0; b < it.nb && ok; ++b, ++g) {
           const int st = g % kStages, round = g / kStages;
-          if (round >= 1 && !wait_bounded(BAR(STFREE + st), (round - 1) & 1, abort_flag, status, limit)) {
-            ok = false;
-            break;
-          }
-          const uint32_t s_khi = smem_u32(stage_ptr(st)), s_vhi = s_khi + Sm::K_BYTES;
-          const uint32_t s_kr = s_khi + 4 * Sm::K_BYTES, s_vr = s_kr + Sm::R_BYTES;
           const int key0 = b * kKeys;
           const int rows = min(kKeys, p.cap - key0);  // residual rows inside this (env, head)
           const uint32_t rbytes = static_cast<uint32_t>(rows) * (HD / 2);
-          mbar_arrive_expect_tx(BAR(FULL + st), 2u * Sm::K_BYTES + 2u * rbytes);
+          // the K tile into its ring, then the V tile into its own
+          for (int ring = 0; ring < 2; ++ring) {
+            if (round >= 1 &&
+                !wait_bounded(BAR((ring ? VFREE : KFREE) + st), (round - 1) & 1, abort_flag, status, limit)) {
+              ok = false;
+              break;
+            }
+            const uint32_t full = BAR((ring ? FULLV : FULLK) + st);
+            const uint32_t s_hi = smem_u32(ring ? vslot(st) : kslot(st));
+            const int64_t row0 = it.krow0 + (ring ? p.kv_rows : 0) + key0;
+            mbar_arrive_expect_tx(full, Sm::K_BYTES + rbytes);
 #pragma unroll
-          for (int kb = 0; kb < KB; ++kb) {
-            tma_load_2d(s_khi + kb * (kKeys * 128), &tmKV, BAR(FULL + st), kb * 64,
-                        static_cast<int>(it.krow0 + key0));
-            tma_load_2d(s_vhi + kb * (kKeys * 128), &tmKV, BAR(FULL + st), kb * 64, static_cast<int>(vrow0 + key0));
+            for (int kb = 0; kb < KB; ++kb)
+              tma_load_2d(s_hi + kb * (kKeys * 128), &tmKV, full, kb * 64, static_cast<int>(row0));
+            bulk_load(s_hi + 2 * Sm::K_BYTES, p.res + row0 * (HD / 2), rbytes, full);
+            const int bit = ring * kStages + st;
+            issued |= 1u << bit;
+            issued_phase = (issued_phase & ~(1u << bit)) | (static_cast<uint32_t>(round & 1) << bit);
           }
-          bulk_load(s_kr, p.res + (it.krow0 + key0) * (HD / 2), rbytes, BAR(FULL + st));
-          bulk_load(s_vr, p.res + (vrow0 + key0) * (HD / 2), rbytes, BAR(FULL + st));
-          issued |= 1u << st;
-          issued_phase = (issued_phase & ~(1u << st)) | (static_cast<uint32_t>(round & 1) << st);
         }
       }
-      for (int st = 0; st < kStages; ++st)
-        if (issued & (1u << st)) wait_drain(BAR(FULL + st), (issued_phase >> st) & 1u, limit);
+      for (int bit = 0; bit < 2 * kStages; ++bit)
+        if (issued & (1u << bit))
+          wait_drain(BAR((bit < kStages ? FULLK : FULLV) + bit % kStages), (issued_phase >> bit) & 1u, limit);
     }
   } else if (warp == 1) {
     if (lane == 0) {
       // ------------------------------------------------------------------ MMA issuer
       const uint32_t IS = idesc_f16(kKeys), IO = idesc_f16(HD, true);
       const uint32_t tQh = tmem + kColQ, tQl = tmem + kColQ + HD / 2;
-      // descriptors of stage 0's tiles; another stage (or k step) adds its byte offset / 16
-      const uint64_t dK0 = sdesc_sw128(smem_u32(stage_ptr(0)));
-      const uint64_t dV0 = sdesc_sw128(smem_u32(stage_ptr(0)) + Sm::K_BYTES, kKeys * 128);
-      constexpr uint64_t kStageStep = Sm::STAGE >> 4, kLoStep = (2 * Sm::K_BYTES) >> 4;
+      // descriptors of slot 0's tiles; another slot (or k step) adds its byte offset / 16
+      const uint64_t dK0 = sdesc_sw128(smem_u32(kslot(0)));
+      const uint64_t dV0 = sdesc_sw128(smem_u32(vslot(0)), kKeys * 128);
+      constexpr uint64_t kSlotStep = Sm::SLOT >> 4, kLoStep = Sm::K_BYTES >> 4;
       bool ok = true;
       // S cursor (item js, block bs, global block gs) and P V cursor (jo, bo, go)
       int js = 0, bs = 0, gs = 0, nbs = get_item(p, 0).nb;
@@ -280,10 +292,11 @@ __global__ void __launch_bounds__(kAtThreads, 1)
       uint32_t spins = 0;
       while (ok && jo < n_my) {
         bool did = false;
-        if (go < gs && mbar_test_wait(BAR(PFULL + (go & 1)), (go >> 1) & 1)) {
+        if (go < gs && mbar_test_wait(BAR(PFULL + (go & 1)), (go >> 1) & 1) &&
+            mbar_test_wait(BAR(CONVV + go % kStages), (go / kStages) & 1)) {
           // O(jo) (+)= P V of block go
           tc_fence_after();
-          const uint64_t dvh = dV0 + (go % kStages) * kStageStep;
+          const uint64_t dvh = dV0 + (go % kStages) * kSlotStep;
           const uint32_t tO = tmem + kColO + (jo & 1) * HD;
           const uint32_t tPh = tmem + kColS + (go & 1) * kKeys, tPl = tPh + kKeys / 2;
 #pragma unroll
@@ -295,7 +308,7 @@ __global__ void __launch_bounds__(kAtThreads, 1)
           }
           tc_commit(BAR(PDONE));
           tc_commit(BAR(SFREE + (go & 1)));
-          tc_commit(BAR(STFREE + go % kStages));
+          tc_commit(BAR(VFREE + go % kStages));
           if (bo == nbo - 1) tc_commit(BAR(ODONE + (jo & 1)));
           ++go;
           if (++bo == nbo) {
@@ -303,12 +316,12 @@ __global__ void __launch_bounds__(kAtThreads, 1)
             if (++jo < n_my) nbo = get_item(p, jo).nb;
           }
           did = true;
-        } else if (js < n_my && mbar_test_wait(BAR(CONV + gs % kStages), (gs / kStages) & 1) &&
+        } else if (js < n_my && mbar_test_wait(BAR(CONVK + gs % kStages), (gs / kStages) & 1) &&
                    (gs < 2 || mbar_test_wait(BAR(SFREE + (gs & 1)), ((gs >> 1) - 1) & 1)) &&
                    (bs > 0 || mbar_test_wait(BAR(QREADY), js & 1))) {
           // S of block gs into buffer gs & 1
           tc_fence_after();
-          const uint64_t dkh = dK0 + (gs % kStages) * kStageStep;
+          const uint64_t dkh = dK0 + (gs % kStages) * kSlotStep;
           const uint32_t tS = tmem + kColS + (gs & 1) * kKeys;
 #pragma unroll
           for (int k = 0; k < HD / 16; ++k) {
@@ -318,6 +331,7 @@ __global__ void __launch_bounds__(kAtThreads, 1)
             mma_ts(tS, tQh + k * 8, dl, IS, 1u);
           }
           tc_commit(BAR(SFULL + (gs & 1)));
+          tc_commit(BAR(KFREE + gs % kStages));
           if (bs == nbs - 1) tc_commit(BAR(QFREE));
           ++gs;
           if (++bs == nbs) {
@@ -502,10 +516,10 @@ __global__ void __launch_bounds__(kAtThreads, 1)
     const uint32_t lane_off = static_cast<uint32_t>(q4 * 32) << 16;
     const int t = threadIdx.x - kWorkWarp0 * 32;
     const int dcols = p.H * HD;
-    constexpr int CH = HD / 8;                                 // 16-byte chunks of one row
-    constexpr int ITER = 2 * kKeys * CH / (32 * kWorkWarps);   // chunks per thread and block
-    constexpr int KSTEP = 32 * kWorkWarps / CH;                // rows between a thread's chunks
-    static_assert((32 * kWorkWarps) % CH == 0 && ITER % 2 == 0, "converter tiling");
+    constexpr int CH = HD / 8;                             // 16-byte chunks of one row
+    constexpr int ITER = kKeys * CH / (32 * kWorkWarps);   // chunks per thread and tile
+    constexpr int KSTEP = 32 * kWorkWarps / CH;            // rows between a thread's chunks
+    static_assert((32 * kWorkWarps) % CH == 0 && ITER >= 1, "converter tiling");
     pdl_wait();  // the queries were written by the q|k|v projection
     // Q rows of an item, times log2(e) / sqrt(HD), -> fp16 pair in TMEM (A operand of S)
     auto write_q = [&](const Item& it) {
@@ -542,45 +556,45 @@ __global__ void __launch_bounds__(kAtThreads, 1)
         for (int c = 0; c < HD; c += 32) asm volatile("prefetch.global.L2 [%0];" ::"l"(qrow + c));
       }
     };
+    // the low part of the tile in `slot` (hi | lo | codes): a thread's chunks all sit in one
+    // column c (the stride over chunks is a multiple of CH), rows key0t, key0t + KSTEP, ...:
+    // loads first, then decode and stores; keys >= live zeroed (hi and lo) when `zero_dead`
+    auto convert = [&](uint8_t* slot, bool zero_dead, int live) {
+      const int c = t % CH, key0t = t / CH;
+      const int coff = (c >> 3) * (kKeys * 128) + key0t * 128 + (((c & 7) ^ (key0t & 7)) << 4);
+      uint4 hv[ITER];
+      uint32_t cv[ITER];
+#pragma unroll
+      for (int i = 0; i < ITER; ++i) {
+        hv[i] = *reinterpret_cast<const uint4*>(slot + coff + i * KSTEP * 128);
+        cv[i] = *reinterpret_cast<const uint32_t*>(slot + 2 * Sm::K_BYTES + (key0t + i * KSTEP) * (HD / 2) + c * 4);
+      }
+#pragma unroll
+      for (int i = 0; i < ITER; ++i) {
+        const int off = coff + i * KSTEP * 128;
+        uint4* lo = reinterpret_cast<uint4*>(slot + Sm::K_BYTES + off);
+        if (zero_dead && key0t + i * KSTEP >= live) {
+          *reinterpret_cast<uint4*>(slot + off) = make_uint4(0u, 0u, 0u, 0u);
+          *lo = make_uint4(0u, 0u, 0u, 0u);
+        } else {
+          *lo = kv_res_lo8(hv[i], cv[i]);
+        }
+      }
+      fence_async_smem();  // the MMAs (async proxy) read what these generic stores wrote
+      __syncwarp();
+    };
     bool ok = true;
     int g = 0;
     for (int j = 0; j < n_my && ok; ++j) {
       const Item it = get_item(p, j);
       for (int b = 0; b < it.nb; ++b, ++g) {
-        const int st = g % kStages;
-        if (!warp_wait(BAR(FULL + st), (g / kStages) & 1, abort_flag, status, limit)) {
+        const int st = g % kStages, ph = (g / kStages) & 1;
+        if (!warp_wait(BAR(FULLK + st), ph, abort_flag, status, limit)) {
           ok = false;
           break;
         }
-        // K_lo, V_lo: a thread's chunks all sit in one column c (the stride over chunks is a
-        // multiple of CH), rows key0t, key0t + KSTEP, ...: loads first, then decode and stores
-        uint8_t* sp = stage_ptr(st);
-        const int live = it.n_keys - b * kKeys;  // keys of this block visible to some row
-        const int c = t % CH, key0t = t / CH;
-        const int coff = (c >> 3) * (kKeys * 128) + key0t * 128 + (((c & 7) ^ (key0t & 7)) << 4);
-        uint4 hv[ITER];
-        uint32_t cv[ITER];
-#pragma unroll
-        for (int i = 0; i < ITER; ++i) {
-          const int w = i / (ITER / 2), key = key0t + (i % (ITER / 2)) * KSTEP;
-          hv[i] = *reinterpret_cast<const uint4*>(sp + w * Sm::K_BYTES + coff + (i % (ITER / 2)) * KSTEP * 128);
-          cv[i] = *reinterpret_cast<const uint32_t*>(sp + 4 * Sm::K_BYTES + w * Sm::R_BYTES + key * (HD / 2) + c * 4);
-        }
-#pragma unroll
-        for (int i = 0; i < ITER; ++i) {
-          const int w = i / (ITER / 2), key = key0t + (i % (ITER / 2)) * KSTEP;
-          const int off = coff + (i % (ITER / 2)) * KSTEP * 128;
-          uint4* lo = reinterpret_cast<uint4*>(sp + (2 + w) * Sm::K_BYTES + off);
-          if (w == 1 && key >= live) {
-            *reinterpret_cast<uint4*>(sp + Sm::K_BYTES + off) = make_uint4(0u, 0u, 0u, 0u);
-            *lo = make_uint4(0u, 0u, 0u, 0u);
-          } else {
-            *lo = kv_res_lo8(hv[i], cv[i]);
-          }
-        }
-        fence_async_smem();  // the MMAs (async proxy) read what these generic stores wrote
-        __syncwarp();
-        if (lane == 0) mbar_arrive(BAR(CONV + st));
+        convert(kslot(st), false, 0);
+        if (lane == 0) mbar_arrive(BAR(CONVK + st));
         if (b == 0) {
           // this item's queries, once the previous item's last S is done
           if (j > 0) {
@@ -593,6 +607,12 @@ __global__ void __launch_bounds__(kAtThreads, 1)
           write_q(it);
           if (j + 1 < n_my) prefetch_q(get_item(p, j + 1));
         }
+        if (!warp_wait(BAR(FULLV + st), ph, abort_flag, status, limit)) {
+          ok = false;
+          break;
+        }
+        convert(vslot(st), true, it.n_keys - b * kKeys);  // keys of this block visible to some row
+        if (lane == 0) mbar_arrive(BAR(CONVV + st));
       }
     }
   }
