@@ -234,6 +234,7 @@ CASES = {
     "attn_score": None,                                        # 6 rows per env after the prefix
     "attn_chunk_res": None,                                    # the same over fp16 + 4-bit residual
     "attn_score_res": None,
+    "attn_score_rows_res": None,                               # the few-row kernel (tiles <= 16 rows)
     # the same prefill shapes on CTA pairs (2-SM MMAs, 256 x 256 tiles)
     "pair_prefill_qkv": (4608, 12288, 4096, 256, 1, True),
     "pair_prefill_down": (4608, 4096, 11008, 256, 1, True),
@@ -254,6 +255,17 @@ CASES = {
     "pair_score_qkv": (384, 12288, 4096, 256, 1, True),
     "pair_score_down": (384, 4096, 11008, 256, 1, True),
     "gemm_score_down_bn256": (384, 4096, 11008, 256, 1, True),
+    # the same in the engine's form: fp16 operands, the activation's high half alone
+    "gemm_score_o_s1_hi_f16": (384, 4096, 4096, 128, 1, False),
+    "gemm_score_o_s2_hi_f16": (384, 4096, 4096, 128, 2, False),
+    "gemm_score_o_bn256_s3_hi_f16": (384, 4096, 4096, 256, 3, False),
+    "gemm_score_down_s1_hi_f16": (384, 4096, 11008, 128, 1, False),
+    "gemm_score_down_s2_hi_f16": (384, 4096, 11008, 128, 2, False),
+    "gemm_score_down_bn256_s3_hi_f16": (384, 4096, 11008, 256, 3, False),
+    "gemm_score_gate_up_bn256_hi_f16": (384, 22016, 4096, 256, 1, False),
+    "gemm_score_gate_up_bn128_hi_f16": (384, 22016, 4096, 128, 1, False),
+    "gemm_score_qkv_bn128_f16": (384, 12288, 4096, 128, 1, True),
+    "gemm_score_qkv_bn256_s2_f16": (384, 12288, 4096, 256, 2, True),
     "gemv_score_o_m128": (128, 4096, 4096, 0, 0, True),
     "gemv_score_down_m128": (128, 4096, 11008, 0, 0, True),
     # decode GEMM at 2x / 4x the weight bytes of the q|k|v step (fixed vs per-byte cost)
@@ -324,7 +336,8 @@ def run_attn_chunk_case(args):
     """Prefill chunk attention of one layer of the bench step: 64 envs, 256 visual + U{16..48}
     text rows each, 32 heads x 128.  attn_chunk / attn_score: the fp16-cache kernel, tiles of
     <= 64 query rows; attn_chunk_res / attn_score_res: the tcgen05 kernel over the fp16 +
-    4-bit residual cache (the engine's form), tiles of <= 128 rows."""
+    4-bit residual cache, tiles of <= 128 rows; attn_score_rows_res: the few-row kernel over the
+    same cache (the engine's score-pass form)."""
     import torch
     import __graft_entry__
     __graft_entry__.build()
@@ -334,6 +347,7 @@ def run_attn_chunk_case(args):
     prefix = (256 + I.randint_i32((B,), 5, 7, 16, 48)).tolist()
     score = args.case.startswith("attn_score")   # the score pass: 6 rows per env after its prefix
     res = args.case.endswith("_res")
+    few = args.case == "attn_score_rows_res"
     tile_rows = 128 if res else 64
     lens = [6] * B if score else prefix
     past = prefix if score else [0] * B
@@ -351,7 +365,10 @@ def run_attn_chunk_case(args):
     ol = torch.empty_like(oh)
 
     def launch():
-        if res:
+        if few:
+            rc = V.vla_op_attn_rows_res(q.data_ptr(), kv.data_ptr(), codes.data_ptr(), B, H, hd, cap, tiles, rows,
+                                        tiles_dev.data_ptr(), oh.data_ptr(), ol.data_ptr())
+        elif res:
             rc = V.vla_op_attn_chunk_res(q.data_ptr(), kv.data_ptr(), codes.data_ptr(), B, H, hd, cap, tiles, rows,
                                          tiles_dev.data_ptr(), oh.data_ptr(), ol.data_ptr())
         else:

@@ -169,6 +169,15 @@ int vla_op_attn_chunk_res(const float* q, const void* kv, const void* kv_res, in
                           int cap, const int32_t* tiles_host, int n_tiles, int rows, int32_t* tiles_dev,
                           void* out_hi, void* out_lo, void* cuda_stream);
 
+/* The same attention for short tiles, the engine's kernel when every tile has at most 16 rows
+ * (the PPO ratio pass of Eq. 2: A - 1 teacher-forced rows per env): arguments as
+ * vla_op_attn_chunk_res, with 1 <= nrows <= 16 per tile (VLA_ERR_ARG otherwise, nothing runs).
+ * mma.sync on one CTA per (tile, head): each cached byte is read once per tile and head, and no
+ * MMA row past the 16th is spent; same results to fp32 rounding order. */
+int vla_op_attn_rows_res(const float* q, const void* kv, const void* kv_res, int max_env, int H, int hd,
+                         int cap, const int32_t* tiles_host, int n_tiles, int rows, int32_t* tiles_dev,
+                         void* out_hi, void* out_lo, void* cuda_stream);
+
 /* Number of SMs the kernels size their persistent grids for (device property). */
 int vla_op_num_sms(void);
 

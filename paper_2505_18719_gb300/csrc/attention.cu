@@ -268,6 +268,286 @@ __global__ void __launch_bounds__(128) attn_chunk_mma_kernel(const float* q,
   }
 }
 
+// ------------------------------------------------------------------ few-row chunk (residual cache)
+// Query tiles of at most 16 rows (the teacher-forced action rows of the score pass, Eq. 2, or any
+// chunk that short) against keys 0..pos of their env, the cache read as fp16 + 4-bit residual
+// (hi + lo, KVLayout).  One CTA per (tile, head), 4 warps: key blocks of 64 staged in shared memory
+// by cp.async (fp16 parts and residual codes, two stages; keys past the tile's last position are
+// zero-filled, never read); warp w takes keys 16w .. 16w+15 of every block with one m16n8k16 row
+// tile (rows past the tile's last repeat its last row and are not written), the low parts decoded
+// from the codes beside each B fragment:
+//   S = Q_hi K_hi + Q_lo K_hi + Q_hi K_lo,   O += P_hi V_hi + P_lo V_hi + P_hi V_lo,
+// online softmax per warp in the exp2 domain (Q pre-scaled by log2(e) / sqrt(hd)); the four warps'
+// (max, sum, O) merge through shared memory at the end.  Each cached byte is read once per (tile,
+// head), against a 128-row tensor-core tile that would spend 7/8 of its MMAs on padding rows.
+template <int HD>
+struct RowsSmem {
+  static constexpr int KB = 64;                 // keys per staged block
+  static constexpr int LD = HD + 8;             // padded fp16 row (halves): ldmatrix rows in distinct banks
+  static constexpr int RB = HD / 2;             // residual bytes of one row
+  static constexpr int RBP = RB + 16;           // padded code row: the fragment reads hit distinct banks
+  static constexpr int PLANE = KB * LD * 2;     // bytes of one staged fp16 block
+  static constexpr int CODES = KB * RBP;        // bytes of one staged code block
+  static constexpr int STAGE = 2 * PLANE + 2 * CODES;  // K | V | K codes | V codes
+  static constexpr int SMEM = 2 * STAGE;
+  static_assert(STAGE % 16 == 0 && 4 * 16 * HD * 4 + 4 * 16 * 2 * 4 <= SMEM, "staging / merge layout");
+};
+
+template <int HD>
+__global__ void __launch_bounds__(128) attn_rows_kernel(const float* q, bf16* out_hi, bf16* out_lo,
+                                                        const AttnTile* tiles, KVLayout kv, int layer, int H,
+                                                        float scale_log2, bool fp16, bool write_lo) {
+  using Sm = RowsSmem<HD>;
+  constexpr int KB = Sm::KB, LD = Sm::LD, RB = Sm::RB, RBP = Sm::RBP, PLANE = Sm::PLANE, STAGE = Sm::STAGE;
+  constexpr int CPR = HD / 8;   // 16-byte chunks of an fp16 row
+  constexpr int NT_D = HD / 8;  // n-tiles over the head dim
+  constexpr int RWP = RBP / 4;  // 32-bit words of a padded code row
+  extern __shared__ __align__(16) uint8_t sm_rows[];
+
+  pdl_launch_dependents();
+  pdl_wait();
+  const AttnTile t = tiles[blockIdx.x];
+  const int head = blockIdx.y;
+  const int d = H * HD;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int g = lane >> 2, tq = lane & 3;
+  const int64_t e0 = static_cast<int64_t>(layer) * kv.layer_stride + static_cast<int64_t>(t.env) * kv.env_stride +
+                     static_cast<int64_t>(head) * kv.head_stride;
+  const f16* kbase = kv.base + e0;
+  const f16* vbase = kbase + kv.kv_stride;
+  const uint8_t* kres = kv.res + e0 / 2;
+  const uint8_t* vres = kres + kv.kv_stride / 2;
+  const int n_keys = t.pos0 + t.nrows;
+  const int n_blocks = (n_keys + KB - 1) / KB;
+  const int last_pos = n_keys - 1;
+
+  auto load_block = [&](int blk, int buf) {
+    const int j0 = blk * KB;
+    const uint32_t s0 = smem_u32(sm_rows + buf * STAGE);
+    for (int i = tid; i < KB * CPR; i += 128) {
+      const int r = i / CPR, c = i - r * CPR;
+      const bool ok = j0 + r < n_keys;
+      const int64_t src = static_cast<int64_t>(ok ? j0 + r : 0) * HD + c * 8;
+      cp_async16(s0 + (r * LD + c * 8) * 2, kbase + src, ok);
+      cp_async16(s0 + PLANE + (r * LD + c * 8) * 2, vbase + src, ok);
+    }
+    for (int i = tid; i < KB * (RB / 16); i += 128) {
+      const int r = i / (RB / 16), c = i - r * (RB / 16);
+      const bool ok = j0 + r < n_keys;
+      const int64_t src = static_cast<int64_t>(ok ? j0 + r : 0) * RB + c * 16;
+      cp_async16(s0 + 2 * PLANE + r * RBP + c * 16, kres + src, ok);
+      cp_async16(s0 + 2 * PLANE + Sm::CODES + r * RBP + c * 16, vres + src, ok);
+    }
+  };
+  load_block(0, 0);
+  cp_async_commit();
+
+  // this thread's two rows (g and g + 8 of the tile) and their positions
+  const int ra = min(g, t.nrows - 1), rb = min(g + 8, t.nrows - 1);
+  const int qpos0 = t.pos0 + ra, qpos1 = t.pos0 + rb;
+  // Q A-fragments from the fp32 rows times log2(e) / sqrt(hd), as fp16 hi / lo pairs
+  uint32_t qh[HD / 16][4], ql[HD / 16][4];
+  {
+    const float* qa = q + static_cast<size_t>(t.row0 + ra) * d + head * HD + 2 * tq;
+    const float* qb = q + static_cast<size_t>(t.row0 + rb) * d + head * HD + 2 * tq;
+#pragma unroll
+    for (int kk = 0; kk < HD / 16; ++kk) {
+      const float2 x0 = __ldcg(reinterpret_cast<const float2*>(qa + kk * 16));
+      const float2 x1 = __ldcg(reinterpret_cast<const float2*>(qb + kk * 16));
+      const float2 x2 = __ldcg(reinterpret_cast<const float2*>(qa + kk * 16 + 8));
+      const float2 x3 = __ldcg(reinterpret_cast<const float2*>(qb + kk * 16 + 8));
+      split_h2(x0.x * scale_log2, x0.y * scale_log2, qh[kk][0], ql[kk][0]);
+      split_h2(x1.x * scale_log2, x1.y * scale_log2, qh[kk][1], ql[kk][1]);
+      split_h2(x2.x * scale_log2, x2.y * scale_log2, qh[kk][2], ql[kk][2]);
+      split_h2(x3.x * scale_log2, x3.y * scale_log2, qh[kk][3], ql[kk][3]);
+    }
+  }
+
+  float o[NT_D][4];
+#pragma unroll
+  for (int i = 0; i < NT_D; ++i) o[i][0] = o[i][1] = o[i][2] = o[i][3] = 0.f;
+  float m0 = -INFINITY, m1 = -INFINITY, l0 = 0.f, l1 = 0.f;
+  const int im = lane >> 3;  // the ldmatrix sub-matrix this lane addresses
+
+  for (int blk = 0; blk < n_blocks; ++blk) {
+    if (blk + 1 < n_blocks) {
+      load_block(blk + 1, (blk + 1) & 1);
+      cp_async_commit();
+      cp_async_wait<1>();
+    } else {
+      cp_async_wait<0>();
+    }
+    __syncthreads();
+    const int k0 = blk * KB + warp * 16;  // this warp's first key
+    if (k0 <= last_pos) {
+      const uint8_t* stg = sm_rows + (blk & 1) * STAGE;
+      const uint32_t ks = smem_u32(stg), vs = ks + PLANE;
+      const uint32_t* kc = reinterpret_cast<const uint32_t*>(stg + 2 * PLANE);
+      const uint32_t* vc = reinterpret_cast<const uint32_t*>(stg + 2 * PLANE + Sm::CODES);
+      float s[2][4];
+#pragma unroll
+      for (int nt = 0; nt < 2; ++nt) {
+        s[nt][0] = s[nt][1] = s[nt][2] = s[nt][3] = 0.f;
+        const int key = warp * 16 + nt * 8 + (lane & 7);
+        // this thread's B elements are in key row warp*16 + nt*8 + g; the codes of dims
+        // 16kk + 2tq (+1) sit in byte tq of the row's word 2kk (+1 for dims + 8)
+        const uint32_t* crow = kc + (warp * 16 + nt * 8 + g) * RWP;
+#pragma unroll
+        for (int kk = 0; kk < HD / 16; kk += 2) {
+          uint32_t b0, b1, b2, b3;
+          const int dim = (kk + (im >> 1)) * 16 + (im & 1) * 8;
+          ldsm_x4(ks + (key * LD + dim) * 2, b0, b1, b2, b3);
+          const uint4 cw = *reinterpret_cast<const uint4*>(crow + 2 * kk);
+          const int sh = 8 * tq;
+          const uint32_t l0b = kv_res_lo2(b0, (cw.x >> sh) & 15u, (cw.x >> (sh + 4)) & 15u);
+          const uint32_t l1b = kv_res_lo2(b1, (cw.y >> sh) & 15u, (cw.y >> (sh + 4)) & 15u);
+          const uint32_t l2b = kv_res_lo2(b2, (cw.z >> sh) & 15u, (cw.z >> (sh + 4)) & 15u);
+          const uint32_t l3b = kv_res_lo2(b3, (cw.w >> sh) & 15u, (cw.w >> (sh + 4)) & 15u);
+          mma16816(s[nt], qh[kk], b0, b1);
+          mma16816(s[nt], ql[kk], b0, b1);
+          mma16816(s[nt], qh[kk], l0b, l1b);
+          mma16816(s[nt], qh[kk + 1], b2, b3);
+          mma16816(s[nt], ql[kk + 1], b2, b3);
+          mma16816(s[nt], qh[kk + 1], l2b, l3b);
+        }
+      }
+      // causal mask, online softmax (row g: c 0, 1; row g + 8: c 2, 3)
+      float mx0 = -INFINITY, mx1 = -INFINITY;
+#pragma unroll
+      for (int nt = 0; nt < 2; ++nt) {
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+          const int kpos = k0 + nt * 8 + 2 * tq + (c & 1);
+          if (kpos > ((c < 2) ? qpos0 : qpos1)) s[nt][c] = -INFINITY;
+        }
+        mx0 = fmaxf(mx0, fmaxf(s[nt][0], s[nt][1]));
+        mx1 = fmaxf(mx1, fmaxf(s[nt][2], s[nt][3]));
+      }
+      mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 1));
+      mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 2));
+      mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 1));
+      mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 2));
+      const float mn0 = fmaxf(m0, mx0), mn1 = fmaxf(m1, mx1);
+      // a row with no visible key yet (in this warp's share) keeps max -inf: reference 0, weights 0
+      const float u0 = mn0 == -INFINITY ? 0.f : mn0, u1 = mn1 == -INFINITY ? 0.f : mn1;
+      const float a0 = exp2f(m0 - u0), a1 = exp2f(m1 - u1);
+      m0 = mn0;
+      m1 = mn1;
+      float ps0 = 0.f, ps1 = 0.f;
+#pragma unroll
+      for (int nt = 0; nt < 2; ++nt) {
+        s[nt][0] = exp2f(s[nt][0] - u0);
+        s[nt][1] = exp2f(s[nt][1] - u0);
+        s[nt][2] = exp2f(s[nt][2] - u1);
+        s[nt][3] = exp2f(s[nt][3] - u1);
+        ps0 += s[nt][0] + s[nt][1];
+        ps1 += s[nt][2] + s[nt][3];
+      }
+      l0 = l0 * a0 + ps0;  // per-thread partial row sums, reduced across the quad at the end
+      l1 = l1 * a1 + ps1;
+#pragma unroll
+      for (int nt = 0; nt < NT_D; ++nt) {
+        o[nt][0] *= a0;
+        o[nt][1] *= a0;
+        o[nt][2] *= a1;
+        o[nt][3] *= a1;
+      }
+      // O += P V: P from the S accumulators as the A operand (keys 0..7 of the warp's 16 in s[0],
+      // 8..15 in s[1]), an fp16 hi / lo pair
+      uint32_t ph[4], pl[4];
+      split_h2(s[0][0], s[0][1], ph[0], pl[0]);
+      split_h2(s[0][2], s[0][3], ph[1], pl[1]);
+      split_h2(s[1][0], s[1][1], ph[2], pl[2]);
+      split_h2(s[1][2], s[1][3], ph[3], pl[3]);
+      // V^T fragments: this thread holds keys 2tq, 2tq + 1 (b0, b2) and 8 + 2tq, 9 + 2tq (b1, b3) of
+      // the warp's 16 at dim 8n + g; that element's code is nibble g of the key row's word n
+      const uint32_t* vrow = vc + (warp * 16 + 2 * tq) * RWP;
+      const int key = warp * 16 + (im & 1) * 8 + (lane & 7);
+      const int sh = 4 * g;
+#pragma unroll
+      for (int nt = 0; nt < NT_D; nt += 2) {
+        uint32_t b0, b1, b2, b3;
+        ldsm_x4_t(vs + (key * LD + (nt + (im >> 1)) * 8) * 2, b0, b1, b2, b3);
+        const uint2 c00 = *reinterpret_cast<const uint2*>(vrow + nt);            // key 2tq
+        const uint2 c01 = *reinterpret_cast<const uint2*>(vrow + RWP + nt);      // key 2tq + 1
+        const uint2 c10 = *reinterpret_cast<const uint2*>(vrow + 8 * RWP + nt);  // key 8 + 2tq
+        const uint2 c11 = *reinterpret_cast<const uint2*>(vrow + 9 * RWP + nt);  // key 9 + 2tq
+        const uint32_t l0b = kv_res_lo2(b0, (c00.x >> sh) & 15u, (c01.x >> sh) & 15u);
+        const uint32_t l1b = kv_res_lo2(b1, (c10.x >> sh) & 15u, (c11.x >> sh) & 15u);
+        const uint32_t l2b = kv_res_lo2(b2, (c00.y >> sh) & 15u, (c01.y >> sh) & 15u);
+        const uint32_t l3b = kv_res_lo2(b3, (c10.y >> sh) & 15u, (c11.y >> sh) & 15u);
+        mma16816(o[nt], ph, b0, b1);
+        mma16816(o[nt], pl, b0, b1);
+        mma16816(o[nt], ph, l0b, l1b);
+        mma16816(o[nt + 1], ph, b2, b3);
+        mma16816(o[nt + 1], pl, b2, b3);
+        mma16816(o[nt + 1], ph, l2b, l3b);
+      }
+    }
+    __syncthreads();  // this buffer is refilled two blocks later
+  }
+
+  // merge the four warps' partials: O [warp][16][HD] and (max, sum) [warp][16] over the stages
+  l0 += __shfl_xor_sync(0xffffffffu, l0, 1);
+  l0 += __shfl_xor_sync(0xffffffffu, l0, 2);
+  l1 += __shfl_xor_sync(0xffffffffu, l1, 1);
+  l1 += __shfl_xor_sync(0xffffffffu, l1, 2);
+  float* mo = reinterpret_cast<float*>(sm_rows);
+  float* mml = mo + 4 * 16 * HD;
+  {
+    float* oa = mo + (warp * 16 + g) * HD + 2 * tq;
+    float* ob = oa + 8 * HD;
+#pragma unroll
+    for (int nt = 0; nt < NT_D; ++nt) {
+      *reinterpret_cast<float2*>(oa + nt * 8) = make_float2(o[nt][0], o[nt][1]);
+      *reinterpret_cast<float2*>(ob + nt * 8) = make_float2(o[nt][2], o[nt][3]);
+    }
+    if (tq == 0) {
+      *reinterpret_cast<float2*>(mml + (warp * 16 + g) * 2) = make_float2(m0, l0);
+      *reinterpret_cast<float2*>(mml + (warp * 16 + g + 8) * 2) = make_float2(m1, l1);
+    }
+  }
+  __syncthreads();
+  constexpr int CPT = HD / 8;  // output columns per thread: 8 threads per row
+  const int row = tid >> 3, c0 = (tid & 7) * CPT;
+  if (row >= t.nrows) return;
+  float mw[4], lw[4], mx = -INFINITY;
+#pragma unroll
+  for (int w = 0; w < 4; ++w) {
+    const float2 ml = *reinterpret_cast<const float2*>(mml + (w * 16 + row) * 2);
+    mw[w] = ml.x;
+    lw[w] = ml.y;
+    mx = fmaxf(mx, ml.x);  // finite: warp 0 holds key 0, visible to every row
+  }
+  float wt[4], lsum = 0.f;
+#pragma unroll
+  for (int w = 0; w < 4; ++w) {
+    wt[w] = exp2f(mw[w] - mx);  // 0 for a warp that saw no visible key of this row
+    lsum += wt[w] * lw[w];
+  }
+  const float inv = 1.f / lsum;
+  uint32_t sat = 0;  // convex combinations of cached values: the fp16 split never saturates
+  uint32_t hi[CPT / 2], lo[CPT / 2];
+#pragma unroll
+  for (int c = 0; c < CPT; c += 2) {
+    float v0 = 0.f, v1 = 0.f;
+#pragma unroll
+    for (int w = 0; w < 4; ++w) {
+      const float2 x = *reinterpret_cast<const float2*>(mo + (w * 16 + row) * HD + c0 + c);
+      v0 += wt[w] * x.x;
+      v1 += wt[w] * x.y;
+    }
+    split_pack2(v0 * inv, v1 * inv, hi[c / 2], lo[c / 2], fp16, sat);
+  }
+  const size_t off = static_cast<size_t>(t.row0 + row) * d + head * HD + c0;
+#pragma unroll
+  for (int i = 0; i < CPT / 8; ++i) {
+    reinterpret_cast<uint4*>(out_hi + off)[i] = make_uint4(hi[4 * i], hi[4 * i + 1], hi[4 * i + 2], hi[4 * i + 3]);
+    if (write_lo)
+      reinterpret_cast<uint4*>(out_lo + off)[i] = make_uint4(lo[4 * i], lo[4 * i + 1], lo[4 * i + 2], lo[4 * i + 3]);
+  }
+}
+
 // ---------------------------------------------------------------------------------- decode
 // One query per (env, head, key range): 16 lanes x 16 bytes read one 128-element fp16 key row
 // (with RES, also its 4-bit residual codes, 4 bytes per lane, and use hi + lo as the cached value),
@@ -500,6 +780,29 @@ int attn_chunk_launch(const float* q, bf16* out_hi, bf16* out_lo, const AttnTile
                             tiles, kv, layer, H, scale_log2, fp16));
   } else {
     return VLA_ERR_UNSUPPORTED;
+  }
+  note_launch();
+  VLA_CUDA_TRY(cudaGetLastError());
+  return VLA_OK;
+}
+
+int attn_rows_launch(const float* q, bf16* out_hi, bf16* out_lo, const AttnTile* tiles, int n_tiles, KVLayout kv,
+                     int layer, int H, int hd, cudaStream_t stream, bool fp16, bool write_lo) {
+  if (n_tiles <= 0) return VLA_OK;
+  if (!kv.res || (hd != 64 && hd != 128)) return VLA_ERR_UNSUPPORTED;
+  if ((reinterpret_cast<uintptr_t>(kv.base) & 15) || (reinterpret_cast<uintptr_t>(kv.res) & 15)) return VLA_ERR_ARG;
+  const float scale_log2 = 1.4426950408889634f / sqrtf(static_cast<float>(hd));
+  const dim3 grid(n_tiles, H);
+  if (hd == 128) {
+    static std::atomic<uint64_t> attr_done{0};
+    VLA_CUDA_TRY(set_smem_limit(attn_rows_kernel<128>, RowsSmem<128>::SMEM, attr_done));
+    VLA_CUDA_TRY(launch_pdl(attn_rows_kernel<128>, grid, dim3(128), RowsSmem<128>::SMEM, stream, q, out_hi, out_lo,
+                            tiles, kv, layer, H, scale_log2, fp16, write_lo));
+  } else {
+    static std::atomic<uint64_t> attr_done{0};
+    VLA_CUDA_TRY(set_smem_limit(attn_rows_kernel<64>, RowsSmem<64>::SMEM, attr_done));
+    VLA_CUDA_TRY(launch_pdl(attn_rows_kernel<64>, grid, dim3(128), RowsSmem<64>::SMEM, stream, q, out_hi, out_lo,
+                            tiles, kv, layer, H, scale_log2, fp16, write_lo));
   }
   note_launch();
   VLA_CUDA_TRY(cudaGetLastError());

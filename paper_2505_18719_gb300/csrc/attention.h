@@ -23,6 +23,13 @@ int attn_chunk_tc_launch(const float* q, bf16* out_hi, bf16* out_lo, const AttnT
                          KVLayout kv, int layer, int H, int hd, uint32_t* status, cudaStream_t stream, bool fp16,
                          int num_sms, bool write_lo);
 
+// The same for tiles of at most 16 rows (kv.res required; not checked on the device: the caller
+// guarantees nrows <= 16), on mma.sync with one CTA per (tile, head): each cached byte is read once
+// per tile and head, with no padding rows beyond 16.  write_lo as attn_chunk_tc_launch.
+constexpr int kAttnRowsMax = 16;
+int attn_rows_launch(const float* q, bf16* out_hi, bf16* out_lo, const AttnTile* tiles, int n_tiles, KVLayout kv,
+                     int layer, int H, int hd, cudaStream_t stream, bool fp16, bool write_lo);
+
 // One query per env row b (rows[b] gives env and position); key range split into equal ranges
 // of at most `chunk` keys (a multiple of 16 at least 16); partials in part_o [B*H*S*hd] f32 and part_ml [B*H*S]
 // (S = ceil(max_ctx/chunk)); counters [B*H] int must be zero at launch and are zero again

@@ -62,19 +62,26 @@ __device__ __forceinline__ uint32_t kv_res_code(float x, f16 hi) {
 // 2^(e - 30) is the value with mantissa and sign cleared (2^(e-15)) times 2^-15.  Exact for
 // e >= 6; below that the term is under 2^-21 in magnitude and comes out as zero or a rounded
 // subnormal.
+// The pair form: h2 two fp16 values, w their 2c in the low bits of each half, or'ed with 0x6400.
+__device__ __forceinline__ uint32_t kv_res_pair(uint32_t h2, uint32_t w) {
+  const uint32_t e = h2 & 0x7C007C00u;
+  const uint32_t c1039 = 0x640F640Fu, c2m15 = 0x02000200u;
+  const __half2 k = __hsub2(*reinterpret_cast<const __half2*>(&w), *reinterpret_cast<const __half2*>(&c1039));
+  const __half2 sc = __hmul2(*reinterpret_cast<const __half2*>(&e), *reinterpret_cast<const __half2*>(&c2m15));
+  const __half2 r = __hmul2(k, sc);
+  return *reinterpret_cast<const uint32_t*>(&r);
+}
 __device__ __forceinline__ uint4 kv_res_lo8(uint4 hi, uint32_t codes) {
   const uint32_t twice_lo = (codes << 1) & 0x1E1E1E1Eu;  // 2c of each byte's low nibble
   const uint32_t twice_hi = (codes >> 3) & 0x1E1E1E1Eu;  // 2c of each byte's high nibble
   auto pair = [&](uint32_t h2, uint32_t sel) {
-    uint32_t w = (__byte_perm(twice_lo, twice_hi, sel) & 0x00FF00FFu) | 0x64006400u;
-    uint32_t e = h2 & 0x7C007C00u;
-    const uint32_t c1039 = 0x640F640Fu, c2m15 = 0x02000200u;
-    const __half2 k = __hsub2(*reinterpret_cast<const __half2*>(&w), *reinterpret_cast<const __half2*>(&c1039));
-    const __half2 sc = __hmul2(*reinterpret_cast<const __half2*>(&e), *reinterpret_cast<const __half2*>(&c2m15));
-    const __half2 r = __hmul2(k, sc);
-    return *reinterpret_cast<const uint32_t*>(&r);
+    return kv_res_pair(h2, (__byte_perm(twice_lo, twice_hi, sel) & 0x00FF00FFu) | 0x64006400u);
   };
   return make_uint4(pair(hi.x, 0x0400u), pair(hi.y, 0x0501u), pair(hi.z, 0x0602u), pair(hi.w, 0x0703u));
+}
+// Low parts of two cached fp16 values h2 (element 0 in the low half) from their codes c0, c1.
+__device__ __forceinline__ uint32_t kv_res_lo2(uint32_t h2, uint32_t c0, uint32_t c1) {
+  return kv_res_pair(h2, (c0 << 1) | (c1 << 17) | 0x64006400u);
 }
 
 // ----------------------------------------------------------------------------- bf16 helpers

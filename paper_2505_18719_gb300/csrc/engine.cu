@@ -359,7 +359,7 @@ struct LastRows {
 // decode == true: one query per env row (rows[b] gives env and position), split-K attention.
 // last != nullptr: the last layer computes q|k|v (the KV cache) for all M rows but attention,
 // O, SwiGLU FFN and the residual only for last->rows, whose output lands in h->h_last.
-int forward_layers(vla_handle* h, int M, const RowInfo* rows_dev, bool decode, int n_tiles,
+int forward_layers(vla_handle* h, int M, const RowInfo* rows_dev, bool decode, int n_tiles, int tile_rows,
                    int max_ctx, const LastRows* last = nullptr) {
   const vla_config& c = h->cfg;
   const int d = c.d_model, F = c.d_ffn, H = c.n_heads, hd = c.head_dim;
@@ -409,9 +409,13 @@ int forward_layers(vla_handle* h, int M, const RowInfo* rows_dev, bool decode, i
       prof_end(h, ev, VLA_KCLASS_ATTN_DECODE, 0, 0);
     } else {
       ev = prof_begin(h, VLA_KCLASS_ATTN_PREFILL);
-      // the low plane of the output only where the o projection reads it
-      rc = attn_chunk_tc_launch(h->q, h->ao, h->ao + pd, h->tiles, n_tiles, h->kvl, l, H, hd, h->status, h->stream,
-                                h->fp16, h->num_sms, gemm_reads_lo(M, kProjO));
+      // the low plane of the output only where the o projection reads it; tiles of at most 16
+      // rows (the score pass) on the few-row kernel
+      rc = tile_rows <= kAttnRowsMax
+               ? attn_rows_launch(h->q, h->ao, h->ao + pd, h->tiles, n_tiles, h->kvl, l, H, hd, h->stream, h->fp16,
+                                  gemm_reads_lo(M, kProjO))
+               : attn_chunk_tc_launch(h->q, h->ao, h->ao + pd, h->tiles, n_tiles, h->kvl, l, H, hd, h->status,
+                                      h->stream, h->fp16, h->num_sms, gemm_reads_lo(M, kProjO));
       prof_end(h, ev, VLA_KCLASS_ATTN_PREFILL, 0, 0);
     }
     if (rc) return fail(h, rc, t_err);
@@ -699,7 +703,7 @@ int vla_prefill(vla_handle* h, int batch, const void* visual, int n_visual, cons
   uint8_t* st = static_cast<uint8_t*>(stage_slot(h, &slot));
   RowInfo* rows = reinterpret_cast<RowInfo*>(st);
   AttnTile* tiles = reinterpret_cast<AttnTile*>(rows + total);
-  int n_tiles = 0;
+  int n_tiles = 0, tile_rows = 0;
   std::vector<int> last(batch);
   int r = 0;
   for (int b = 0; b < batch; ++b) {
@@ -708,8 +712,10 @@ int vla_prefill(vla_handle* h, int batch, const void* visual, int n_visual, cons
     if (h->has_pending[b]) rows[r++] = RowInfo{b, pos++, ROW_TOKEN, b};
     for (int j = 0; j < n_visual; ++j) rows[r++] = RowInfo{b, pos++, ROW_VISUAL, b * n_visual + j};
     for (int j = 0; j < lengths[b]; ++j) rows[r++] = RowInfo{b, pos++, ROW_TEXT, b * max_len + j};
-    for (int t0 = 0; t0 < chunk[b]; t0 += 128)
+    for (int t0 = 0; t0 < chunk[b]; t0 += 128) {
       tiles[n_tiles++] = AttnTile{b, r0 + t0, std::min(128, chunk[b] - t0), h->len[b] + t0};
+      tile_rows = std::max(tile_rows, std::min(128, chunk[b] - t0));
+    }
     last[b] = r - 1;
   }
   int* sidx = reinterpret_cast<int*>(tiles + n_tiles);
@@ -737,7 +743,7 @@ int vla_prefill(vla_handle* h, int batch, const void* visual, int n_visual, cons
   prof_end(h, ev, VLA_KCLASS_OTHER, 0, 6.0 * total * c.d_model);
   if (rc) return fail(h, rc, t_err);
   // the last layer runs past q|k|v only for each env's final row, straight into h_last
-  if ((rc = forward_layers(h, static_cast<int>(total), h->rows, false, n_tiles, 0, &lr))) return rc;
+  if ((rc = forward_layers(h, static_cast<int>(total), h->rows, false, n_tiles, tile_rows, 0, &lr))) return rc;
 
   for (int b = 0; b < batch; ++b) {
     h->len[b] += chunk[b];
@@ -811,7 +817,7 @@ int vla_decode_actions(vla_handle* h, const float* uniforms, float temperature, 
       rc = assemble_launch(rows_i, B, nullptr, nullptr, h->fed, h->embed, d, c.vocab, h->h, h->status, h->stream);
       prof_end(h, ev, VLA_KCLASS_OTHER, 0, 6.0 * B * d);
       if (rc) return fail(h, rc, t_err);
-      if ((rc = forward_layers(h, B, rows_i, true, 0, max_len_p + i))) return rc;
+      if ((rc = forward_layers(h, B, rows_i, true, 0, 0, max_len_p + i))) return rc;
     }
     ha.h = (i == 0) ? h->h_last : h->h;
     ha.step = i;
@@ -873,7 +879,7 @@ int vla_score_actions(vla_handle* h, const int32_t* tokens, float temperature, f
     rc = assemble_launch(h->rows, M, nullptr, nullptr, tokens, h->embed, d, c.vocab, h->h, h->status, h->stream);
     prof_end(h, ev, VLA_KCLASS_OTHER, 0, 6.0 * M * d);
     if (rc) return fail(h, rc, t_err);
-    if ((rc = forward_layers(h, M, h->rows, false, n_tiles, 0))) return rc;
+    if ((rc = forward_layers(h, M, h->rows, false, n_tiles, n, 0))) return rc;
   }
   // head inputs: row b*A = prefill's last hidden, rows b*A+1+j = chunk rows
   if (cudaMemcpy2DAsync(h->head_in, static_cast<size_t>(A) * d * sizeof(float), h->h_last, d * sizeof(float),
@@ -1361,6 +1367,37 @@ int vla_op_attn_chunk_res(const float* q, const void* kv, const void* kv_res, in
                                       false, query_num_sms(), true);
   if (rc != VLA_OK && rc != VLA_ERR_CUDA)
     return set_err(nullptr, rc, "vla_op_attn_chunk_res: unsupported arguments or misaligned buffers");
+  return rc;
+}
+
+int vla_op_attn_rows_res(const float* q, const void* kv, const void* kv_res, int max_env, int H, int hd, int cap,
+                         const int32_t* tiles_host, int n_tiles, int rows, int32_t* tiles_dev, void* out_hi,
+                         void* out_lo, void* cuda_stream) {
+  if (!q || !kv || !kv_res || !tiles_host || !tiles_dev || !out_hi || !out_lo || max_env < 1 || H < 1 || cap < 1 ||
+      n_tiles < 1 || rows < 1 || (hd != 64 && hd != 128))
+    return set_err(nullptr, VLA_ERR_ARG, "vla_op_attn_rows_res: bad argument");
+  for (int i = 0; i < n_tiles; ++i) {
+    const int32_t* t = tiles_host + 4 * i;
+    if (t[0] < 0 || t[0] >= max_env || t[2] < 1 || t[2] > kAttnRowsMax || t[3] < 0 || t[3] + t[2] > cap ||
+        t[1] < 0 || t[1] + t[2] > rows)
+      return set_err(nullptr, VLA_ERR_ARG, "vla_op_attn_rows_res: tile outside the buffers or over 16 rows");
+  }
+  cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
+  if (cudaMemcpyAsync(tiles_dev, tiles_host, static_cast<size_t>(n_tiles) * 4 * sizeof(int32_t),
+                      cudaMemcpyHostToDevice, st) != cudaSuccess)
+    return cuda_fail(cudaGetLastError(), "vla_op_attn_rows_res: tile copy");
+  KVLayout L{};
+  L.base = static_cast<f16*>(const_cast<void*>(kv));
+  L.res = static_cast<uint8_t*>(const_cast<void*>(kv_res));
+  L.cap = cap;
+  L.head_stride = static_cast<int64_t>(cap) * hd;
+  L.kv_stride = static_cast<int64_t>(H) * L.head_stride;
+  L.env_stride = 2 * L.kv_stride;
+  L.layer_stride = static_cast<int64_t>(max_env) * L.env_stride;
+  const int rc = attn_rows_launch(q, static_cast<bf16*>(out_hi), static_cast<bf16*>(out_lo),
+                                  reinterpret_cast<const AttnTile*>(tiles_dev), n_tiles, L, 0, H, hd, st, false, true);
+  if (rc != VLA_OK && rc != VLA_ERR_CUDA)
+    return set_err(nullptr, rc, "vla_op_attn_rows_res: unsupported arguments or misaligned buffers");
   return rc;
 }
 

@@ -106,6 +106,7 @@ def load(path: str = LIB_PATH):
         "vla_op_attn_chunk": (i32, [vp, vp, i32, i32, i32, i32, vp, i32, i32, vp, vp, vp, vp]),
         "vla_op_rmsnorm": (i32, [vp, i32, i32, i32, vp, f32, vp, vp, i32, vp]),
         "vla_op_attn_chunk_res": (i32, [vp, vp, vp, i32, i32, i32, i32, vp, i32, i32, vp, vp, vp, vp]),
+        "vla_op_attn_rows_res": (i32, [vp, vp, vp, i32, i32, i32, i32, vp, i32, i32, vp, vp, vp, vp]),
         "vla_op_read_status": (i32, [vp, ctypes.POINTER(u32)]),
         "vla_test_inject_launch_error": (i32, [i64, i32]),
         "vla_test_set_wait_limit_ns": (i32, [ctypes.c_uint64]),
@@ -289,6 +290,16 @@ def vla_op_attn_chunk_res(q_ptr, kv_ptr, res_ptr, max_env, H, hd, cap, tiles, ro
     return load().vla_op_attn_chunk_res(q_ptr or None, kv_ptr or None, res_ptr or None, max_env, H, hd, cap, arr,
                                         len(tiles), rows, tiles_dev_ptr or None, out_hi_ptr or None,
                                         out_lo_ptr or None, stream or None)
+
+
+def vla_op_attn_rows_res(q_ptr, kv_ptr, res_ptr, max_env, H, hd, cap, tiles, rows, tiles_dev_ptr, out_hi_ptr,
+                         out_lo_ptr, stream=0) -> int:
+    """tiles: host sequence of (env, row0, nrows <= 16, pos0); res: the cache's 4-bit codes."""
+    flat = [int(x) for t in tiles for x in t]
+    arr = (ctypes.c_int32 * len(flat))(*flat)
+    return load().vla_op_attn_rows_res(q_ptr or None, kv_ptr or None, res_ptr or None, max_env, H, hd, cap, arr,
+                                       len(tiles), rows, tiles_dev_ptr or None, out_hi_ptr or None,
+                                       out_lo_ptr or None, stream or None)
 
 
 def vla_op_num_sms() -> int:

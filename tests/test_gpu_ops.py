@@ -429,6 +429,57 @@ def test_chunk_attention_tc_matches_fp64(hd):
                                    tiles_dev.data_ptr(), oh.data_ptr(), ol.data_ptr()) == V.VLA_ERR_ARG
 
 
+@pytest.mark.parametrize("hd", [128, 64])
+def test_attn_rows_res_matches_fp64(hd):
+    """The few-row chunk attention (tiles of <= 16 rows) vs brute-force causal softmax attention in
+    fp64 over the cached values (fp16 + residual): 1..16 rows after 0..300 cached positions, tiles
+    crossing a 64-key block boundary, the context reaching the last cache position, NaN past each
+    env's context; a 17-row tile is rejected on the host."""
+    H, cap, max_env = 3, 316, 7
+    chunks = [(0, 0, 1), (1, 0, 16), (2, 7, 5), (3, 300, 16), (4, 100, 6), (5, 60, 9), (6, 63, 1)]
+    rows = sum(n for _, _, n in chunks)
+    x = (I.normal_bf16((max_env, 2, H, cap, hd), 95, hd, 1.0).float()
+         + I.normal_bf16((max_env, 2, H, cap, hd), 95, 7 + hd, 2.0 ** -9).float()).numpy()
+    hi, packed, value = _encode_res4(x)
+    for env, past, n in chunks:
+        hi[env, :, :, past + n:] = np.float16("nan")
+    q = I.normal_bf16((rows, H * hd), 95, 1000 + hd, 1.0).float()
+    tiles, qpos, qenv = [], [], []
+    r = 0
+    for env, past, n in chunks:
+        tiles.append((env, r, n, past))
+        qpos += [past + i for i in range(n)]
+        qenv += [env] * n
+        r += n
+    tiles_dev = torch.zeros(len(tiles) * 4, dtype=torch.int32, device="cuda")
+    oh = torch.full((rows, H * hd), float("nan"), dtype=torch.bfloat16, device="cuda")
+    ol = torch.full_like(oh, float("nan"))
+    qd, kvd, rsd = q.cuda(), torch.from_numpy(hi).cuda(), torch.from_numpy(packed).cuda()
+    rc = V.vla_op_attn_rows_res(qd.data_ptr(), kvd.data_ptr(), rsd.data_ptr(), max_env, H, hd, cap, tiles, rows,
+                                tiles_dev.data_ptr(), oh.data_ptr(), ol.data_ptr())
+    assert rc == 0, V.vla_last_error(None)
+    out = oh.cpu().double() + ol.cpu().double()
+    kv64 = torch.from_numpy(value)
+    kvhi = torch.from_numpy(hi.astype(np.float64))
+    err = err_hi = 0.0
+    for i in range(rows):
+        env, p = qenv[i], qpos[i]
+        for hh in range(H):
+            qi = q[i, hh * hd:(hh + 1) * hd].double()
+            o = out[i, hh * hd:(hh + 1) * hd]
+            K, Vv = kv64[env, 0, hh, :p + 1], kv64[env, 1, hh, :p + 1]
+            w = torch.softmax(K @ qi / math.sqrt(hd), dim=0)
+            err = max(err, float((o - w @ Vv).abs().max()))
+            Kh, Vh = kvhi[env, 0, hh, :p + 1], kvhi[env, 1, hh, :p + 1]
+            wh = torch.softmax(Kh @ qi / math.sqrt(hd), dim=0)
+            err_hi = max(err_hi, float((o - wh @ Vh).abs().max()))
+    assert err < 1e-4, err
+    assert err_hi > 4 * err, (err, err_hi)   # the residual is read, not just the fp16 part
+    bad = [(0, 0, 17, 0)]
+    assert V.vla_op_attn_rows_res(qd.data_ptr(), kvd.data_ptr(), rsd.data_ptr(), max_env, H, hd, cap, bad, rows,
+                                  tiles_dev.data_ptr(), oh.data_ptr(), ol.data_ptr()) == V.VLA_ERR_ARG
+
+
 def _decode_res4(hi: np.ndarray, packed: np.ndarray) -> np.ndarray:
     """The cached values from the fp16 parts and their packed 4-bit codes, from the definition:
     hi + (2c - 15) ulp(hi) / 32 with ulp(hi) = 2^(e-25) (biased exponent e >= 1) or 2^-24."""
@@ -439,23 +490,31 @@ def _decode_res4(hi: np.ndarray, packed: np.ndarray) -> np.ndarray:
     return hi.astype(np.float64) + (2.0 * c - 15.0) * np.ldexp(1.0, np.maximum(e, 1) - 30)
 
 
-@pytest.mark.parametrize("score", [False, True])
-def test_chunk_attention_tc_full_size_sampled(score):
+@pytest.mark.parametrize("score,growing", [(False, False), (True, False), (False, True), (True, True)])
+def test_chunk_attention_tc_full_size_sampled(score, growing):
     """The engine's chunk attention at the bench step's size: 64 envs x 32 heads x 128, contexts
     of 256 + U{16..48} positions in a 320-position cache.  Prefill: each env's whole context as
     one chunk in tiles of <= 128 rows (192 tiles, 6144 (tile, head) items, ~41 per persistent
     CTA); score: 6 rows after the context (64 tiles, 2048 items).  Random fp16 parts and residual
-    codes, NaN past each env's last position; sampled (row, head) outputs vs fp64 brute force."""
+    codes, NaN past each env's last position; sampled (row, head) outputs vs fp64 brute force.
+    growing: logits rising by ~0.2 per key position (dimension 0 of every key grows along the
+    sequence, every query has 8 there), so each 64-key block's maximum exceeds the running one
+    by far more than the kernel's rescale threshold and O is rescaled at every block, while the
+    S products of the following blocks are already in flight."""
     B, H, hd, cap = 64, 32, 128, 320
     ctx = (256 + I.randint_i32((B,), 97, 3, 16, 49)).tolist()
     lens = [6] * B if score else [c - 6 for c in ctx]
     past = [c - 6 for c in ctx] if score else [0] * B
     hi = I.normal_bf16((B, 2, H, cap, hd), 97, 1, 1.0).float().half().numpy()
+    if growing:
+        hi[:, 0, :, :, 0] = (0.21 * np.arange(cap)).astype(np.float16)
     packed = I.randint_i32((B, 2, H, cap, hd // 2), 97, 2, 0, 256).to(torch.uint8).numpy()
     for b in range(B):
         hi[b, :, :, past[b] + lens[b]:] = np.float16("nan")
     rows = sum(lens)
     q = I.normal_bf16((rows, H * hd), 97, 4, 1.0).float()
+    if growing:
+        q[:, ::hd] = 8.0
     tiles, row_env, row_pos, tile_of_row = [], [], [], []
     r = 0
     for b, n in enumerate(lens):
@@ -472,8 +531,16 @@ def test_chunk_attention_tc_full_size_sampled(score):
     assert V.vla_op_attn_chunk_res(qd.data_ptr(), kvd.data_ptr(), rsd.data_ptr(), B, H, hd, cap, tiles, rows,
                                    tiles_dev.data_ptr(), oh.data_ptr(), ol.data_ptr()) == 0
     assert V.vla_op_read_status() == (0, 0)
-    out = oh.cpu().double() + ol.cpu().double()
-    assert torch.isfinite(out).all()
+    outs = [oh.cpu().double() + ol.cpu().double()]
+    if score:
+        # the few-row kernel the engine runs on these tiles
+        oh.fill_(float("nan"))
+        ol.fill_(float("nan"))
+        assert V.vla_op_attn_rows_res(qd.data_ptr(), kvd.data_ptr(), rsd.data_ptr(), B, H, hd, cap, tiles, rows,
+                                      tiles_dev.data_ptr(), oh.data_ptr(), ol.data_ptr()) == 0
+        outs.append(oh.cpu().double() + ol.cpu().double())
+    for out in outs:
+        assert torch.isfinite(out).all()
     rng = np.random.default_rng(11)
     picks = [(int(i), int(h)) for i, h in zip(rng.integers(0, rows, 48), rng.integers(0, H, 48))]
     picks += [(t[1] + t[2] - 1, (k * 7) % H) for k, t in enumerate(tiles[::9])]   # tiles' last rows
@@ -486,7 +553,8 @@ def test_chunk_attention_tc_full_size_sampled(score):
         s = K @ qi / math.sqrt(hd)
         w = np.exp(s - s.max())
         ref = (w / w.sum()) @ Vv
-        err = max(err, float(np.abs(out[i, h * hd:(h + 1) * hd].numpy() - ref).max()))
+        for out in outs:
+            err = max(err, float(np.abs(out[i, h * hd:(h + 1) * hd].numpy() - ref).max()))
     assert err < 1e-4, err
 
 
