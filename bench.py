@@ -64,7 +64,9 @@ def phase_work(sh, past, chunk):
     except that the last layer only needs q|k|v for all rows (KV cache) and the rest for each
     env's final row; attention FLOPs are the causal ones.  Decode bytes are, per forward, all
     weights + the K/V each env reads (positions 0..pos) and writes + the 256 head rows.
-    Score: one weight stream, K/V reads of the 6 teacher-forced rows, 2 P flops per row."""
+    Score: one weight stream, K/V reads of the 6 teacher-forced rows, 2 P flops per row; its
+    projections (384 rows) are tensor-bound, so the pass's floor is max(projection flops at the
+    tensor peak, weights at HBM speed) + the K/V reads at HBM speed."""
     d, F, L = sh.d_model, sh.d_ffn, sh.n_layers
     per_layer = 4 * d * d + 3 * F * d
     qkv_params = 3 * d * d
@@ -87,7 +89,8 @@ def phase_work(sh, past, chunk):
     sc_bytes = w_bytes + sum((p + n) * kv_tok for p in P) + B * n * kv_tok + 2.0 * 256 * d
     sc_flops = 2.0 * params * B * n + L * sum(2.0 * d * (2 * n * p + n * (n + 1)) for p in P)
     return {"prefill_flops": flops_pre, "prefill_flops_all_rows": flops_pre_formula,
-            "decode_bytes": dec_bytes, "score_bytes": sc_bytes, "score_flops": sc_flops, "rows": T}
+            "decode_bytes": dec_bytes, "score_bytes": sc_bytes, "score_flops": sc_flops,
+            "score_gemm_flops": 2.0 * params * B * n, "score_weight_bytes": w_bytes + 2.0 * 256 * d, "rows": T}
 
 
 def peaks():
@@ -733,6 +736,12 @@ def main():
                                "unit": "GB/s", "frac": sw["score_bytes"] / (t_sc / 1e3) / 1e9 / hbm,
                                "tflops": sw["score_flops"] / (t_sc / 1e3) / 1e12,
                                "peak_kind": f"{peak_kind} HBM copy"}
+        # projections tensor-bound at 384 rows: floor = max(their flops at the sustained tensor
+        # peak, the weights at HBM speed) + the K/V reads at HBM speed
+        floor_ms = 1e3 * (max(sw["score_gemm_flops"] / (tf_sus * 1e12), sw["score_weight_bytes"] / (hbm * 1e9))
+                          + (sw["score_bytes"] - sw["score_weight_bytes"]) / (hbm * 1e9))
+        phase_roof["score"]["floor_ms"] = floor_ms
+        phase_roof["score"]["frac_of_floor"] = floor_ms / t_sc
 
     n_gpus = world
     acts = wl.turns * B * A                     # action tokens per step

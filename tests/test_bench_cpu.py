@@ -44,6 +44,9 @@ def test_score_work_64_envs():
     wl, lens, w = _work("7b_b64_ragged_score")
     assert abs(w["score_flops"] / 1e12 - 4.97) < 0.1                 # 2 P x 384 rows + attention
     assert abs(w["score_bytes"] / 1e9 - (12.95 + 12.6)) < 0.5          # weights + cached K/V
+    # the projections alone: 2 P x 64 envs x 6 rows; the weights (+ the 256 head rows)
+    assert abs(w["score_gemm_flops"] - 2.0 * P7B * 64 * 6) < 1.0
+    assert abs(w["score_weight_bytes"] - (2.0 * P7B + 2.0 * 256 * 4096)) < 1.0
 
 
 def test_both_arms_share_the_config():
