@@ -289,20 +289,22 @@ struct RowsSmem {
   static constexpr int PLANE = KB * LD * 2;     // bytes of one staged fp16 block
   static constexpr int CODES = KB * RBP;        // bytes of one staged code block
   static constexpr int STAGE = 2 * PLANE + 2 * CODES;  // K | V | K codes | V codes
-  static constexpr int SMEM = 2 * STAGE;
-  static_assert(STAGE % 16 == 0 && 4 * 16 * HD * 4 + 4 * 16 * 2 * 4 <= SMEM, "staging / merge layout");
+  static constexpr int QPLANE = 16 * LD * 2;            // the tile's 16 query rows, fp16 (hi or lo)
+  static constexpr int SMEM = STAGE + 2 * QPLANE;       // one stage: four CTAs share an SM
+  static_assert(STAGE % 16 == 0 && 4 * 16 * HD * 4 + 4 * 16 * 2 * 4 <= STAGE, "staging / merge layout");
 };
 
 template <int HD>
-__global__ void __launch_bounds__(128) attn_rows_kernel(const float* q, bf16* out_hi, bf16* out_lo,
-                                                        const AttnTile* tiles, KVLayout kv, int layer, int H,
-                                                        float scale_log2, bool fp16, bool write_lo) {
+__global__ void __launch_bounds__(128, 4) attn_rows_kernel(const float* q, bf16* out_hi, bf16* out_lo,
+                                                           const AttnTile* tiles, KVLayout kv, int layer, int H,
+                                                           float scale_log2, bool fp16, bool write_lo) {
   using Sm = RowsSmem<HD>;
-  constexpr int KB = Sm::KB, LD = Sm::LD, RB = Sm::RB, RBP = Sm::RBP, PLANE = Sm::PLANE, STAGE = Sm::STAGE;
+  constexpr int KB = Sm::KB, LD = Sm::LD, RB = Sm::RB, RBP = Sm::RBP, PLANE = Sm::PLANE;
   constexpr int CPR = HD / 8;   // 16-byte chunks of an fp16 row
   constexpr int NT_D = HD / 8;  // n-tiles over the head dim
   constexpr int RWP = RBP / 4;  // 32-bit words of a padded code row
   extern __shared__ __align__(16) uint8_t sm_rows[];
+  uint8_t* qs = sm_rows + Sm::STAGE;  // Q_hi [16][LD], then Q_lo [16][LD]
 
   pdl_launch_dependents();
   pdl_wait();
@@ -321,9 +323,9 @@ __global__ void __launch_bounds__(128) attn_rows_kernel(const float* q, bf16* ou
   const int n_blocks = (n_keys + KB - 1) / KB;
   const int last_pos = n_keys - 1;
 
-  auto load_block = [&](int blk, int buf) {
+  auto load_block = [&](int blk) {
     const int j0 = blk * KB;
-    const uint32_t s0 = smem_u32(sm_rows + buf * STAGE);
+    const uint32_t s0 = smem_u32(sm_rows);
     for (int i = tid; i < KB * CPR; i += 128) {
       const int r = i / CPR, c = i - r * CPR;
       const bool ok = j0 + r < n_keys;
@@ -339,29 +341,36 @@ __global__ void __launch_bounds__(128) attn_rows_kernel(const float* q, bf16* ou
       cp_async16(s0 + 2 * PLANE + Sm::CODES + r * RBP + c * 16, vres + src, ok);
     }
   };
-  load_block(0, 0);
+  load_block(0);
   cp_async_commit();
 
-  // this thread's two rows (g and g + 8 of the tile) and their positions
-  const int ra = min(g, t.nrows - 1), rb = min(g + 8, t.nrows - 1);
-  const int qpos0 = t.pos0 + ra, qpos1 = t.pos0 + rb;
-  // Q A-fragments from the fp32 rows times log2(e) / sqrt(hd), as fp16 hi / lo pairs
-  uint32_t qh[HD / 16][4], ql[HD / 16][4];
+  // the tile's 16 query rows (rows past the last repeat it) times log2(e) / sqrt(hd), as fp16
+  // hi / lo planes: 8 threads per row, HD / 8 values each
   {
-    const float* qa = q + static_cast<size_t>(t.row0 + ra) * d + head * HD + 2 * tq;
-    const float* qb = q + static_cast<size_t>(t.row0 + rb) * d + head * HD + 2 * tq;
+    constexpr int QPT = HD / 8;
+    const int row = tid >> 3, c0 = (tid & 7) * QPT;
+    const float* qr = q + static_cast<size_t>(t.row0 + min(row, t.nrows - 1)) * d + head * HD + c0;
+    float4 x[QPT / 4];
 #pragma unroll
-    for (int kk = 0; kk < HD / 16; ++kk) {
-      const float2 x0 = __ldcg(reinterpret_cast<const float2*>(qa + kk * 16));
-      const float2 x1 = __ldcg(reinterpret_cast<const float2*>(qb + kk * 16));
-      const float2 x2 = __ldcg(reinterpret_cast<const float2*>(qa + kk * 16 + 8));
-      const float2 x3 = __ldcg(reinterpret_cast<const float2*>(qb + kk * 16 + 8));
-      split_h2(x0.x * scale_log2, x0.y * scale_log2, qh[kk][0], ql[kk][0]);
-      split_h2(x1.x * scale_log2, x1.y * scale_log2, qh[kk][1], ql[kk][1]);
-      split_h2(x2.x * scale_log2, x2.y * scale_log2, qh[kk][2], ql[kk][2]);
-      split_h2(x3.x * scale_log2, x3.y * scale_log2, qh[kk][3], ql[kk][3]);
+    for (int i = 0; i < QPT / 4; ++i) x[i] = __ldcg(reinterpret_cast<const float4*>(qr) + i);
+    uint32_t hi[QPT / 2], lo[QPT / 2];
+#pragma unroll
+    for (int i = 0; i < QPT / 4; ++i) {
+      split_h2(x[i].x * scale_log2, x[i].y * scale_log2, hi[2 * i], lo[2 * i]);
+      split_h2(x[i].z * scale_log2, x[i].w * scale_log2, hi[2 * i + 1], lo[2 * i + 1]);
+    }
+#pragma unroll
+    for (int i = 0; i < QPT / 8; ++i) {
+      reinterpret_cast<uint4*>(qs + (row * LD + c0) * 2)[i] = make_uint4(hi[4 * i], hi[4 * i + 1], hi[4 * i + 2], hi[4 * i + 3]);
+      reinterpret_cast<uint4*>(qs + Sm::QPLANE + (row * LD + c0) * 2)[i] =
+          make_uint4(lo[4 * i], lo[4 * i + 1], lo[4 * i + 2], lo[4 * i + 3]);
     }
   }
+  // this thread's two rows (g and g + 8 of the tile) and their positions
+  const int qpos0 = t.pos0 + min(g, t.nrows - 1), qpos1 = t.pos0 + min(g + 8, t.nrows - 1);
+  const uint32_t qh_s = smem_u32(qs), ql_s = qh_s + Sm::QPLANE;
+  // A-fragment address of this lane: row lane % 16, columns + 8 for lanes 16..31
+  const uint32_t qa_off = ((lane & 15) * LD + (lane >> 4) * 8) * 2;
 
   float o[NT_D][4];
 #pragma unroll
@@ -370,45 +379,43 @@ __global__ void __launch_bounds__(128) attn_rows_kernel(const float* q, bf16* ou
   const int im = lane >> 3;  // the ldmatrix sub-matrix this lane addresses
 
   for (int blk = 0; blk < n_blocks; ++blk) {
-    if (blk + 1 < n_blocks) {
-      load_block(blk + 1, (blk + 1) & 1);
-      cp_async_commit();
-      cp_async_wait<1>();
-    } else {
-      cp_async_wait<0>();
-    }
+    cp_async_wait<0>();
     __syncthreads();
     const int k0 = blk * KB + warp * 16;  // this warp's first key
     if (k0 <= last_pos) {
-      const uint8_t* stg = sm_rows + (blk & 1) * STAGE;
-      const uint32_t ks = smem_u32(stg), vs = ks + PLANE;
-      const uint32_t* kc = reinterpret_cast<const uint32_t*>(stg + 2 * PLANE);
-      const uint32_t* vc = reinterpret_cast<const uint32_t*>(stg + 2 * PLANE + Sm::CODES);
+      const uint32_t ks = smem_u32(sm_rows), vs = ks + PLANE;
+      const uint32_t* kc = reinterpret_cast<const uint32_t*>(sm_rows + 2 * PLANE);
+      const uint32_t* vc = reinterpret_cast<const uint32_t*>(sm_rows + 2 * PLANE + Sm::CODES);
       float s[2][4];
 #pragma unroll
-      for (int nt = 0; nt < 2; ++nt) {
-        s[nt][0] = s[nt][1] = s[nt][2] = s[nt][3] = 0.f;
-        const int key = warp * 16 + nt * 8 + (lane & 7);
-        // this thread's B elements are in key row warp*16 + nt*8 + g; the codes of dims
-        // 16kk + 2tq (+1) sit in byte tq of the row's word 2kk (+1 for dims + 8)
-        const uint32_t* crow = kc + (warp * 16 + nt * 8 + g) * RWP;
+      for (int nt = 0; nt < 2; ++nt) s[nt][0] = s[nt][1] = s[nt][2] = s[nt][3] = 0.f;
 #pragma unroll
-        for (int kk = 0; kk < HD / 16; kk += 2) {
+      for (int kk = 0; kk < HD / 16; kk += 2) {
+        uint32_t qh0[4], ql0[4], qh1[4], ql1[4];
+        ldsm_x4(qh_s + qa_off + kk * 32, qh0[0], qh0[1], qh0[2], qh0[3]);
+        ldsm_x4(ql_s + qa_off + kk * 32, ql0[0], ql0[1], ql0[2], ql0[3]);
+        ldsm_x4(qh_s + qa_off + kk * 32 + 32, qh1[0], qh1[1], qh1[2], qh1[3]);
+        ldsm_x4(ql_s + qa_off + kk * 32 + 32, ql1[0], ql1[1], ql1[2], ql1[3]);
+#pragma unroll
+        for (int nt = 0; nt < 2; ++nt) {
+          // this thread's B elements are in key row warp*16 + nt*8 + g; the codes of dims
+          // 16kk + 2tq (+1) sit in byte tq of the row's word 2kk (+1 for dims + 8)
           uint32_t b0, b1, b2, b3;
+          const int key = warp * 16 + nt * 8 + (lane & 7);
           const int dim = (kk + (im >> 1)) * 16 + (im & 1) * 8;
           ldsm_x4(ks + (key * LD + dim) * 2, b0, b1, b2, b3);
-          const uint4 cw = *reinterpret_cast<const uint4*>(crow + 2 * kk);
+          const uint4 cw = *reinterpret_cast<const uint4*>(kc + (warp * 16 + nt * 8 + g) * RWP + 2 * kk);
           const int sh = 8 * tq;
           const uint32_t l0b = kv_res_lo2(b0, (cw.x >> sh) & 15u, (cw.x >> (sh + 4)) & 15u);
           const uint32_t l1b = kv_res_lo2(b1, (cw.y >> sh) & 15u, (cw.y >> (sh + 4)) & 15u);
           const uint32_t l2b = kv_res_lo2(b2, (cw.z >> sh) & 15u, (cw.z >> (sh + 4)) & 15u);
           const uint32_t l3b = kv_res_lo2(b3, (cw.w >> sh) & 15u, (cw.w >> (sh + 4)) & 15u);
-          mma16816(s[nt], qh[kk], b0, b1);
-          mma16816(s[nt], ql[kk], b0, b1);
-          mma16816(s[nt], qh[kk], l0b, l1b);
-          mma16816(s[nt], qh[kk + 1], b2, b3);
-          mma16816(s[nt], ql[kk + 1], b2, b3);
-          mma16816(s[nt], qh[kk + 1], l2b, l3b);
+          mma16816(s[nt], qh0, b0, b1);
+          mma16816(s[nt], ql0, b0, b1);
+          mma16816(s[nt], qh0, l0b, l1b);
+          mma16816(s[nt], qh1, b2, b3);
+          mma16816(s[nt], ql1, b2, b3);
+          mma16816(s[nt], qh1, l2b, l3b);
         }
       }
       // causal mask, online softmax (row g: c 0, 1; row g + 8: c 2, 3)
@@ -484,7 +491,11 @@ __global__ void __launch_bounds__(128) attn_rows_kernel(const float* q, bf16* ou
         mma16816(o[nt + 1], ph, l2b, l3b);
       }
     }
-    __syncthreads();  // this buffer is refilled two blocks later
+    __syncthreads();  // every warp is done with the stage: the next block's copies may land
+    if (blk + 1 < n_blocks) {
+      load_block(blk + 1);
+      cp_async_commit();
+    }
   }
 
   // merge the four warps' partials: O [warp][16][HD] and (max, sum) [warp][16] over the stages
