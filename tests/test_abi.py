@@ -66,6 +66,18 @@ def test_host_argument_errors_without_gpu(lib):
     assert lib.vla_op_rmsnorm(None, 0, 0, 0, None, 1e-6, None, None, 1, None) == V.VLA_ERR_ARG
     assert "vla_op_rmsnorm" in V.vla_last_error(None)
     assert lib.vla_op_read_status(None, None) == V.VLA_ERR_ARG
+    # the chunk attentions check their tiles on the host before any copy or launch: a tile over
+    # the kernel's row limit, outside the env range or past the cache capacity, and null buffers
+    rows_res = lambda tiles, max_env=2, cap=64: V.vla_op_attn_rows_res(16, 16, 16, max_env, 2, 128, cap, tiles, 32,
+                                                                        16, 16, 16)
+    assert rows_res([(0, 0, 17, 0)]) == V.VLA_ERR_ARG                 # 17 rows > 16
+    assert "16 rows" in V.vla_last_error(None)
+    assert rows_res([(2, 0, 4, 0)]) == V.VLA_ERR_ARG                  # env >= max_env
+    assert rows_res([(0, 0, 4, 62)]) == V.VLA_ERR_ARG                 # pos0 + nrows > cap
+    assert rows_res([(0, 30, 4, 0)]) == V.VLA_ERR_ARG                 # row0 + nrows > rows
+    assert V.vla_op_attn_rows_res(0, 16, 16, 2, 2, 128, 64, [(0, 0, 4, 0)], 32, 16, 16, 16) == V.VLA_ERR_ARG
+    assert V.vla_op_attn_rows_res(16, 16, 16, 2, 2, 96, 64, [(0, 0, 4, 0)], 32, 16, 16, 16) == V.VLA_ERR_ARG
+    assert V.vla_op_attn_chunk_res(16, 16, 16, 2, 2, 128, 64, [(0, 0, 129, 0)], 200, 16, 16, 16) == V.VLA_ERR_ARG
     # failure-injection hooks: argument checks, and arming / disarming touch no device
     assert lib.vla_test_inject_launch_error(-1, 701) == V.VLA_ERR_ARG
     assert lib.vla_test_inject_launch_error(3, 0) == V.VLA_ERR_ARG
