@@ -357,6 +357,7 @@ struct LastRows {
 
 // All decoder layers over M rows already assembled in h->h (Llama-2 layer, §3.1).
 // decode == true: one query per env row (rows[b] gives env and position), split-K attention.
+// Otherwise n_tiles attention tiles in h->tiles, the largest of tile_rows rows.
 // last != nullptr: the last layer computes q|k|v (the KV cache) for all M rows but attention,
 // O, SwiGLU FFN and the residual only for last->rows, whose output lands in h->h_last.
 int forward_layers(vla_handle* h, int M, const RowInfo* rows_dev, bool decode, int n_tiles, int tile_rows,
