@@ -271,11 +271,13 @@ __global__ void __launch_bounds__(128) attn_chunk_mma_kernel(const float* q,
 // ------------------------------------------------------------------ few-row chunk (residual cache)
 // Query tiles of at most 16 rows (the teacher-forced action rows of the score pass, Eq. 2, or any
 // chunk that short) against keys 0..pos of their env, the cache read as fp16 + 4-bit residual
-// (hi + lo, KVLayout).  One CTA per (tile, head), 4 warps: key blocks of 64 staged in shared memory
-// by cp.async (fp16 parts and residual codes, two stages; keys past the tile's last position are
-// zero-filled, never read); warp w takes keys 16w .. 16w+15 of every block with one m16n8k16 row
-// tile (rows past the tile's last repeat its last row and are not written), the low parts decoded
-// from the codes beside each B fragment:
+// (hi + lo, KVLayout).  One CTA per (tile, head), 4 warps, 128 registers and one 45 KB stage so
+// that four CTAs share an SM (the other CTAs' blocks are in flight while one computes): key
+// blocks of 64 staged in shared memory by cp.async (fp16 parts and residual codes; keys past the
+// tile's last position are zero-filled, never read), the tile's query rows as an fp16 pair in
+// shared memory (ldmatrix A fragments); warp w takes keys 16w .. 16w+15 of every block with one
+// m16n8k16 row tile (rows past the tile's last repeat its last row and are not written), the low
+// parts decoded from the codes beside each B fragment:
 //   S = Q_hi K_hi + Q_lo K_hi + Q_hi K_lo,   O += P_hi V_hi + P_lo V_hi + P_hi V_lo,
 // online softmax per warp in the exp2 domain (Q pre-scaled by log2(e) / sqrt(hd)); the four warps'
 // (max, sum, O) merge through shared memory at the end.  Each cached byte is read once per (tile,
